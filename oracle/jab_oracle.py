@@ -1,0 +1,325 @@
+"""Float64 CPU oracle for the joint attention-block loss L_JAB and its STE/LSQ scale gradient.
+
+TEST INFRASTRUCTURE ONLY. Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline /
+reference legs may import or run this module. The product path (the C-ABI library and its
+Python binding) never imports it, and it never imports the product path.
+
+Plain, slow, obviously correct: numpy in float64, one step of the paper per function, no
+blocking, fusion or reordering beyond what the definitions state. numpy's matmul is used as a
+library primitive for the projection and the attention products.
+
+What it computes (paper: Section 2.1 Eq. 2, Section 2.2 Eq. 3, App. B "Effective weight of the
+KL term", App. B "Joint STE fine-tuning" Eq. 13, App. C "Models and scope"):
+
+  1. quantizer          v = fl32(w / s), q = clip(round_half_even(v), -qmax, qmax), w_hat = q*s
+  2. joint projection   [Q | K | V] = X W^T  (W = [W_Q; W_K; W_V] in nn.Linear layout)
+  3. RoPE               rotate-half on every Q and K head, positions 0..T-1 per sequence
+  4. attention          A = softmax(Q K^T / sqrt(d_h) + M) V, causal M, GQA head map
+  5. loss               L = ||A(X; W) - A(X; w_hat)||_F^2 / (B * T * Hq * d_h)   (MSE term)
+  6. backward           dL/dw_hat by the attention VJP, then the LSQ rule for dL/ds.
+
+Readings of points the paper leaves open (each is stated where it is used):
+  R1  w/s is the IEEE fp32 quotient and round() is round-half-to-even.
+  R2  the code range is symmetric [-qmax, qmax], qmax = 2^(b-1) - 1.
+  R3  the MSE term is an element-wise mean over B*T*(Hq*d_h) entries; SSE is also returned.
+  R4  only the MSE term (lambda_KL = 0) is on this path.
+  R5  the LSQ branch tests |v| <= qmax on the unrounded quotient v.
+  R6  n_w in (n_w * qmax)^(-1/2) is the group size G; it is exposed as kappa.
+  R7  RoPE is the rotate-half convention with inv_freq_j = theta^(-2j/d_h).
+  R8  GQA: query head h reads key/value head floor(h / (Hq / Hkv)).
+  R9  an all-zero group gets scale 1 at absmax init (any positive scale gives code 0).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+__all__ = [
+    "qmax_of", "expand_groups", "fp32_quotient", "quantize", "init_scales_absmax",
+    "init_scales_minmse", "project", "rope_tables", "apply_rope", "apply_rope_transpose",
+    "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
+    "jab_loss_and_grad", "lsq_factor", "default_kappa",
+]
+
+
+# --------------------------------------------------------------------------------------------
+# 1. Quantizer (Section 2.1, Eq. 2)
+# --------------------------------------------------------------------------------------------
+
+def qmax_of(bits: int) -> int:
+    """qmax = 2^(b-1) - 1 (Eq. 2). b=2 gives the symmetric code set {-1, 0, 1} (reading R2)."""
+    if bits < 2:
+        raise ValueError("bits must be >= 2")
+    return (1 << (bits - 1)) - 1
+
+
+def expand_groups(s: np.ndarray, group_size: int) -> np.ndarray:
+    """One scale per (output row, group): s[o, g] applies to columns g*G .. g*G+G-1 (Section 2.1)."""
+    return np.repeat(np.asarray(s), group_size, axis=1)
+
+
+def fp32_quotient(w: np.ndarray, s_full: np.ndarray) -> np.ndarray:
+    """v = w / s as an IEEE single-precision quotient (reading R1), returned as float64.
+
+    w holds bf16 values and s fp32 values; both convert to float32 exactly.
+    """
+    w32 = np.asarray(w, dtype=np.float32)
+    s32 = np.asarray(s_full, dtype=np.float32)
+    return (w32 / s32).astype(np.float64)
+
+
+def quantize(w: np.ndarray, s: np.ndarray, bits: int, group_size: int):
+    """Eq. 2: Q(w) = clip(round(w/s), -qmax, qmax) * s with a per-(row, group) scale.
+
+    Returns (codes int8, w_hat float64, v float64). w_hat = q * s is exact in float64
+    (|q| < 2^7 times a 24-bit significand).
+    """
+    w = np.asarray(w, dtype=np.float64)
+    s = np.asarray(s, dtype=np.float64)
+    if not np.all(np.isfinite(s)) or np.any(s <= 0):
+        raise ValueError("scales must be finite and > 0")
+    qm = qmax_of(bits)
+    s_full = expand_groups(s, group_size)
+    v = fp32_quotient(w, s_full)
+    q = np.clip(np.rint(v), -qm, qm)          # np.rint rounds half to even
+    w_hat = q * s_full
+    return q.astype(np.int8), w_hat, v
+
+
+def init_scales_absmax(w: np.ndarray, bits: int, group_size: int) -> np.ndarray:
+    """Starting scale max_{i in g} |w[o, i]| / qmax per group, as an fp32 quotient (reading R9)."""
+    w = np.asarray(w, dtype=np.float64)
+    D, d = w.shape
+    amax = np.abs(w).reshape(D, d // group_size, group_size).max(axis=2)
+    s = (amax.astype(np.float32) / np.float32(qmax_of(bits))).astype(np.float32)
+    s[amax == 0] = np.float32(1.0)
+    return s
+
+
+def init_scales_minmse(w: np.ndarray, bits: int, group_size: int, n_grid: int = 80) -> np.ndarray:
+    """Per-group min-MSE grid search over shrunken absmax scales (the warm-start scales).
+
+    Candidates s_k = fl32(s_0 * (100 - k) / 100) for k = 0 .. n_grid-1 (product and quotient
+    in float64, then one rounding to fp32); the chosen scale minimises sum_{i in g}
+    (Q(w_i; s_k) - w_i)^2, ties going to the smallest k.
+    """
+    w = np.asarray(w, dtype=np.float64)
+    D, d = w.shape
+    ng = d // group_size
+    s0 = init_scales_absmax(w, bits, group_size).astype(np.float64)
+    best_err = np.full((D, ng), np.inf)
+    best_s = s0.astype(np.float32).copy()
+    qm = qmax_of(bits)
+    wg = w.reshape(D, ng, group_size)
+    for k in range(n_grid):
+        sk = (s0 * (100 - k) / 100.0).astype(np.float32)
+        v = (wg.astype(np.float32) / sk[:, :, None]).astype(np.float64)
+        q = np.clip(np.rint(v), -qm, qm)
+        err = ((q * sk[:, :, None].astype(np.float64) - wg) ** 2).sum(axis=2)
+        better = err < best_err
+        best_err = np.where(better, err, best_err)
+        best_s = np.where(better, sk, best_s)
+    return best_s.astype(np.float32)
+
+
+# --------------------------------------------------------------------------------------------
+# 2-4. Block forward: projection, RoPE, causal GQA attention (Section 2.1; App. C)
+# --------------------------------------------------------------------------------------------
+
+def project(x: np.ndarray, w: np.ndarray) -> np.ndarray:
+    """Joint projection [Q | K | V] = X W^T with W in nn.Linear layout [D, d] (Section 2.1)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x @ np.asarray(w, dtype=np.float64).T
+
+
+def rope_tables(T: int, head_dim: int, theta: float):
+    """cos/sin [T, d_h/2] of phi = t * theta^(-2j/d_h) (reading R7)."""
+    j = np.arange(head_dim // 2, dtype=np.float64)
+    inv_freq = theta ** (-2.0 * j / head_dim)
+    phi = np.arange(T, dtype=np.float64)[:, None] * inv_freq[None, :]
+    return np.cos(phi), np.sin(phi)
+
+
+def apply_rope(x: np.ndarray, cos: np.ndarray, sin: np.ndarray) -> np.ndarray:
+    """Rotate-half RoPE on x [B, T, H, d_h]:  x'_j = x_j cos - x_{j+h} sin,
+    x'_{j+h} = x_{j+h} cos + x_j sin, with h = d_h/2 and the angle of pair j at position t."""
+    h = x.shape[-1] // 2
+    c = cos[None, :, None, :]
+    s = sin[None, :, None, :]
+    x1, x2 = x[..., :h], x[..., h:]
+    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def apply_rope_transpose(g: np.ndarray, cos: np.ndarray, sin: np.ndarray) -> np.ndarray:
+    """Transpose (= inverse) of the RoPE rotation, applied to gradients."""
+    h = g.shape[-1] // 2
+    c = cos[None, :, None, :]
+    s = sin[None, :, None, :]
+    g1, g2 = g[..., :h], g[..., h:]
+    return np.concatenate([g1 * c + g2 * s, g2 * c - g1 * s], axis=-1)
+
+
+def split_heads(qkv: np.ndarray, n_q_heads: int, n_kv_heads: int, head_dim: int):
+    """[B, T, D] -> Q [B,T,Hq,d_h], K [B,T,Hkv,d_h], V [B,T,Hkv,d_h] (rows Q, then K, then V)."""
+    B, T, _ = qkv.shape
+    nq = n_q_heads * head_dim
+    nk = n_kv_heads * head_dim
+    q = qkv[:, :, :nq].reshape(B, T, n_q_heads, head_dim)
+    k = qkv[:, :, nq:nq + nk].reshape(B, T, n_kv_heads, head_dim)
+    v = qkv[:, :, nq + nk:nq + 2 * nk].reshape(B, T, n_kv_heads, head_dim)
+    return q, k, v
+
+
+def _kv_head(h: int, n_q_heads: int, n_kv_heads: int) -> int:
+    """GQA head map (reading R8)."""
+    return h // (n_q_heads // n_kv_heads)
+
+
+def causal_gqa_attention(q, k, v, scale: float, return_p: bool = False):
+    """A = softmax(Q K^T * scale + M) V per (sequence, query head), causal mask M (Section 2.1).
+
+    q [B,T,Hq,d_h], k/v [B,T,Hkv,d_h] -> O [B,T,Hq,d_h]; optionally P [B,Hq,T,T] and the
+    row log-sum-exp [B,Hq,T] of the scaled scores.
+    """
+    B, T, Hq, dh = q.shape
+    Hkv = k.shape[2]
+    mask = np.triu(np.ones((T, T), dtype=bool), k=1)      # j > t is masked
+    out = np.empty((B, T, Hq, dh))
+    P_all = np.empty((B, Hq, T, T)) if return_p else None
+    lse = np.empty((B, Hq, T))
+    for b in range(B):
+        for h in range(Hq):
+            g = _kv_head(h, Hq, Hkv)
+            S = (q[b, :, h, :] @ k[b, :, g, :].T) * scale
+            S = np.where(mask, -np.inf, S)
+            m = S.max(axis=1, keepdims=True)
+            E = np.exp(S - m)
+            Z = E.sum(axis=1, keepdims=True)
+            P = E / Z
+            out[b, :, h, :] = P @ v[b, :, g, :]
+            lse[b, h, :] = (m + np.log(Z))[:, 0]
+            if return_p:
+                P_all[b, h] = P
+    return out, P_all, lse
+
+
+def _softmax_scale(desc) -> float:
+    sc = float(desc.get("softmax_scale", 0.0) or 0.0)
+    return sc if sc > 0 else 1.0 / np.sqrt(desc["head_dim"])
+
+
+def block_forward(x: np.ndarray, w: np.ndarray, desc: dict, return_parts: bool = False):
+    """Attention output A(X; W) [B, T, Hq*d_h] of one block (merged heads, pre-o_proj)."""
+    B, T, _ = x.shape
+    Hq, Hkv, dh = desc["n_q_heads"], desc["n_kv_heads"], desc["head_dim"]
+    qkv = project(x, w)
+    q, k, v = split_heads(qkv, Hq, Hkv, dh)
+    if desc.get("use_rope", False):
+        cos, sin = rope_tables(T, dh, float(desc.get("rope_theta", 10000.0)))
+        q = apply_rope(q, cos, sin)
+        k = apply_rope(k, cos, sin)
+    o, P, lse = causal_gqa_attention(q, k, v, _softmax_scale(desc), return_p=return_parts)
+    a = o.reshape(B, T, Hq * dh)
+    if return_parts:
+        return a, dict(q=q, k=k, v=v, o=o, P=P, lse=lse)
+    return a
+
+
+# --------------------------------------------------------------------------------------------
+# 5. Loss (Section 2.2, Eq. 3, MSE term; App. B "Effective weight of the KL term")
+# --------------------------------------------------------------------------------------------
+
+def jab_loss(x, w, s, bits: int, desc: dict, a_ref=None):
+    """L_JAB MSE term for one candidate (reading R3, R4).
+
+    a_ref is the teacher output A(X; W) with the float (bf16) weights; it is computed here when
+    not given. Returns dict(loss, sse, sse_parts [B, Hq], codes, w_hat).
+    """
+    G = desc["group_size"]
+    codes, w_hat, _ = quantize(w, s, bits, G)
+    if a_ref is None:
+        a_ref = block_forward(x, w, desc)
+    a_hat = block_forward(x, w_hat, desc)
+    B, T, _ = a_ref.shape
+    Hq, dh = desc["n_q_heads"], desc["head_dim"]
+    err = (a_hat - a_ref).reshape(B, T, Hq, dh)
+    sse_parts = (err ** 2).sum(axis=(1, 3))
+    sse = float(sse_parts.sum())
+    return dict(loss=sse / (B * T * Hq * dh), sse=sse, sse_parts=sse_parts, codes=codes,
+                w_hat=w_hat, a_ref=a_ref, a_hat=a_hat)
+
+
+# --------------------------------------------------------------------------------------------
+# 6. Backward: attention VJP, STE on w_hat, LSQ rule on s (App. B "Joint STE fine-tuning", Eq. 13)
+# --------------------------------------------------------------------------------------------
+
+def attention_vjp(q, k, v, P, dO, scale: float):
+    """Vector-Jacobian product of causal GQA attention.
+
+    dV = P^T dO, dP = dO V^T, dS = P * (dP - rowsum(dP * P)), dQ = dS K * scale,
+    dK = dS^T Q * scale; key/value gradients are summed over the query heads of a group.
+    """
+    B, T, Hq, dh = q.shape
+    Hkv = k.shape[2]
+    dq = np.zeros_like(q)
+    dk = np.zeros_like(k)
+    dv = np.zeros_like(v)
+    for b in range(B):
+        for h in range(Hq):
+            g = _kv_head(h, Hq, Hkv)
+            Ph = P[b, h]
+            dOh = dO[b, :, h, :]
+            dv[b, :, g, :] += Ph.T @ dOh
+            dP = dOh @ v[b, :, g, :].T
+            dS = Ph * (dP - (dP * Ph).sum(axis=1, keepdims=True))
+            dq[b, :, h, :] = (dS @ k[b, :, g, :]) * scale
+            dk[b, :, g, :] += (dS.T @ q[b, :, h, :]) * scale
+    return dq, dk, dv
+
+
+def lsq_factor(v: np.ndarray, bits: int) -> np.ndarray:
+    """Eq. 13: d w_hat / d s = q - v if |v| <= qmax, else sign(v) * qmax (reading R5)."""
+    qm = qmax_of(bits)
+    q = np.clip(np.rint(v), -qm, qm)
+    return np.where(np.abs(v) <= qm, q - v, np.sign(v) * qm)
+
+
+def default_kappa(bits: int, group_size: int) -> float:
+    """LSQ gradient scale (n_w * qmax)^(-1/2) with n_w = G (reading R6)."""
+    return 1.0 / np.sqrt(group_size * qmax_of(bits))
+
+
+def jab_loss_and_grad(x, w, s, bits: int, desc: dict, a_ref=None, kappa: float = 1.0):
+    """L_JAB and its gradient w.r.t. the per-group scales (STE on weights, LSQ on scales).
+
+    Returns dict(loss, sse, grad_s [D, d/G] = kappa * sum_{i in g} dL/dw_hat[o,i] * r[o,i],
+    grad_w_hat [D, d] = dL/dw_hat (the STE weight gradient, d w_hat / d w = 1)).
+    kappa <= 0 selects default_kappa(bits, G).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    G = desc["group_size"]
+    Hq, Hkv, dh = desc["n_q_heads"], desc["n_kv_heads"], desc["head_dim"]
+    B, T, d = x.shape
+    codes, w_hat, v = quantize(w, s, bits, G)
+    if a_ref is None:
+        a_ref = block_forward(x, w, desc)
+    a_hat, parts = block_forward(x, w_hat, desc, return_parts=True)
+    n_el = B * T * Hq * dh
+    diff = a_hat - a_ref
+    sse = float((diff ** 2).sum())
+    dO = (2.0 / n_el) * diff.reshape(B, T, Hq, dh)
+    dq, dk, dv = attention_vjp(parts["q"], parts["k"], parts["v"], parts["P"], dO,
+                               _softmax_scale(desc))
+    if desc.get("use_rope", False):
+        cos, sin = rope_tables(T, dh, float(desc.get("rope_theta", 10000.0)))
+        dq = apply_rope_transpose(dq, cos, sin)
+        dk = apply_rope_transpose(dk, cos, sin)
+    dqkv = np.concatenate([dq.reshape(B, T, Hq * dh), dk.reshape(B, T, Hkv * dh),
+                           dv.reshape(B, T, Hkv * dh)], axis=2)
+    grad_w_hat = dqkv.reshape(B * T, -1).T @ x.reshape(B * T, d)      # [D, d]
+    r = lsq_factor(v, bits)
+    if kappa is None or kappa <= 0:
+        kappa = default_kappa(bits, G)
+    D = grad_w_hat.shape[0]
+    grad_s = kappa * (grad_w_hat * r).reshape(D, d // G, G).sum(axis=2)
+    return dict(loss=sse / n_el, sse=sse, grad_s=grad_s, grad_w_hat=grad_w_hat, codes=codes,
+                w_hat=w_hat, a_ref=a_ref, a_hat=a_hat, lse=parts["lse"])

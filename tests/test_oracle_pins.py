@@ -1,0 +1,365 @@
+"""Pins of the float64 oracle against what the paper and the mathematics fix (CPU only).
+
+Each test names the passage it follows. None of them re-types the oracle's own formula:
+they use hand-worked values, closed forms, invariances, brute force and finite differences.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+from oracle import jab_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _desc(d, Hq, Hkv, dh, G, rope=False, theta=10000.0):
+    return dict(d_model=d, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=dh, group_size=G,
+                use_rope=rope, rope_theta=theta, softmax_scale=0.0)
+
+
+def _bf16(a):
+    """Round float64 values to bf16 (round-to-nearest-even), returned as float64."""
+    a32 = np.asarray(a, dtype=np.float32)
+    u = a32.view(np.uint32).astype(np.uint64)
+    u = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
+    return u.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def _tiny(seed=0, B=2, T=6, d=8, Hq=2, Hkv=1, dh=4, G=4, rope=False, w_std=0.3):
+    rng = np.random.default_rng(seed)
+    desc = _desc(d, Hq, Hkv, dh, G, rope)
+    D = (Hq + 2 * Hkv) * dh
+    x = _bf16(rng.standard_normal((B, T, d)))
+    w = _bf16(rng.standard_normal((D, d)) * w_std)
+    return desc, x, w
+
+
+# ------------------------------------------------------------------ quantizer (Eq. 2, Eq. 13)
+
+def test_quantizer_golden_worked_examples():
+    with open(os.path.join(GOLDEN, "quantizer_worked.json")) as f:
+        fx = json.load(f)
+    for case in fx["cases"]:
+        w = np.array([case["w"]])
+        n = w.shape[1]
+        s = np.array([[case["scale"]]], dtype=np.float32)
+        codes, w_hat, v = O.quantize(w, s, case["bits"], n)
+        assert codes[0].tolist() == case["codes"]
+        np.testing.assert_array_equal(w_hat[0], case["w_hat"])
+        np.testing.assert_array_equal(O.lsq_factor(v, case["bits"])[0], case["lsq"])
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 5, 8])
+def test_quantizer_brute_force_nearest_grid_point(bits):
+    """Eq. 2 equals the nearest point of {-qmax..qmax} to the fp32 quotient, ties to even."""
+    rng = np.random.default_rng(bits)
+    G = 16
+    w = _bf16(rng.standard_normal((6, 64)) * 0.02)
+    s = O.init_scales_absmax(w, bits, G) * np.float32(0.7)   # push some codes past the clamp
+    codes, w_hat, v = O.quantize(w, s, bits, G)
+    qm = (1 << (bits - 1)) - 1
+    grid = np.arange(-qm, qm + 1)
+    for idx in np.ndindex(w.shape):
+        dist = np.abs(v[idx] - grid)
+        best = np.flatnonzero(dist == dist.min())
+        pick = best[0] if len(best) == 1 else [b for b in best if grid[b] % 2 == 0][0]
+        assert codes[idx] == grid[pick], (idx, v[idx])
+    assert codes.min() >= -qm and codes.max() <= qm
+    assert (codes == qm).any() or (codes == -qm).any()
+
+
+def test_quantizer_error_bound_idempotence_and_grid():
+    rng = np.random.default_rng(1)
+    G, bits = 8, 3
+    w = _bf16(rng.standard_normal((4, 32)) * 0.05)
+    s = O.init_scales_absmax(w, bits, G)
+    codes, w_hat, v = O.quantize(w, s, bits, G)
+    s_full = np.repeat(s.astype(np.float64), G, axis=1)
+    inside = np.abs(v) <= (1 << (bits - 1)) - 1
+    assert np.all(np.abs(w_hat - w)[inside] <= s_full[inside] / 2 * (1 + 1e-6))
+    codes2, w_hat2, _ = O.quantize(w_hat, s, bits, G)          # Q(Q(w)) = Q(w)
+    np.testing.assert_array_equal(codes2, codes)
+    np.testing.assert_array_equal(w_hat2, w_hat)
+    # weights built on the grid (powers-of-two scales, exact in bf16) reproduce their codes
+    q = rng.integers(-3, 4, size=(4, 32))
+    s_grid = np.full((4, 4), 2.0 ** -6, dtype=np.float32)
+    w_grid = q * 2.0 ** -6
+    c3, wh3, _ = O.quantize(w_grid, s_grid, bits, G)
+    np.testing.assert_array_equal(c3, q)
+    np.testing.assert_array_equal(wh3, w_grid)
+
+
+def test_absmax_scale_init_maps_group_max_to_qmax():
+    rng = np.random.default_rng(2)
+    w = _bf16(rng.standard_normal((3, 16)) * 0.02)
+    w[1, 8:] = 0.0                                   # all-zero group
+    for bits in (2, 3, 8):
+        s = O.init_scales_absmax(w, bits, 8)
+        codes, _, _ = O.quantize(w, s, bits, 8)
+        qm = (1 << (bits - 1)) - 1
+        for o in range(3):
+            for g in range(2):
+                grp = np.abs(w[o, g * 8:(g + 1) * 8])
+                if grp.max() == 0:
+                    assert s[o, g] == 1.0 and not codes[o, g * 8:(g + 1) * 8].any()
+                else:
+                    assert np.abs(codes[o, g * 8:(g + 1) * 8]).max() == qm
+
+
+def test_minmse_scale_search_brute_force():
+    """Warm-start scales: the chosen scale attains the minimum over all candidates."""
+    rng = np.random.default_rng(3)
+    bits, G = 2, 8
+    w = _bf16(rng.standard_normal((3, 16)) * 0.02)
+    s = O.init_scales_minmse(w, bits, G)
+    s0 = O.init_scales_absmax(w, bits, G).astype(np.float64)
+    for o in range(3):
+        for g in range(2):
+            grp = w[o, g * G:(g + 1) * G]
+            errs = []
+            for k in range(80):
+                sk = np.float32(s0[o, g] * (100 - k) / 100.0)
+                c, wh, _ = O.quantize(grp[None], np.array([[sk]]), bits, G)
+                errs.append(((wh[0] - grp) ** 2).sum())
+            k_best = int(np.argmin(errs))
+            assert s[o, g] == np.float32(s0[o, g] * (100 - k_best) / 100.0)
+            assert errs[k_best] <= errs[0]
+
+
+# ------------------------------------------------------------------ attention (Section 2.1)
+
+def test_attention_golden_worked_example():
+    with open(os.path.join(GOLDEN, "attention_worked.json")) as f:
+        fx = json.load(f)
+    desc = _desc(3, 1, 1, 1, 3)
+    a = O.block_forward(np.array([fx["x"]]), np.array(fx["w"]), desc)
+    np.testing.assert_allclose(a[0, :, 0], fx["a"], rtol=0, atol=1e-14)
+    for case in fx["rope"]["cases"]:
+        dh = case["head_dim"]
+        cos, sin = O.rope_tables(case["t"] + 1, dh, 10000.0)
+        x = np.zeros((1, case["t"] + 1, 1, dh))
+        x[0, case["t"], 0] = case["x"]
+        out = O.apply_rope(x, cos, sin)[0, case["t"], 0]
+        np.testing.assert_allclose(out, case["out"], atol=1e-14)
+
+
+def test_softmax_rows_and_causal_support():
+    desc, x, w = _tiny(rope=True)
+    a, parts = O.block_forward(x, w, desc, return_parts=True)
+    P = parts["P"]
+    np.testing.assert_allclose(P.sum(axis=-1), 1.0, atol=1e-13)
+    assert (P >= 0).all()
+    T = x.shape[1]
+    assert np.all(P[..., np.triu_indices(T, 1)[0], np.triu_indices(T, 1)[1]] == 0)
+
+
+def test_zero_query_weights_give_causal_running_mean():
+    """W_Q = 0: every score is 0, so token t averages V over positions 0..t (GQA map h -> h//r)."""
+    desc, x, w = _tiny(Hq=4, Hkv=2, dh=4, d=8, rope=True)
+    w = w.copy()
+    w[:16] = 0.0                                       # all query rows
+    a = O.block_forward(x, w, desc)
+    B, T, _ = x.shape
+    v = (x @ w[24:32].T).reshape(B, T, 2, 4)           # V rows follow 16 Q rows and 8 K rows
+    counts = np.arange(1, T + 1)[None, :, None, None]
+    mean = np.cumsum(v, axis=1) / counts
+    expect = np.concatenate([mean[:, :, h // 2] for h in range(4)], axis=-1)
+    np.testing.assert_allclose(a, expect, atol=1e-13)
+
+
+def test_causal_invariance_to_future_tokens():
+    desc, x, w = _tiny(T=8, rope=True)
+    s = O.init_scales_absmax(w, 3, desc["group_size"])
+    r1 = O.jab_loss(x, w, s, 3, desc)
+    x2 = x.copy()
+    x2[:, 5:] = _bf16(np.random.default_rng(9).standard_normal(x2[:, 5:].shape))
+    r2 = O.jab_loss(x2, w, s, 3, desc)
+    np.testing.assert_array_equal(r1["a_ref"][:, :5], r2["a_ref"][:, :5])
+    np.testing.assert_array_equal(r1["a_hat"][:, :5], r2["a_hat"][:, :5])
+    assert not np.allclose(r1["a_ref"][:, 5:], r2["a_ref"][:, 5:])
+
+
+def test_query_key_scaling_invariance_with_rope():
+    """L_JAB depends on (W_Q, W_K) only through the scores; W_Q*c, W_K/c leaves A unchanged."""
+    desc, x, w = _tiny(rope=True)
+    a = O.block_forward(x, w, desc)
+    w2 = w.copy()
+    w2[:8] *= 4.0          # Q rows (Hq*dh = 8)
+    w2[8:12] /= 4.0        # K rows
+    np.testing.assert_allclose(O.block_forward(x, w2, desc), a, atol=1e-13)
+
+
+def test_per_head_linear_invariance_without_rope():
+    """Section 2.3 / App. B: W_Q -> W_Q R, W_K -> W_K R^{-T} per head leaves L_JAB unchanged."""
+    for Hq, Hkv in ((2, 2), (4, 2)):
+        desc, x, w = _tiny(Hq=Hq, Hkv=Hkv, dh=4, d=8)
+        a = O.block_forward(x, w, desc)
+        rng = np.random.default_rng(5)
+        w2 = w.copy()
+        r = Hq // Hkv
+        for g in range(Hkv):
+            R = rng.standard_normal((4, 4)) + 3 * np.eye(4)
+            for h in range(g * r, (g + 1) * r):
+                w2[h * 4:(h + 1) * 4] = R.T @ w[h * 4:(h + 1) * 4]           # Q_h -> Q_h R
+            k0 = Hq * 4 + g * 4
+            w2[k0:k0 + 4] = np.linalg.inv(R) @ w[k0:k0 + 4]                   # K_g -> K_g R^{-T}
+        np.testing.assert_allclose(O.block_forward(x, w2, desc), a, atol=1e-11)
+
+
+def test_scalar_head_toy_example_exact_zero_damage():
+    """App. B, d_head = 1: delta_q = eps q with delta_k = -eps/(1+eps) k reproduces q k^T exactly,
+    so the joint loss is zero although both matrices moved."""
+    desc, x, w = _tiny(Hq=1, Hkv=1, dh=1, d=4, G=4)
+    eps = 0.25
+    w2 = w.copy()
+    w2[0] = w[0] * (1 + eps)
+    w2[1] = w[1] - eps / (1 + eps) * w[1]
+    a, a2 = O.block_forward(x, w, desc), O.block_forward(x, w2, desc)
+    np.testing.assert_allclose(a2, a, atol=1e-14)
+
+
+def test_hessian_null_space_dimension_at_float_point():
+    """Section 2.3: the per-head invariance gives H_L a null space of dimension >= n_head*d_head^2.
+
+    At w*, H = 2 J^T J / n (Eq. 5 with lambda_KL = 0), so the null space is that of the Jacobian
+    J = dA/dw, computed here by central differences on a block with more outputs than weights.
+    """
+    for Hq, dh in ((1, 2), (2, 2)):
+        desc = _desc(3, Hq, Hq, dh, 3)
+        rng = np.random.default_rng(11)
+        x = rng.standard_normal((2, 16, 3))
+        D = 3 * Hq * dh
+        w = rng.standard_normal((D, 3)) * 0.7
+        n_w = w.size
+        J = np.empty((2 * 16 * Hq * dh, n_w))
+        h = 1e-5
+        for i in range(n_w):
+            e = np.zeros(n_w)
+            e[i] = h
+            ap = O.block_forward(x, w + e.reshape(w.shape), desc)
+            am = O.block_forward(x, w - e.reshape(w.shape), desc)
+            J[:, i] = ((ap - am) / (2 * h)).ravel()
+        sv = np.linalg.svd(J, compute_uv=False)
+        null = int((sv < 1e-6 * sv[0]).sum())
+        assert null >= Hq * dh * dh, (Hq, dh, sv)
+
+
+# ------------------------------------------------------------------ loss (Section 2.2, Eq. 3)
+
+def test_loss_zero_when_weights_on_grid():
+    desc, x, _ = _tiny(rope=True)
+    rng = np.random.default_rng(4)
+    D, d = 16, 8
+    q = rng.integers(-3, 4, size=(D, d))
+    s = np.full((D, d // 4), 2.0 ** -4, dtype=np.float32)
+    w = q * 2.0 ** -4
+    r = O.jab_loss(x, w, s, 3, desc)
+    assert r["loss"] == 0.0 and r["sse"] == 0.0
+    g = O.jab_loss_and_grad(x, w, s, 3, desc)
+    assert g["loss"] == 0.0 and not g["grad_s"].any()
+
+
+def test_single_token_closed_form():
+    """T = 1: softmax over one key is 1, so A = V; L = ||X (W_V_hat - W_V)^T||^2 / (B Hq d_h)
+    mapped through the GQA head map, and the Q/K scale gradients are exactly zero."""
+    desc, x, w = _tiny(T=1, Hq=4, Hkv=2, dh=4, rope=True)
+    s = O.init_scales_absmax(w, 2, 4)
+    r = O.jab_loss_and_grad(x, w, s, 2, desc, kappa=1.0)
+    _, w_hat, _ = O.quantize(w, s, 2, 4)
+    dv = (x[:, 0] @ (w_hat[24:32] - w[24:32]).T).reshape(-1, 2, 4)   # [B, Hkv, dh]
+    sse = sum(((dv[:, h // 2]) ** 2).sum() for h in range(4))
+    np.testing.assert_allclose(r["sse"], sse, rtol=1e-12)
+    np.testing.assert_allclose(r["loss"], sse / (x.shape[0] * 4 * 4), rtol=1e-12)
+    assert not r["grad_s"][:24].any()
+
+
+def test_loss_quadratic_at_float_point():
+    """Eq. 5: L_JAB is zero and stationary at w*, so L(w* + eps*Delta) / eps^2 tends to
+    ||J_A Delta||^2 / n, with J_A Delta a central-difference directional derivative."""
+    desc, x, w = _tiny(rope=True)
+    rng = np.random.default_rng(6)
+    delta = rng.standard_normal(w.shape) * 0.05
+    a0 = O.block_forward(x, w, desc)
+    n = a0.size
+    ratios = []
+    for eps in (1e-3, 1e-4):
+        ratios.append(((O.block_forward(x, w + eps * delta, desc) - a0) ** 2).sum() / n / eps ** 2)
+    h = 1e-6
+    jvp = (O.block_forward(x, w + h * delta, desc) - O.block_forward(x, w - h * delta, desc)) / (2 * h)
+    gn = (jvp ** 2).sum() / n
+    np.testing.assert_allclose(ratios[1], gn, rtol=1e-3)
+    np.testing.assert_allclose(ratios[0], ratios[1], rtol=3e-2)
+
+
+def test_loss_shrinks_with_bits():
+    """Finer grids shrink the error: L(b) strictly decreases over b = 2..8 on a random block."""
+    desc, x, w = _tiny(T=8, rope=True, w_std=0.5)
+    losses = [O.jab_loss(x, w, O.init_scales_absmax(w, b, 4), b, desc)["loss"] for b in (2, 3, 4, 5, 8)]
+    assert all(l1 > l2 for l1, l2 in zip(losses, losses[1:])), losses
+
+
+# ------------------------------------------------------------------ gradients (Eq. 13)
+
+def _loss_at_w_hat(x, w_hat, desc, a_ref):
+    return ((O.block_forward(x, w_hat, desc) - a_ref) ** 2).sum() / a_ref.size
+
+
+@pytest.mark.parametrize("rope,Hq,Hkv", [(False, 2, 2), (True, 2, 1)])
+def test_weight_gradient_matches_finite_differences(rope, Hq, Hkv):
+    """STE weight gradient dL/dw_hat (Eq. 13, d w_hat / d w = 1) against central differences."""
+    desc, x, w = _tiny(rope=rope, Hq=Hq, Hkv=Hkv, T=5)
+    s = O.init_scales_absmax(w, 3, 4)
+    g = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=1.0)
+    a_ref, w_hat = g["a_ref"], g["w_hat"]
+    h = 1e-6
+    rng = np.random.default_rng(7)
+    idx = [tuple(i) for i in rng.integers(0, [w.shape[0], w.shape[1]], size=(24, 2))]
+    for i in idx:
+        wp, wm = w_hat.copy(), w_hat.copy()
+        wp[i] += h
+        wm[i] -= h
+        fd = (_loss_at_w_hat(x, wp, desc, a_ref) - _loss_at_w_hat(x, wm, desc, a_ref)) / (2 * h)
+        np.testing.assert_allclose(g["grad_w_hat"][i], fd, rtol=1e-5, atol=1e-11)
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+def test_scale_gradient_matches_lsq_surrogate_finite_differences(bits):
+    """LSQ rule (Eq. 13) against central differences of the frozen-code surrogate
+    w_hat(s') = s' q + w (1 - s'/s) where |v| <= qmax, and s' sign(v) qmax elsewhere: its
+    derivative at s' = s is exactly the rule, so FD of L(w_hat(s')) must equal grad_s (kappa=1)."""
+    desc, x, w = _tiny(rope=True, T=5)
+    G = 4
+    s = O.init_scales_absmax(w, bits, G) * np.float32(0.8)
+    g = O.jab_loss_and_grad(x, w, s, bits, desc, kappa=1.0)
+    codes, w_hat, v = O.quantize(w, s, bits, G)
+    qm = (1 << (bits - 1)) - 1
+    inside = np.abs(v) <= qm
+    a_ref = g["a_ref"]
+    h = 1e-7
+    for o in range(w.shape[0]):
+        for gi in range(w.shape[1] // G):
+            cols = slice(gi * G, (gi + 1) * G)
+
+            def surrogate(sp):
+                wh = w_hat.copy()
+                qv = codes[o, cols].astype(np.float64)
+                wv = w[o, cols]
+                ins = inside[o, cols]
+                wh[o, cols] = np.where(ins, sp * qv + wv * (1 - sp / float(s[o, gi])),
+                                       sp * np.sign(v[o, cols]) * qm)
+                return _loss_at_w_hat(x, wh, desc, a_ref)
+
+            s0 = float(s[o, gi])
+            fd = (surrogate(s0 + h) - surrogate(s0 - h)) / (2 * h)
+            np.testing.assert_allclose(g["grad_s"][o, gi], fd, rtol=2e-5, atol=1e-12)
+
+
+def test_kappa_is_a_pure_multiplier_and_default():
+    desc, x, w = _tiny(rope=True)
+    s = O.init_scales_absmax(w, 3, 4)
+    g1 = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=1.0)
+    g2 = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=0.0)
+    np.testing.assert_allclose(g2["grad_s"], g1["grad_s"] / np.sqrt(4 * 3), rtol=1e-14)
+    assert O.default_kappa(3, 128) == 1 / np.sqrt(128 * 3)
