@@ -1,0 +1,147 @@
+/*
+ * jab.h -- C ABI of the GB300 (sm_103a) library for the joint attention-block loss L_JAB.
+ *
+ * L_JAB (Section 2.2, Eq. 3, MSE term) compares the causal, GQA, RoPE attention output of one
+ * transformer block computed with its float weights, A(X; W), against the same block computed with
+ * the joint [W_Q | W_K | W_V] fake-quantised at b bits (Section 2.1, Eq. 2):
+ *
+ *     L_JAB(w_hat) = ||A(X; W) - A(X; w_hat)||_F^2 / (B * T * Hq * d_h)
+ *
+ * and its gradient w.r.t. the per-(row, group) scales uses the straight-through estimator on the
+ * weights and the LSQ rule on the scales (App. B "Joint STE fine-tuning", Eq. 13).
+ *
+ * Conventions shared by every entry point
+ *  - Pointers named *_dev are device pointers owned by the caller; the library never frees or
+ *    retains them after the call is enqueued. Host arrays are named *_host.
+ *  - Every entry point that takes a workspace uses only the caller's workspace `ws` (size from
+ *    jab_workspace_size) for scratch. It allocates no device memory.
+ *  - Calls are asynchronous on `stream`. Host-side argument checks return an error immediately and
+ *    enqueue nothing. Problems found on the device (non-finite or non-positive scales, fp16 range
+ *    overflow, a bounded wait that timed out) set a per-device flag that jab_get_device_status reads.
+ *  - Layouts are row-major. The joint weight uses the nn.Linear layout: row o is output feature o,
+ *    rows [0, Hq*d_h) are W_Q, then Hkv*d_h rows of W_K, then Hkv*d_h rows of W_V (a transpose would
+ *    quantise along the wrong axis). Groups of G consecutive input columns share one scale.
+ *  - bf16 and fp16 tensors are passed as `const void*` holding IEEE-754 binary16 / bfloat16 bits.
+ *  - Supported shapes: head_dim in {64, 128}; d_model a multiple of 64; group_size a multiple of 64
+ *    dividing d_model; n_q_heads a multiple of n_kv_heads; (Hq + 2 Hkv) * head_dim a multiple of 128;
+ *    any B >= 1 and T >= 1 with B * T <= 2^31. Other shapes return JAB_ERR_UNSUPPORTED. Device
+ *    pointers must be 16-byte aligned and the workspace 256-byte aligned.
+ *  - The tensor-core operands of the forward path are fp16 (X and w_hat are converted from their
+ *    bf16 inputs on the device); accumulation is fp32; the loss is summed in fp64.
+ */
+#ifndef JAB_H_
+#define JAB_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same handle type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* jab_stream_t;
+
+typedef enum {
+  JAB_OK = 0,
+  JAB_ERR_INVALID_ARG = 1,   /* NULL pointer, bad size, misaligned pointer, workspace too small   */
+  JAB_ERR_UNSUPPORTED = 2,   /* shape outside the supported set above                            */
+  JAB_ERR_CUDA = 3,          /* a CUDA runtime call or kernel launch failed                      */
+  JAB_ERR_NONFINITE = 4,     /* device: scale <= 0 or non-finite, or a non-finite result          */
+  JAB_ERR_RANGE = 5,         /* device: an input value is outside the fp16 range (|x| > 65504)   */
+  JAB_ERR_TIMEOUT = 6        /* device: a bounded wait in a pipelined kernel gave up             */
+} jab_status;
+
+/* One attention block. Section 2.1 (d, d_head), App. C (Mistral-7B: GQA, RoPE theta = 1e4). */
+typedef struct {
+  int32_t d_model;      /* d: input features of X and columns of W                               */
+  int32_t n_q_heads;    /* Hq                                                                     */
+  int32_t n_kv_heads;   /* Hkv; query head h reads key/value head h / (Hq / Hkv)                  */
+  int32_t head_dim;     /* d_h                                                                    */
+  int32_t group_size;   /* G: input columns per scale                                             */
+  int32_t use_rope;     /* 0: no RoPE (GPT-2); 1: rotate-half RoPE on Q and K, positions 0..T-1    */
+  float rope_theta;     /* RoPE base; inv_freq_j = theta^(-2j/d_h)                                 */
+  float softmax_scale;  /* <= 0 selects 1/sqrt(d_h) (Section 2.1)                                  */
+} jab_block_desc;
+
+/* Bytes of workspace the calls below need for this block, B sequences of T tokens, n_cand candidates
+ * per jab_loss_forward call, with_bwd != 0 for jab_loss_backward_scales. Returns 0 on invalid input.
+ * One workspace sized with (n_cand = max, with_bwd = 1) serves every entry point. */
+size_t jab_workspace_size(const jab_block_desc* desc, int32_t B, int32_t T, int32_t n_cand,
+                          int32_t with_bwd);
+
+/* Teacher pass (Section 2.2: A(X) of the unmodified block; App. B, decision 3: teacher and student
+ * see the same X). Computes A(X; W) once per block; its cost is shared by every candidate.
+ *   X_dev          bf16 [B, T, d_model]
+ *   W_dev          bf16 [(Hq + 2 Hkv) * d_h, d_model]   (nn.Linear layout, see above)
+ *   A_ref_dev      out fp32 [B, T, Hq * d_h]            merged heads, pre-o_proj
+ *   lse_dev        out fp32 [B, Hq, T] or NULL          log-sum-exp of each softmax row
+ *   a_sqnorm_dev   out fp64 [1] or NULL                 ||A_ref||_F^2 (for eps^A = sqrt(SSE/||A||^2)) */
+jab_status jab_reference_forward(const jab_block_desc* desc, int32_t B, int32_t T,
+                                 const void* X_dev, const void* W_dev, float* A_ref_dev,
+                                 float* lse_dev, double* a_sqnorm_dev, void* ws, size_t ws_bytes,
+                                 jab_stream_t stream);
+
+/* Forward L_JAB (Eq. 3, MSE term) for n_cand candidate (bits, scales) pairs of the same block, e.g.
+ * the bit widths scored for the knapsack (Section 2.4). X is read once for all candidates.
+ *   bits_host      int32 [n_cand], each in [2, 8]
+ *   scales_host    host array [n_cand] of device pointers, each fp32 [(Hq+2Hkv)*d_h, d_model/G] > 0
+ *   loss_dev       out fp64 [n_cand]                    SSE_c / (B * T * Hq * d_h)
+ *   sse_parts_dev  out fp64 [n_cand, B, Hq] or NULL     SSE of each (candidate, sequence, query head) */
+jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                            const void* W_dev, const float* A_ref_dev, int32_t n_cand,
+                            const int32_t* bits_host, const float* const* scales_host,
+                            double* loss_dev, double* sse_parts_dev, void* ws, size_t ws_bytes,
+                            jab_stream_t stream);
+
+/* Forward L_JAB and its gradient w.r.t. the scales for one candidate (App. B "Joint STE fine-tuning",
+ * Eq. 13): d w_hat / d w = 1 (STE) and d w_hat / d s = q - v if |v| <= qmax, else sign(v) qmax, with
+ * v = w / s.
+ *   grad_scales_dev out fp32 [(Hq+2Hkv)*d_h, d_model/G] = kappa * sum_{i in group} dL/dw_hat[o,i] * r[o,i]
+ *   kappa          <= 0 selects the LSQ factor (G * qmax)^(-1/2); 1 gives the raw rule
+ *   loss_dev       out fp64 [1] */
+jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                    int32_t bits, const float* scales_dev, float kappa,
+                                    double* loss_dev, float* grad_scales_dev, void* ws,
+                                    size_t ws_bytes, jab_stream_t stream);
+
+/* Quantiser alone (Section 2.1, Eq. 2): v = fl32(w / s), q = clip(round-half-even(v), -qmax, qmax).
+ *   codes_dev      out int8 [(Hq+2Hkv)*d_h, d_model] or NULL
+ *   w_hat_dev      out fp32 [(Hq+2Hkv)*d_h, d_model] or NULL   fl32(q * s) */
+jab_status jab_quantize(const jab_block_desc* desc, int32_t bits, const void* W_dev,
+                        const float* scales_dev, int8_t* codes_dev, float* w_hat_dev,
+                        jab_stream_t stream);
+
+/* Starting scales. mode 0: max_{i in g}|w| / qmax (an all-zero group gets 1). mode 1: the per-group
+ * min-MSE search over s_k = fl32(s_0 * (100 - k) / 100), k = 0..79, minimising
+ * sum_{i in g} (Q(w_i; s_k) - w_i)^2 (ties to the smallest k).
+ *   scales_dev     out fp32 [(Hq+2Hkv)*d_h, d_model/G] */
+jab_status jab_init_scales(const jab_block_desc* desc, int32_t bits, int32_t mode,
+                           const void* W_dev, float* scales_dev, jab_stream_t stream);
+
+/* Synchronises `stream`, then returns and clears the device-side status of the current device
+ * (JAB_OK if no kernel reported a problem since the last call). */
+jab_status jab_get_device_status(jab_stream_t stream);
+
+/* ---- Instrumentation (not part of the method): per-launch-site device time with CUDA events. ----
+ * jab_timing_enable(1) makes every later entry-point call record a CUDA event pair on its stream
+ * around each of its kernel launch sites. jab_timing_collect synchronises those events and folds
+ * them into per-site totals; jab_timing_get(i, ...) reads site i (0 <= i < jab_timing_count()):
+ * its name, the summed device time in ms, the number of recorded ranges and the number of kernels
+ * launched. jab_timing_reset clears the totals. Host-side state, guarded by a mutex. */
+jab_status jab_timing_enable(int32_t on);
+jab_status jab_timing_collect(void);
+int32_t jab_timing_count(void);
+jab_status jab_timing_get(int32_t i, const char** name, double* total_ms, int64_t* ranges,
+                          int64_t* kernels);
+jab_status jab_timing_reset(void);
+
+/* Static, NUL-terminated description of a status code. */
+const char* jab_status_string(jab_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* JAB_H_ */

@@ -1,0 +1,218 @@
+"""ctypes binding of libjab.so (include/jab.h). Argument marshalling only.
+
+Each function has the name of its C entry point, takes torch tensors where the C function takes
+device pointers, checks dtype / device / contiguity (the C side checks shapes, alignment and
+workspace size), calls the library on the current CUDA stream (or the one given), and raises
+JabError on a non-OK status.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+JAB_OK = 0
+_STATUS_NAMES = {0: "JAB_OK", 1: "JAB_ERR_INVALID_ARG", 2: "JAB_ERR_UNSUPPORTED", 3: "JAB_ERR_CUDA",
+                 4: "JAB_ERR_NONFINITE", 5: "JAB_ERR_RANGE", 6: "JAB_ERR_TIMEOUT"}
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def lib_path() -> str:
+    return os.path.join(_HERE, "libjab.so")
+
+
+class JabError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = int(status)
+        super().__init__(f"{where}: {_STATUS_NAMES.get(self.status, self.status)} "
+                         f"({jab_status_string(self.status)})")
+
+
+class BlockDesc(ctypes.Structure):
+    """jab_block_desc: one attention block (Section 2.1; App. C)."""
+
+    _fields_ = [("d_model", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("group_size", ctypes.c_int32), ("use_rope", ctypes.c_int32),
+                ("rope_theta", ctypes.c_float), ("softmax_scale", ctypes.c_float)]
+
+    def as_dict(self) -> dict:
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
+def desc_from_shape(shape, group_size: int) -> BlockDesc:
+    """BlockDesc from a workloads.BlockShape-like object (d_model, heads, head_dim, RoPE)."""
+    return BlockDesc(shape.d_model, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, group_size,
+                     1 if shape.use_rope else 0, float(shape.rope_theta), 0.0)
+
+
+_P = ctypes.c_void_p
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libjab.so; raises if it has not been built (there is no fallback)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = lib_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with `python -m paper_2609_34866_gb300.build` "
+                           "or __graft_entry__.build()")
+    L = ctypes.CDLL(path)
+    D = ctypes.POINTER(BlockDesc)
+    i32, f32, sz = ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+    L.jab_workspace_size.argtypes = [D, i32, i32, i32, i32]
+    L.jab_workspace_size.restype = sz
+    L.jab_reference_forward.argtypes = [D, i32, i32, _P, _P, _P, _P, _P, _P, sz, _P]
+    L.jab_loss_forward.argtypes = [D, i32, i32, _P, _P, _P, i32, ctypes.POINTER(i32),
+                                   ctypes.POINTER(_P), _P, _P, _P, sz, _P]
+    L.jab_loss_backward_scales.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P, _P, sz, _P]
+    L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
+    L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
+    L.jab_get_device_status.argtypes = [_P]
+    L.jab_status_string.argtypes = [i32]
+    L.jab_status_string.restype = ctypes.c_char_p
+    L.jab_timing_enable.argtypes = [i32]
+    L.jab_timing_collect.argtypes = []
+    L.jab_timing_count.argtypes = []
+    L.jab_timing_count.restype = i32
+    L.jab_timing_get.argtypes = [i32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_double),
+                                 ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    L.jab_timing_reset.argtypes = []
+    for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_backward_scales",
+               "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
+               "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
+        getattr(L, fn).restype = i32
+    _LIB = L
+    return L
+
+
+def jab_status_string(status: int) -> str:
+    try:
+        return lib().jab_status_string(int(status)).decode()
+    except RuntimeError:
+        return _STATUS_NAMES.get(int(status), "unknown")
+
+
+def _ptr(t: Optional[torch.Tensor], dtype=None, name="tensor") -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(status: int, where: str):
+    if status != JAB_OK:
+        raise JabError(status, where)
+
+
+def jab_workspace_size(desc: BlockDesc, B: int, T: int, n_cand: int = 1, with_bwd: bool = True) -> int:
+    return int(lib().jab_workspace_size(ctypes.byref(desc), B, T, n_cand, 1 if with_bwd else 0))
+
+
+class Workspace:
+    """A caller-owned device workspace (a uint8 torch tensor) sized by jab_workspace_size."""
+
+    def __init__(self, desc: BlockDesc, B: int, T: int, n_cand: int = 1, with_bwd: bool = True,
+                 device=None):
+        self.nbytes = jab_workspace_size(desc, B, T, n_cand, with_bwd)
+        if self.nbytes == 0:
+            raise JabError(1, "jab_workspace_size")
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8,
+                               device=device or torch.device("cuda", torch.cuda.current_device()))
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+
+def jab_reference_forward(desc, B, T, X, W, A_ref, ws: Workspace, lse=None, a_sqnorm=None,
+                          stream=None):
+    st = lib().jab_reference_forward(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), _ptr(lse, torch.float32, "lse"),
+        _ptr(a_sqnorm, torch.float64, "a_sqnorm"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_reference_forward")
+
+
+def jab_loss_forward(desc, B, T, X, W, A_ref, bits: Sequence[int], scales: Sequence[torch.Tensor],
+                     loss, ws: Workspace, sse_parts=None, stream=None):
+    n = len(bits)
+    if len(scales) != n:
+        raise ValueError("bits and scales must have the same length")
+    bits_arr = (ctypes.c_int32 * n)(*[int(b) for b in bits])
+    sc_arr = (ctypes.c_void_p * n)(*[_ptr(s, torch.float32, "scales") for s in scales])
+    st = lib().jab_loss_forward(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), n, bits_arr, sc_arr,
+        _ptr(loss, torch.float64, "loss"), _ptr(sse_parts, torch.float64, "sse_parts"), ws.ptr,
+        ws.nbytes, _stream(stream))
+    _check(st, "jab_loss_forward")
+
+
+def jab_loss_backward_scales(desc, B, T, X, W, A_ref, bits: int, scales, kappa: float, loss,
+                             grad_scales, ws: Workspace, stream=None):
+    st = lib().jab_loss_backward_scales(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), int(bits), _ptr(scales, torch.float32, "scales"),
+        float(kappa), _ptr(loss, torch.float64, "loss"),
+        _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_loss_backward_scales")
+
+
+def jab_quantize(desc, bits, W, scales, codes=None, w_hat=None, stream=None):
+    st = lib().jab_quantize(ctypes.byref(desc), int(bits), _ptr(W, torch.bfloat16, "W"),
+                            _ptr(scales, torch.float32, "scales"), _ptr(codes, torch.int8, "codes"),
+                            _ptr(w_hat, torch.float32, "w_hat"), _stream(stream))
+    _check(st, "jab_quantize")
+
+
+def jab_init_scales(desc, bits, mode, W, scales, stream=None):
+    st = lib().jab_init_scales(ctypes.byref(desc), int(bits), int(mode),
+                               _ptr(W, torch.bfloat16, "W"), _ptr(scales, torch.float32, "scales"),
+                               _stream(stream))
+    _check(st, "jab_init_scales")
+
+
+def jab_get_device_status(stream=None) -> int:
+    """Synchronises the stream and returns (and clears) the device-side status word."""
+    return int(lib().jab_get_device_status(_stream(stream)))
+
+
+def jab_timing_enable(on: bool = True):
+    _check(lib().jab_timing_enable(1 if on else 0), "jab_timing_enable")
+
+
+def jab_timing_reset():
+    _check(lib().jab_timing_reset(), "jab_timing_reset")
+
+
+def jab_timing_read() -> dict:
+    """Synchronises the recorded events; returns {site: (total_ms, ranges, kernels)}."""
+    L = lib()
+    _check(L.jab_timing_collect(), "jab_timing_collect")
+    out = {}
+    for i in range(L.jab_timing_count()):
+        name = ctypes.c_char_p()
+        ms = ctypes.c_double()
+        rng = ctypes.c_int64()
+        nk = ctypes.c_int64()
+        _check(L.jab_timing_get(i, ctypes.byref(name), ctypes.byref(ms), ctypes.byref(rng),
+                                ctypes.byref(nk)), "jab_timing_get")
+        out[name.value.decode()] = (ms.value, rng.value, nk.value)
+    return out

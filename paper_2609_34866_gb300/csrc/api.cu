@@ -1,0 +1,329 @@
+// C ABI of libjab (include/jab.h): argument validation, workspace carving and kernel sequencing.
+// Every step of the computation runs in the kernels of this library; there is no host fallback.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "path.h"
+#include "timing.h"
+#include "workspace.h"
+
+namespace jab {
+
+__device__ int g_status;  // one per device context: first device-side problem since the last read
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+int* g_status_ptr[kMaxDevices] = {};
+int g_sms[kMaxDevices] = {};
+
+jab_status device_info(int** status, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return JAB_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_status_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return JAB_ERR_CUDA;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return JAB_ERR_CUDA;
+    g_status_ptr[dev] = static_cast<int*>(p);
+    g_sms[dev] = n;
+  }
+  *status = g_status_ptr[dev];
+  *sms = g_sms[dev];
+  return JAB_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+jab_status check_desc(const jab_block_desc* d) {
+  if (d == nullptr) return JAB_ERR_INVALID_ARG;
+  if (d->d_model <= 0 || d->n_q_heads <= 0 || d->n_kv_heads <= 0 || d->head_dim <= 0 ||
+      d->group_size <= 0)
+    return JAB_ERR_INVALID_ARG;
+  if (d->use_rope && !(d->rope_theta > 0.f)) return JAB_ERR_INVALID_ARG;
+  if (d->n_q_heads % d->n_kv_heads != 0) return JAB_ERR_UNSUPPORTED;
+  if (d->head_dim != 64 && d->head_dim != 128) return JAB_ERR_UNSUPPORTED;
+  if (d->d_model % 64 != 0 || d->group_size % 64 != 0 || d->d_model % d->group_size != 0)
+    return JAB_ERR_UNSUPPORTED;
+  if (block_rows(d) % 128 != 0) return JAB_ERR_UNSUPPORTED;
+  return JAB_OK;
+}
+
+jab_status check_bt(int32_t B, int32_t T) {
+  if (B < 1 || T < 1) return JAB_ERR_INVALID_ARG;
+  if ((int64_t)B * T > (int64_t)1 << 31) return JAB_ERR_UNSUPPORTED;
+  return JAB_OK;
+}
+
+float softmax_scale(const jab_block_desc* d) {
+  return d->softmax_scale > 0.f ? d->softmax_scale : (float)(1.0 / sqrt((double)d->head_dim));
+}
+
+#define JAB_TRY(expr)                                   \
+  do {                                                  \
+    if ((expr) != cudaSuccess) return JAB_ERR_CUDA;     \
+  } while (0)
+
+// A timed launch site: `nk` kernels launched by `expr` on stream `st`.
+#define JAB_SITE(name, nk, expr)                        \
+  do {                                                  \
+    TimedSite site_(name, st, nk);                      \
+    if ((expr) != cudaSuccess) return JAB_ERR_CUDA;     \
+  } while (0)
+
+// Projection X W^T (+ RoPE) for C candidates stacked along the output dimension.
+jab_status run_projection(const jab_block_desc* d, int64_t N, int T, int C, const void* x16,
+                          const void* w16, void* qkv, const float* cos_t, const float* sin_t,
+                          cudaStream_t st) {
+  const int D = (int)block_rows(d);
+  const int n_rot = d->use_rope ? (d->n_q_heads + d->n_kv_heads) * d->head_dim : 0;
+  if (use_tc_path())
+    JAB_SITE("proj_gemm", 1, launch_proj_gemm_tc(x16, w16, qkv, N, C * D, d->d_model, D, n_rot, d->head_dim, T,
+                                cos_t, sin_t, st));
+  else
+    JAB_SITE("proj_gemm", 1, launch_proj_gemm_simple(x16, w16, qkv, N, C * D, d->d_model, D, n_rot, d->head_dim, T,
+                                    cos_t, sin_t, st));
+  return JAB_OK;
+}
+
+AttnLaunch attn_launch(const jab_block_desc* d, int B, int T, int C, char* ws,
+                       const Workspace& wp, int* status, cudaStream_t st) {
+  AttnLaunch L{};
+  L.qkv = ws + wp.qkv;
+  L.D = (int)block_rows(d);
+  L.ldq = (int64_t)C * L.D;
+  L.B = B;
+  L.T = T;
+  L.Hq = d->n_q_heads;
+  L.Hkv = d->n_kv_heads;
+  L.dh = d->head_dim;
+  L.C = C;
+  L.scale = softmax_scale(d);
+  L.nP = (T + kPartRows - 1) / kPartRows;
+  L.part = reinterpret_cast<double*>(ws + wp.part);
+  L.status = status;
+  L.stream = st;
+  return L;
+}
+
+}  // namespace
+}  // namespace jab
+
+using namespace jab;
+
+extern "C" {
+
+size_t jab_workspace_size(const jab_block_desc* desc, int32_t B, int32_t T, int32_t n_cand,
+                          int32_t with_bwd) {
+  if (check_desc(desc) != JAB_OK || check_bt(B, T) != JAB_OK || n_cand < 1) return 0;
+  return plan_workspace(desc, B, T, n_cand, with_bwd != 0).total;
+}
+
+jab_status jab_reference_forward(const jab_block_desc* desc, int32_t B, int32_t T,
+                                 const void* X_dev, const void* W_dev, float* A_ref_dev,
+                                 float* lse_dev, double* a_sqnorm_dev, void* ws, size_t ws_bytes,
+                                 jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (!X_dev || !W_dev || !A_ref_dev || !ws) return JAB_ERR_INVALID_ARG;
+  if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) ||
+      (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, B, T, 1, false);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
+  float* cos_t = reinterpret_cast<float*>(w + wp.rope);
+  float* sin_t = cos_t + (int64_t)T * (dh / 2);
+  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
+  JAB_SITE("quantize", 1, launch_quantize(W_dev, nullptr, D, dm, desc->group_size, 0, w + wp.w16, nullptr, nullptr,
+                          status, sms, st));
+  if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
+  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, st)) !=
+      JAB_OK)
+    return s;
+  AttnLaunch L = attn_launch(desc, B, T, 1, w, wp, status, st);
+  L.a_out = A_ref_dev;
+  L.lse = lse_dev;
+  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 0) : launch_attn_fwd_simple(L, 0));
+  if (a_sqnorm_dev)
+    JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0, a_sqnorm_dev, nullptr, st));
+  return JAB_OK;
+}
+
+jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                            const void* W_dev, const float* A_ref_dev, int32_t n_cand,
+                            const int32_t* bits_host, const float* const* scales_host,
+                            double* loss_dev, double* sse_parts_dev, void* ws, size_t ws_bytes,
+                            jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (n_cand < 1 || !bits_host || !scales_host || !X_dev || !W_dev || !A_ref_dev || !loss_dev ||
+      !ws)
+    return JAB_ERR_INVALID_ARG;
+  if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) ||
+      (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  for (int c = 0; c < n_cand; ++c) {
+    if (bits_host[c] < 2 || bits_host[c] > 8 || scales_host[c] == nullptr)
+      return JAB_ERR_INVALID_ARG;
+    if (!aligned16(scales_host[c])) return JAB_ERR_INVALID_ARG;
+  }
+  const Workspace wp = plan_workspace(desc, B, T, n_cand, false);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
+  float* cos_t = reinterpret_cast<float*>(w + wp.rope);
+  float* sin_t = cos_t + (int64_t)T * (dh / 2);
+  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
+  for (int c = 0; c < n_cand; ++c)
+    JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_host[c], D, dm, desc->group_size, bits_host[c],
+                            w + wp.w16 + (size_t)c * D * dm * 2, nullptr, nullptr, status, sms, st));
+  if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
+  if ((s = run_projection(desc, N, T, n_cand, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t,
+                          st)) != JAB_OK)
+    return s;
+  AttnLaunch L = attn_launch(desc, B, T, n_cand, w, wp, status, st);
+  L.a_ref = A_ref_dev;
+  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 1) : launch_attn_fwd_simple(L, 1));
+  const double inv_n = 1.0 / ((double)N * desc->n_q_heads * dh);
+  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, n_cand, B, desc->n_q_heads, L.nP, inv_n, loss_dev,
+                             sse_parts_dev, st));
+  return JAB_OK;
+}
+
+jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                    int32_t bits, const float* scales_dev, float kappa,
+                                    double* loss_dev, float* grad_scales_dev, void* ws,
+                                    size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (bits < 2 || bits > 8 || !X_dev || !W_dev || !A_ref_dev || !scales_dev || !loss_dev ||
+      !grad_scales_dev || !ws)
+    return JAB_ERR_INVALID_ARG;
+  if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) || !aligned16(scales_dev) ||
+      !aligned16(grad_scales_dev) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, B, T, 1, true);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
+  const int G = desc->group_size;
+  float* cos_t = reinterpret_cast<float*>(w + wp.rope);
+  float* sin_t = cos_t + (int64_t)T * (dh / 2);
+  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
+  JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, dm, st));
+  JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_dev, D, dm, G, bits, w + wp.w16, nullptr, nullptr, status,
+                          sms, st));
+  if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
+  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, st)) !=
+      JAB_OK)
+    return s;
+  AttnLaunch L = attn_launch(desc, B, T, 1, w, wp, status, st);
+  L.a_ref = A_ref_dev;
+  L.lse = reinterpret_cast<float*>(w + wp.lse);
+  L.d_o = w + wp.d_o;
+  L.dvec = reinterpret_cast<float*>(w + wp.dvec);
+  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 2) : launch_attn_fwd_simple(L, 2));
+  const double n_el = (double)N * desc->n_q_heads * dh;
+  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el, loss_dev, nullptr,
+                             st));
+  JAB_SITE("attn_bwd", 2, use_tc_path() ? launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt)
+                        : launch_attn_bwd_simple(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt));
+  const double k = kappa > 0.f ? (double)kappa : 1.0 / sqrt((double)G * qmax_of(bits));
+  const float coef = (float)(k * 2.0 / n_el);
+  JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
+  if (use_tc_path())
+    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, w + wp.xt, W_dev, scales_dev, N, D, dm, G, bits, coef,
+                                grad_scales_dev, st));
+  else
+    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_simple(w + wp.dqkvt, w + wp.xt, W_dev, scales_dev, N, D, dm, G, bits,
+                                    coef, grad_scales_dev, st));
+  JAB_SITE("check_finite", 1, launch_check_finite(grad_scales_dev, (int64_t)D * (dm / G), status, st));
+  return JAB_OK;
+}
+
+jab_status jab_quantize(const jab_block_desc* desc, int32_t bits, const void* W_dev,
+                        const float* scales_dev, int8_t* codes_dev, float* w_hat_dev,
+                        jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if (bits < 2 || bits > 8 || !W_dev || !scales_dev || (!codes_dev && !w_hat_dev))
+    return JAB_ERR_INVALID_ARG;
+  if (!aligned16(W_dev) || !aligned16(scales_dev) || (codes_dev && !aligned16(codes_dev)) ||
+      (w_hat_dev && !aligned16(w_hat_dev)))
+    return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  JAB_TRY(launch_quantize(W_dev, scales_dev, (int)block_rows(desc), desc->d_model,
+                          desc->group_size, bits, nullptr, codes_dev, w_hat_dev, status, sms,
+                          reinterpret_cast<cudaStream_t>(stream)));
+  return JAB_OK;
+}
+
+jab_status jab_init_scales(const jab_block_desc* desc, int32_t bits, int32_t mode,
+                           const void* W_dev, float* scales_dev, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if (bits < 2 || bits > 8 || (mode != 0 && mode != 1) || !W_dev || !scales_dev)
+    return JAB_ERR_INVALID_ARG;
+  JAB_TRY(launch_init_scales(W_dev, (int)block_rows(desc), desc->d_model, desc->group_size, bits,
+                             mode, scales_dev, reinterpret_cast<cudaStream_t>(stream)));
+  return JAB_OK;
+}
+
+jab_status jab_get_device_status(jab_stream_t stream) {
+  int* status;
+  int sms;
+  jab_status s = device_info(&status, &sms);
+  if (s != JAB_OK) return s;
+  JAB_TRY(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
+  int v = 0;
+  JAB_TRY(cudaMemcpyFromSymbol(&v, g_status, sizeof(int)));
+  const int zero = 0;
+  JAB_TRY(cudaMemcpyToSymbol(g_status, &zero, sizeof(int)));
+  return static_cast<jab_status>(v);
+}
+
+const char* jab_status_string(jab_status status) {
+  switch (status) {
+    case JAB_OK: return "ok";
+    case JAB_ERR_INVALID_ARG: return "invalid argument";
+    case JAB_ERR_UNSUPPORTED: return "unsupported shape";
+    case JAB_ERR_CUDA: return "CUDA error";
+    case JAB_ERR_NONFINITE: return "non-finite or non-positive value";
+    case JAB_ERR_RANGE: return "input outside the fp16 range";
+    case JAB_ERR_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,64 @@
+// Shared device helpers for the JAB kernels (sm_103a).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/jab.h"
+
+namespace jab {
+
+using half_t = __half;
+using bf16_t = __nv_bfloat16;
+
+// Records the first device-side problem in the per-device status word (0 = OK).
+__device__ __forceinline__ void report(int* status, int code) {
+  if (status != nullptr) atomicCAS(status, 0, code);
+}
+
+__host__ __device__ __forceinline__ int qmax_of(int bits) { return (1 << (bits - 1)) - 1; }
+
+// Eq. 2 with reading R1: v = fl32(w / s) (IEEE round-to-nearest division), q = clip(rint(v)).
+__device__ __forceinline__ float quant_code(float w, float s, int qmax, float* v_out) {
+  const float v = __fdiv_rn(w, s);
+  float q = rintf(v);  // round half to even
+  q = fminf(fmaxf(q, -(float)qmax), (float)qmax);
+  if (v_out) *v_out = v;
+  return q;
+}
+
+// Eq. 13: d w_hat / d s = q - v if |v| <= qmax, else sign(v) * qmax.
+__device__ __forceinline__ float lsq_factor(float w, float s, int qmax) {
+  float v;
+  const float q = quant_code(w, s, qmax, &v);
+  return (fabsf(v) <= (float)qmax) ? (q - v) : copysignf((float)qmax, v);
+}
+
+__device__ __forceinline__ double warp_sum(double x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// Block-wide sum in a fixed order (deterministic); every thread gets the result.
+template <int NT>
+__device__ __forceinline__ double block_sum(double x, double* smem /* >= NT/32 */) {
+  x = warp_sum(x);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) smem[w] = x;
+  __syncthreads();
+  double t = 0.0;
+#pragma unroll
+  for (int i = 0; i < NT / 32; ++i) t += smem[i];
+  return t;
+}
+
+}  // namespace jab

@@ -1,0 +1,48 @@
+// Loss reduction (Eq. 3, MSE term): per-tile fp64 partials -> SSE per (candidate, sequence, head)
+// and L = SSE / (B T Hq d_h). Fixed summation order, so repeated calls give identical bits.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace jab {
+
+__global__ void __launch_bounds__(256) loss_reduce_kernel(const double* __restrict__ part, int B,
+                                                          int Hq, int nP, double inv_n,
+                                                          double* __restrict__ out,
+                                                          double* __restrict__ parts_out) {
+  __shared__ double red[8];
+  const int c = blockIdx.x;
+  const int nbh = B * Hq;
+  double acc = 0.0;
+  for (int i = threadIdx.x; i < nbh; i += blockDim.x) {
+    const double* p = part + ((int64_t)c * nbh + i) * nP;
+    double s = 0.0;
+    for (int k = 0; k < nP; ++k) s += p[k];
+    if (parts_out) parts_out[(int64_t)c * nbh + i] = s;
+    acc += s;
+  }
+  const double tot = block_sum<256>(acc, red);
+  if (threadIdx.x == 0) out[c] = tot * inv_n;
+}
+
+__global__ void check_finite_kernel(const float* __restrict__ x, int64_t n, int* status) {
+  bool bad = false;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    bad |= !isfinite(x[i]);
+  if (__syncthreads_or(bad) && threadIdx.x == 0) report(status, JAB_ERR_NONFINITE);
+}
+
+cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
+                               double* out, double* parts_out, cudaStream_t st) {
+  loss_reduce_kernel<<<C, 256, 0, st>>>(part, B, Hq, nP, inv_n, out, parts_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_check_finite(const float* x, int64_t n, int* status, cudaStream_t st) {
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > 1024) blocks = 1024;
+  check_finite_kernel<<<(unsigned)blocks, 256, 0, st>>>(x, n, status);
+  return cudaGetLastError();
+}
+
+}  // namespace jab

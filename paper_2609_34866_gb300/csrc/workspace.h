@@ -1,0 +1,66 @@
+// Layout of the caller-provided workspace (host-side arithmetic only).
+#pragma once
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/jab.h"
+
+namespace jab {
+
+constexpr int kPartRows = 64;  // query rows per loss partial (one partial per (c, b, h, 64 rows))
+
+struct Workspace {
+  // byte offsets into ws; SIZE_MAX when absent
+  size_t x16;      // fp16 [N, d]            X converted for the fp16 tensor-core path
+  size_t w16;      // fp16 [C, D, d]         w_hat per candidate (or W for the teacher)
+  size_t qkv;      // fp16 [N, C*D]          projected, RoPE-rotated Q|K|V for every candidate
+  size_t rope;     // fp32 [2, T, d_h/2]     cos then sin
+  size_t part;     // fp64 [C, B, Hq, nP]    per-tile partial sums (SSE or ||A||^2)
+  size_t status;   // int32 [4]              reserved
+  // backward only
+  size_t xt;       // bf16 [d, N]            X transposed (K-major operand of the weight gradient)
+  size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
+  size_t lse;      // fp32 [B, Hq, T]        student log-sum-exp
+  size_t dvec;     // fp32 [B, Hq, T]        rowsum(dO * O)
+  size_t dqkvt;    // bf16 [D, N]            dL/d[Q|K|V] (pre-RoPE), transposed
+  size_t total;
+};
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+inline int64_t block_rows(const jab_block_desc* d) {
+  return (int64_t)(d->n_q_heads + 2 * d->n_kv_heads) * d->head_dim;
+}
+
+inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, int64_t C,
+                                bool bwd) {
+  Workspace w;
+  const int64_t N = B * T, D = block_rows(d), dm = d->d_model, dh = d->head_dim;
+  const int64_t nP = (T + kPartRows - 1) / kPartRows;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  w.status = take(64);
+  w.x16 = take((size_t)N * dm * 2);
+  w.w16 = take((size_t)C * D * dm * 2);
+  w.qkv = take((size_t)N * C * D * 2);
+  w.rope = take((size_t)2 * T * (dh / 2) * 4);
+  w.part = take((size_t)C * B * d->n_q_heads * nP * 8);
+  if (bwd) {
+    w.xt = take((size_t)N * dm * 2);
+    w.d_o = take((size_t)N * d->n_q_heads * dh * 2);
+    w.lse = take((size_t)B * d->n_q_heads * T * 4);
+    w.dvec = take((size_t)B * d->n_q_heads * T * 4);
+    w.dqkvt = take((size_t)D * N * 2);
+  } else {
+    w.xt = w.d_o = w.lse = w.dvec = w.dqkvt = SIZE_MAX;
+  }
+  w.total = off;
+  return w;
+}
+
+}  // namespace jab

@@ -1,0 +1,94 @@
+"""Shared helpers of the GPU parity tests: run the C-ABI path and the float64 oracle on the same
+seeded inputs and compare. Test infrastructure only."""
+from __future__ import annotations
+
+from dataclasses import replace
+
+import numpy as np
+import torch
+
+from oracle import jab_oracle as O
+from workloads import BlockShape, Workload, WORKLOADS, make_x, make_block_weights
+
+# Tolerances (stated in the spec bars): attention-output error <= 1e-2 of its RMS, L_JAB
+# relative error <= 1e-2, scale-gradient cosine >= 0.999; integer codes bit-exact.
+A_TOL = 1e-2
+L_TOL = 1e-2
+COS_MIN = 0.999
+
+
+def J():
+    import paper_2609_34866_gb300 as mod
+    return mod
+
+
+def oracle_desc(shape: BlockShape, G: int) -> dict:
+    return dict(d_model=shape.d_model, n_q_heads=shape.n_q_heads, n_kv_heads=shape.n_kv_heads,
+                head_dim=shape.head_dim, group_size=G, use_rope=shape.use_rope,
+                rope_theta=shape.rope_theta, softmax_scale=0.0)
+
+
+def np64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def cosine(a, b) -> float:
+    a = np.asarray(a, np.float64).ravel()
+    b = np.asarray(b, np.float64).ravel()
+    return float(a @ b / (np.linalg.norm(a) * np.linalg.norm(b)))
+
+
+# Small cases: several 64/128-row tiles plus a ragged tail, GQA ratios 1, 2 and 4, both head
+# sizes, both group sizes, RoPE on and off.
+SMALL_CASES = {
+    "gpt2_T200": (WORKLOADS["gpt2_sweep"], 2, 200, 128),
+    "mistral_T130": (WORKLOADS["mistral_block"], 1, 130, 128),
+    "mistral_G64_T70": (WORKLOADS["mistral_ste_long"], 2, 70, 64),
+    "gqa2_T257": (replace(WORKLOADS["mistral_block"],
+                          shape=BlockShape(512, 4, 2, 128, True, 10000.0)), 1, 257, 64),
+    "dh64_gqa4_T65": (replace(WORKLOADS["gpt2_smoke"],
+                              shape=BlockShape(256, 4, 1, 64, True, 500.0)), 2, 65, 128),
+    "gpt2_T1": (WORKLOADS["gpt2_smoke"], 3, 1, 128),
+}
+
+
+class Case:
+    """Seeded inputs of one case, on the GPU and as float64 arrays for the oracle."""
+
+    def __init__(self, wl: Workload, B: int, T: int, G: int, block: int = 0):
+        self.wl, self.B, self.T, self.G = wl, B, T, G
+        self.shape = wl.shape
+        self.desc = J().desc_from_shape(wl.shape, G)
+        self.odesc = oracle_desc(wl.shape, G)
+        x = make_x(wl, batch=B, seq_len=T)
+        w = make_block_weights(wl, block)
+        self.X = x.cuda()
+        self.W = w.cuda()
+        self.x64 = np64(x)
+        self.w64 = np64(w)
+        self.D = wl.shape.d_out
+        self.Hq = wl.shape.n_q_heads
+        self.dh = wl.shape.head_dim
+        self._a_ref_np = None
+
+    def workspace(self, n_cand=1, with_bwd=True):
+        return J().Workspace(self.desc, self.B, self.T, n_cand, with_bwd)
+
+    def gpu_teacher(self, ws=None):
+        ws = ws or self.workspace()
+        A = torch.empty((self.B, self.T, self.Hq * self.dh), dtype=torch.float32, device="cuda")
+        lse = torch.empty((self.B, self.Hq, self.T), dtype=torch.float32, device="cuda")
+        sq = torch.zeros(1, dtype=torch.float64, device="cuda")
+        J().jab_reference_forward(self.desc, self.B, self.T, self.X, self.W, A, ws, lse=lse,
+                                  a_sqnorm=sq)
+        return A, lse, sq
+
+    def oracle_teacher(self):
+        if self._a_ref_np is None:
+            self._a_ref_np = O.block_forward(self.x64, self.w64, self.odesc)
+        return self._a_ref_np
+
+    def gpu_scales(self, bits: int, mode: int = 0) -> torch.Tensor:
+        s = torch.empty((self.D, self.shape.d_model // self.G), dtype=torch.float32, device="cuda")
+        J().jab_init_scales(self.desc, bits, mode, self.W, s)
+        return s
