@@ -82,12 +82,12 @@ float softmax_scale(const jab_block_desc* d) {
 // Projection X W^T (+ RoPE) for C candidates stacked along the output dimension.
 jab_status run_projection(const jab_block_desc* d, int64_t N, int T, int C, const void* x16,
                           const void* w16, void* qkv, const float* cos_t, const float* sin_t,
-                          cudaStream_t st) {
+                          int* status, cudaStream_t st) {
   const int D = (int)block_rows(d);
   const int n_rot = d->use_rope ? (d->n_q_heads + d->n_kv_heads) * d->head_dim : 0;
   if (use_tc_path())
-    JAB_SITE("proj_gemm", 1, launch_proj_gemm_tc(x16, w16, qkv, N, C * D, d->d_model, D, n_rot, d->head_dim, T,
-                                cos_t, sin_t, st));
+    JAB_SITE("proj_gemm", 1, launch_proj_gemm_tc(x16, w16, qkv, N, C * D, d->d_model, D, n_rot,
+                                                 d->head_dim, T, cos_t, sin_t, status, st));
   else
     JAB_SITE("proj_gemm", 1, launch_proj_gemm_simple(x16, w16, qkv, N, C * D, d->d_model, D, n_rot, d->head_dim, T,
                                     cos_t, sin_t, st));
@@ -153,7 +153,7 @@ jab_status jab_reference_forward(const jab_block_desc* desc, int32_t B, int32_t 
   JAB_SITE("quantize", 1, launch_quantize(W_dev, nullptr, D, dm, desc->group_size, 0, w + wp.w16, nullptr, nullptr,
                           status, sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
-  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, st)) !=
+  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, status, st)) !=
       JAB_OK)
     return s;
   AttnLaunch L = attn_launch(desc, B, T, 1, w, wp, status, st);
@@ -201,7 +201,7 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
                             w + wp.w16 + (size_t)c * D * dm * 2, nullptr, nullptr, status, sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
   if ((s = run_projection(desc, N, T, n_cand, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t,
-                          st)) != JAB_OK)
+                          status, st)) != JAB_OK)
     return s;
   AttnLaunch L = attn_launch(desc, B, T, n_cand, w, wp, status, st);
   L.a_ref = A_ref_dev;
@@ -239,11 +239,11 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   float* cos_t = reinterpret_cast<float*>(w + wp.rope);
   float* sin_t = cos_t + (int64_t)T * (dh / 2);
   JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
-  JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, dm, st));
+  JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, wp.ldt, dm, st));
   JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_dev, D, dm, G, bits, w + wp.w16, nullptr, nullptr, status,
                           sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
-  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, st)) !=
+  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, w + wp.qkv, cos_t, sin_t, status, st)) !=
       JAB_OK)
     return s;
   AttnLaunch L = attn_launch(desc, B, T, 1, w, wp, status, st);
@@ -251,6 +251,7 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   L.lse = reinterpret_cast<float*>(w + wp.lse);
   L.d_o = w + wp.d_o;
   L.dvec = reinterpret_cast<float*>(w + wp.dvec);
+  L.ldt = wp.ldt;
   JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 2) : launch_attn_fwd_simple(L, 2));
   const double n_el = (double)N * desc->n_q_heads * dh;
   JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el, loss_dev, nullptr,
@@ -261,11 +262,13 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   const float coef = (float)(k * 2.0 / n_el);
   JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
   if (use_tc_path())
-    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, w + wp.xt, W_dev, scales_dev, N, D, dm, G, bits, coef,
-                                grad_scales_dev, st));
+    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, w + wp.xt, wp.ldt, W_dev, scales_dev,
+                                                 N, D, dm, G, bits, coef, grad_scales_dev, status,
+                                                 st));
   else
-    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_simple(w + wp.dqkvt, w + wp.xt, W_dev, scales_dev, N, D, dm, G, bits,
-                                    coef, grad_scales_dev, st));
+    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_simple(w + wp.dqkvt, w + wp.xt, wp.ldt, W_dev,
+                                                     scales_dev, N, D, dm, G, bits, coef,
+                                                     grad_scales_dev, st));
   JAB_SITE("check_finite", 1, launch_check_finite(grad_scales_dev, (int64_t)D * (dm / G), status, st));
   return JAB_OK;
 }

@@ -108,9 +108,11 @@ __global__ void __launch_bounds__(256) attn_fwd_simple_kernel(AttnArgs a) {
     }
     m = mt;
   }
-  const float inv_l = 1.f / l;
+  // Explicitly rounded ops: the teacher (mode 0) and the student (modes 1, 2) must produce the same
+  // bits for the same inputs, so no FMA contraction may differ between the modes.
+  const float inv_l = __fdiv_rn(1.f, l);
 #pragma unroll
-  for (int k = 0; k < DQ; ++k) o[k] *= inv_l;
+  for (int k = 0; k < DQ; ++k) o[k] = __fmul_rn(o[k], inv_l);
   const float lse = (m + log2f(l)) * kLn2;
   const int64_t orow = (rowbase + te) * (int64_t)(a.Hq * DH) + (int64_t)h * DH + qd * DQ;
   double acc = 0.0;
@@ -127,7 +129,7 @@ __global__ void __launch_bounds__(256) attn_fwd_simple_kernel(AttnArgs a) {
     float sq = 0.f, dsum = 0.f;
 #pragma unroll
     for (int k = 0; k < DQ; ++k) {
-      const float e = o[k] - a.a_ref[orow + k];
+      const float e = __fsub_rn(o[k], a.a_ref[orow + k]);
       sq += e * e;
       if (MODE == 2) {
         const half_t e16 = __float2half_rn(e);
@@ -314,7 +316,7 @@ cudaError_t launch_attn_bwd_simple(const AttnLaunch& L, const float* cos_t, cons
                                    int use_rope, void* dqkvt) {
   AttnArgs a{(const half_t*)L.qkv, L.ldq, L.D, L.B, L.T, L.Hq, L.Hkv, L.scale, L.nP, L.part,
              L.a_ref, L.a_out, L.lse, (half_t*)L.d_o, L.dvec, L.status};
-  const int64_t N = (int64_t)L.B * L.T;
+  const int64_t N = L.ldt;  // row pitch of dQKV^T
   dim3 gq((unsigned)((L.T + 63) / 64), (unsigned)L.Hq, (unsigned)L.B);
   dim3 gk((unsigned)((L.T + 63) / 64), (unsigned)L.Hkv, (unsigned)L.B);
   if (L.dh == 128) {

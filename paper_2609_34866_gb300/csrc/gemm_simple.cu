@@ -97,9 +97,9 @@ __global__ void __launch_bounds__(256) proj_gemm_simple_kernel(
 // Tile 64 (o) x 64 (i) x 32 (n), 256 threads, thread owns rows ty + 16 a, columns tx + 16 b.
 // The 64 columns of a tile lie in one quantisation group (G is a multiple of 64).
 __global__ void __launch_bounds__(256) wgrad_lsq_simple_kernel(
-    const bf16_t* __restrict__ dqkvt, const bf16_t* __restrict__ xt, const bf16_t* __restrict__ w,
-    const float* __restrict__ s, int64_t N, int D, int d, int G, int bits, float coef,
-    float* __restrict__ ds) {
+    const bf16_t* __restrict__ dqkvt, const bf16_t* __restrict__ xt, int64_t ldt,
+    const bf16_t* __restrict__ w, const float* __restrict__ s, int64_t N, int D, int d, int G,
+    int bits, float coef, float* __restrict__ ds) {
   __shared__ float As[32][64 + 1];
   __shared__ float Bs[32][64 + 1];
   __shared__ float red[64][17];
@@ -110,15 +110,15 @@ __global__ void __launch_bounds__(256) wgrad_lsq_simple_kernel(
   for (int a = 0; a < 4; ++a)
 #pragma unroll
     for (int b = 0; b < 4; ++b) acc[a][b] = 0.f;
-  const bool vec = (N % 8) == 0;
+  const bool vec = (ldt % 8) == 0;
   for (int64_t n0 = 0; n0 < N; n0 += 32) {
     {  // 64 rows x 32 n of each operand: thread loads 8 consecutive n of one row
       const int r = tid >> 2, nn = (tid & 3) * 8;
       const int64_t n = n0 + nn;
       float va[8], vb[8];
-      if (vec && n + 8 <= N) {  // 16-byte loads need row starts aligned: N % 8 == 0
-        uint4 ua = *reinterpret_cast<const uint4*>(dqkvt + (int64_t)(o0 + r) * N + n);
-        uint4 ub = *reinterpret_cast<const uint4*>(xt + (int64_t)(i0 + r) * N + n);
+      if (vec && n + 8 <= N) {  // 16-byte loads need row starts aligned: ldt % 8 == 0
+        uint4 ua = *reinterpret_cast<const uint4*>(dqkvt + (int64_t)(o0 + r) * ldt + n);
+        uint4 ub = *reinterpret_cast<const uint4*>(xt + (int64_t)(i0 + r) * ldt + n);
         const bf16_t* ha = reinterpret_cast<const bf16_t*>(&ua);
         const bf16_t* hb = reinterpret_cast<const bf16_t*>(&ub);
 #pragma unroll
@@ -130,8 +130,8 @@ __global__ void __launch_bounds__(256) wgrad_lsq_simple_kernel(
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const bool ok = n + e < N;
-          va[e] = ok ? __bfloat162float(dqkvt[(int64_t)(o0 + r) * N + n + e]) : 0.f;
-          vb[e] = ok ? __bfloat162float(xt[(int64_t)(i0 + r) * N + n + e]) : 0.f;
+          va[e] = ok ? __bfloat162float(dqkvt[(int64_t)(o0 + r) * ldt + n + e]) : 0.f;
+          vb[e] = ok ? __bfloat162float(xt[(int64_t)(i0 + r) * ldt + n + e]) : 0.f;
         }
       }
 #pragma unroll
@@ -189,11 +189,11 @@ cudaError_t launch_proj_gemm_simple(const void* A, const void* Bw, void* C, int6
   return cudaGetLastError();
 }
 
-cudaError_t launch_wgrad_lsq_simple(const void* dqkvt, const void* xt, const void* w,
+cudaError_t launch_wgrad_lsq_simple(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
                                     const float* s, int64_t N, int D, int d, int G, int bits,
                                     float coef, float* ds, cudaStream_t st) {
   dim3 grid((unsigned)(d / 64), (unsigned)(D / 64));
-  wgrad_lsq_simple_kernel<<<grid, 256, 0, st>>>((const bf16_t*)dqkvt, (const bf16_t*)xt,
+  wgrad_lsq_simple_kernel<<<grid, 256, 0, st>>>((const bf16_t*)dqkvt, (const bf16_t*)xt, ldt,
                                                 (const bf16_t*)w, s, N, D, d, G, bits, coef, ds);
   return cudaGetLastError();
 }

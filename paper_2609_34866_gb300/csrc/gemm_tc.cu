@@ -1,0 +1,428 @@
+// Tensor-core (tcgen05) GEMMs of the L_JAB path on sm_103a.
+//
+//   C[m, n] = sum_k A[m, k] B[n, k]        A, B K-major 16-bit, fp32 accumulation in TMEM
+//
+// Persistent, warp-specialised kernel, one CTA per SM:
+//   warp 0      TMA producer: 128x64 A tile and 256x64 B tile per stage, 4-stage mbarrier ring
+//   warp 1      TMEM owner and UMMA issuer (one thread): 4 x tcgen05.mma M128 N256 K16 per stage
+//   warps 2..5  epilogue: tcgen05.ld of the 128 x 256 fp32 accumulator, one TMEM lane per thread
+// Two accumulators (2 x 256 TMEM columns) let the epilogue of one tile overlap the next mainloop.
+//
+// Epilogues:
+//   projection  [Q|K|V] = X w_hat^T: rotate-half RoPE on the Q and K heads (partner column +-d_h/2
+//               lives in the same thread's row), fp16 store.
+//   wgrad       G = dQKV^T X (K = tokens, split-K): ds[o, g] += coef * sum_{i in g} G[o,i] r[o,i]
+//               with the LSQ factor r of Eq. 13 recomputed from w and s; G is never stored.
+#include <cudaTypedefs.h>
+
+#include "path.h"
+#include "tc.cuh"
+
+namespace jab {
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int NUM_THREADS = 192;
+constexpr uint32_t TMEM_COLS = 2 * BN;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+
+enum EpiKind { kEpiRope = 0, kEpiLsq = 1 };
+
+struct GemmParams {
+  int64_t M;
+  int Nn, K;
+  int num_m, num_n, splits, k_blocks, group_m;
+  int* status;
+  // projection epilogue
+  half_t* C;
+  int D, n_rot, dh, T;
+  const float* cos_t;
+  const float* sin_t;
+  // LSQ epilogue
+  const bf16_t* w;
+  const float* s;
+  int d, G, bits;
+  float coef;
+  float* ds;
+};
+
+struct Bars {
+  uint64_t full[STAGES], empty[STAGES], tfull[2], tempty[2], drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ void decode_unit(const GemmParams& p, int unit, int& mb, int& nb,
+                                            int& ks) {
+  const int tiles = p.num_m * p.num_n;
+  ks = unit / tiles;
+  const int t = unit - ks * tiles;
+  const int span = p.group_m * p.num_n;
+  const int grp = t / span;
+  const int first_m = grp * p.group_m;
+  const int gm = min(p.group_m, p.num_m - first_m);
+  const int local = t - grp * span;
+  mb = first_m + local % gm;
+  nb = local / gm;
+}
+
+__device__ __forceinline__ void k_range(const GemmParams& p, int ks, int& kb0, int& kb1) {
+  kb0 = (int)((int64_t)p.k_blocks * ks / p.splits);
+  kb1 = (int)((int64_t)p.k_blocks * (ks + 1) / p.splits);
+}
+
+// Waits for a barrier phase while draining at exit: time-bounded, ignores the abort flag.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = tc::globaltimer();
+  while (!tc::mbar_test(bar, parity)) {
+    if (tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
+  }
+}
+
+__device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, int mb, int nb,
+                                         int row) {
+  const int64_t m = (int64_t)mb * BM + row;
+  const bool row_ok = m < p.M;
+  const int t = row_ok ? (int)(m % p.T) : 0;
+  const int half = p.dh >> 1;
+#pragma unroll 1
+  for (int pr = 0; pr < BN / 64; ++pr) {
+    const int c1 = (p.dh == 128) ? (pr >> 1) * 4 + (pr & 1) : pr * 2;
+    const int c2 = c1 + half / 32;
+    const int col1 = nb * BN + c1 * 32;
+    if (col1 >= p.Nn) continue;  // uniform over the warp
+    uint32_t ra[32], rb[32];
+    __syncwarp();  // tcgen05.ld is warp-collective (.sync.aligned)
+    tc::tmem_ld32(taddr + c1 * 32, ra);
+    tc::tmem_ld32(taddr + c2 * 32, rb);
+    tc::tmem_ld_wait();
+    float a[32], b[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      a[i] = __uint_as_float(ra[i]);
+      b[i] = __uint_as_float(rb[i]);
+    }
+    const int o = col1 % p.D;
+    if (p.n_rot > 0 && o < p.n_rot) {
+      const int jj0 = o % p.dh;
+      const float4* cp = reinterpret_cast<const float4*>(p.cos_t + (int64_t)t * half + jj0);
+      const float4* sp = reinterpret_cast<const float4*>(p.sin_t + (int64_t)t * half + jj0);
+#pragma unroll
+      for (int v = 0; v < 8; ++v) {
+        const float4 c4 = __ldg(cp + v), s4 = __ldg(sp + v);
+        const float cs[4] = {c4.x, c4.y, c4.z, c4.w}, sn[4] = {s4.x, s4.y, s4.z, s4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int i = v * 4 + e;
+          const float x1 = a[i], x2 = b[i];
+          a[i] = x1 * cs[e] - x2 * sn[e];
+          b[i] = x2 * cs[e] + x1 * sn[e];
+        }
+      }
+    }
+    if (row_ok) {
+      uint4* d1 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1);
+      uint4* d2 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1 + half);
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        uint4 u1, u2;
+        __half2* h1 = reinterpret_cast<__half2*>(&u1);
+        __half2* h2 = reinterpret_cast<__half2*>(&u2);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          h1[e] = __floats2half2_rn(a[v * 8 + 2 * e], a[v * 8 + 2 * e + 1]);
+          h2[e] = __floats2half2_rn(b[v * 8 + 2 * e], b[v * 8 + 2 * e + 1]);
+        }
+        d1[v] = u1;
+        d2[v] = u2;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int mb, int nb,
+                                        int row) {
+  const int o = mb * BM + row;  // M = D is a multiple of 128: every row is valid
+  const int qmax = qmax_of(p.bits);
+  const int ng = p.d / p.G;
+  float part = 0.f;
+  int cur = -1;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int i0 = nb * BN + c * 32;
+    if (i0 >= p.Nn) break;  // uniform over the warp
+    uint32_t r[32];
+    __syncwarp();
+    tc::tmem_ld32(taddr + c * 32, r);
+    tc::tmem_ld_wait();
+    const int g = i0 / p.G;
+    const float sc = __ldg(p.s + (int64_t)o * ng + g);
+    const uint4* wp = reinterpret_cast<const uint4*>(p.w + (int64_t)o * p.d + i0);
+    float acc = 0.f;
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const uint4 u = __ldg(wp + v);
+      const bf16_t* wb = reinterpret_cast<const bf16_t*>(&u);
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        acc = fmaf(__uint_as_float(r[v * 8 + e]), lsq_factor(__bfloat162float(wb[e]), sc, qmax),
+                   acc);
+    }
+    if (g != cur) {
+      if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
+      part = 0.f;
+      cur = g;
+    }
+    part += acc;
+  }
+  if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
+}
+
+template <int EPI, bool BF16>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  Bars* bars = reinterpret_cast<Bars*>(smem + STAGES * STAGE_BYTES);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int total = p.num_m * p.num_n * p.splits;
+  volatile int* abort = &bars->abort;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      tc::mbar_init(&bars->full[s], 1);
+      tc::mbar_init(&bars->empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(&bars->tfull[a], 1);
+      tc::mbar_init(&bars->tempty[a], 4);
+    }
+    tc::mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tmA);
+    tc::prefetch_tmap(&tmB);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = bars->tmem_base;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, last_parity = 0;  // per-stage bitmasks for the exit drain
+      for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x) {
+        int mb, nb, ks, kb0, kb1;
+        decode_unit(p, unit, mb, nb, ks);
+        k_range(p, ks, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!tc::mbar_wait(&bars->empty[stage], phase ^ 1, abort, p.status)) break;
+          uint8_t* sa = smem + stage * STAGE_BYTES;
+          tc::mbar_expect_tx(&bars->full[stage], STAGE_BYTES);
+          tc::tma_load_2d(sa, &tmA, &bars->full[stage], kb * BK, mb * BM);
+          tc::tma_load_2d(sa + A_BYTES, &tmB, &bars->full[stage], kb * BK, nb * BN);
+          issued |= 1u << stage;
+          last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (*abort)  // let every issued copy land before the CTA's shared memory is released
+        for (int s = 0; s < STAGES; ++s)
+          if (issued & (1u << s)) drain_wait(&bars->full[s], (last_parity >> s) & 1);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------- UMMA issuer
+      constexpr uint32_t IDESC = tc::idesc_f16(BF16, BM, BN);
+      int stage = 0, it = 0;
+      uint32_t phase = 0;
+      for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x, ++it) {
+        int mb, nb, ks, kb0, kb1;
+        decode_unit(p, unit, mb, nb, ks);
+        k_range(p, ks, kb0, kb1);
+        const int acc = it & 1;
+        const uint32_t aphase = (it >> 1) & 1;
+        if (!tc::mbar_wait(&bars->tempty[acc], aphase ^ 1, abort, p.status)) break;
+        tc::fence_after_sync();
+        const uint32_t d_tmem = tmem + acc * BN;
+        bool ok = true;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!tc::mbar_wait(&bars->full[stage], phase, abort, p.status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t a0 = tc::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t b0 = a0 + A_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc::umma_f16(d_tmem, tc::sdesc_kmajor_sw128(a0 + k * 32),
+                         tc::sdesc_kmajor_sw128(b0 + k * 32), IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&bars->empty[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc::umma_commit(&bars->tfull[acc]);
+      }
+      tc::umma_commit(&bars->drain);  // every MMA of this CTA has completed once this flips
+      drain_wait(&bars->drain, 0);
+    }
+  } else {  // ---------------- epilogue warps 2..5
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int row = q * 32 + lane;
+    int it = 0;
+    for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x, ++it) {
+      int mb, nb, ks;
+      decode_unit(p, unit, mb, nb, ks);
+      const int acc = it & 1;
+      const uint32_t aphase = (it >> 1) & 1;
+      if (!tc::mbar_wait(&bars->tfull[acc], aphase, abort, p.status)) break;
+      tc::fence_after_sync();
+      const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + acc * BN;
+      if (EPI == kEpiRope)
+        epi_rope(p, taddr, mb, nb, row);
+      else
+        epi_lsq(p, taddr, mb, nb, row);
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->tempty[acc]);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }();
+  return fn;
+}
+
+// Row-major [outer, inner] 16-bit matrix with row pitch `pitch` elements; box = box_outer rows of
+// 64 elements (128 B, the swizzle span).
+bool make_tmap(CUtensorMap* m, const void* base, bool bf16, uint64_t inner, uint64_t outer,
+               uint64_t pitch, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15u) || (pitch * 2) % 16) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2,
+            const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+template <int EPI, bool BF16>
+cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmParams& p,
+                        cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI, BF16>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int total = p.num_m * p.num_n * p.splits;
+  const int grid = std::min(total, sm_count());
+  gemm_tc_kernel<EPI, BF16><<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
+                                int D, int n_rot, int dh, int T, const float* cos_t,
+                                const float* sin_t, int* status, cudaStream_t st) {
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, A, false, K, M, K, BM) || !make_tmap(&tb, Bw, false, K, Nn, K, BN))
+    return cudaErrorInvalidValue;
+  GemmParams p{};
+  p.M = M;
+  p.Nn = Nn;
+  p.K = K;
+  p.num_m = (int)((M + BM - 1) / BM);
+  p.num_n = (Nn + BN - 1) / BN;
+  p.splits = 1;
+  p.k_blocks = K / BK;
+  p.group_m = 32;
+  p.status = status;
+  p.C = static_cast<half_t*>(C);
+  p.D = D;
+  p.n_rot = n_rot;
+  p.dh = dh;
+  p.T = T;
+  p.cos_t = cos_t;
+  p.sin_t = sin_t;
+  return launch_gemm<kEpiRope, false>(ta, tb, p, st);
+}
+
+cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
+                                const float* s, int64_t N, int D, int d, int G, int bits,
+                                float coef, float* ds, int* status, cudaStream_t st) {
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, xt, true, N, d, ldt, BN))
+    return cudaErrorInvalidValue;
+  GemmParams p{};
+  p.M = D;
+  p.Nn = d;
+  p.K = (int)std::min<int64_t>(N, INT32_MAX);
+  p.num_m = D / BM;
+  p.num_n = (d + BN - 1) / BN;
+  p.k_blocks = (int)((N + BK - 1) / BK);
+  const int tiles = p.num_m * p.num_n;
+  const int sms = sm_count();
+  int splits = 1;  // enough units for >= 4 waves, each at least 16 k-blocks long
+  while (tiles * splits < 4 * sms && p.k_blocks / (splits * 2) >= 16) splits *= 2;
+  p.splits = splits;
+  p.group_m = 8;
+  p.status = status;
+  p.w = static_cast<const bf16_t*>(w);
+  p.s = s;
+  p.d = d;
+  p.G = G;
+  p.bits = bits;
+  p.coef = coef;
+  p.ds = ds;
+  return launch_gemm<kEpiLsq, true>(ta, tb, p, st);
+}
+
+}  // namespace jab

@@ -18,13 +18,14 @@ struct AttnLaunch {
   float* lse;           // fp32 [B, Hq, T] or null
   void* d_o;            // fp16 [N, Hq*dh] (backward)
   float* dvec;          // fp32 [B, Hq, T] (backward)
+  int64_t ldt;          // row pitch of the transposed dQKV^T (backward)
   int* status;
   cudaStream_t stream;
 };
 
 // prep.cu
 cudaError_t launch_convert_x(const void* x, void* xh, int64_t n, int* status, int sms, cudaStream_t st);
-cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int d, cudaStream_t st);
+cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int64_t ldt, int d, cudaStream_t st);
 cudaError_t launch_quantize(const void* w, const float* s, int D, int d, int G, int bits, void* w16,
                             int8_t* codes, float* w_hat32, int* status, int sms, cudaStream_t st);
 cudaError_t launch_init_scales(const void* w, int D, int d, int G, int bits, int mode, float* s_out,
@@ -35,9 +36,9 @@ cudaError_t launch_rope_table(int T, int dh, double theta, float* cos_t, float* 
 cudaError_t launch_proj_gemm_simple(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
                                     int D, int n_rot, int dh, int T, const float* cos_t,
                                     const float* sin_t, cudaStream_t st);
-cudaError_t launch_wgrad_lsq_simple(const void* dqkvt, const void* xt, const void* w, const float* s,
-                                    int64_t N, int D, int d, int G, int bits, float coef, float* ds,
-                                    cudaStream_t st);
+cudaError_t launch_wgrad_lsq_simple(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
+                                    const float* s, int64_t N, int D, int d, int G, int bits,
+                                    float coef, float* ds, cudaStream_t st);
 
 // attn_simple.cu
 cudaError_t launch_attn_fwd_simple(const AttnLaunch& L, int mode);

@@ -22,10 +22,10 @@ inline bool use_tc_path() {
 // gemm_tc.cu
 cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
                                 int D, int n_rot, int dh, int T, const float* cos_t,
-                                const float* sin_t, cudaStream_t st);
-cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, const void* w, const float* s,
-                                int64_t N, int D, int d, int G, int bits, float coef, float* ds,
-                                cudaStream_t st);
+                                const float* sin_t, int* status, cudaStream_t st);
+cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
+                                const float* s, int64_t N, int D, int d, int G, int bits,
+                                float coef, float* ds, int* status, cudaStream_t st);
 // attn_tc.cu
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);
 cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,

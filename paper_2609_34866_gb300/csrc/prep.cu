@@ -31,7 +31,7 @@ __global__ void convert_x_kernel(const uint4* __restrict__ x, uint4* __restrict_
 
 // X [N, d] bf16 -> X^T [d, N] bf16 through a 64x64 shared-memory tile.
 __global__ void transpose_bf16_kernel(const bf16_t* __restrict__ x, bf16_t* __restrict__ xt,
-                                      int64_t N, int d) {
+                                      int64_t N, int64_t ldt, int d) {
   __shared__ bf16_t tile[64][65];
   const int64_t n0 = (int64_t)blockIdx.x * 64;
   const int c0 = blockIdx.y * 64;
@@ -44,7 +44,7 @@ __global__ void transpose_bf16_kernel(const bf16_t* __restrict__ x, bf16_t* __re
   for (int r = threadIdx.y; r < 64; r += blockDim.y) {
     const int c = c0 + r;
     const int64_t n = n0 + threadIdx.x;
-    if (n < N && c < d) xt[(int64_t)c * N + n] = tile[threadIdx.x][r];
+    if (n < N && c < d) xt[(int64_t)c * ldt + n] = tile[threadIdx.x][r];
   }
 }
 
@@ -167,9 +167,10 @@ cudaError_t launch_convert_x(const void* x, void* xh, int64_t n, int* status, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int d, cudaStream_t st) {
+cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int64_t ldt, int d,
+                               cudaStream_t st) {
   dim3 grid((unsigned)((N + 63) / 64), (unsigned)((d + 63) / 64));
-  transpose_bf16_kernel<<<grid, dim3(64, 8), 0, st>>>((const bf16_t*)x, (bf16_t*)xt, N, d);
+  transpose_bf16_kernel<<<grid, dim3(64, 8), 0, st>>>((const bf16_t*)x, (bf16_t*)xt, N, ldt, d);
   return cudaGetLastError();
 }
 
