@@ -107,7 +107,8 @@ AttnLaunch attn_launch(const jab_block_desc* d, int B, int T, int C, char* ws,
   L.dh = d->head_dim;
   L.C = C;
   L.scale = softmax_scale(d);
-  L.nP = (T + kPartRows - 1) / kPartRows;
+  const int rows = use_tc_path() ? attn_fwd_tc_rows() : kPartRows;  // rows per loss partial
+  L.nP = (T + rows - 1) / rows;
   L.part = reinterpret_cast<double*>(ws + wp.part);
   L.status = status;
   L.stream = st;

@@ -3,7 +3,6 @@
 
 namespace jab {
 
-cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) { return launch_attn_fwd_simple(L, mode); }
 cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
                                int use_rope, void* dqkvt) {
   return launch_attn_bwd_simple(L, cos_t, sin_t, use_rope, dqkvt);

@@ -120,8 +120,10 @@ def test_backward_parity(name, bits):
                             kappa=1.0)
     assert abs(loss.item() - r["loss"]) <= L_TOL * r["loss"]
     g = grad.cpu().numpy()
-    if c.T == 1:   # softmax over one key: Q and K scale gradients vanish exactly
-        assert not g[: (c.Hq + c.shape.n_kv_heads) * c.dh].any()
+    if c.T == 1:   # softmax over one key: Q and K scale gradients vanish (here to fp32 rounding:
+        # dP - rowsum(dO * O) cancels only up to the summation order of the two dot products)
+        nqk = (c.Hq + c.shape.n_kv_heads) * c.dh
+        assert np.abs(g[:nqk]).max() <= 1e-4 * np.abs(g[nqk:]).max()
     assert cosine(g, r["grad_s"]) >= COS_MIN, cosine(g, r["grad_s"])
     # kappa <= 0 selects (G qmax)^(-1/2): a pure multiplier
     grad2 = torch.empty_like(s)
