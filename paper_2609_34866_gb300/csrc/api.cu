@@ -109,6 +109,7 @@ AttnLaunch attn_launch(const jab_block_desc* d, int B, int T, int C, char* ws,
   L.scale = softmax_scale(d);
   const int rows = use_tc_path() ? attn_fwd_tc_rows() : kPartRows;  // rows per loss partial
   L.nP = (T + rows - 1) / rows;
+  L.lse_pitch = T;
   L.part = reinterpret_cast<double*>(ws + wp.part);
   L.status = status;
   L.stream = st;
@@ -253,6 +254,7 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   L.d_o = w + wp.d_o;
   L.dvec = reinterpret_cast<float*>(w + wp.dvec);
   L.ldt = wp.ldt;
+  L.lse_pitch = (int)wp.tp;
   JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 2) : launch_attn_fwd_simple(L, 2));
   const double n_el = (double)N * desc->n_q_heads * dh;
   JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el, loss_dev, nullptr,

@@ -1,0 +1,620 @@
+// Tensor-core (tcgen05) backward of causal GQA attention for the STE gradient of L_JAB, sm_103a.
+//
+// Inputs from the forward (mode 2): dO = O - A_ref (fp16; the factor 2/n is applied to the scale
+// gradient at the end), the row log-sum-exp and D = rowsum(dO * O). P is recomputed tile by tile:
+//   P = exp(S - lse),  dP = dO V^T,  dS = P * (dP - D)
+//   dV = P^T dO,  dK = scale * dS^T Q,  dQ = scale * dS K        (summed over the GQA group for K, V)
+// Two kernels, no atomics:
+//   dkdv  one CTA per (128-key block, KV head, sequence); loops over the query heads of the group and
+//         over 64-query blocks: S^T = K Q^T, dP^T = V dO^T into double-buffered TMEM, P^T and dS^T
+//         rows (fp16) to shared memory, dV += P^T dO and dK += dS^T Q accumulated in TMEM.
+//   dq    one CTA per (128 query rows, query head, sequence); loops over 64-key blocks: S = Q K^T,
+//         dP = dO V^T, dS (fp16) to shared memory, dQ += dS K in TMEM.
+// Warp roles as in the forward: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..5 one row per
+// thread. The epilogues apply the transpose of RoPE to dQ and dK and write dQKV^T (bf16, [D, ldt]),
+// the K-major operand of the weight-gradient GEMM.
+#include <cudaTypedefs.h>
+
+#include "path.h"
+#include "tc.cuh"
+
+namespace jab {
+namespace {
+
+constexpr int NUM_THREADS = 192;
+constexpr int STAGES = 3;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct BwdParams {
+  int T, B, Hq, Hkv, lse_pitch;
+  int qcol0, kcol0, vcol0;  // column offsets of Q, K, V heads in the QKV matrix
+  int64_t ldt;
+  float scale, sl2;
+  const float* lse;
+  const float* dvec;
+  const float* cos_t;
+  const float* sin_t;
+  int use_rope;
+  bf16_t* dqkvt;
+  int* status;
+};
+
+struct BwdBars {
+  uint64_t fixed_full, ld_full[STAGES], ld_empty[STAGES], s_full[2], s_empty[2];
+  uint64_t p_full, p_empty, o_full, drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = tc::globaltimer();
+  while (!tc::mbar_test(bar, parity))
+    if (tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
+}
+
+__device__ __forceinline__ void init_bars(BwdBars* bars) {
+  tc::mbar_init(&bars->fixed_full, 1);
+  for (int i = 0; i < STAGES; ++i) {
+    tc::mbar_init(&bars->ld_full[i], 1);
+    tc::mbar_init(&bars->ld_empty[i], 1);
+  }
+  for (int i = 0; i < 2; ++i) {
+    tc::mbar_init(&bars->s_full[i], 1);
+    tc::mbar_init(&bars->s_empty[i], 4);
+  }
+  tc::mbar_init(&bars->p_full, 4);
+  tc::mbar_init(&bars->p_empty, 1);
+  tc::mbar_init(&bars->o_full, 1);
+  tc::mbar_init(&bars->drain, 1);
+  bars->abort = 0;
+  tc::fence_mbar_init();
+}
+
+// 64 fp16 values (one 128-byte row of a K-major, 128-byte-swizzled operand tile) to shared memory.
+__device__ __forceinline__ void store_row64(uint8_t* base, int row, const float (&v)[64]) {
+#pragma unroll
+  for (int c8 = 0; c8 < 8; ++c8) {
+    uint4 u;
+    __half2* hp = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(v[c8 * 8 + 2 * e], v[c8 * 8 + 2 * e + 1]);
+    *reinterpret_cast<uint4*>(base + row * 128 + ((c8 ^ (row & 7)) << 4)) = u;
+  }
+}
+
+// Writes this thread's TMEM row of DH gradient columns, times `mul`, optionally through the transpose
+// of RoPE at position `pos`, as bf16 to dst[dim * ldt] (one column of dQKV^T).
+template <int DH>
+__device__ __forceinline__ void write_grad_row(uint32_t taddr, float mul, bool rope, int pos,
+                                               const float* cos_t, const float* sin_t,
+                                               bf16_t* dst, int64_t ldt, bool valid) {
+  constexpr int HALF = DH / 2;
+#pragma unroll 1
+  for (int pr = 0; pr < HALF / 32; ++pr) {
+    const int c1 = pr, c2 = pr + HALF / 32;
+    uint32_t ra[32], rb[32];
+    __syncwarp();
+    tc::tmem_ld32(taddr + c1 * 32, ra);
+    tc::tmem_ld32(taddr + c2 * 32, rb);
+    tc::tmem_ld_wait();
+    if (!valid) continue;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      float g1 = __uint_as_float(ra[i]) * mul, g2 = __uint_as_float(rb[i]) * mul;
+      if (rope) {
+        const int jj = c1 * 32 + i;
+        const float cs = __ldg(cos_t + (int64_t)pos * HALF + jj);
+        const float sn = __ldg(sin_t + (int64_t)pos * HALF + jj);
+        const float x1 = g1, x2 = g2;
+        g1 = x1 * cs + x2 * sn;
+        g2 = x2 * cs - x1 * sn;
+      }
+      dst[(int64_t)(c1 * 32 + i) * ldt] = __float2bfloat16_rn(g1);
+      dst[(int64_t)(c2 * 32 + i) * ldt] = __float2bfloat16_rn(g2);
+    }
+  }
+}
+
+// ================================================================================ dK, dV
+template <int DH>
+struct DkdvLayout {
+  static constexpr int BK = 128, BQ = 64;
+  static constexpr int KCHUNK = BK * 128;  // 64 columns of a 128-row tile
+  static constexpr int QCHUNK = BQ * 128;  // 64 columns of a 64-row tile
+  static constexpr int K_OFF = 0;
+  static constexpr int V_OFF = K_OFF + BK * DH * 2;
+  static constexpr int ST_OFF = V_OFF + BK * DH * 2;
+  static constexpr int ST_Q = 0, ST_DO = BQ * DH * 2, ST_LSE = 2 * BQ * DH * 2,
+                       ST_D = ST_LSE + BQ * 4, ST_BYTES = ST_D + BQ * 4;
+  static constexpr int ST_STRIDE = (ST_BYTES + 1023) / 1024 * 1024;
+  static constexpr int P_OFF = ST_OFF + STAGES * ST_STRIDE;
+  static constexpr int DS_OFF = P_OFF + BK * BQ * 2;
+  static constexpr int BAR_OFF = DS_OFF + BK * BQ * 2;
+  static constexpr int USED = BAR_OFF + 256 + 1024;
+  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+};
+
+template <int DH>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_kv,
+                            const __grid_constant__ CUtensorMap tm_q,
+                            const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
+  using L = DkdvLayout<DH>;
+  constexpr int BK = L::BK, BQ = L::BQ;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  BwdBars* bars = reinterpret_cast<BwdBars*>(smem + L::BAR_OFF);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &bars->abort;
+
+  const int kb = blockIdx.z, g = blockIdx.x, b = blockIdx.y;  // key block slowest: longest first
+  const int r = p.Hq / p.Hkv;
+  const int nq = (p.T + BQ - 1) / BQ;
+  const int i0 = (kb * BK) / BQ;
+  const int per_head = nq - i0;
+  const int n_it = r * per_head;
+  const int row0 = b * p.T;
+
+  if (threadIdx.x == 0) {
+    init_bars(bars);
+    tc::prefetch_tmap(&tm_kv);
+    tc::prefetch_tmap(&tm_q);
+    tc::prefetch_tmap(&tm_do);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&bars->tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = bars->tmem_base;
+  constexpr uint32_t DV_COL = 256, DK_COL = 256 + DH;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ------------------------------------------------------------- TMA
+      uint32_t issued = 0, last_par = 0;
+      tc::mbar_expect_tx(&bars->fixed_full, 2 * BK * DH * 2);
+      for (int ch = 0; ch < DH / 64; ++ch) {
+        tc::tma_load_2d(smem + L::K_OFF + ch * L::KCHUNK, &tm_kv, &bars->fixed_full,
+                        p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
+        tc::tma_load_2d(smem + L::V_OFF + ch * L::KCHUNK, &tm_kv, &bars->fixed_full,
+                        p.vcol0 + g * DH + ch * 64, row0 + kb * BK);
+      }
+      for (int it = 0; it < n_it; ++it) {
+        const int st = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        const int h = g * r + it / per_head, i = i0 + it % per_head;
+        if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
+        uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
+        tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
+        for (int ch = 0; ch < DH / 64; ++ch) {
+          tc::tma_load_2d(sbase + L::ST_Q + ch * L::QCHUNK, &tm_q, &bars->ld_full[st],
+                          p.qcol0 + h * DH + ch * 64, row0 + i * BQ);
+          tc::tma_load_2d(sbase + L::ST_DO + ch * L::QCHUNK, &tm_do, &bars->ld_full[st],
+                          h * DH + ch * 64, row0 + i * BQ);
+        }
+        const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + i * BQ;
+        tc::bulk_load(sbase + L::ST_LSE, p.lse + lrow, BQ * 4, &bars->ld_full[st]);
+        tc::bulk_load(sbase + L::ST_D, p.dvec + lrow, BQ * 4, &bars->ld_full[st]);
+        issued |= 1u << st;
+        last_par = (last_par & ~(1u << st)) | (ph << st);
+      }
+      if (*abort) {
+        drain_wait(&bars->fixed_full, 0);
+        for (int st = 0; st < STAGES; ++st)
+          if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ------------------------------------------------------------- UMMA
+      constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
+      constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
+      const uint32_t k_base = tc::smem_u32(smem + L::K_OFF);
+      const uint32_t v_base = tc::smem_u32(smem + L::V_OFF);
+      const uint32_t p_base = tc::smem_u32(smem + L::P_OFF);
+      const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
+      bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
+      auto issue_grad = [&](int jt) -> bool {
+        if (!tc::mbar_wait(&bars->p_full, jt & 1, abort, p.status)) return false;
+        tc::fence_after_sync();
+        const int st = jt % STAGES;
+        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+#pragma unroll
+        for (int k = 0; k < BQ / 16; ++k) {
+          const uint32_t acc = (jt > 0 || k > 0) ? 1u : 0u;
+          tc::umma_f16(tmem + DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
+                       tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::QCHUNK, 1024), ID_G,
+                       acc);
+          tc::umma_f16(tmem + DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
+                       tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::QCHUNK, 1024), ID_G,
+                       acc);
+        }
+        tc::umma_commit(&bars->ld_empty[st]);
+        tc::umma_commit(&bars->p_empty);
+        return true;
+      };
+      for (int it = 0; ok && it < n_it; ++it) {
+        const int st = it % STAGES;
+        const int sbuf = it & 1;
+        if (!tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status)) break;
+        if (!tc::mbar_wait(&bars->s_empty[sbuf], ((it >> 1) & 1) ^ 1, abort, p.status)) break;
+        tc::fence_after_sync();
+        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
+          const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
+          tc::umma_f16(tmem + sbuf * BQ, tc::sdesc_kmajor_sw128(k_base + ko),
+                       tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
+          tc::umma_f16(tmem + 128 + sbuf * BQ, tc::sdesc_kmajor_sw128(v_base + ko),
+                       tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&bars->s_full[sbuf]);
+        if (it > 0 && !issue_grad(it - 1)) break;
+        if (it == n_it - 1 && issue_grad(it)) tc::umma_commit(&bars->o_full);
+      }
+      tc::umma_commit(&bars->drain);
+      drain_wait(&bars->drain, 0);
+    }
+  } else {  // --------------------------------------------------------------------- elementwise
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int key = kb * BK + row;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    bool ok = true;
+    for (int it = 0; it < n_it; ++it) {
+      const int st = it % STAGES;
+      const int sbuf = it & 1;
+      const int i = i0 + it % per_head;
+      if (!tc::mbar_wait(&bars->s_full[sbuf], (it >> 1) & 1, abort, p.status) ||
+          !tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      tc::fence_after_sync();
+      float s[BQ], dp[BQ];
+#pragma unroll
+      for (int ch = 0; ch < BQ / 32; ++ch) {
+        uint32_t ra[32], rb[32];
+        __syncwarp();
+        tc::tmem_ld32(tmem + lane_base + sbuf * BQ + ch * 32, ra);
+        tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BQ + ch * 32, rb);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          s[ch * 32 + e] = __uint_as_float(ra[e]);
+          dp[ch * 32 + e] = __uint_as_float(rb[e]);
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
+      const uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
+      const float* lse_s = reinterpret_cast<const float*>(sbase + L::ST_LSE);
+      const float* d_s = reinterpret_cast<const float*>(sbase + L::ST_D);
+#pragma unroll
+      for (int c = 0; c < BQ; ++c) {
+        const int q = i * BQ + c;
+        const bool valid = q < p.T && q >= key;
+        const float pv = valid ? exp2f(s[c] * p.sl2 - lse_s[c] * kLog2e) : 0.f;
+        s[c] = pv;
+        dp[c] = valid ? pv * (dp[c] - d_s[c]) : 0.f;
+      }
+      if (!tc::mbar_wait(&bars->p_empty, (it & 1) ^ 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      store_row64(smem + L::P_OFF, row, s);
+      store_row64(smem + L::DS_OFF, row, dp);
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->p_full);
+    }
+    if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
+      tc::fence_after_sync();
+      const bool valid = key < p.T;
+      const int64_t n = (int64_t)row0 + (valid ? key : 0);
+      write_grad_row<DH>(tmem + lane_base + DV_COL, 1.f, false, 0, p.cos_t, p.sin_t,
+                         p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt + n, p.ldt, valid);
+      write_grad_row<DH>(tmem + lane_base + DK_COL, p.scale, p.use_rope != 0, valid ? key : 0,
+                         p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt + n,
+                         p.ldt, valid);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// ================================================================================ dQ
+template <int DH>
+struct DqLayout {
+  static constexpr int BQ = 128, BK = 64;
+  static constexpr int QCHUNK = BQ * 128;
+  static constexpr int KCHUNK = BK * 128;
+  static constexpr int Q_OFF = 0;
+  static constexpr int DO_OFF = Q_OFF + BQ * DH * 2;
+  static constexpr int ST_OFF = DO_OFF + BQ * DH * 2;
+  static constexpr int ST_K = 0, ST_V = BK * DH * 2, ST_BYTES = 2 * BK * DH * 2;
+  static constexpr int DS_OFF = ST_OFF + STAGES * ST_BYTES;
+  static constexpr int BAR_OFF = DS_OFF + BQ * BK * 2;
+  static constexpr int USED = BAR_OFF + 256 + 1024;
+  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+};
+
+template <int DH>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    attn_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+                          const __grid_constant__ CUtensorMap tm_kv,
+                          const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
+  using L = DqLayout<DH>;
+  constexpr int BQ = L::BQ, BK = L::BK;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  BwdBars* bars = reinterpret_cast<BwdBars*>(smem + L::BAR_OFF);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &bars->abort;
+
+  const int nqb = (p.T + BQ - 1) / BQ;
+  const int qb = nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
+  const int h = blockIdx.x, b = blockIdx.y;
+  const int g = h / (p.Hq / p.Hkv);
+  const int q0 = qb * BQ;
+  const int n_kb = (min(q0 + BQ, p.T) + BK - 1) / BK;
+  const int row0 = b * p.T;
+
+  if (threadIdx.x == 0) {
+    init_bars(bars);
+    tc::prefetch_tmap(&tm_q);
+    tc::prefetch_tmap(&tm_kv);
+    tc::prefetch_tmap(&tm_do);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&bars->tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = bars->tmem_base;
+  constexpr uint32_t DQ_COL = 256;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ------------------------------------------------------------- TMA
+      uint32_t issued = 0, last_par = 0;
+      tc::mbar_expect_tx(&bars->fixed_full, 2 * BQ * DH * 2);
+      for (int ch = 0; ch < DH / 64; ++ch) {
+        tc::tma_load_2d(smem + L::Q_OFF + ch * L::QCHUNK, &tm_q, &bars->fixed_full,
+                        p.qcol0 + h * DH + ch * 64, row0 + q0);
+        tc::tma_load_2d(smem + L::DO_OFF + ch * L::QCHUNK, &tm_do, &bars->fixed_full,
+                        h * DH + ch * 64, row0 + q0);
+      }
+      for (int j = 0; j < n_kb; ++j) {
+        const int st = j % STAGES;
+        const uint32_t ph = (j / STAGES) & 1;
+        if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
+        uint8_t* sbase = smem + L::ST_OFF + st * L::ST_BYTES;
+        tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
+        for (int ch = 0; ch < DH / 64; ++ch) {
+          tc::tma_load_2d(sbase + L::ST_K + ch * L::KCHUNK, &tm_kv, &bars->ld_full[st],
+                          p.kcol0 + g * DH + ch * 64, row0 + j * BK);
+          tc::tma_load_2d(sbase + L::ST_V + ch * L::KCHUNK, &tm_kv, &bars->ld_full[st],
+                          p.vcol0 + g * DH + ch * 64, row0 + j * BK);
+        }
+        issued |= 1u << st;
+        last_par = (last_par & ~(1u << st)) | (ph << st);
+      }
+      if (*abort) {
+        drain_wait(&bars->fixed_full, 0);
+        for (int st = 0; st < STAGES; ++st)
+          if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ------------------------------------------------------------- UMMA
+      constexpr uint32_t ID_S = tc::idesc_f16(false, BQ, BK);
+      constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
+      const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
+      const uint32_t do_base = tc::smem_u32(smem + L::DO_OFF);
+      const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
+      bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
+      auto issue_dq = [&](int jj) -> bool {
+        if (!tc::mbar_wait(&bars->p_full, jj & 1, abort, p.status)) return false;
+        tc::fence_after_sync();
+        const int st = jj % STAGES;
+        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          tc::umma_f16(tmem + DQ_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
+                       tc::sdesc_mnmajor_sw128(sb + L::ST_K + k * 16 * 128, L::KCHUNK, 1024), ID_G,
+                       (jj > 0 || k > 0) ? 1u : 0u);
+        tc::umma_commit(&bars->ld_empty[st]);
+        tc::umma_commit(&bars->p_empty);
+        return true;
+      };
+      for (int j = 0; ok && j < n_kb; ++j) {
+        const int st = j % STAGES;
+        const int sbuf = j & 1;
+        if (!tc::mbar_wait(&bars->ld_full[st], (j / STAGES) & 1, abort, p.status)) break;
+        if (!tc::mbar_wait(&bars->s_empty[sbuf], ((j >> 1) & 1) ^ 1, abort, p.status)) break;
+        tc::fence_after_sync();
+        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
+          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
+          tc::umma_f16(tmem + sbuf * BK, tc::sdesc_kmajor_sw128(q_base + qo),
+                       tc::sdesc_kmajor_sw128(sb + L::ST_K + ko), ID_S, k > 0 ? 1u : 0u);
+          tc::umma_f16(tmem + 128 + sbuf * BK, tc::sdesc_kmajor_sw128(do_base + qo),
+                       tc::sdesc_kmajor_sw128(sb + L::ST_V + ko), ID_S, k > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&bars->s_full[sbuf]);
+        if (j > 0 && !issue_dq(j - 1)) break;
+        if (j == n_kb - 1 && issue_dq(j)) tc::umma_commit(&bars->o_full);
+      }
+      tc::umma_commit(&bars->drain);
+      drain_wait(&bars->drain, 0);
+    }
+  } else {  // --------------------------------------------------------------------- elementwise
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int t = q0 + row;
+    const bool valid_row = t < p.T;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + (valid_row ? t : 0);
+    const float lse2 = valid_row ? p.lse[lrow] * kLog2e : 0.f;
+    const float drow = valid_row ? p.dvec[lrow] : 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_kb; ++j) {
+      const int sbuf = j & 1;
+      if (!tc::mbar_wait(&bars->s_full[sbuf], (j >> 1) & 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      tc::fence_after_sync();
+      float s[BK], dp[BK];
+#pragma unroll
+      for (int ch = 0; ch < BK / 32; ++ch) {
+        uint32_t ra[32], rb[32];
+        __syncwarp();
+        tc::tmem_ld32(tmem + lane_base + sbuf * BK + ch * 32, ra);
+        tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BK + ch * 32, rb);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          s[ch * 32 + e] = __uint_as_float(ra[e]);
+          dp[ch * 32 + e] = __uint_as_float(rb[e]);
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
+#pragma unroll
+      for (int c = 0; c < BK; ++c) {
+        const int kk = j * BK + c;
+        const bool valid = valid_row && kk <= t;
+        const float pv = valid ? exp2f(s[c] * p.sl2 - lse2) : 0.f;
+        dp[c] = valid ? pv * (dp[c] - drow) : 0.f;
+      }
+      if (!tc::mbar_wait(&bars->p_empty, (j & 1) ^ 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      store_row64(smem + L::DS_OFF, row, dp);
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->p_full);
+    }
+    if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
+      tc::fence_after_sync();
+      const int64_t n = (int64_t)row0 + (valid_row ? t : 0);
+      write_grad_row<DH>(tmem + lane_base + DQ_COL, p.scale, p.use_rope != 0, valid_row ? t : 0,
+                         p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.qcol0 + h * DH) * p.ldt + n, p.ldt,
+                         valid_row);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// ================================================================================ host
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }();
+  return fn;
+}
+
+bool tmap_rows(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <typename K>
+cudaError_t set_smem(K kernel, int bytes, bool& done) {
+  if (done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done = true;
+  return e;
+}
+
+template <int DH>
+cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
+  const int64_t N = (int64_t)L.B * L.T;
+  CUtensorMap kv128, q64, do64, q128, kv64, do128;
+  if (!tmap_rows(&kv128, L.qkv, L.ldq, N, 128) || !tmap_rows(&q64, L.qkv, L.ldq, N, 64) ||
+      !tmap_rows(&do64, L.d_o, (uint64_t)L.Hq * DH, N, 64) ||
+      !tmap_rows(&q128, L.qkv, L.ldq, N, 128) || !tmap_rows(&kv64, L.qkv, L.ldq, N, 64) ||
+      !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128))
+    return cudaErrorInvalidValue;
+  static bool a1 = false, a2 = false;
+  cudaError_t e = set_smem(attn_bwd_dkdv_tc_kernel<DH>, DkdvLayout<DH>::SMEM, a1);
+  if (e != cudaSuccess) return e;
+  e = set_smem(attn_bwd_dq_tc_kernel<DH>, DqLayout<DH>::SMEM, a2);
+  if (e != cudaSuccess) return e;
+  dim3 g1((unsigned)L.Hkv, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
+  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, q64, do64, p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  dim3 g2((unsigned)L.Hq, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
+  attn_bwd_dq_tc_kernel<DH><<<g2, NUM_THREADS, DqLayout<DH>::SMEM, L.stream>>>(q128, kv64, do128, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
+                               int use_rope, void* dqkvt) {
+  BwdParams p{};
+  p.T = L.T;
+  p.B = L.B;
+  p.Hq = L.Hq;
+  p.Hkv = L.Hkv;
+  p.lse_pitch = L.lse_pitch;
+  p.qcol0 = 0;
+  p.kcol0 = L.Hq * L.dh;
+  p.vcol0 = (L.Hq + L.Hkv) * L.dh;
+  p.ldt = L.ldt;
+  p.scale = L.scale;
+  p.sl2 = L.scale * kLog2e;
+  p.lse = L.lse;
+  p.dvec = L.dvec;
+  p.cos_t = cos_t;
+  p.sin_t = sin_t;
+  p.use_rope = use_rope;
+  p.dqkvt = static_cast<bf16_t*>(dqkvt);
+  p.status = L.status;
+  if ((reinterpret_cast<uintptr_t>(L.lse) & 15u) || (reinterpret_cast<uintptr_t>(L.dvec) & 15u) ||
+      (L.lse_pitch % 64) != 0)
+    return cudaErrorInvalidValue;
+  return L.dh == 128 ? launch_bwd<128>(L, p) : launch_bwd<64>(L, p);
+}
+
+}  // namespace jab

@@ -27,6 +27,7 @@ struct AttnArgs {
   half_t* d_o;          // mode 2: e = A_hat - A_ref, fp16 [N, Hq*d_h]
   float* dvec;          // mode 2: rowsum(dO * O) [B, Hq, T]
   int* status;
+  int lse_pitch;        // row pitch of lse / dvec
 };
 
 __device__ __forceinline__ float quad_sum(float x) {
@@ -140,10 +141,10 @@ __global__ void __launch_bounds__(256) attn_fwd_simple_kernel(AttnArgs a) {
     acc = valid ? (double)sq : 0.0;
     if (MODE == 2) {
       dsum = quad_sum(dsum);
-      if (valid && qd == 0) a.dvec[((int64_t)b * a.Hq + h) * a.T + t] = dsum;
+      if (valid && qd == 0) a.dvec[((int64_t)b * a.Hq + h) * a.lse_pitch + t] = dsum;
     }
   }
-  if (a.lse != nullptr && MODE != 1 && valid && qd == 0) a.lse[((int64_t)b * a.Hq + h) * a.T + t] = lse;
+  if (a.lse != nullptr && MODE != 1 && valid && qd == 0) a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + t] = lse;
   const double tot = block_sum<256>(acc, red);
   if (threadIdx.x == 0)
     a.part[(((int64_t)c * a.B + b) * a.Hq + h) * a.nP + qb] = tot;
@@ -176,8 +177,8 @@ __global__ void __launch_bounds__(256) attn_bwd_dq_simple_kernel(AttnArgs a, con
     dO[k] = __half2float(a.d_o[orow + k]);
     dq[k] = 0.f;
   }
-  const float lse2 = a.lse[((int64_t)b * a.Hq + h) * a.T + te] * kLog2e;
-  const float Dt = a.dvec[((int64_t)b * a.Hq + h) * a.T + te];
+  const float lse2 = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + te] * kLog2e;
+  const float Dt = a.dvec[((int64_t)b * a.Hq + h) * a.lse_pitch + te];
   for (int kb = 0; kb <= qb; ++kb) {
     const int rows = min(64, a.T - kb * 64);
     __syncthreads();
@@ -254,8 +255,8 @@ __global__ void __launch_bounds__(256) attn_bwd_dkdv_simple_kernel(AttnArgs a, c
       load_tile<DH>(Os, dOp, (int64_t)a.Hq * DH, rowbase + qb * 64, rows);
       if (threadIdx.x < 64) {
         const int tq = min(qb * 64 + (int)threadIdx.x, a.T - 1);
-        Ls[threadIdx.x] = a.lse[((int64_t)b * a.Hq + h) * a.T + tq] * kLog2e;
-        Ds[threadIdx.x] = a.dvec[((int64_t)b * a.Hq + h) * a.T + tq];
+        Ls[threadIdx.x] = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + tq] * kLog2e;
+        Ds[threadIdx.x] = a.dvec[((int64_t)b * a.Hq + h) * a.lse_pitch + tq];
       }
       __syncthreads();
       for (int i = 0; i < 64; ++i) {
@@ -300,7 +301,7 @@ __global__ void __launch_bounds__(256) attn_bwd_dkdv_simple_kernel(AttnArgs a, c
 // ---------------------------------------------------------------- launchers
 cudaError_t launch_attn_fwd_simple(const AttnLaunch& L, int mode) {
   AttnArgs a{(const half_t*)L.qkv, L.ldq, L.D, L.B, L.T, L.Hq, L.Hkv, L.scale, L.nP, L.part,
-             L.a_ref, L.a_out, L.lse, (half_t*)L.d_o, L.dvec, L.status};
+             L.a_ref, L.a_out, L.lse, (half_t*)L.d_o, L.dvec, L.status, L.lse_pitch};
   dim3 grid((unsigned)((L.T + 63) / 64), (unsigned)L.Hq, (unsigned)(L.B * L.C));
 #define JAB_FWD(DH_, M_) attn_fwd_simple_kernel<DH_, M_><<<grid, 256, 0, L.stream>>>(a)
   if (L.dh == 128) {
@@ -315,7 +316,7 @@ cudaError_t launch_attn_fwd_simple(const AttnLaunch& L, int mode) {
 cudaError_t launch_attn_bwd_simple(const AttnLaunch& L, const float* cos_t, const float* sin_t,
                                    int use_rope, void* dqkvt) {
   AttnArgs a{(const half_t*)L.qkv, L.ldq, L.D, L.B, L.T, L.Hq, L.Hkv, L.scale, L.nP, L.part,
-             L.a_ref, L.a_out, L.lse, (half_t*)L.d_o, L.dvec, L.status};
+             L.a_ref, L.a_out, L.lse, (half_t*)L.d_o, L.dvec, L.status, L.lse_pitch};
   const int64_t N = L.ldt;  // row pitch of dQKV^T
   dim3 gq((unsigned)((L.T + 63) / 64), (unsigned)L.Hq, (unsigned)L.B);
   dim3 gk((unsigned)((L.T + 63) / 64), (unsigned)L.Hkv, (unsigned)L.B);

@@ -51,7 +51,7 @@ struct FwdBars {
 };
 
 struct FwdParams {
-  int T, B, Hq, Hkv, D, nqb, nP;
+  int T, B, Hq, Hkv, D, nqb, nP, lse_pitch;
   float sl2;  // softmax scale * log2(e)
   double* part;
   const float* a_ref;
@@ -79,9 +79,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
 
-  const int qb = p.nqb - 1 - (int)blockIdx.x;  // longest rows first
-  const int h = blockIdx.y;
-  const int b = (int)blockIdx.z % p.B, c = (int)blockIdx.z / p.B;
+  const int qb = p.nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
+  const int h = blockIdx.x;
+  const int b = (int)blockIdx.y % p.B, c = (int)blockIdx.y / p.B;
   const int g = h / (p.Hq / p.Hkv);
   const int q0 = qb * BQ;
   const int nkb = min(qb + 1, (p.T + BKV - 1) / BKV);
@@ -328,8 +328,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (valid) {
         if (MODE != 1 && p.lse != nullptr)
-          p.lse[((int64_t)b * p.Hq + h) * p.T + t] = (m + log2f(l)) * kLn2;
-        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.T + t] = dsum;
+          p.lse[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = (m + log2f(l)) * kLn2;
+        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = dsum;
         acc = (double)sq;
       }
     }
@@ -401,6 +401,7 @@ cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) {
   p.D = L.D;
   p.nqb = (L.T + BQ - 1) / BQ;
   p.nP = L.nP;
+  p.lse_pitch = L.lse_pitch;
   p.sl2 = L.scale * kLog2e;
   p.part = L.part;
   p.a_ref = L.a_ref;
@@ -409,7 +410,7 @@ cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) {
   p.d_o = static_cast<half_t*>(L.d_o);
   p.dvec = L.dvec;
   p.status = L.status;
-  dim3 grid((unsigned)p.nqb, (unsigned)L.Hq, (unsigned)(L.B * L.C));
+  dim3 grid((unsigned)L.Hq, (unsigned)(L.B * L.C), (unsigned)p.nqb);
 #define JAB_FWD(DH_, M_) return launch_fwd<DH_, M_>(tm, p, grid, L.stream)
   if (L.dh == 128) {
     if (mode == 0) JAB_FWD(128, 0);

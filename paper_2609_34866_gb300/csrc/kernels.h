@@ -19,6 +19,7 @@ struct AttnLaunch {
   void* d_o;            // fp16 [N, Hq*dh] (backward)
   float* dvec;          // fp32 [B, Hq, T] (backward)
   int64_t ldt;          // row pitch of the transposed dQKV^T (backward)
+  int lse_pitch;        // row pitch of lse and dvec ([B, Hq, lse_pitch])
   int* status;
   cudaStream_t stream;
 };

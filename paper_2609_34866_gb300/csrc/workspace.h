@@ -21,10 +21,11 @@ struct Workspace {
   // backward only
   size_t xt;       // bf16 [d, ldt]          X transposed (K-major operand of the weight gradient)
   size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
-  size_t lse;      // fp32 [B, Hq, T]        student log-sum-exp
-  size_t dvec;     // fp32 [B, Hq, T]        rowsum(dO * O)
+  size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp (Tp = T rounded up to 64)
+  size_t dvec;     // fp32 [B, Hq, Tp]       rowsum(dO * O)
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
   int64_t ldt;     // row pitch (elements) of xt and dqkvt: N rounded up to 64
+  int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 64
   size_t total;
 };
 
@@ -40,6 +41,7 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
   const int64_t N = B * T, D = block_rows(d), dm = d->d_model, dh = d->head_dim;
   const int64_t nP = (T + kPartRows - 1) / kPartRows;
   w.ldt = (N + 63) / 64 * 64;
+  w.tp = (T + 63) / 64 * 64;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t o = off;
@@ -55,8 +57,8 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
   if (bwd) {
     w.xt = take((size_t)w.ldt * dm * 2);
     w.d_o = take((size_t)N * d->n_q_heads * dh * 2);
-    w.lse = take((size_t)B * d->n_q_heads * T * 4);
-    w.dvec = take((size_t)B * d->n_q_heads * T * 4);
+    w.lse = take((size_t)B * d->n_q_heads * w.tp * 4);
+    w.dvec = take((size_t)B * d->n_q_heads * w.tp * 4);
     w.dqkvt = take((size_t)D * w.ldt * 2);
   } else {
     w.xt = w.d_o = w.lse = w.dvec = w.dqkvt = SIZE_MAX;
