@@ -1,7 +1,8 @@
 // Tensor-core (tcgen05) backward of causal GQA attention for the STE gradient of L_JAB, sm_103a.
 //
 // Inputs from the forward (mode 2): dO = O - A_ref (fp16; the factor 2/n is applied to the scale
-// gradient at the end), the row log-sum-exp and D = rowsum(dO * O). P is recomputed tile by tile:
+// gradient at the end), the row log-sum-exp in log2 units and D = rowsum(dO * O). P is recomputed
+// tile by tile:
 //   P = exp(S - lse),  dP = dO V^T,  dS = P * (dP - D)
 //   dV = P^T dO,  dK = scale * dS^T Q,  dQ = scale * dS K        (summed over the GQA group for K, V)
 // Two kernels, no atomics:
@@ -10,8 +11,8 @@
 //         rows (fp16) to shared memory, dV += P^T dO and dK += dS^T Q accumulated in TMEM.
 //   dq    one CTA per (128 query rows, query head, sequence); loops over 64-key blocks: S = Q K^T,
 //         dP = dO V^T, dS (fp16) to shared memory, dQ += dS K in TMEM.
-// Warp roles as in the forward: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..5 one row per
-// thread. The epilogues apply the transpose of RoPE to dQ and dK and write dQKV^T (bf16, [D, ldt]),
+// Warp roles: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..9 elementwise: two warps per
+// TMEM lane quarter, each thread owning one row and half of the columns of the S / dP tile. The epilogues apply the transpose of RoPE to dQ and dK and write dQKV^T (bf16, [D, ldt]),
 // the K-major operand of the weight-gradient GEMM.
 #include <cudaTypedefs.h>
 
@@ -21,7 +22,8 @@
 namespace jab {
 namespace {
 
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise (2 per lane quarter)
+constexpr int EW_WARPS = 8;
 constexpr int STAGES = 3;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -60,9 +62,9 @@ __device__ __forceinline__ void init_bars(BwdBars* bars) {
   }
   for (int i = 0; i < 2; ++i) {
     tc::mbar_init(&bars->s_full[i], 1);
-    tc::mbar_init(&bars->s_empty[i], 4);
+    tc::mbar_init(&bars->s_empty[i], EW_WARPS);
   }
-  tc::mbar_init(&bars->p_full, 4);
+  tc::mbar_init(&bars->p_full, EW_WARPS);
   tc::mbar_init(&bars->p_empty, 1);
   tc::mbar_init(&bars->o_full, 1);
   tc::mbar_init(&bars->drain, 1);
@@ -70,27 +72,32 @@ __device__ __forceinline__ void init_bars(BwdBars* bars) {
   tc::fence_mbar_init();
 }
 
-// 64 fp16 values (one 128-byte row of a K-major, 128-byte-swizzled operand tile) to shared memory.
-__device__ __forceinline__ void store_row64(uint8_t* base, int row, const float (&v)[64]) {
+// 32 fp16 values, half of one 128-byte row of a K-major, 128-byte-swizzled operand tile (16-byte
+// chunks 4*half .. 4*half+3), to shared memory.
+__device__ __forceinline__ void store_half_row(uint8_t* base, int row, int half,
+                                               const float (&v)[32]) {
 #pragma unroll
-  for (int c8 = 0; c8 < 8; ++c8) {
+  for (int k = 0; k < 4; ++k) {
     uint4 u;
     __half2* hp = reinterpret_cast<__half2*>(&u);
 #pragma unroll
-    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(v[c8 * 8 + 2 * e], v[c8 * 8 + 2 * e + 1]);
+    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(v[k * 8 + 2 * e], v[k * 8 + 2 * e + 1]);
+    const int c8 = half * 4 + k;
     *reinterpret_cast<uint4*>(base + row * 128 + ((c8 ^ (row & 7)) << 4)) = u;
   }
 }
 
 // Writes this thread's TMEM row of DH gradient columns, times `mul`, optionally through the transpose
 // of RoPE at position `pos`, as bf16 to dst[dim * ldt] (one column of dQKV^T).
+// Only the 32-column pairs (pr, pr + DH/64) with pr in [pr0, pr1) are handled by this thread.
 template <int DH>
 __device__ __forceinline__ void write_grad_row(uint32_t taddr, float mul, bool rope, int pos,
                                                const float* cos_t, const float* sin_t,
-                                               bf16_t* dst, int64_t ldt, bool valid) {
+                                               bf16_t* dst, int64_t ldt, bool valid, int pr0,
+                                               int pr1) {
   constexpr int HALF = DH / 2;
 #pragma unroll 1
-  for (int pr = 0; pr < HALF / 32; ++pr) {
+  for (int pr = pr0; pr < pr1; ++pr) {
     const int c1 = pr, c2 = pr + HALF / 32;
     uint32_t ra[32], rb[32];
     __syncwarp();
@@ -258,10 +265,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else {  // --------------------------------------------------------------------- elementwise
+  } else {  // ------------------------------------------------ elementwise: row = key, 32 queries
     const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
     const int key = kb * BK + row;
+    const int col0 = half * 32;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     bool ok = true;
     for (int it = 0; it < n_it; ++it) {
@@ -274,40 +283,41 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc::fence_after_sync();
-      float s[BQ], dp[BQ];
-#pragma unroll
-      for (int ch = 0; ch < BQ / 32; ++ch) {
-        uint32_t ra[32], rb[32];
-        __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + sbuf * BQ + ch * 32, ra);
-        tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BQ + ch * 32, rb);
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          s[ch * 32 + e] = __uint_as_float(ra[e]);
-          dp[ch * 32 + e] = __uint_as_float(rb[e]);
-        }
-      }
+      uint32_t rs[32], rd[32];
+      __syncwarp();
+      tc::tmem_ld32(tmem + lane_base + sbuf * BQ + col0, rs);
+      tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BQ + col0, rd);
+      tc::tmem_ld_wait();
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
       const uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
-      const float* lse_s = reinterpret_cast<const float*>(sbase + L::ST_LSE);
-      const float* d_s = reinterpret_cast<const float*>(sbase + L::ST_D);
+      const float* lse2 = reinterpret_cast<const float*>(sbase + L::ST_LSE) + col0;
+      const float* dd = reinterpret_cast<const float*>(sbase + L::ST_D) + col0;
+      const int q0 = i * BQ + col0;
+      float pv[32], dsv[32];
+      if (q0 >= kb * BK + BK - 1 && q0 + 31 < p.T) {  // every (key, query) pair is visible
 #pragma unroll
-      for (int c = 0; c < BQ; ++c) {
-        const int q = i * BQ + c;
-        const bool valid = q < p.T && q >= key;
-        const float pv = valid ? exp2f(s[c] * p.sl2 - lse_s[c] * kLog2e) : 0.f;
-        s[c] = pv;
-        dp[c] = valid ? pv * (dp[c] - d_s[c]) : 0.f;
+        for (int c = 0; c < 32; ++c) {
+          pv[c] = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2[c]));
+          dsv[c] = pv[c] * (__uint_as_float(rd[c]) - dd[c]);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const int q = q0 + c;
+          const bool valid = q < p.T && q >= key;
+          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2[c]));
+          pv[c] = valid ? e : 0.f;
+          dsv[c] = valid ? e * (__uint_as_float(rd[c]) - dd[c]) : 0.f;
+        }
       }
       if (!tc::mbar_wait(&bars->p_empty, (it & 1) ^ 1, abort, p.status)) {
         ok = false;
         break;
       }
-      store_row64(smem + L::P_OFF, row, s);
-      store_row64(smem + L::DS_OFF, row, dp);
+      store_half_row(smem + L::P_OFF, row, half, pv);
+      store_half_row(smem + L::DS_OFF, row, half, dsv);
       tc::fence_proxy_async_smem();
       tc::fence_before_sync();
       __syncwarp();
@@ -317,11 +327,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::fence_after_sync();
       const bool valid = key < p.T;
       const int64_t n = (int64_t)row0 + (valid ? key : 0);
+      const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
       write_grad_row<DH>(tmem + lane_base + DV_COL, 1.f, false, 0, p.cos_t, p.sin_t,
-                         p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt + n, p.ldt, valid);
+                         p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt + n, p.ldt, valid, pr0, pr1);
       write_grad_row<DH>(tmem + lane_base + DK_COL, p.scale, p.use_rope != 0, valid ? key : 0,
                          p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt + n,
-                         p.ldt, valid);
+                         p.ldt, valid, pr0, pr1);
     }
   }
   tc::fence_before_sync();
@@ -463,14 +474,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else {  // --------------------------------------------------------------------- elementwise
+  } else {  // ------------------------------------------------ elementwise: row = query, 32 keys
     const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
     const int t = q0 + row;
+    const int col0 = half * 32;
     const bool valid_row = t < p.T;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + (valid_row ? t : 0);
-    const float lse2 = valid_row ? p.lse[lrow] * kLog2e : 0.f;
+    const float lse2 = valid_row ? p.lse[lrow] : INFINITY;  // P = 0 on rows past T
     const float drow = valid_row ? p.dvec[lrow] : 0.f;
     bool ok = true;
     for (int j = 0; j < n_kb; ++j) {
@@ -480,35 +493,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc::fence_after_sync();
-      float s[BK], dp[BK];
-#pragma unroll
-      for (int ch = 0; ch < BK / 32; ++ch) {
-        uint32_t ra[32], rb[32];
-        __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + sbuf * BK + ch * 32, ra);
-        tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BK + ch * 32, rb);
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          s[ch * 32 + e] = __uint_as_float(ra[e]);
-          dp[ch * 32 + e] = __uint_as_float(rb[e]);
-        }
-      }
+      uint32_t rs[32], rd[32];
+      __syncwarp();
+      tc::tmem_ld32(tmem + lane_base + sbuf * BK + col0, rs);
+      tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BK + col0, rd);
+      tc::tmem_ld_wait();
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
+      const int k0 = j * BK + col0;
+      float dsv[32];
+      if (k0 + 31 <= q0) {  // every key of this slice is visible to every row of the CTA
 #pragma unroll
-      for (int c = 0; c < BK; ++c) {
-        const int kk = j * BK + c;
-        const bool valid = valid_row && kk <= t;
-        const float pv = valid ? exp2f(s[c] * p.sl2 - lse2) : 0.f;
-        dp[c] = valid ? pv * (dp[c] - drow) : 0.f;
+        for (int c = 0; c < 32; ++c) {
+          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2));
+          dsv[c] = e * (__uint_as_float(rd[c]) - drow);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2));
+          dsv[c] = (k0 + c <= t) ? e * (__uint_as_float(rd[c]) - drow) : 0.f;
+        }
       }
       if (!tc::mbar_wait(&bars->p_empty, (j & 1) ^ 1, abort, p.status)) {
         ok = false;
         break;
       }
-      store_row64(smem + L::DS_OFF, row, dp);
+      store_half_row(smem + L::DS_OFF, row, half, dsv);
       tc::fence_proxy_async_smem();
       tc::fence_before_sync();
       __syncwarp();
@@ -517,9 +529,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
       tc::fence_after_sync();
       const int64_t n = (int64_t)row0 + (valid_row ? t : 0);
+      const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
       write_grad_row<DH>(tmem + lane_base + DQ_COL, p.scale, p.use_rope != 0, valid_row ? t : 0,
                          p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.qcol0 + h * DH) * p.ldt + n, p.ldt,
-                         valid_row);
+                         valid_row, pr0, pr1);
     }
   }
   tc::fence_before_sync();

@@ -50,7 +50,7 @@ __device__ __forceinline__ void load_tile(half_t (*dst)[DH], const half_t* src, 
 }
 
 // MODE 0: teacher (write A and lse, partial ||A||^2); 1: loss (partial SSE); 2: loss + backward
-// inputs (dO = e in fp16, lse, rowsum(dO * O)).
+// inputs (dO = e in fp16, lse in log2 units, rowsum(dO * O)).
 template <int DH, int MODE>
 __global__ void __launch_bounds__(256) attn_fwd_simple_kernel(AttnArgs a) {
   constexpr int DQ = DH / 4;
@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(256) attn_fwd_simple_kernel(AttnArgs a) {
   const float inv_l = __fdiv_rn(1.f, l);
 #pragma unroll
   for (int k = 0; k < DQ; ++k) o[k] = __fmul_rn(o[k], inv_l);
-  const float lse = (m + log2f(l)) * kLn2;
+  const float lse = MODE == 2 ? m + log2f(l) : (m + log2f(l)) * kLn2;  // mode 2: log2 units
   const int64_t orow = (rowbase + te) * (int64_t)(a.Hq * DH) + (int64_t)h * DH + qd * DQ;
   double acc = 0.0;
   if (MODE == 0) {
@@ -177,7 +177,7 @@ __global__ void __launch_bounds__(256) attn_bwd_dq_simple_kernel(AttnArgs a, con
     dO[k] = __half2float(a.d_o[orow + k]);
     dq[k] = 0.f;
   }
-  const float lse2 = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + te] * kLog2e;
+  const float lse2 = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + te];  // log2 units
   const float Dt = a.dvec[((int64_t)b * a.Hq + h) * a.lse_pitch + te];
   for (int kb = 0; kb <= qb; ++kb) {
     const int rows = min(64, a.T - kb * 64);
@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(256) attn_bwd_dkdv_simple_kernel(AttnArgs a, c
       load_tile<DH>(Os, dOp, (int64_t)a.Hq * DH, rowbase + qb * 64, rows);
       if (threadIdx.x < 64) {
         const int tq = min(qb * 64 + (int)threadIdx.x, a.T - 1);
-        Ls[threadIdx.x] = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + tq] * kLog2e;
+        Ls[threadIdx.x] = a.lse[((int64_t)b * a.Hq + h) * a.lse_pitch + tq];
         Ds[threadIdx.x] = a.dvec[((int64_t)b * a.Hq + h) * a.lse_pitch + tq];
       }
       __syncthreads();

@@ -6,13 +6,15 @@
 //                 S_j = Q K_j^T            M128 N128 K=d_h     A, B K-major (smem)
 //                 O  += P_j V_j            M128 N=d_h K128     A = P (smem, K-major), B = V MN-major
 //               S is double-buffered in TMEM so S_{j+1} runs while the softmax works on S_j.
-//   warps 2..5  softmax, one query row per thread: tcgen05.ld of the S row, causal mask, online
+//   warps 2..9  softmax, two warps per TMEM lane quarter: a thread owns one query row and half of
+//               its 128 scores (the halves exchange row maxima through shared memory): tcgen05.ld of
+//               the S row, causal mask, online
 //               softmax in the log2 domain with lazy rescaling (O is rescaled in TMEM only when the
 //               running max grows by more than 2^8), P in fp16 to shared memory; after the last
 //               block the epilogue of the calling mode:
 //                 mode 0 (teacher)  A_ref = O (fp32), lse, partial ||A||^2
 //                 mode 1 (loss)     partial SSE = sum (O - A_ref)^2                     (Eq. 3)
-//                 mode 2 (loss+bwd) also dO = O - A_ref (fp16), lse, D = rowsum(dO * O)
+//                 mode 2 (loss+bwd) also dO = O - A_ref (fp16), lse in log2 units, D = rowsum(dO * O)
 // The SSE partials are per (candidate, sequence, head, 128-row block), fp64, reduced in fixed order.
 #include <cudaTypedefs.h>
 
@@ -23,7 +25,8 @@ namespace jab {
 namespace {
 
 constexpr int BQ = 128, BKV = 128;
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;  // warp 0 TMA, warp 1 UMMA, warps 2..9 softmax (2 per lane quarter)
+constexpr int EW_WARPS = 8;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleLog2 = 8.f;  // rescale O only when the row max grows by more than 2^8
@@ -38,7 +41,7 @@ struct FwdLayout {
   static constexpr int P_OFF = V_OFF + 2 * TILE;
   static constexpr int P_BYTES = BQ * BKV * 2;
   static constexpr int BAR_OFF = P_OFF + P_BYTES;
-  static constexpr int USED = BAR_OFF + 256 + 1024;
+  static constexpr int USED = BAR_OFF + 8192 + 1024;
   // At least half of the SM's shared memory, so that one CTA (and its 512 TMEM columns) owns the SM.
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
 };
@@ -47,8 +50,38 @@ struct FwdBars {
   uint64_t q_full, kv_full[2], kv_empty[2], s_full[2], s_empty[2], p_full, p_empty, o_full, drain;
   uint32_t tmem_base;
   int abort;
-  double red[4];
+  double red[EW_WARPS];
+  float xmax[2][2][BQ];  // [iteration parity][column half][row]: partial row maxima
+  float xl[2][BQ];       // partial row sums, exchanged once at the end
+  float xd[2][BQ];       // partial rowsum(dO * O)
+  int flag[2][BQ];       // [column half][row]: sequence number of the last value posted
 };
+
+// Pair exchange between the two threads that own the halves of one row: post a value under a
+// monotonically increasing sequence number, then read the partner's value of the same number.
+// The wait is time-bounded like every mbarrier wait (no barrier that could hang if one side left).
+__device__ __forceinline__ void pair_post(FwdBars* bars, int half, int row, int seq) {
+  __threadfence_block();
+  reinterpret_cast<volatile int*>(&bars->flag[half][row])[0] = seq;
+}
+__device__ __forceinline__ void pair_wait(FwdBars* bars, int half, int row, int seq,
+                                          volatile int* abort, int* status) {
+  volatile int* f = &bars->flag[half ^ 1][row];
+  if (*f < seq) {
+    const uint64_t t0 = tc::globaltimer();
+    for (uint32_t it = 0; *f < seq; ++it) {
+      if ((it & 63u) == 0) {
+        if (*abort) break;
+        if (tc::globaltimer() - t0 > tc::kWaitLimitNs) {
+          *abort = 1;
+          report(status, JAB_ERR_TIMEOUT);
+          break;
+        }
+      }
+    }
+  }
+  __threadfence_block();
+}
 
 struct FwdParams {
   int T, B, Hq, Hkv, D, nqb, nP, lse_pitch;
@@ -96,9 +129,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::mbar_init(&bars->kv_full[i], 1);
       tc::mbar_init(&bars->kv_empty[i], 1);
       tc::mbar_init(&bars->s_full[i], 1);
-      tc::mbar_init(&bars->s_empty[i], 4);
+      tc::mbar_init(&bars->s_empty[i], EW_WARPS);
     }
-    tc::mbar_init(&bars->p_full, 4);
+    tc::mbar_init(&bars->p_full, EW_WARPS);
     tc::mbar_init(&bars->p_empty, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
@@ -106,6 +139,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm);
   }
+  for (int i = threadIdx.x; i < 2 * BQ; i += blockDim.x) (&bars->flag[0][0])[i] = 0;
   if (warp == 1) {
     tc::tmem_alloc(&bars->tmem_base, 512);
     tc::tmem_relinquish();
@@ -190,8 +224,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {  // ------------------------------------------------------------------------ softmax
     const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
     const int t = q0 + row;
+    const int col0 = half * (BKV / 2);  // this thread's 64 score columns
+    const int ocol0 = half * (DH / 2);  // and DH/2 output columns
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     uint8_t* pbuf = smem + L::P_OFF;
     float m = -INFINITY, l = 0.f;
@@ -203,12 +240,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc::fence_after_sync();
-      float s[BKV];
+      float s[BKV / 2];
 #pragma unroll
-      for (int ch = 0; ch < BKV / 32; ++ch) {
+      for (int ch = 0; ch < BKV / 64; ++ch) {
         uint32_t r[32];
         __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + sb * BKV + ch * 32, r);
+        tc::tmem_ld32(tmem + lane_base + sb * BKV + col0 + ch * 32, r);
         tc::tmem_ld_wait();
 #pragma unroll
         for (int i = 0; i < 32; ++i) s[ch * 32 + i] = __uint_as_float(r[i]) * p.sl2;
@@ -216,26 +253,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->s_empty[sb]);
-      const int k0 = j * BKV;
-      if (k0 + BKV - 1 > q0 || k0 + BKV > p.T) {  // diagonal or ragged block: mask
+      const int k0 = j * BKV + col0;
+      if (k0 + BKV / 2 - 1 > q0 || k0 + BKV / 2 > p.T) {  // diagonal or ragged block: mask
 #pragma unroll
-        for (int i = 0; i < BKV; ++i)
+        for (int i = 0; i < BKV / 2; ++i)
           if (k0 + i > t || k0 + i >= p.T) s[i] = -INFINITY;
       }
-      float mx = s[0];
+      float mx8[8];  // 8 independent partial maxima: a short dependency chain
 #pragma unroll
-      for (int i = 1; i < BKV; ++i) mx = fmaxf(mx, s[i]);
+      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+      for (int i = 8; i < BKV / 2; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
+      const float pmax = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      bars->xmax[sb][half][row] = pmax;
+      pair_post(bars, half, row, j + 1);
+      pair_wait(bars, half, row, j + 1, abort, p.status);
+      const float mx = fmaxf(pmax, reinterpret_cast<volatile float*>(&bars->xmax[sb][half ^ 1][row])[0]);
       const float m_new = fmaxf(m, mx);
       const bool resc = m_new > m + kRescaleLog2;
       const float m_use = resc ? m_new : m;
-      const float alpha = resc ? exp2f(m - m_new) : 1.f;
-      float rs = 0.f;
+      const float alpha = resc ? tc::fast_exp2(m - m_new) : 1.f;
+      float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int i = 0; i < BKV; ++i) {
-        s[i] = exp2f(s[i] - m_use);
-        rs += s[i];
+      for (int i = 0; i < BKV / 2; ++i) {
+        s[i] = tc::fast_exp2(s[i] - m_use);
+        rs8[i & 7] += s[i];
       }
-      l = l * alpha + rs;
+      l = l * alpha + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
       m = m_use;
       // P_{j-1} V_{j-1} must be complete before O is rescaled or the P buffer is overwritten.
       if (!tc::mbar_wait(&bars->p_empty, (j & 1) ^ 1, abort, p.status)) {
@@ -245,25 +290,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::fence_after_sync();
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
 #pragma unroll
-        for (int ch = 0; ch < DH / 32; ++ch) {
+        for (int ch = 0; ch < DH / 64; ++ch) {
           uint32_t r[32];
           __syncwarp();
-          tc::tmem_ld32(tmem + lane_base + O_COL + ch * 32, r);
+          tc::tmem_ld32(tmem + lane_base + O_COL + ocol0 + ch * 32, r);
           tc::tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-          tc::tmem_st32(tmem + lane_base + O_COL + ch * 32, r);
+          tc::tmem_st32(tmem + lane_base + O_COL + ocol0 + ch * 32, r);
         }
         tc::tmem_st_wait();
       }
+      uint8_t* prow = pbuf + half * (BQ * 128) + row * 128;  // this half = one 64-key swizzle chunk
 #pragma unroll
-      for (int cc = 0; cc < BKV / 8; ++cc) {
+      for (int c8 = 0; c8 < 8; ++c8) {
         uint4 u;
         __half2* hp = reinterpret_cast<__half2*>(&u);
 #pragma unroll
-        for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(s[cc * 8 + 2 * e], s[cc * 8 + 2 * e + 1]);
-        const int kc = cc >> 3, c8 = cc & 7;
-        *reinterpret_cast<uint4*>(pbuf + kc * (BQ * 128) + row * 128 + ((c8 ^ (row & 7)) << 4)) = u;
+        for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(s[c8 * 8 + 2 * e], s[c8 * 8 + 2 * e + 1]);
+        *reinterpret_cast<uint4*>(prow + ((c8 ^ (row & 7)) << 4)) = u;
       }
       tc::fence_proxy_async_smem();
       tc::fence_before_sync();
@@ -272,17 +317,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     // ---------------------------------------------------------------- epilogue
     double acc = 0.0;
+    bars->xl[half][row] = l;
+    pair_post(bars, half, row, nkb + 1);
+    pair_wait(bars, half, row, nkb + 1, abort, p.status);
+    l += reinterpret_cast<volatile float*>(&bars->xl[half ^ 1][row])[0];
     if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
       tc::fence_after_sync();
       const bool valid = t < p.T;
       const float inv_l = __fdiv_rn(1.f, l);
-      const int64_t orow = ((int64_t)row0 + (valid ? t : 0)) * (int64_t)(p.Hq * DH) + h * DH;
+      const int64_t orow = ((int64_t)row0 + (valid ? t : 0)) * (int64_t)(p.Hq * DH) + h * DH + ocol0;
       float sq = 0.f, dsum = 0.f;
 #pragma unroll 1
-      for (int ch = 0; ch < DH / 32; ++ch) {
+      for (int ch = 0; ch < DH / 64; ++ch) {
         uint32_t r[32];
         __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + O_COL + ch * 32, r);
+        tc::tmem_ld32(tmem + lane_base + O_COL + ocol0 + ch * 32, r);
         tc::tmem_ld_wait();
         float o[32];
 #pragma unroll
@@ -326,19 +375,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      if (valid) {
-        if (MODE != 1 && p.lse != nullptr)
-          p.lse[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = (m + log2f(l)) * kLn2;
-        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = dsum;
-        acc = (double)sq;
+      if (MODE == 2) {
+        bars->xd[half][row] = dsum;
+        pair_post(bars, half, row, nkb + 2);
+        pair_wait(bars, half, row, nkb + 2, abort, p.status);
+        dsum += reinterpret_cast<volatile float*>(&bars->xd[half ^ 1][row])[0];
       }
+      if (valid && half == 0) {
+        if (MODE != 1 && p.lse != nullptr)
+          p.lse[((int64_t)b * p.Hq + h) * p.lse_pitch + t] =
+              MODE == 2 ? m + log2f(l) : (m + log2f(l)) * kLn2;  // mode 2: log2 units
+        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = dsum;
+      }
+      if (valid) acc = (double)sq;
     }
     acc = warp_sum(acc);
-    if (lane == 0) bars->red[quarter] = acc;
-    tc::named_bar_sync(1, 128);
-    if (warp == 2 && lane == 0)
-      p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb] =
-          bars->red[0] + bars->red[1] + bars->red[2] + bars->red[3];
+    if (lane == 0) bars->red[warp - 2] = acc;
+    tc::named_bar_sync(1, EW_WARPS * 32);
+    if (warp == 2 && lane == 0) {
+      double tot = 0.0;
+      for (int w = 0; w < EW_WARPS; ++w) tot += bars->red[w];
+      p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb] = tot;
+    }
   }
   tc::fence_before_sync();
   __syncthreads();

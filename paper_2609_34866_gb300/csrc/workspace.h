@@ -21,7 +21,7 @@ struct Workspace {
   // backward only
   size_t xt;       // bf16 [d, ldt]          X transposed (K-major operand of the weight gradient)
   size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
-  size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp (Tp = T rounded up to 64)
+  size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 64)
   size_t dvec;     // fp32 [B, Hq, Tp]       rowsum(dO * O)
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
   int64_t ldt;     // row pitch (elements) of xt and dqkvt: N rounded up to 64
