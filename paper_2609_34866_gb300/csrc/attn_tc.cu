@@ -407,6 +407,338 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ============================================================================ head-pair kernel
+// Two query heads of one KV group per CTA (GQA: they read the same K and V), 128 query rows each,
+// keys in blocks of 64 through a 3-stage K/V ring. Per head: S double-buffered in TMEM (2 x 64
+// columns), O in TMEM (128 columns), P in shared memory; four softmax warps per head, one row per
+// thread. Every K/V byte loaded feeds twice the tensor work of the single-head kernel.
+constexpr int PBQ = 128, PBK = 64, PSTAGES = 3;
+
+template <int DH>
+struct PairLayout {
+  static constexpr int QTILE = PBQ * DH * 2;
+  static constexpr int QCHUNK = PBQ * 128;
+  static constexpr int KVTILE = PBK * DH * 2;
+  static constexpr int KVCHUNK = PBK * 128;
+  static constexpr int Q_OFF = 0;
+  static constexpr int KV_OFF = Q_OFF + 2 * QTILE;
+  static constexpr int STAGE = 2 * KVTILE;  // K then V
+  static constexpr int P_OFF = KV_OFF + PSTAGES * STAGE;
+  static constexpr int PTILE = PBQ * PBK * 2;
+  static constexpr int BAR_OFF = P_OFF + 2 * PTILE;
+  static constexpr int USED = BAR_OFF + 512 + 1024;
+  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+};
+
+struct PairBars {
+  uint64_t q_full, kv_full[PSTAGES], kv_empty[PSTAGES];
+  uint64_t s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], o_full[2], drain;
+  uint32_t tmem_base;
+  int abort;
+  double red[EW_WARPS];
+};
+
+template <int DH, int MODE>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    attn_fwd_pair_kernel(const __grid_constant__ CUtensorMap tm_q,
+                         const __grid_constant__ CUtensorMap tm_kv, const FwdParams p) {
+  using L = PairLayout<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  PairBars* bars = reinterpret_cast<PairBars*>(smem + L::BAR_OFF);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &bars->abort;
+
+  const int qb = p.nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
+  const int h0 = 2 * (int)blockIdx.x;
+  const int b = (int)blockIdx.y % p.B, c = (int)blockIdx.y / p.B;
+  const int g = h0 / (p.Hq / p.Hkv);
+  const int q0 = qb * PBQ;
+  const int nkb = (min(q0 + PBQ, p.T) + PBK - 1) / PBK;
+  const int row0 = b * p.T;
+  const int kcol = c * p.D + (p.Hq + g) * DH;
+  const int vcol = c * p.D + (p.Hq + p.Hkv + g) * DH;
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bars->q_full, 1);
+    for (int i = 0; i < PSTAGES; ++i) {
+      tc::mbar_init(&bars->kv_full[i], 1);
+      tc::mbar_init(&bars->kv_empty[i], 1);
+    }
+    for (int hd = 0; hd < 2; ++hd) {
+      for (int i = 0; i < 2; ++i) {
+        tc::mbar_init(&bars->s_full[hd][i], 1);
+        tc::mbar_init(&bars->s_empty[hd][i], 4);
+      }
+      tc::mbar_init(&bars->p_full[hd], 4);
+      tc::mbar_init(&bars->p_empty[hd], 1);
+      tc::mbar_init(&bars->o_full[hd], 1);
+    }
+    tc::mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tm_q);
+    tc::prefetch_tmap(&tm_kv);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&bars->tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = bars->tmem_base;
+  auto s_col = [](int hd, int sb) { return (uint32_t)((hd * 2 + sb) * PBK); };
+  auto o_col = [](int hd) { return (uint32_t)(4 * PBK + hd * 128); };
+
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------------------------------------------------------- TMA
+      uint32_t issued = 0, last_par = 0;
+      tc::mbar_expect_tx(&bars->q_full, 2 * L::QTILE);
+      for (int hd = 0; hd < 2; ++hd)
+        for (int ch = 0; ch < DH / 64; ++ch)
+          tc::tma_load_2d(smem + L::Q_OFF + hd * L::QTILE + ch * L::QCHUNK, &tm_q, &bars->q_full,
+                          c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
+      for (int j = 0; j < nkb; ++j) {
+        const int st = j % PSTAGES;
+        const uint32_t ph = (j / PSTAGES) & 1;
+        if (!tc::mbar_wait(&bars->kv_empty[st], ph ^ 1, abort, p.status)) break;
+        uint8_t* sbase = smem + L::KV_OFF + st * L::STAGE;
+        tc::mbar_expect_tx(&bars->kv_full[st], L::STAGE);
+        for (int ch = 0; ch < DH / 64; ++ch) {
+          tc::tma_load_2d(sbase + ch * L::KVCHUNK, &tm_kv, &bars->kv_full[st], kcol + ch * 64,
+                          row0 + j * PBK);
+          tc::tma_load_2d(sbase + L::KVTILE + ch * L::KVCHUNK, &tm_kv, &bars->kv_full[st],
+                          vcol + ch * 64, row0 + j * PBK);
+        }
+        issued |= 1u << st;
+        last_par = (last_par & ~(1u << st)) | (ph << st);
+      }
+      if (*abort) {
+        drain_wait(&bars->q_full, 0);
+        for (int st = 0; st < PSTAGES; ++st)
+          if (issued & (1u << st)) drain_wait(&bars->kv_full[st], (last_par >> st) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------------------------------------------------------- UMMA
+      constexpr uint32_t ID_S = tc::idesc_f16(false, PBQ, PBK);
+      constexpr uint32_t ID_PV = tc::idesc_f16(false, PBQ, DH) | (1u << 16);  // B = V, MN-major
+      bool ok = tc::mbar_wait(&bars->q_full, 0, abort, p.status);
+      auto issue_pv = [&](int hd, int jj) -> bool {
+        if (!tc::mbar_wait(&bars->p_full[hd], jj & 1, abort, p.status)) return false;
+        tc::fence_after_sync();
+        const uint32_t v_base =
+            tc::smem_u32(smem + L::KV_OFF + (jj % PSTAGES) * L::STAGE + L::KVTILE);
+        const uint32_t p_base = tc::smem_u32(smem + L::P_OFF + hd * L::PTILE);
+#pragma unroll
+        for (int k = 0; k < PBK / 16; ++k)
+          tc::umma_f16(tmem + o_col(hd), tc::sdesc_kmajor_sw128(p_base + k * 32),
+                       tc::sdesc_mnmajor_sw128(v_base + k * 16 * 128, L::KVCHUNK, 1024), ID_PV,
+                       (jj > 0 || k > 0) ? 1u : 0u);
+        tc::umma_commit(&bars->p_empty[hd]);
+        if (hd == 1) tc::umma_commit(&bars->kv_empty[jj % PSTAGES]);
+        return true;
+      };
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int st = j % PSTAGES, sb = j & 1;
+        if (!tc::mbar_wait(&bars->kv_full[st], (j / PSTAGES) & 1, abort, p.status)) break;
+        const uint32_t k_base = tc::smem_u32(smem + L::KV_OFF + st * L::STAGE);
+        for (int hd = 0; hd < 2 && ok; ++hd) {
+          if (!tc::mbar_wait(&bars->s_empty[hd][sb], ((j >> 1) & 1) ^ 1, abort, p.status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF + hd * L::QTILE);
+#pragma unroll
+          for (int k = 0; k < DH / 16; ++k)
+            tc::umma_f16(tmem + s_col(hd, sb),
+                         tc::sdesc_kmajor_sw128(q_base + (k >> 2) * L::QCHUNK + (k & 3) * 32),
+                         tc::sdesc_kmajor_sw128(k_base + (k >> 2) * L::KVCHUNK + (k & 3) * 32),
+                         ID_S, k > 0 ? 1u : 0u);
+          tc::umma_commit(&bars->s_full[hd][sb]);
+        }
+        if (!ok) break;
+        if (j > 0 && (!issue_pv(0, j - 1) || !issue_pv(1, j - 1))) break;
+        if (j == nkb - 1) {
+          for (int hd = 0; hd < 2; ++hd)
+            if (issue_pv(hd, j)) tc::umma_commit(&bars->o_full[hd]);
+        }
+      }
+      tc::umma_commit(&bars->drain);
+      drain_wait(&bars->drain, 0);
+    }
+  } else {  // ------------------------------------------------------------------------ softmax
+    const int hd = (warp - 2) >> 2;
+    const int h = h0 + hd;
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int t = q0 + row;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    uint8_t* prow = smem + L::P_OFF + hd * L::PTILE + row * 128;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      const int sb = j & 1;
+      if (!tc::mbar_wait(&bars->s_full[hd][sb], (j >> 1) & 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      tc::fence_after_sync();
+      float s[PBK];
+#pragma unroll
+      for (int ch = 0; ch < PBK / 32; ++ch) {
+        uint32_t r[32];
+        __syncwarp();
+        tc::tmem_ld32(tmem + lane_base + s_col(hd, sb) + ch * 32, r);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) s[ch * 32 + i] = __uint_as_float(r[i]) * p.sl2;
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->s_empty[hd][sb]);
+      const int k0 = j * PBK;
+      if (k0 + PBK - 1 > q0 || k0 + PBK > p.T) {  // diagonal or ragged block: mask
+#pragma unroll
+        for (int i = 0; i < PBK; ++i)
+          if (k0 + i > t || k0 + i >= p.T) s[i] = -INFINITY;
+      }
+      float mx8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+      for (int i = 8; i < PBK; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      const float m_new = fmaxf(m, mx);
+      const bool resc = m_new > m + kRescaleLog2;
+      const float m_use = resc ? m_new : m;
+      const float alpha = resc ? tc::fast_exp2(m - m_new) : 1.f;
+      float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < PBK; ++i) {
+        s[i] = tc::fast_exp2(s[i] - m_use);
+        rs8[i & 7] += s[i];
+      }
+      l = l * alpha + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
+      m = m_use;
+      // P V of the previous block must be complete before O is rescaled or P is overwritten.
+      if (!tc::mbar_wait(&bars->p_empty[hd], (j & 1) ^ 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+      tc::fence_after_sync();
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+#pragma unroll
+        for (int ch = 0; ch < DH / 32; ++ch) {
+          uint32_t r[32];
+          __syncwarp();
+          tc::tmem_ld32(tmem + lane_base + o_col(hd) + ch * 32, r);
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+          tc::tmem_st32(tmem + lane_base + o_col(hd) + ch * 32, r);
+        }
+        tc::tmem_st_wait();
+      }
+#pragma unroll
+      for (int c8 = 0; c8 < 8; ++c8) {
+        uint4 u;
+        __half2* hp = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(s[c8 * 8 + 2 * e], s[c8 * 8 + 2 * e + 1]);
+        *reinterpret_cast<uint4*>(prow + ((c8 ^ (row & 7)) << 4)) = u;
+      }
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->p_full[hd]);
+    }
+    // ---------------------------------------------------------------- epilogue
+    double acc = 0.0;
+    if (ok && tc::mbar_wait(&bars->o_full[hd], 0, abort, p.status)) {
+      tc::fence_after_sync();
+      const bool valid = t < p.T;
+      const float inv_l = __fdiv_rn(1.f, l);
+      const int64_t orow = ((int64_t)row0 + (valid ? t : 0)) * (int64_t)(p.Hq * DH) + h * DH;
+      float sq = 0.f, dsum = 0.f;
+#pragma unroll 1
+      for (int ch = 0; ch < DH / 32; ++ch) {
+        uint32_t r[32];
+        __syncwarp();
+        tc::tmem_ld32(tmem + lane_base + o_col(hd) + ch * 32, r);
+        tc::tmem_ld_wait();
+        float o[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] = __fmul_rn(__uint_as_float(r[i]), inv_l);
+        if (!valid) continue;
+        if (MODE == 0) {
+          float4* dst = reinterpret_cast<float4*>(p.a_out + orow + ch * 32);
+#pragma unroll
+          for (int v = 0; v < 8; ++v) {
+            dst[v] = make_float4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
+            sq += o[4 * v] * o[4 * v] + o[4 * v + 1] * o[4 * v + 1] + o[4 * v + 2] * o[4 * v + 2] +
+                  o[4 * v + 3] * o[4 * v + 3];
+          }
+        } else {
+          const float4* ar = reinterpret_cast<const float4*>(p.a_ref + orow + ch * 32);
+          float e[32];
+#pragma unroll
+          for (int v = 0; v < 8; ++v) {
+            const float4 a4 = __ldg(ar + v);
+            e[4 * v] = __fsub_rn(o[4 * v], a4.x);
+            e[4 * v + 1] = __fsub_rn(o[4 * v + 1], a4.y);
+            e[4 * v + 2] = __fsub_rn(o[4 * v + 2], a4.z);
+            e[4 * v + 3] = __fsub_rn(o[4 * v + 3], a4.w);
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) sq += e[i] * e[i];
+          if (MODE == 2) {
+            uint4* dst = reinterpret_cast<uint4*>(p.d_o + orow + ch * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+              uint4 u;
+              __half2* hp = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                hp[k] = __floats2half2_rn(e[v * 8 + 2 * k], e[v * 8 + 2 * k + 1]);
+                const float2 f = __half22float2(hp[k]);
+                dsum += f.x * o[v * 8 + 2 * k] + f.y * o[v * 8 + 2 * k + 1];
+              }
+              dst[v] = u;
+            }
+          }
+        }
+      }
+      if (valid) {
+        if (MODE != 1 && p.lse != nullptr)
+          p.lse[((int64_t)b * p.Hq + h) * p.lse_pitch + t] =
+              MODE == 2 ? m + log2f(l) : (m + log2f(l)) * kLn2;  // mode 2: log2 units
+        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = dsum;
+        acc = (double)sq;
+      }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) bars->red[warp - 2] = acc;
+    tc::named_bar_sync(1, EW_WARPS * 32);
+    if (quarter == 0 && lane == 0) {  // one thread per head
+      const int w0 = hd * 4;
+      p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb] =
+          bars->red[w0] + bars->red[w0 + 1] + bars->red[w0 + 2] + bars->red[w0 + 3];
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     void* f = nullptr;
@@ -418,6 +750,21 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
   }();
   return fn;
+}
+
+template <int DH, int MODE>
+cudaError_t launch_fwd_pair(const CUtensorMap& tq, const CUtensorMap& tkv, const FwdParams& p,
+                            dim3 grid, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_pair_kernel<DH, MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         PairLayout<DH>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  attn_fwd_pair_kernel<DH, MODE><<<grid, NUM_THREADS, PairLayout<DH>::SMEM, st>>>(tq, tkv, p);
+  return cudaGetLastError();
 }
 
 template <int DH, int MODE>
@@ -468,6 +815,25 @@ cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) {
   p.d_o = static_cast<half_t*>(L.d_o);
   p.dvec = L.dvec;
   p.status = L.status;
+  if ((L.Hq / L.Hkv) % 2 == 0) {  // head pairs of one KV group share every K/V tile
+    CUtensorMap tkv;
+    cuuint32_t box64[2] = {64, (cuuint32_t)PBK};
+    if (fn(&tkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(L.qkv), dims, strides, box64,
+           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    dim3 pgrid((unsigned)(L.Hq / 2), (unsigned)(L.B * L.C), (unsigned)p.nqb);
+#define JAB_FWD2(DH_, M_) return launch_fwd_pair<DH_, M_>(tm, tkv, p, pgrid, L.stream)
+    if (L.dh == 128) {
+      if (mode == 0) JAB_FWD2(128, 0);
+      if (mode == 1) JAB_FWD2(128, 1);
+      JAB_FWD2(128, 2);
+    }
+    if (mode == 0) JAB_FWD2(64, 0);
+    if (mode == 1) JAB_FWD2(64, 1);
+    JAB_FWD2(64, 2);
+#undef JAB_FWD2
+  }
   dim3 grid((unsigned)L.Hq, (unsigned)(L.B * L.C), (unsigned)p.nqb);
 #define JAB_FWD(DH_, M_) return launch_fwd<DH_, M_>(tm, p, grid, L.stream)
   if (L.dh == 128) {
