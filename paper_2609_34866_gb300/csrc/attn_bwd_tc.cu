@@ -87,14 +87,13 @@ __device__ __forceinline__ void store_half_row(uint8_t* base, int row, int half,
   }
 }
 
-// Writes this thread's TMEM row of DH gradient columns, times `mul`, optionally through the transpose
-// of RoPE at position `pos`, as bf16 to dst[dim * ldt] (one column of dQKV^T).
-// Only the 32-column pairs (pr, pr + DH/64) with pr in [pr0, pr1) are handled by this thread.
+// Stages this thread's TMEM row of DH gradient columns, times `mul`, optionally through the
+// transpose of RoPE at position `pos`, into tile[dim][row] (bf16, 128 rows per dim). Only the
+// 32-column pairs (pr, pr + DH/64) with pr in [pr0, pr1) are handled by this thread.
 template <int DH>
-__device__ __forceinline__ void write_grad_row(uint32_t taddr, float mul, bool rope, int pos,
+__device__ __forceinline__ void stage_grad_row(uint32_t taddr, float mul, bool rope, int pos,
                                                const float* cos_t, const float* sin_t,
-                                               bf16_t* dst, int64_t ldt, bool valid, int pr0,
-                                               int pr1) {
+                                               bf16_t* tile, int row, int pr0, int pr1) {
   constexpr int HALF = DH / 2;
 #pragma unroll 1
   for (int pr = pr0; pr < pr1; ++pr) {
@@ -104,7 +103,6 @@ __device__ __forceinline__ void write_grad_row(uint32_t taddr, float mul, bool r
     tc::tmem_ld32(taddr + c1 * 32, ra);
     tc::tmem_ld32(taddr + c2 * 32, rb);
     tc::tmem_ld_wait();
-    if (!valid) continue;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
       float g1 = __uint_as_float(ra[i]) * mul, g2 = __uint_as_float(rb[i]) * mul;
@@ -116,8 +114,31 @@ __device__ __forceinline__ void write_grad_row(uint32_t taddr, float mul, bool r
         g1 = x1 * cs + x2 * sn;
         g2 = x2 * cs - x1 * sn;
       }
-      dst[(int64_t)(c1 * 32 + i) * ldt] = __float2bfloat16_rn(g1);
-      dst[(int64_t)(c2 * 32 + i) * ldt] = __float2bfloat16_rn(g2);
+      tile[(c1 * 32 + i) * 128 + row] = __float2bfloat16_rn(g1);
+      tile[(c2 * 32 + i) * 128 + row] = __float2bfloat16_rn(g2);
+    }
+  }
+}
+
+// Cooperative store of tile[DH][128] to dst[d * ldt + n0 + r] for r < nvalid: 16-byte vectors when
+// the token offset is 8-aligned (consecutive threads cover consecutive 16-byte chunks of a dim
+// row), element-wise otherwise.
+template <int DH>
+__device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int64_t ldt, int64_t n0,
+                                           int nvalid, int tid, int nthreads) {
+  if ((n0 & 7) == 0) {
+    for (int idx = tid; idx < DH * 16; idx += nthreads) {
+      const int d = idx >> 4, r0 = (idx & 15) * 8;
+      bf16_t* o = dst + (int64_t)d * ldt + n0 + r0;
+      if (r0 + 8 <= nvalid)
+        *reinterpret_cast<uint4*>(o) = *reinterpret_cast<const uint4*>(tile + d * 128 + r0);
+      else
+        for (int r = r0; r < nvalid; ++r) o[r - r0] = tile[d * 128 + r];
+    }
+  } else {
+    for (int idx = tid; idx < DH * 128; idx += nthreads) {
+      const int d = idx >> 7, r = idx & 127;
+      if (r < nvalid) dst[(int64_t)d * ldt + n0 + r] = tile[d * 128 + r];
     }
   }
 }
@@ -222,45 +243,58 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t v_base = tc::smem_u32(smem + L::V_OFF);
       const uint32_t p_base = tc::smem_u32(smem + L::P_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
+      // Event-driven issue: S^T / dP^T of block ns go out as soon as their K/V stage has landed and
+      // their TMEM buffer is free (up to two blocks ahead), the gradient MMAs of block ng as soon as
+      // its P^T and dS^T are in shared memory.
       bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
-      auto issue_grad = [&](int jt) -> bool {
-        if (!tc::mbar_wait(&bars->p_full, jt & 1, abort, p.status)) return false;
-        tc::fence_after_sync();
-        const int st = jt % STAGES;
-        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+      int ns = 0, ng = 0;
+      tc::Watchdog wd;
+      while (ok && ng < n_it) {
+        bool prog = false;
+        if (ns < n_it && ns <= ng + 2) {
+          const int st = ns % STAGES, sbuf = ns & 1;
+          if (tc::mbar_ready(&bars->ld_full[st], (ns / STAGES) & 1) &&
+              tc::mbar_ready(&bars->s_empty[sbuf], ((ns >> 1) & 1) ^ 1)) {
+            tc::fence_after_sync();
+            const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
 #pragma unroll
-        for (int k = 0; k < BQ / 16; ++k) {
-          const uint32_t acc = (jt > 0 || k > 0) ? 1u : 0u;
-          tc::umma_f16(tmem + DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
-                       tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::QCHUNK, 1024), ID_G,
-                       acc);
-          tc::umma_f16(tmem + DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
-                       tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::QCHUNK, 1024), ID_G,
-                       acc);
+            for (int k = 0; k < DH / 16; ++k) {
+              const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
+              const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
+              tc::umma_f16(tmem + sbuf * BQ, tc::sdesc_kmajor_sw128(k_base + ko),
+                           tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16(tmem + 128 + sbuf * BQ, tc::sdesc_kmajor_sw128(v_base + ko),
+                           tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
+            }
+            tc::umma_commit(&bars->s_full[sbuf]);
+            ++ns;
+            prog = true;
+          }
         }
-        tc::umma_commit(&bars->ld_empty[st]);
-        tc::umma_commit(&bars->p_empty);
-        return true;
-      };
-      for (int it = 0; ok && it < n_it; ++it) {
-        const int st = it % STAGES;
-        const int sbuf = it & 1;
-        if (!tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status)) break;
-        if (!tc::mbar_wait(&bars->s_empty[sbuf], ((it >> 1) & 1) ^ 1, abort, p.status)) break;
-        tc::fence_after_sync();
-        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+        if (ng < ns && tc::mbar_ready(&bars->p_full, ng & 1)) {
+          tc::fence_after_sync();
+          const int st = ng % STAGES;
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
 #pragma unroll
-        for (int k = 0; k < DH / 16; ++k) {
-          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
-          const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
-          tc::umma_f16(tmem + sbuf * BQ, tc::sdesc_kmajor_sw128(k_base + ko),
-                       tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
-          tc::umma_f16(tmem + 128 + sbuf * BQ, tc::sdesc_kmajor_sw128(v_base + ko),
-                       tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
+          for (int k = 0; k < BQ / 16; ++k) {
+            const uint32_t acc = (ng > 0 || k > 0) ? 1u : 0u;
+            tc::umma_f16(tmem + DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
+                         tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::QCHUNK, 1024),
+                         ID_G, acc);
+            tc::umma_f16(tmem + DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
+                         tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::QCHUNK, 1024),
+                         ID_G, acc);
+          }
+          tc::umma_commit(&bars->ld_empty[st]);
+          tc::umma_commit(&bars->p_empty);
+          if (ng == n_it - 1) tc::umma_commit(&bars->o_full);
+          ++ng;
+          prog = true;
         }
-        tc::umma_commit(&bars->s_full[sbuf]);
-        if (it > 0 && !issue_grad(it - 1)) break;
-        if (it == n_it - 1 && issue_grad(it)) tc::umma_commit(&bars->o_full);
+        if (prog)
+          wd.progress();
+        else if (!wd.tick(abort, p.status))
+          ok = false;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
@@ -323,16 +357,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->p_full);
     }
-    if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
+    // Epilogue: dV and dK rows (transpose of RoPE on dK) staged transposed in the now idle stage
+    // buffers, then stored as dQKV^T columns with coalesced 16-byte stores.
+    const bool have = ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status);
+    bf16_t* tv = reinterpret_cast<bf16_t*>(smem + L::ST_OFF);
+    bf16_t* tk = tv + DH * 128;
+    const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
+    if (have) {
       tc::fence_after_sync();
-      const bool valid = key < p.T;
-      const int64_t n = (int64_t)row0 + (valid ? key : 0);
-      const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
-      write_grad_row<DH>(tmem + lane_base + DV_COL, 1.f, false, 0, p.cos_t, p.sin_t,
-                         p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt + n, p.ldt, valid, pr0, pr1);
-      write_grad_row<DH>(tmem + lane_base + DK_COL, p.scale, p.use_rope != 0, valid ? key : 0,
-                         p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt + n,
-                         p.ldt, valid, pr0, pr1);
+      stage_grad_row<DH>(tmem + lane_base + DV_COL, 1.f, false, 0, p.cos_t, p.sin_t, tv, row, pr0,
+                         pr1);
+      stage_grad_row<DH>(tmem + lane_base + DK_COL, p.scale, p.use_rope != 0,
+                         key < p.T ? key : 0, p.cos_t, p.sin_t, tk, row, pr0, pr1);
+    }
+    tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
+    if (have) {
+      const int nvalid = min(BK, p.T - kb * BK);
+      const int64_t n0 = (int64_t)row0 + kb * BK;
+      const int tid = threadIdx.x - 64;
+      store_tile<DH>(tv, p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
+                     EW_WARPS * 32);
+      store_tile<DH>(tk, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
+                     EW_WARPS * 32);
     }
   }
   tc::fence_before_sync();
@@ -437,39 +483,49 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t do_base = tc::smem_u32(smem + L::DO_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
       bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
-      auto issue_dq = [&](int jj) -> bool {
-        if (!tc::mbar_wait(&bars->p_full, jj & 1, abort, p.status)) return false;
-        tc::fence_after_sync();
-        const int st = jj % STAGES;
-        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+      int ns = 0, ng = 0;  // next S / dP block, next dQ block (event-driven, as in dkdv)
+      tc::Watchdog wd;
+      while (ok && ng < n_kb) {
+        bool prog = false;
+        if (ns < n_kb && ns <= ng + 2) {
+          const int st = ns % STAGES, sbuf = ns & 1;
+          if (tc::mbar_ready(&bars->ld_full[st], (ns / STAGES) & 1) &&
+              tc::mbar_ready(&bars->s_empty[sbuf], ((ns >> 1) & 1) ^ 1)) {
+            tc::fence_after_sync();
+            const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k)
-          tc::umma_f16(tmem + DQ_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
-                       tc::sdesc_mnmajor_sw128(sb + L::ST_K + k * 16 * 128, L::KCHUNK, 1024), ID_G,
-                       (jj > 0 || k > 0) ? 1u : 0u);
-        tc::umma_commit(&bars->ld_empty[st]);
-        tc::umma_commit(&bars->p_empty);
-        return true;
-      };
-      for (int j = 0; ok && j < n_kb; ++j) {
-        const int st = j % STAGES;
-        const int sbuf = j & 1;
-        if (!tc::mbar_wait(&bars->ld_full[st], (j / STAGES) & 1, abort, p.status)) break;
-        if (!tc::mbar_wait(&bars->s_empty[sbuf], ((j >> 1) & 1) ^ 1, abort, p.status)) break;
-        tc::fence_after_sync();
-        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
-#pragma unroll
-        for (int k = 0; k < DH / 16; ++k) {
-          const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
-          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
-          tc::umma_f16(tmem + sbuf * BK, tc::sdesc_kmajor_sw128(q_base + qo),
-                       tc::sdesc_kmajor_sw128(sb + L::ST_K + ko), ID_S, k > 0 ? 1u : 0u);
-          tc::umma_f16(tmem + 128 + sbuf * BK, tc::sdesc_kmajor_sw128(do_base + qo),
-                       tc::sdesc_kmajor_sw128(sb + L::ST_V + ko), ID_S, k > 0 ? 1u : 0u);
+            for (int k = 0; k < DH / 16; ++k) {
+              const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
+              const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
+              tc::umma_f16(tmem + sbuf * BK, tc::sdesc_kmajor_sw128(q_base + qo),
+                           tc::sdesc_kmajor_sw128(sb + L::ST_K + ko), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16(tmem + 128 + sbuf * BK, tc::sdesc_kmajor_sw128(do_base + qo),
+                           tc::sdesc_kmajor_sw128(sb + L::ST_V + ko), ID_S, k > 0 ? 1u : 0u);
+            }
+            tc::umma_commit(&bars->s_full[sbuf]);
+            ++ns;
+            prog = true;
+          }
         }
-        tc::umma_commit(&bars->s_full[sbuf]);
-        if (j > 0 && !issue_dq(j - 1)) break;
-        if (j == n_kb - 1 && issue_dq(j)) tc::umma_commit(&bars->o_full);
+        if (ng < ns && tc::mbar_ready(&bars->p_full, ng & 1)) {
+          tc::fence_after_sync();
+          const int st = ng % STAGES;
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc::umma_f16(tmem + DQ_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
+                         tc::sdesc_mnmajor_sw128(sb + L::ST_K + k * 16 * 128, L::KCHUNK, 1024),
+                         ID_G, (ng > 0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&bars->ld_empty[st]);
+          tc::umma_commit(&bars->p_empty);
+          if (ng == n_kb - 1) tc::umma_commit(&bars->o_full);
+          ++ng;
+          prog = true;
+        }
+        if (prog)
+          wd.progress();
+        else if (!wd.tick(abort, p.status))
+          ok = false;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
@@ -526,14 +582,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->p_full);
     }
-    if (ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status)) {
+    // Epilogue: dQ rows (transpose of RoPE) staged transposed in the idle stage buffers, then
+    // stored as dQKV^T columns with coalesced 16-byte stores.
+    const bool have = ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status);
+    bf16_t* tq = reinterpret_cast<bf16_t*>(smem + L::ST_OFF);
+    const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
+    if (have) {
       tc::fence_after_sync();
-      const int64_t n = (int64_t)row0 + (valid_row ? t : 0);
-      const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
-      write_grad_row<DH>(tmem + lane_base + DQ_COL, p.scale, p.use_rope != 0, valid_row ? t : 0,
-                         p.cos_t, p.sin_t, p.dqkvt + (int64_t)(p.qcol0 + h * DH) * p.ldt + n, p.ldt,
-                         valid_row, pr0, pr1);
+      stage_grad_row<DH>(tmem + lane_base + DQ_COL, p.scale, p.use_rope != 0, valid_row ? t : 0,
+                         p.cos_t, p.sin_t, tq, row, pr0, pr1);
     }
+    tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
+    if (have)
+      store_tile<DH>(tq, p.dqkvt + (int64_t)(p.qcol0 + h * DH) * p.ldt, p.ldt,
+                     (int64_t)row0 + q0, min(BQ, p.T - q0), threadIdx.x - 64, EW_WARPS * 32);
   }
   tc::fence_before_sync();
   __syncthreads();
