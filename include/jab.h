@@ -49,7 +49,9 @@ typedef enum {
   JAB_ERR_CUDA = 3,          /* a CUDA runtime call or kernel launch failed                      */
   JAB_ERR_NONFINITE = 4,     /* device: scale <= 0 or non-finite, or a non-finite result          */
   JAB_ERR_RANGE = 5,         /* device: an input value is outside the fp16 range (|x| > 65504)   */
-  JAB_ERR_TIMEOUT = 6        /* device: a bounded wait in a pipelined kernel gave up             */
+  JAB_ERR_TIMEOUT = 6,       /* device: a bounded wait in a pipelined kernel gave up             */
+  JAB_ERR_SCRATCH_LIMIT = 7  /* jab_loss_forward_noalloc: the problem needs more scratch than the
+                                fixed JAB_NOALLOC_SCRATCH_BYTES                                    */
 } jab_status;
 
 /* One attention block. Section 2.1 (d, d_head), App. C (Mistral-7B: GQA, RoPE theta = 1e4). */
@@ -119,6 +121,26 @@ jab_status jab_quantize(const jab_block_desc* desc, int32_t bits, const void* W_
  *   scales_dev     out fp32 [(Hq+2Hkv)*d_h, d_model/G] */
 jab_status jab_init_scales(const jab_block_desc* desc, int32_t bits, int32_t mode,
                            const void* W_dev, float* scales_dev, jab_stream_t stream);
+
+/* Bytes of the fixed device scratch array behind jab_loss_forward_noalloc (64 MiB). */
+#define JAB_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
+
+/* jab_loss_forward without a caller workspace, for callers that cannot allocate device memory (all
+ * of it reserved up front by another allocator, or allocation forbidden where the loss is needed).
+ * The paper has no counterpart: this is a deployment convenience around the same computation.
+ * Arguments and results are those of jab_loss_forward minus ws / ws_bytes; the scratch is one
+ * file-scope device array of JAB_NOALLOC_SCRATCH_BYTES that every GPU loading this library holds
+ * until the process exits. Problems whose jab_workspace_size(desc, B, T, n_cand, 0) exceeds it
+ * return JAB_ERR_SCRATCH_LIMIT (e.g. a GPT-2-sized block with a few candidates and a few thousand
+ * tokens fits; a full Mistral-sized calibration batch does not). The first call on a device looks
+ * up the array's device address (cudaGetSymbolAddress), so make that first call before any stream
+ * capture. No memory is allocated or freed by any call. All calls share the one array: calls that
+ * overlap on the GPU (different streams, no ordering between them) race on it; serialise them. */
+jab_status jab_loss_forward_noalloc(const jab_block_desc* desc, int32_t B, int32_t T,
+                                   const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                   int32_t n_cand, const int32_t* bits_host,
+                                   const float* const* scales_host, double* loss_dev,
+                                   double* sse_parts_dev, jab_stream_t stream);
 
 /* Synchronises `stream`, then returns and clears the device-side status of the current device
  * (JAB_OK if no kernel reported a problem since the last call). */

@@ -15,7 +15,8 @@ import torch
 
 JAB_OK = 0
 _STATUS_NAMES = {0: "JAB_OK", 1: "JAB_ERR_INVALID_ARG", 2: "JAB_ERR_UNSUPPORTED", 3: "JAB_ERR_CUDA",
-                 4: "JAB_ERR_NONFINITE", 5: "JAB_ERR_RANGE", 6: "JAB_ERR_TIMEOUT"}
+                 4: "JAB_ERR_NONFINITE", 5: "JAB_ERR_RANGE", 6: "JAB_ERR_TIMEOUT",
+                 7: "JAB_ERR_SCRATCH_LIMIT"}
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -70,6 +71,8 @@ def lib() -> ctypes.CDLL:
     L.jab_reference_forward.argtypes = [D, i32, i32, _P, _P, _P, _P, _P, _P, sz, _P]
     L.jab_loss_forward.argtypes = [D, i32, i32, _P, _P, _P, i32, ctypes.POINTER(i32),
                                    ctypes.POINTER(_P), _P, _P, _P, sz, _P]
+    L.jab_loss_forward_noalloc.argtypes = [D, i32, i32, _P, _P, _P, i32, ctypes.POINTER(i32),
+                                           ctypes.POINTER(_P), _P, _P, _P]
     L.jab_loss_backward_scales.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P, _P, sz, _P]
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
@@ -83,7 +86,8 @@ def lib() -> ctypes.CDLL:
     L.jab_timing_get.argtypes = [i32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_double),
                                  ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
     L.jab_timing_reset.argtypes = []
-    for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_backward_scales",
+    for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
+               "jab_loss_backward_scales",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
         getattr(L, fn).restype = i32
@@ -163,6 +167,24 @@ def jab_loss_forward(desc, B, T, X, W, A_ref, bits: Sequence[int], scales: Seque
         _ptr(loss, torch.float64, "loss"), _ptr(sse_parts, torch.float64, "sse_parts"), ws.ptr,
         ws.nbytes, _stream(stream))
     _check(st, "jab_loss_forward")
+
+
+def jab_loss_forward_noalloc(desc, B, T, X, W, A_ref, bits: Sequence[int],
+                             scales: Sequence[torch.Tensor], loss, sse_parts=None, stream=None):
+    """jab_loss_forward on the library's fixed device scratch (no workspace argument): for callers
+    that cannot allocate device memory. Raises JabError(JAB_ERR_SCRATCH_LIMIT) when the problem
+    needs more scratch than JAB_NOALLOC_SCRATCH_BYTES."""
+    n = len(bits)
+    if len(scales) != n:
+        raise ValueError("bits and scales must have the same length")
+    bits_arr = (ctypes.c_int32 * n)(*[int(b) for b in bits])
+    sc_arr = (ctypes.c_void_p * n)(*[_ptr(s, torch.float32, "scales") for s in scales])
+    st = lib().jab_loss_forward_noalloc(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), n, bits_arr, sc_arr,
+        _ptr(loss, torch.float64, "loss"), _ptr(sse_parts, torch.float64, "sse_parts"),
+        _stream(stream))
+    _check(st, "jab_loss_forward_noalloc")
 
 
 def jab_loss_backward_scales(desc, B, T, X, W, A_ref, bits: int, scales, kappa: float, loss,

@@ -328,6 +328,7 @@ const char* jab_status_string(jab_status status) {
     case JAB_ERR_NONFINITE: return "non-finite or non-positive value";
     case JAB_ERR_RANGE: return "input outside the fp16 range";
     case JAB_ERR_TIMEOUT: return "device wait timed out";
+    case JAB_ERR_SCRATCH_LIMIT: return "problem larger than the fixed no-allocation scratch";
   }
   return "unknown status";
 }
