@@ -31,6 +31,7 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
+from paper_2609_34866_gb300.multi import dist_env, max_over_ranks  # noqa: E402
 from workloads import WORKLOADS, make_block_weights, make_x  # noqa: E402
 
 METRIC = "JAB candidate-loss evals/s (fwd+STE bwd), Mistral-7B-shaped attention block"
@@ -132,13 +133,6 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def dist_env():
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return world, rank, local
-
-
 def config_of(wl):
     s = wl.shape
     return {"workload": wl.name, "batch": wl.batch, "seq_len": wl.seq_len, "d_model": s.d_model,
@@ -233,13 +227,6 @@ def run_ours(args, wl):
         if world > 1:
             torch.distributed.barrier()
 
-    def max_over_ranks(x):
-        if world > 1:
-            t = torch.tensor([x], dtype=torch.float64, device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            return t.item()
-        return x
-
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -261,7 +248,7 @@ def run_ours(args, wl):
     barrier()
     J.jab_timing_enable(False)
     sites = J.jab_timing_read()
-    ms = max_over_ranks(e0.elapsed_time(e1))
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
     if J.jab_get_device_status() != 0:
         raise RuntimeError("device status set in the timed region")
     ms_step = ms / args.steps
@@ -289,11 +276,18 @@ def run_ours(args, wl):
         achieved = amount / (per_launch_ms / 1e3) / 1e9
         bound, peak, unit = "hbm", pk["hbm"], "GB/s"
         peak_note = f"{pk['source']} HBM copy bandwidth"
-    traffic = None
+    traffic = None  # DRAM bytes per launch from an ncu capture, only while the kernel source is unchanged
     tfile = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tfile):
+        import hashlib
         with open(tfile) as f:
-            traffic = json.load(f).get(f"{dom}@{wl.name}@{'tc' if tc else 'simple'}")
+            ent = json.load(f).get(f"{dom}@{wl.name}@B{wl.batch}xT{wl.seq_len}@{'tc' if tc else 'simple'}")
+        if ent:
+            csrc = os.path.join(ROOT, "paper_2609_34866_gb300", "csrc")
+            same = all(hashlib.sha256(open(os.path.join(csrc, fn), "rb").read()).hexdigest()[:16] == h
+                       for fn, h in ent.get("csrc_sha256_16", {}).items()
+                       if os.path.exists(os.path.join(csrc, fn)))
+            traffic = ent["bytes_per_launch"] if same else None
     roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
                 "frac": achieved / peak, "traffic": traffic, "kernel": dom,
                 "launch_ms": per_launch_ms, "peak_source": peak_note}
@@ -310,7 +304,7 @@ def run_ours(args, wl):
         fwd_step()
     e1.record(st)
     torch.cuda.synchronize()
-    fwd_ms = max_over_ranks(e0.elapsed_time(e1))
+    fwd_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     fwd_value = world * args.steps / (fwd_ms / 1e3)
 
     # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed region
@@ -337,7 +331,7 @@ def run_ours(args, wl):
             e2e_step()
         e1.record(st)
         torch.cuda.synchronize()
-        e2e_ms = max_over_ranks(e0.elapsed_time(e1))
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
         h2d = sum(t.numel() * t.element_size() for t in (hX, hW, hA, hS))
         d2h = hL.numel() * 8 + hG.numel() * 4
         e2e = {"value": world * args.steps / (e2e_ms / 1e3), "unit": "evals/s",
@@ -346,8 +340,11 @@ def run_ours(args, wl):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        dt, sample = oracle_sample(wl, 1)
-        cpu = {"value": 1.0 / (dt * wl.batch), "unit": "evals/s", "cores": os.cpu_count(),
+        # a bounded sample of ~10-20 s of oracle work: size it from one sequence's time
+        dt1, _ = oracle_sample(wl, 1)
+        k = max(1, min(wl.batch, int(np.ceil(12.0 / max(dt1, 1e-3)))))
+        dt, sample = oracle_sample(wl, k) if k > 1 else (dt1, _)
+        cpu = {"value": k / (dt * wl.batch), "unit": "evals/s", "cores": os.cpu_count(),
                "kind": "oracle", "sample": sample, "seconds": dt}
 
     if world > 1:
@@ -381,10 +378,15 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="mistral_block", choices=sorted(WORKLOADS))
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's sequence count (smaller cases for profiling)")
+    ap.add_argument("--seq-len", type=int, default=None, help="override the workload's sequence length")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     wl = WORKLOADS[args.workload]
+    if args.batch is not None or args.seq_len is not None:
+        wl = wl.with_batch(args.batch or wl.batch, args.seq_len)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)

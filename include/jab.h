@@ -142,6 +142,12 @@ jab_status jab_loss_forward_noalloc(const jab_block_desc* desc, int32_t B, int32
                                    const float* const* scales_host, double* loss_dev,
                                    double* sse_parts_dev, jab_stream_t stream);
 
+/* Failure-path self-test (not part of the method): launches one CTA that waits, with the bounded
+ * mbarrier wait of every pipelined kernel, on a barrier phase nothing completes. After the wait's
+ * 2-second limit the kernel sets JAB_ERR_TIMEOUT in the device status and returns; the context
+ * stays usable. Read the result with jab_get_device_status. */
+jab_status jab_selftest_wait_timeout(jab_stream_t stream);
+
 /* Synchronises `stream`, then returns and clears the device-side status of the current device
  * (JAB_OK if no kernel reported a problem since the last call). */
 jab_status jab_get_device_status(jab_stream_t stream);

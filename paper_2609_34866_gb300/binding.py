@@ -77,6 +77,7 @@ def lib() -> ctypes.CDLL:
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
     L.jab_get_device_status.argtypes = [_P]
+    L.jab_selftest_wait_timeout.argtypes = [_P]
     L.jab_status_string.argtypes = [i32]
     L.jab_status_string.restype = ctypes.c_char_p
     L.jab_timing_enable.argtypes = [i32]
@@ -89,6 +90,7 @@ def lib() -> ctypes.CDLL:
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
                "jab_loss_backward_scales",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
+               "jab_selftest_wait_timeout",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
         getattr(L, fn).restype = i32
     _LIB = L
@@ -209,6 +211,11 @@ def jab_init_scales(desc, bits, mode, W, scales, stream=None):
                                _ptr(W, torch.bfloat16, "W"), _ptr(scales, torch.float32, "scales"),
                                _stream(stream))
     _check(st, "jab_init_scales")
+
+
+def jab_selftest_wait_timeout(stream=None):
+    """Launches the bounded-wait self-test kernel (its wait runs out after 2 s)."""
+    _check(lib().jab_selftest_wait_timeout(_stream(stream)), "jab_selftest_wait_timeout")
 
 
 def jab_get_device_status(stream=None) -> int:

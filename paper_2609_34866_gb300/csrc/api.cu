@@ -41,6 +41,16 @@ jab_status device_info(int** status, int* sms) {
   return JAB_OK;
 }
 
+}  // namespace
+
+// The device status word of the current device (for kernels launched outside this file).
+jab_status device_status_ptr(int** status) {
+  int sms = 0;
+  return device_info(status, &sms);
+}
+
+namespace {
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 jab_status check_desc(const jab_block_desc* d) {

@@ -192,3 +192,15 @@ def test_error_paths():
     J().jab_loss_forward(c.desc, c.B, c.T, X, c.W, A, [3], [s], loss, ws)
     assert J().jab_get_device_status() == 5
     assert J().jab_get_device_status() == 0
+
+
+def test_bounded_wait_times_out_and_context_survives():
+    """A pipelined kernel's wait on a barrier that never flips gives up after its limit, reports
+    JAB_ERR_TIMEOUT through the status word, and later calls still work (no fault, no hang)."""
+    J().jab_get_device_status()
+    J().jab_selftest_wait_timeout()
+    assert J().jab_get_device_status() == 6
+    c = case("gpt2_T1")
+    A, _, _ = c.gpu_teacher()
+    assert J().jab_get_device_status() == 0
+    np.testing.assert_allclose(np64(A), c.oracle_teacher(), rtol=0, atol=1e-2 * np.abs(c.oracle_teacher()).max())
