@@ -391,20 +391,70 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ================================================================================ dQ
+// Persistent: one CTA per SM walks a longest-first list of (128 query rows, query head, sequence)
+// tiles with 128-key blocks, so every UMMA is M128 N128. TMEM: S = Q K^T (128 columns) and
+// dP = dO V^T (128) single-buffered, and two dQ accumulators (2 x 128) so that the next tile's
+// MMAs run while the elementwise warps finish the previous tile's epilogue. K has a 2-stage ring
+// (read by S and later by dQ), V a single buffer (read only by dP); the next tile's Q and dO load
+// as soon as the current tile's last S/dP has completed.
 template <int DH>
 struct DqLayout {
-  static constexpr int BQ = 128, BK = 64;
-  static constexpr int QCHUNK = BQ * 128;
-  static constexpr int KCHUNK = BK * 128;
+  static constexpr int BQ = 128, BK = 128;
+  static constexpr int CHUNK = 128 * 128;  // 64 columns of a 128-row tile
+  static constexpr int TILE = 128 * DH * 2;
   static constexpr int Q_OFF = 0;
-  static constexpr int DO_OFF = Q_OFF + BQ * DH * 2;
-  static constexpr int ST_OFF = DO_OFF + BQ * DH * 2;
-  static constexpr int ST_K = 0, ST_V = BK * DH * 2, ST_BYTES = 2 * BK * DH * 2;
-  static constexpr int DS_OFF = ST_OFF + STAGES * ST_BYTES;
-  static constexpr int BAR_OFF = DS_OFF + BQ * BK * 2;
+  static constexpr int DO_OFF = Q_OFF + TILE;
+  static constexpr int K_OFF = DO_OFF + TILE;  // 2 stages
+  static constexpr int V_OFF = K_OFF + 2 * TILE;
+  static constexpr int DS_OFF = V_OFF + TILE;  // dS, and the epilogue's staging tile
+  static constexpr int DS_BYTES = BQ * BK * 2;
+  static constexpr int BAR_OFF = DS_OFF + DS_BYTES;
   static constexpr int USED = BAR_OFF + 256 + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
 };
+
+struct DqBars {
+  uint64_t qdo_full, qdo_empty, k_full[2], k_empty[2], v_full, v_empty, s_full, s_empty;
+  uint64_t p_full, p_empty, o_full[2], o_empty[2], drain;
+  uint32_t tmem_base;
+  int abort;
+  int ew_count;  // arrivals at the elementwise warps' epilogue barrier
+};
+
+// Time-bounded barrier of the 8 elementwise warps (epoch-numbered; no hardware barrier that could
+// hang if a warp left early).
+__device__ __forceinline__ void ew_barrier(DqBars* bars, int epoch, volatile int* abort,
+                                           int* status) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) {
+    __threadfence_block();
+    atomicAdd(&bars->ew_count, 1);
+    volatile int* c = &bars->ew_count;
+    const uint64_t t0 = tc::globaltimer();
+    for (uint32_t it = 0; *c < EW_WARPS * epoch; ++it) {
+      if ((it & 63u) == 0) {
+        if (*abort) break;
+        if (tc::globaltimer() - t0 > tc::kWaitLimitNs) {
+          *abort = 1;
+          report(status, JAB_ERR_TIMEOUT);
+          break;
+        }
+      }
+    }
+    __threadfence_block();
+  }
+  __syncwarp();
+}
+
+struct DqTile {
+  int qb, h, b;
+};
+// Tile n of the longest-first order: query blocks from the last (most keys) to the first.
+__device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
+  const int per_qb = Hq * B;
+  const int r = n % per_qb;
+  return DqTile{nqb - 1 - n / per_qb, r % Hq, r / Hq};
+}
 
 template <int DH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -416,20 +466,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  BwdBars* bars = reinterpret_cast<BwdBars*>(smem + L::BAR_OFF);
+  DqBars* bars = reinterpret_cast<DqBars*>(smem + L::BAR_OFF);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
 
   const int nqb = (p.T + BQ - 1) / BQ;
-  const int qb = nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
-  const int h = blockIdx.x, b = blockIdx.y;
-  const int g = h / (p.Hq / p.Hkv);
-  const int q0 = qb * BQ;
-  const int n_kb = (min(q0 + BQ, p.T) + BK - 1) / BK;
-  const int row0 = b * p.T;
+  const int n_tiles = nqb * p.Hq * p.B;
+  auto n_kb_of = [&](const DqTile& tl) { return (min(tl.qb * BQ + BQ, p.T) + BK - 1) / BK; };
 
   if (threadIdx.x == 0) {
-    init_bars(bars);
+    tc::mbar_init(&bars->qdo_full, 1);
+    tc::mbar_init(&bars->qdo_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&bars->k_full[i], 1);
+      tc::mbar_init(&bars->k_empty[i], 1);
+      tc::mbar_init(&bars->o_full[i], 1);
+      tc::mbar_init(&bars->o_empty[i], EW_WARPS);
+    }
+    tc::mbar_init(&bars->v_full, 1);
+    tc::mbar_init(&bars->v_empty, 1);
+    tc::mbar_init(&bars->s_full, 1);
+    tc::mbar_init(&bars->s_empty, EW_WARPS);
+    tc::mbar_init(&bars->p_full, EW_WARPS);
+    tc::mbar_init(&bars->p_empty, 1);
+    tc::mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    bars->ew_count = 0;
+    tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_q);
     tc::prefetch_tmap(&tm_kv);
     tc::prefetch_tmap(&tm_do);
@@ -442,37 +505,50 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
-  constexpr uint32_t DQ_COL = 256;
+  constexpr uint32_t S_COL = 0, DP_COL = 128, DQ_COL = 256;
 
   if (warp == 0) {
     if (lane == 0) {  // ------------------------------------------------------------- TMA
-      uint32_t issued = 0, last_par = 0;
-      tc::mbar_expect_tx(&bars->fixed_full, 2 * BQ * DH * 2);
-      for (int ch = 0; ch < DH / 64; ++ch) {
-        tc::tma_load_2d(smem + L::Q_OFF + ch * L::QCHUNK, &tm_q, &bars->fixed_full,
-                        p.qcol0 + h * DH + ch * 64, row0 + q0);
-        tc::tma_load_2d(smem + L::DO_OFF + ch * L::QCHUNK, &tm_do, &bars->fixed_full,
-                        h * DH + ch * 64, row0 + q0);
-      }
-      for (int j = 0; j < n_kb; ++j) {
-        const int st = j % STAGES;
-        const uint32_t ph = (j / STAGES) & 1;
-        if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
-        uint8_t* sbase = smem + L::ST_OFF + st * L::ST_BYTES;
-        tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
+      uint32_t J = 0;  // key blocks loaded so far (all tiles)
+      int n = 0;
+      bool qdo_issued = false, v_issued = false;
+      uint32_t k_issued = 0, k_par = 0, qdo_par = 0, v_par = 0;
+      for (int tile = blockIdx.x; tile < n_tiles && !*abort; tile += gridDim.x, ++n) {
+        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+        const int row0 = tl.b * p.T, g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
+        if (!tc::mbar_wait(&bars->qdo_empty, (n & 1) ^ 1, abort, p.status)) break;
+        tc::mbar_expect_tx(&bars->qdo_full, 2 * L::TILE);
         for (int ch = 0; ch < DH / 64; ++ch) {
-          tc::tma_load_2d(sbase + L::ST_K + ch * L::KCHUNK, &tm_kv, &bars->ld_full[st],
-                          p.kcol0 + g * DH + ch * 64, row0 + j * BK);
-          tc::tma_load_2d(sbase + L::ST_V + ch * L::KCHUNK, &tm_kv, &bars->ld_full[st],
-                          p.vcol0 + g * DH + ch * 64, row0 + j * BK);
+          tc::tma_load_2d(smem + L::Q_OFF + ch * L::CHUNK, &tm_q, &bars->qdo_full,
+                          p.qcol0 + tl.h * DH + ch * 64, row0 + tl.qb * BQ);
+          tc::tma_load_2d(smem + L::DO_OFF + ch * L::CHUNK, &tm_do, &bars->qdo_full,
+                          tl.h * DH + ch * 64, row0 + tl.qb * BQ);
         }
-        issued |= 1u << st;
-        last_par = (last_par & ~(1u << st)) | (ph << st);
+        qdo_issued = true;
+        qdo_par = n & 1;
+        for (int j = 0; j < nkb; ++j, ++J) {
+          const int st = J & 1;
+          if (!tc::mbar_wait(&bars->k_empty[st], ((J >> 1) & 1) ^ 1, abort, p.status)) break;
+          tc::mbar_expect_tx(&bars->k_full[st], L::TILE);
+          for (int ch = 0; ch < DH / 64; ++ch)
+            tc::tma_load_2d(smem + L::K_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv,
+                            &bars->k_full[st], p.kcol0 + g * DH + ch * 64, row0 + j * BK);
+          k_issued |= 1u << st;
+          k_par = (k_par & ~(1u << st)) | (((J >> 1) & 1u) << st);
+          if (!tc::mbar_wait(&bars->v_empty, (J & 1) ^ 1, abort, p.status)) break;
+          tc::mbar_expect_tx(&bars->v_full, L::TILE);
+          for (int ch = 0; ch < DH / 64; ++ch)
+            tc::tma_load_2d(smem + L::V_OFF + ch * L::CHUNK, &tm_kv, &bars->v_full,
+                            p.vcol0 + g * DH + ch * 64, row0 + j * BK);
+          v_issued = true;
+          v_par = J & 1;
+        }
       }
       if (*abort) {
-        drain_wait(&bars->fixed_full, 0);
-        for (int st = 0; st < STAGES; ++st)
-          if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
+        if (qdo_issued) drain_wait(&bars->qdo_full, qdo_par);
+        for (int st = 0; st < 2; ++st)
+          if (k_issued & (1u << st)) drain_wait(&bars->k_full[st], (k_par >> st) & 1);
+        if (v_issued) drain_wait(&bars->v_full, v_par);
       }
     }
   } else if (warp == 1) {
@@ -481,121 +557,163 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
       const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
       const uint32_t do_base = tc::smem_u32(smem + L::DO_OFF);
+      const uint32_t v_base = tc::smem_u32(smem + L::V_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
-      bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
-      int ns = 0, ng = 0;  // next S / dP block, next dQ block (event-driven, as in dkdv)
+      bool ok = true;
+      uint32_t Js = 0, Jg = 0;  // S/dP blocks and dQ blocks issued so far (all tiles)
+      int n = 0;
       tc::Watchdog wd;
-      while (ok && ng < n_kb) {
-        bool prog = false;
-        if (ns < n_kb && ns <= ng + 2) {
-          const int st = ns % STAGES, sbuf = ns & 1;
-          if (tc::mbar_ready(&bars->ld_full[st], (ns / STAGES) & 1) &&
-              tc::mbar_ready(&bars->s_empty[sbuf], ((ns >> 1) & 1) ^ 1)) {
+      for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++n) {
+        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+        const int nkb = n_kb_of(tl);
+        const uint32_t acc = DQ_COL + (n & 1) * 128;
+        if (!tc::mbar_wait(&bars->qdo_full, n & 1, abort, p.status) ||
+            !tc::mbar_wait(&bars->o_empty[n & 1], ((n >> 1) & 1) ^ 1, abort, p.status)) {
+          ok = false;
+          break;
+        }
+        // Event-driven issue: S/dP of block ns as soon as K_ns, V_ns have landed and the
+        // elementwise warps have read the previous S/dP; dQ of block ng once its dS is written.
+        int ns = 0, ng = 0;
+        while (ok && ng < nkb) {
+          bool prog = false;
+          if (ns < nkb && ns <= ng + 1 && tc::mbar_ready(&bars->k_full[Js & 1], (Js >> 1) & 1) &&
+              tc::mbar_ready(&bars->v_full, Js & 1) && tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
             tc::fence_after_sync();
-            const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Js & 1) * L::TILE);
 #pragma unroll
             for (int k = 0; k < DH / 16; ++k) {
-              const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
-              const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
-              tc::umma_f16(tmem + sbuf * BK, tc::sdesc_kmajor_sw128(q_base + qo),
-                           tc::sdesc_kmajor_sw128(sb + L::ST_K + ko), ID_S, k > 0 ? 1u : 0u);
-              tc::umma_f16(tmem + 128 + sbuf * BK, tc::sdesc_kmajor_sw128(do_base + qo),
-                           tc::sdesc_kmajor_sw128(sb + L::ST_V + ko), ID_S, k > 0 ? 1u : 0u);
+              const uint32_t off = (k >> 2) * L::CHUNK + (k & 3) * 32;
+              tc::umma_f16(tmem + S_COL, tc::sdesc_kmajor_sw128(q_base + off),
+                           tc::sdesc_kmajor_sw128(k_base + off), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16(tmem + DP_COL, tc::sdesc_kmajor_sw128(do_base + off),
+                           tc::sdesc_kmajor_sw128(v_base + off), ID_S, k > 0 ? 1u : 0u);
             }
-            tc::umma_commit(&bars->s_full[sbuf]);
+            tc::umma_commit(&bars->s_full);
+            tc::umma_commit(&bars->v_empty);
             ++ns;
+            ++Js;
+            if (ns == nkb) tc::umma_commit(&bars->qdo_empty);  // Q, dO free for the next tile
             prog = true;
           }
-        }
-        if (ng < ns && tc::mbar_ready(&bars->p_full, ng & 1)) {
-          tc::fence_after_sync();
-          const int st = ng % STAGES;
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_BYTES);
+          if (ng < ns && tc::mbar_ready(&bars->p_full, Jg & 1)) {
+            tc::fence_after_sync();
+            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Jg & 1) * L::TILE);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            tc::umma_f16(tmem + DQ_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
-                         tc::sdesc_mnmajor_sw128(sb + L::ST_K + k * 16 * 128, L::KCHUNK, 1024),
-                         ID_G, (ng > 0 || k > 0) ? 1u : 0u);
-          tc::umma_commit(&bars->ld_empty[st]);
-          tc::umma_commit(&bars->p_empty);
-          if (ng == n_kb - 1) tc::umma_commit(&bars->o_full);
-          ++ng;
-          prog = true;
+            for (int k = 0; k < BK / 16; ++k)
+              tc::umma_f16(tmem + acc,
+                           tc::sdesc_kmajor_sw128(ds_base + (k >> 2) * (BQ * 128) + (k & 3) * 32),
+                           tc::sdesc_mnmajor_sw128(k_base + k * 16 * 128, L::CHUNK, 1024), ID_G,
+                           (ng > 0 || k > 0) ? 1u : 0u);
+            tc::umma_commit(&bars->k_empty[Jg & 1]);
+            tc::umma_commit(&bars->p_empty);
+            ++ng;
+            ++Jg;
+            if (ng == nkb) tc::umma_commit(&bars->o_full[n & 1]);
+            prog = true;
+          }
+          if (prog)
+            wd.progress();
+          else if (!wd.tick(abort, p.status))
+            ok = false;
         }
-        if (prog)
-          wd.progress();
-        else if (!wd.tick(abort, p.status))
-          ok = false;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else {  // ------------------------------------------------ elementwise: row = query, 32 keys
+  } else {  // ------------------------------------------------ elementwise: row = query, 64 keys
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
     const int row = quarter * 32 + lane;
-    const int t = q0 + row;
-    const int col0 = half * 32;
-    const bool valid_row = t < p.T;
+    const int col0 = half * 64;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + (valid_row ? t : 0);
-    const float lse2 = valid_row ? p.lse[lrow] : INFINITY;  // P = 0 on rows past T
-    const float drow = valid_row ? p.dvec[lrow] : 0.f;
-    bool ok = true;
-    for (int j = 0; j < n_kb; ++j) {
-      const int sbuf = j & 1;
-      if (!tc::mbar_wait(&bars->s_full[sbuf], (j >> 1) & 1, abort, p.status)) {
-        ok = false;
-        break;
-      }
-      tc::fence_after_sync();
-      uint32_t rs[32], rd[32];
-      __syncwarp();
-      tc::tmem_ld32(tmem + lane_base + sbuf * BK + col0, rs);
-      tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BK + col0, rd);
-      tc::tmem_ld_wait();
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
-      const int k0 = j * BK + col0;
-      float dsv[32];
-      if (k0 + 31 <= q0) {  // every key of this slice is visible to every row of the CTA
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2));
-          dsv[c] = e * (__uint_as_float(rd[c]) - drow);
-        }
-      } else {
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2));
-          dsv[c] = (k0 + c <= t) ? e * (__uint_as_float(rd[c]) - drow) : 0.f;
-        }
-      }
-      if (!tc::mbar_wait(&bars->p_empty, (j & 1) ^ 1, abort, p.status)) {
-        ok = false;
-        break;
-      }
-      store_half_row(smem + L::DS_OFF, row, half, dsv);
-      tc::fence_proxy_async_smem();
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->p_full);
-    }
-    // Epilogue: dQ rows (transpose of RoPE) staged transposed in the idle stage buffers, then
-    // stored as dQKV^T columns with coalesced 16-byte stores.
-    const bool have = ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status);
-    bf16_t* tq = reinterpret_cast<bf16_t*>(smem + L::ST_OFF);
+    uint8_t* dsrow = smem + L::DS_OFF + half * (BQ * 128) + row * 128;  // one 64-key swizzle chunk
+    bf16_t* stage = reinterpret_cast<bf16_t*>(smem + L::DS_OFF);
     const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
-    if (have) {
+    bool ok = true;
+    uint32_t J = 0;
+    int n = 0, epoch = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++n) {
+      const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+      const int nkb = n_kb_of(tl);
+      const int q0 = tl.qb * BQ, t = q0 + row, row0 = tl.b * p.T;
+      const bool valid_row = t < p.T;
+      const int64_t lrow = ((int64_t)tl.b * p.Hq + tl.h) * p.lse_pitch + (valid_row ? t : 0);
+      const float lse2 = valid_row ? p.lse[lrow] : INFINITY;  // P = 0 on rows past T
+      const float drow = valid_row ? p.dvec[lrow] : 0.f;
+      for (int j = 0; ok && j < nkb; ++j, ++J) {
+        if (!tc::mbar_wait(&bars->s_full, J & 1, abort, p.status)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        float sv[64], dp[64];
+#pragma unroll
+        for (int ch = 0; ch < 2; ++ch) {
+          uint32_t rs[32], rd[32];
+          __syncwarp();
+          tc::tmem_ld32(tmem + lane_base + S_COL + col0 + ch * 32, rs);
+          tc::tmem_ld32(tmem + lane_base + DP_COL + col0 + ch * 32, rd);
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            sv[ch * 32 + e] = __uint_as_float(rs[e]);
+            dp[ch * 32 + e] = __uint_as_float(rd[e]);
+          }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->s_empty);
+        const int k0 = j * BK + col0;
+        if (k0 + 63 <= q0) {  // every key of this slice is visible to every row of the tile
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            dp[c] = tc::fast_exp2(fmaf(sv[c], p.sl2, -lse2)) * (dp[c] - drow);
+        } else {
+#pragma unroll
+          for (int c = 0; c < 64; ++c) {
+            const float e = tc::fast_exp2(fmaf(sv[c], p.sl2, -lse2));
+            dp[c] = (k0 + c <= t) ? e * (dp[c] - drow) : 0.f;
+          }
+        }
+        if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
+          ok = false;
+          break;
+        }
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          uint4 u;
+          __half2* hp = reinterpret_cast<__half2*>(&u);
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            hp[e] = __floats2half2_rn(dp[c8 * 8 + 2 * e], dp[c8 * 8 + 2 * e + 1]);
+          *reinterpret_cast<uint4*>(dsrow + ((c8 ^ (row & 7)) << 4)) = u;
+        }
+        tc::fence_proxy_async_smem();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->p_full);
+      }
+      if (!ok) break;
+      // Epilogue: dQ rows (transpose of RoPE) staged transposed in the dS buffer (free until this
+      // tile's successor writes its first dS, which these same warps do next), then stored as
+      // dQKV^T columns with coalesced 16-byte stores.
+      if (!tc::mbar_wait(&bars->o_full[n & 1], (n >> 1) & 1, abort, p.status) ||
+          !tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
       tc::fence_after_sync();
-      stage_grad_row<DH>(tmem + lane_base + DQ_COL, p.scale, p.use_rope != 0, valid_row ? t : 0,
-                         p.cos_t, p.sin_t, tq, row, pr0, pr1);
-    }
-    tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
-    if (have)
-      store_tile<DH>(tq, p.dqkvt + (int64_t)(p.qcol0 + h * DH) * p.ldt, p.ldt,
+      stage_grad_row<DH>(tmem + lane_base + DQ_COL + (n & 1) * 128, p.scale, p.use_rope != 0,
+                         valid_row ? t : 0, p.cos_t, p.sin_t, stage, row, pr0, pr1);
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->o_empty[n & 1]);  // dQ accumulator reusable
+      ew_barrier(bars, ++epoch, abort, p.status);
+      store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
                      (int64_t)row0 + q0, min(BQ, p.T - q0), threadIdx.x - 64, EW_WARPS * 32);
+      ew_barrier(bars, ++epoch, abort, p.status);
+    }
   }
   tc::fence_before_sync();
   __syncthreads();
@@ -643,10 +761,9 @@ cudaError_t set_smem(K kernel, int bytes, bool& done) {
 template <int DH>
 cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   const int64_t N = (int64_t)L.B * L.T;
-  CUtensorMap kv128, q64, do64, q128, kv64, do128;
+  CUtensorMap kv128, q64, do64, do128;
   if (!tmap_rows(&kv128, L.qkv, L.ldq, N, 128) || !tmap_rows(&q64, L.qkv, L.ldq, N, 64) ||
       !tmap_rows(&do64, L.d_o, (uint64_t)L.Hq * DH, N, 64) ||
-      !tmap_rows(&q128, L.qkv, L.ldq, N, 128) || !tmap_rows(&kv64, L.qkv, L.ldq, N, 64) ||
       !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128))
     return cudaErrorInvalidValue;
   static bool a1 = false, a2 = false;
@@ -658,8 +775,12 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, q64, do64, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  dim3 g2((unsigned)L.Hq, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
-  attn_bwd_dq_tc_kernel<DH><<<g2, NUM_THREADS, DqLayout<DH>::SMEM, L.stream>>>(q128, kv64, do128, p);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t dq_tiles = (int64_t)((L.T + 127) / 128) * L.Hq * L.B;
+  const unsigned g2 = (unsigned)std::min<int64_t>(dq_tiles, sms > 0 ? sms : 1);
+  attn_bwd_dq_tc_kernel<DH><<<g2, NUM_THREADS, DqLayout<DH>::SMEM, L.stream>>>(kv128, kv128, do128, p);
   return cudaGetLastError();
 }
 
