@@ -117,7 +117,7 @@ AttnLaunch attn_launch(const jab_block_desc* d, int B, int T, int C, char* ws,
   L.dh = d->head_dim;
   L.C = C;
   L.scale = softmax_scale(d);
-  const int rows = use_tc_path() ? attn_fwd_tc_rows() : kPartRows;  // rows per loss partial
+  const int rows = use_tc_path() ? attn_fwd_tc_rows(d->n_q_heads, d->n_kv_heads) : kPartRows;
   L.nP = (T + rows - 1) / rows;
   L.lse_pitch = T;
   L.part = reinterpret_cast<double*>(ws + wp.part);

@@ -18,6 +18,8 @@
 // The SSE partials are per (candidate, sequence, head, 128-row block), fp64, reduced in fixed order.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+
 #include "path.h"
 #include "tc.cuh"
 
@@ -84,7 +86,7 @@ __device__ __forceinline__ void pair_wait(FwdBars* bars, int half, int row, int 
 }
 
 struct FwdParams {
-  int T, B, Hq, Hkv, D, nqb, nP, lse_pitch;
+  int T, B, C, Hq, Hkv, D, nqb, nP, lse_pitch;
   float sl2;  // softmax scale * log2(e)
   double* part;
   const float* a_ref;
@@ -408,79 +410,136 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ============================================================================ head-pair kernel
-// Two query heads of one KV group per CTA (GQA: they read the same K and V), 128 query rows each,
-// keys in blocks of 64 through a 3-stage K/V ring. Per head: S double-buffered in TMEM (2 x 64
-// columns), O in TMEM (128 columns), P in shared memory; four softmax warps per head, one row per
-// thread. Every K/V byte loaded feeds twice the tensor work of the single-head kernel.
-constexpr int PBQ = 128, PBK = 64, PSTAGES = 3;
+// Persistent: one CTA per SM walks a longest-first list of tiles. A tile is 64 query rows of two
+// query heads of one KV group (GQA: both read the same K and V) stacked into the 128 rows of every
+// UMMA: TMEM lane r < 64 is row q0 + r of head h0, lane 64 + r is row q0 + r of head h0 + 1.
+// Keys come in blocks of 128 so that both products are M128 N128 UMMAs with the A operand in tensor
+// memory (TS form), the shape that runs the tensor pipe at full rate on sm_103a:
+//   S_j = Q K_j^T     A = Q (TMEM, copied from the TMA-loaded smem tile by tcgen05.cp), B = K_j
+//   O  += P_j V_j     A = P_j (TMEM, fp16 pairs written by the softmax threads), B = V_j (smem,
+//                     MN-major)
+// TMEM columns: S double-buffered at 0 / 128, O at 256 (DH columns), Q (DH / 2 columns) and P
+// (64 columns) after it. S_{j+2} is issued as soon as the softmax has read S_j out of its buffer, so
+// the tensor pipe computes the next scores while the softmax of block j runs.
+//   warp 0      TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages, one
+//               block ahead of V), V ring (2 stages)
+//   warp 1      TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
+//   warps 2..9  softmax, two warps per TMEM lane quarter: a thread owns one stacked row and one half
+//               (64 keys) of each S block; the halves agree on the row maximum through shared memory.
+//               Lazy rescaling as in the single-head kernel. Epilogue: O is read out of TMEM (and
+//               released to the next tile) at once, then staged through shared memory so that A_ref
+//               loads and dO / A stores are coalesced.
+constexpr int SQ = 64, SKB = 128, SK_ST = 2, SV_ST = 2;
 
-template <int DH>
-struct PairLayout {
-  static constexpr int QTILE = PBQ * DH * 2;
-  static constexpr int QCHUNK = PBQ * 128;
-  static constexpr int KVTILE = PBK * DH * 2;
-  static constexpr int KVCHUNK = PBK * 128;
-  static constexpr int Q_OFF = 0;
-  static constexpr int KV_OFF = Q_OFF + 2 * QTILE;
-  static constexpr int STAGE = 2 * KVTILE;  // K then V
-  static constexpr int P_OFF = KV_OFF + PSTAGES * STAGE;
-  static constexpr int PTILE = PBQ * PBK * 2;
-  static constexpr int BAR_OFF = P_OFF + 2 * PTILE;
-  static constexpr int USED = BAR_OFF + 512 + 1024;
-  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
-};
-
-struct PairBars {
-  uint64_t q_full, kv_full[PSTAGES], kv_empty[PSTAGES];
-  uint64_t s_full[2][2], s_empty[2][2], p_full[2], p_empty[2], o_full[2], drain;
+struct StackBars {
+  uint64_t q_full, q_empty, k_full[SK_ST], k_empty[SK_ST], v_full[SV_ST], v_empty[SV_ST];
+  uint64_t s_full[2], s_empty[2], p_full, pv_done, o_full, o_empty, drain;
   uint32_t tmem_base;
   int abort;
   double red[EW_WARPS];
+  float xv[2][2][128];  // [sequence parity][half][row]: values exchanged between the two halves
+  int flag[2][128];     // [half][row]: sequence number of the last value posted
 };
+
+template <int DH>
+struct StackLayout {
+  static constexpr int CHUNK = 128 * 128;  // 64 columns of a 128-row tile (128-byte swizzle)
+  static constexpr int TILE = 128 * DH * 2;
+  static constexpr int Q_OFF = 0;
+  static constexpr int K_OFF = Q_OFF + TILE;
+  static constexpr int V_OFF = K_OFF + SK_ST * TILE;
+  static constexpr int EPI_OFF = V_OFF + SV_ST * TILE;  // per softmax warp: 32 x 32 fp32
+  static constexpr int BAR_OFF = EPI_OFF + EW_WARPS * 4096;
+  static constexpr int USED = BAR_OFF + (int)sizeof(StackBars) + 1024;
+  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+  static constexpr uint32_t S_COL = 0, O_COL = 2 * SKB, Q_COL = 2 * SKB + DH,
+                            P_COL = 2 * SKB + DH + DH / 2;
+  static_assert(P_COL + SKB / 2 <= 512, "TMEM budget");
+};
+
+struct StackTile {
+  int hp, bc, qb, nkb;
+};
+
+// Tile k of the longest-first order: query blocks from the last (most key blocks) to the first.
+__device__ __forceinline__ StackTile stack_tile(int k, int pairs, int BC, int nqb, int T) {
+  StackTile t;
+  t.hp = k % pairs;
+  t.bc = (k / pairs) % BC;
+  t.qb = nqb - 1 - k / (pairs * BC);
+  t.nkb = (min((t.qb + 1) * SQ, T) + SKB - 1) / SKB;
+  return t;
+}
+
+// Exchange one float with the thread that owns the other half of the same row. `seq` counts this
+// thread's exchanges; values alternate between two slots, which is enough because neither side can
+// post twice without reading the other's post in between. The wait is time-bounded.
+__device__ __forceinline__ float half_exchange(StackBars* bars, int half, int row, int& seq, float v,
+                                               volatile int* abort, int* status) {
+  ++seq;
+  bars->xv[seq & 1][half][row] = v;
+  __threadfence_block();
+  reinterpret_cast<volatile int*>(&bars->flag[half][row])[0] = seq;
+  volatile int* f = &bars->flag[half ^ 1][row];
+  if (*f < seq) {
+    const uint64_t t0 = tc::globaltimer();
+    for (uint32_t it = 0; *f < seq; ++it) {
+      if ((it & 63u) == 0) {
+        if (*abort) break;
+        if (tc::globaltimer() - t0 > tc::kWaitLimitNs) {
+          *abort = 1;
+          report(status, JAB_ERR_TIMEOUT);
+          break;
+        }
+      }
+    }
+  }
+  __threadfence_block();
+  return reinterpret_cast<volatile float*>(&bars->xv[seq & 1][half ^ 1][row])[0];
+}
 
 template <int DH, int MODE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_fwd_pair_kernel(const __grid_constant__ CUtensorMap tm_q,
                          const __grid_constant__ CUtensorMap tm_kv, const FwdParams p) {
-  using L = PairLayout<DH>;
+  using L = StackLayout<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  PairBars* bars = reinterpret_cast<PairBars*>(smem + L::BAR_OFF);
+  StackBars* bars = reinterpret_cast<StackBars*>(smem + L::BAR_OFF);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
-
-  const int qb = p.nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
-  const int h0 = 2 * (int)blockIdx.x;
-  const int b = (int)blockIdx.y % p.B, c = (int)blockIdx.y / p.B;
-  const int g = h0 / (p.Hq / p.Hkv);
-  const int q0 = qb * PBQ;
-  const int nkb = (min(q0 + PBQ, p.T) + PBK - 1) / PBK;
-  const int row0 = b * p.T;
-  const int kcol = c * p.D + (p.Hq + g) * DH;
-  const int vcol = c * p.D + (p.Hq + p.Hkv + g) * DH;
+  const int pairs = p.Hq / 2, BC = p.B * p.C;
+  const int nqb = (p.T + SQ - 1) / SQ;
+  const int ntiles = pairs * BC * nqb;
+  const int ratio = p.Hq / p.Hkv;
 
   if (threadIdx.x == 0) {
     tc::mbar_init(&bars->q_full, 1);
-    for (int i = 0; i < PSTAGES; ++i) {
-      tc::mbar_init(&bars->kv_full[i], 1);
-      tc::mbar_init(&bars->kv_empty[i], 1);
+    tc::mbar_init(&bars->q_empty, 1);
+    for (int i = 0; i < SK_ST; ++i) {
+      tc::mbar_init(&bars->k_full[i], 1);
+      tc::mbar_init(&bars->k_empty[i], 1);
     }
-    for (int hd = 0; hd < 2; ++hd) {
-      for (int i = 0; i < 2; ++i) {
-        tc::mbar_init(&bars->s_full[hd][i], 1);
-        tc::mbar_init(&bars->s_empty[hd][i], 4);
-      }
-      tc::mbar_init(&bars->p_full[hd], 4);
-      tc::mbar_init(&bars->p_empty[hd], 1);
-      tc::mbar_init(&bars->o_full[hd], 1);
+    for (int i = 0; i < SV_ST; ++i) {
+      tc::mbar_init(&bars->v_full[i], 1);
+      tc::mbar_init(&bars->v_empty[i], 1);
     }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&bars->s_full[i], 1);
+      tc::mbar_init(&bars->s_empty[i], EW_WARPS);
+    }
+    tc::mbar_init(&bars->p_full, EW_WARPS);
+    tc::mbar_init(&bars->pv_done, 1);
+    tc::mbar_init(&bars->o_full, 1);
+    tc::mbar_init(&bars->o_empty, EW_WARPS);
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_q);
     tc::prefetch_tmap(&tm_kv);
   }
+  for (int i = threadIdx.x; i < 2 * 128; i += blockDim.x) (&bars->flag[0][0])[i] = 0;
   if (warp == 1) {
     tc::tmem_alloc(&bars->tmem_base, 512);
     tc::tmem_relinquish();
@@ -489,245 +548,343 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
-  auto s_col = [](int hd, int sb) { return (uint32_t)((hd * 2 + sb) * PBK); };
-  auto o_col = [](int hd) { return (uint32_t)(4 * PBK + hd * 128); };
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------------------------------------------------------- TMA
-      uint32_t issued = 0, last_par = 0;
-      tc::mbar_expect_tx(&bars->q_full, 2 * L::QTILE);
-      for (int hd = 0; hd < 2; ++hd)
+      int gk = 0, gv = 0, tc_ = 0;
+      uint32_t kiss = 0, kpar = 0, viss = 0, vpar = 0, qiss = 0, qpar = 0;
+      bool ok = true;
+      auto load_k = [&](int kcol, int krow) -> bool {
+        const int st = gk % SK_ST;
+        const uint32_t ph = (gk / SK_ST) & 1;
+        if (!tc::mbar_wait(&bars->k_empty[st], ph ^ 1, abort, p.status)) return false;
+        tc::mbar_expect_tx(&bars->k_full[st], L::TILE);
         for (int ch = 0; ch < DH / 64; ++ch)
-          tc::tma_load_2d(smem + L::Q_OFF + hd * L::QTILE + ch * L::QCHUNK, &tm_q, &bars->q_full,
-                          c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
-      for (int j = 0; j < nkb; ++j) {
-        const int st = j % PSTAGES;
-        const uint32_t ph = (j / PSTAGES) & 1;
-        if (!tc::mbar_wait(&bars->kv_empty[st], ph ^ 1, abort, p.status)) break;
-        uint8_t* sbase = smem + L::KV_OFF + st * L::STAGE;
-        tc::mbar_expect_tx(&bars->kv_full[st], L::STAGE);
-        for (int ch = 0; ch < DH / 64; ++ch) {
-          tc::tma_load_2d(sbase + ch * L::KVCHUNK, &tm_kv, &bars->kv_full[st], kcol + ch * 64,
-                          row0 + j * PBK);
-          tc::tma_load_2d(sbase + L::KVTILE + ch * L::KVCHUNK, &tm_kv, &bars->kv_full[st],
-                          vcol + ch * 64, row0 + j * PBK);
+          tc::tma_load_2d(smem + L::K_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv, &bars->k_full[st],
+                          kcol + ch * 64, krow);
+        kiss |= 1u << st;
+        kpar = (kpar & ~(1u << st)) | (ph << st);
+        ++gk;
+        return true;
+      };
+      auto load_v = [&](int vcol, int vrow) -> bool {
+        const int st = gv % SV_ST;
+        const uint32_t ph = (gv / SV_ST) & 1;
+        if (!tc::mbar_wait(&bars->v_empty[st], ph ^ 1, abort, p.status)) return false;
+        tc::mbar_expect_tx(&bars->v_full[st], L::TILE);
+        for (int ch = 0; ch < DH / 64; ++ch)
+          tc::tma_load_2d(smem + L::V_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv, &bars->v_full[st],
+                          vcol + ch * 64, vrow);
+        viss |= 1u << st;
+        vpar = (vpar & ~(1u << st)) | (ph << st);
+        ++gv;
+        return true;
+      };
+      for (int k = blockIdx.x; ok && k < ntiles; k += gridDim.x, ++tc_) {
+        const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
+        const int b = tl.bc % p.B, c = tl.bc / p.B, h0 = 2 * tl.hp, g = h0 / ratio;
+        const int row0 = b * p.T, q0 = tl.qb * SQ;
+        const int kcol = c * p.D + (p.Hq + g) * DH, vcol = c * p.D + (p.Hq + p.Hkv + g) * DH;
+        if (!tc::mbar_wait(&bars->q_empty, (tc_ & 1) ^ 1, abort, p.status)) break;
+        tc::mbar_expect_tx(&bars->q_full, L::TILE);
+        for (int ch = 0; ch < DH / 64; ++ch)
+          for (int hd = 0; hd < 2; ++hd)
+            tc::tma_load_2d(smem + L::Q_OFF + ch * L::CHUNK + hd * SQ * 128, &tm_q, &bars->q_full,
+                            c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
+        qiss = 1;
+        qpar = tc_ & 1;
+        if (MODE != 0) {  // the epilogue reads these A_ref rows (both heads: 2 DH fp32, contiguous)
+          const int nr = min(SQ, p.T - q0);
+          for (int r = 0; r < nr; ++r)
+            tc::prefetch_l2(p.a_ref + ((int64_t)row0 + q0 + r) * (int64_t)(p.Hq * DH) + h0 * DH,
+                            2 * DH * 4);
         }
-        issued |= 1u << st;
-        last_par = (last_par & ~(1u << st)) | (ph << st);
+        for (int j = 0; j < tl.nkb; ++j) {  // K runs one block ahead of V
+          if (!load_k(kcol, row0 + j * SKB)) { ok = false; break; }
+          if (j > 0 && !load_v(vcol, row0 + (j - 1) * SKB)) { ok = false; break; }
+        }
+        if (ok && !load_v(vcol, row0 + (tl.nkb - 1) * SKB)) ok = false;
       }
       if (*abort) {
-        drain_wait(&bars->q_full, 0);
-        for (int st = 0; st < PSTAGES; ++st)
-          if (issued & (1u << st)) drain_wait(&bars->kv_full[st], (last_par >> st) & 1);
+        if (qiss) drain_wait(&bars->q_full, qpar);
+        for (int st = 0; st < SK_ST; ++st)
+          if (kiss & (1u << st)) drain_wait(&bars->k_full[st], (kpar >> st) & 1);
+        for (int st = 0; st < SV_ST; ++st)
+          if (viss & (1u << st)) drain_wait(&bars->v_full[st], (vpar >> st) & 1);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------------------------------------------------------- UMMA
-      constexpr uint32_t ID_S = tc::idesc_f16(false, PBQ, PBK);
-      constexpr uint32_t ID_PV = tc::idesc_f16(false, PBQ, DH) | (1u << 16);  // B = V, MN-major
-      bool ok = tc::mbar_wait(&bars->q_full, 0, abort, p.status);
-      auto issue_pv = [&](int hd, int jj) -> bool {
-        if (!tc::mbar_wait(&bars->p_full[hd], jj & 1, abort, p.status)) return false;
+      constexpr uint32_t ID_S = tc::idesc_f16(false, 128, SKB);
+      constexpr uint32_t ID_PV = tc::idesc_f16(false, 128, DH) | (1u << 16);  // B = V, MN-major
+      int g0 = 0, tc_ = 0;
+      bool ok = true;
+      // S of global block gg into buffer gg & 1, once the softmax has read S_{gg-2} out of it.
+      auto issue_s = [&](int gg) -> bool {
+        const int ks = gg % SK_ST, sb = gg & 1;
+        if (!tc::mbar_wait(&bars->k_full[ks], (gg / SK_ST) & 1, abort, p.status)) return false;
+        if (!tc::mbar_wait(&bars->s_empty[sb], ((gg >> 1) & 1) ^ 1, abort, p.status)) return false;
         tc::fence_after_sync();
-        const uint32_t v_base =
-            tc::smem_u32(smem + L::KV_OFF + (jj % PSTAGES) * L::STAGE + L::KVTILE);
-        const uint32_t p_base = tc::smem_u32(smem + L::P_OFF + hd * L::PTILE);
+        const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + ks * L::TILE);
 #pragma unroll
-        for (int k = 0; k < PBK / 16; ++k)
-          tc::umma_f16(tmem + o_col(hd), tc::sdesc_kmajor_sw128(p_base + k * 32),
-                       tc::sdesc_mnmajor_sw128(v_base + k * 16 * 128, L::KVCHUNK, 1024), ID_PV,
-                       (jj > 0 || k > 0) ? 1u : 0u);
-        tc::umma_commit(&bars->p_empty[hd]);
-        if (hd == 1) tc::umma_commit(&bars->kv_empty[jj % PSTAGES]);
+        for (int kk = 0; kk < DH / 16; ++kk)
+          tc::umma_f16_ts(tmem + L::S_COL + sb * SKB, tmem + L::Q_COL + kk * 8,
+                          tc::sdesc_kmajor_sw128(k_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32),
+                          ID_S, kk > 0 ? 1u : 0u);
+        tc::umma_commit(&bars->s_full[sb]);
+        tc::umma_commit(&bars->k_empty[ks]);
         return true;
       };
-      for (int j = 0; ok && j < nkb; ++j) {
-        const int st = j % PSTAGES, sb = j & 1;
-        if (!tc::mbar_wait(&bars->kv_full[st], (j / PSTAGES) & 1, abort, p.status)) break;
-        const uint32_t k_base = tc::smem_u32(smem + L::KV_OFF + st * L::STAGE);
-        for (int hd = 0; hd < 2 && ok; ++hd) {
-          if (!tc::mbar_wait(&bars->s_empty[hd][sb], ((j >> 1) & 1) ^ 1, abort, p.status)) {
-            ok = false;
-            break;
-          }
-          tc::fence_after_sync();
-          const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF + hd * L::QTILE);
+      auto issue_pv = [&](int gg, bool first) -> bool {
+        const int vs = gg % SV_ST;
+        if (!tc::mbar_wait(&bars->v_full[vs], (gg / SV_ST) & 1, abort, p.status)) return false;
+        if (!tc::mbar_wait(&bars->p_full, gg & 1, abort, p.status)) return false;
+        if (first && tc_ > 0 && !tc::mbar_wait(&bars->o_empty, (tc_ - 1) & 1, abort, p.status))
+          return false;
+        tc::fence_after_sync();
+        const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + vs * L::TILE);
 #pragma unroll
-          for (int k = 0; k < DH / 16; ++k)
-            tc::umma_f16(tmem + s_col(hd, sb),
-                         tc::sdesc_kmajor_sw128(q_base + (k >> 2) * L::QCHUNK + (k & 3) * 32),
-                         tc::sdesc_kmajor_sw128(k_base + (k >> 2) * L::KVCHUNK + (k & 3) * 32),
-                         ID_S, k > 0 ? 1u : 0u);
-          tc::umma_commit(&bars->s_full[hd][sb]);
+        for (int k = 0; k < SKB / 16; ++k)
+          tc::umma_f16_ts(tmem + L::O_COL, tmem + L::P_COL + k * 8,
+                          tc::sdesc_mnmajor_sw128(v_base + k * 16 * 128, L::CHUNK, 1024), ID_PV,
+                          (!first || k > 0) ? 1u : 0u);
+        tc::umma_commit(&bars->pv_done);
+        tc::umma_commit(&bars->v_empty[vs]);
+        return true;
+      };
+      for (int k = blockIdx.x; ok && k < ntiles; k += gridDim.x, ++tc_) {
+        const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
+        // Q of this tile into TMEM once the previous tile's last S (which read the old Q) is done.
+        if (g0 > 0 &&
+            !tc::mbar_wait(&bars->s_full[(g0 - 1) & 1], ((g0 - 1) >> 1) & 1, abort, p.status))
+          break;
+        if (!tc::mbar_wait(&bars->q_full, tc_ & 1, abort, p.status)) break;
+        tc::fence_after_sync();
+        {
+          const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)
+            tc::tmem_cp_128x256b(tmem + L::Q_COL + kk * 8,
+                                 tc::sdesc_kmajor_sw128(q_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
+          tc::umma_commit(&bars->q_empty);
+        }
+        // S runs two blocks ahead of P V.
+        ok = issue_s(g0) && (tl.nkb < 2 || issue_s(g0 + 1));
+        for (int j = 0; ok && j < tl.nkb; ++j) {
+          if (j + 2 < tl.nkb && !issue_s(g0 + j + 2)) { ok = false; break; }
+          if (!issue_pv(g0 + j, j == 0)) { ok = false; break; }
         }
         if (!ok) break;
-        if (j > 0 && (!issue_pv(0, j - 1) || !issue_pv(1, j - 1))) break;
-        if (j == nkb - 1) {
-          for (int hd = 0; hd < 2; ++hd)
-            if (issue_pv(hd, j)) tc::umma_commit(&bars->o_full[hd]);
-        }
+        tc::umma_commit(&bars->o_full);
+        g0 += tl.nkb;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
   } else {  // ------------------------------------------------------------------------ softmax
-    const int hd = (warp - 2) >> 2;
-    const int h = h0 + hd;
     const int quarter = warp & 3;
-    const int row = quarter * 32 + lane;
-    const int t = q0 + row;
+    const int half = (warp - 2) >> 2;
+    const int row = quarter * 32 + lane;  // stacked row = TMEM lane
+    const int hd = row >> 6;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    uint8_t* prow = smem + L::P_OFF + hd * L::PTILE + row * 128;
-    float m = -INFINITY, l = 0.f;
-    bool ok = true;
-    for (int j = 0; j < nkb; ++j) {
-      const int sb = j & 1;
-      if (!tc::mbar_wait(&bars->s_full[hd][sb], (j >> 1) & 1, abort, p.status)) {
-        ok = false;
-        break;
-      }
-      tc::fence_after_sync();
-      float s[PBK];
-#pragma unroll
-      for (int ch = 0; ch < PBK / 32; ++ch) {
-        uint32_t r[32];
-        __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + s_col(hd, sb) + ch * 32, r);
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 32; ++i) s[ch * 32 + i] = __uint_as_float(r[i]) * p.sl2;
-      }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->s_empty[hd][sb]);
-      const int k0 = j * PBK;
-      if (k0 + PBK - 1 > q0 || k0 + PBK > p.T) {  // diagonal or ragged block: mask
-#pragma unroll
-        for (int i = 0; i < PBK; ++i)
-          if (k0 + i > t || k0 + i >= p.T) s[i] = -INFINITY;
-      }
-      float mx8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = s[i];
-#pragma unroll
-      for (int i = 8; i < PBK; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      const float m_new = fmaxf(m, mx);
-      const bool resc = m_new > m + kRescaleLog2;
-      const float m_use = resc ? m_new : m;
-      const float alpha = resc ? tc::fast_exp2(m - m_new) : 1.f;
-      float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int i = 0; i < PBK; ++i) {
-        s[i] = tc::fast_exp2(s[i] - m_use);
-        rs8[i & 7] += s[i];
-      }
-      l = l * alpha + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
-      m = m_use;
-      // P V of the previous block must be complete before O is rescaled or P is overwritten.
-      if (!tc::mbar_wait(&bars->p_empty[hd], (j & 1) ^ 1, abort, p.status)) {
-        ok = false;
-        break;
-      }
-      tc::fence_after_sync();
-      if (j > 0 && __any_sync(0xffffffffu, resc)) {
-#pragma unroll
-        for (int ch = 0; ch < DH / 32; ++ch) {
-          uint32_t r[32];
+    float* stg = reinterpret_cast<float*>(smem + L::EPI_OFF + (warp - 2) * 4096);
+    int g = 0, tc_ = 0, seq = 0;
+    for (int k = blockIdx.x; k < ntiles; k += gridDim.x, ++tc_) {
+      if (*abort) break;
+      const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
+      const int b = tl.bc % p.B, c = tl.bc / p.B;
+      const int h = 2 * tl.hp + hd;
+      const int q0 = tl.qb * SQ;
+      const int t = q0 + (row & 63);
+      const int row0 = b * p.T;
+      float m = -INFINITY, l = 0.f;
+      bool ok = true;
+      for (int j = 0; j < tl.nkb; ++j, ++g) {
+        const int sb = g & 1;
+        if (!tc::mbar_wait(&bars->s_full[sb], (g >> 1) & 1, abort, p.status)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        float s[64];
+        {
+          uint32_t r0[32], r1[32];
           __syncwarp();
-          tc::tmem_ld32(tmem + lane_base + o_col(hd) + ch * 32, r);
+          tc::tmem_ld32(tmem + lane_base + L::S_COL + sb * SKB + half * 64, r0);
+          tc::tmem_ld32(tmem + lane_base + L::S_COL + sb * SKB + half * 64 + 32, r1);
           tc::tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-          tc::tmem_st32(tmem + lane_base + o_col(hd) + ch * 32, r);
+          for (int i = 0; i < 32; ++i) {
+            s[i] = __uint_as_float(r0[i]);
+            s[32 + i] = __uint_as_float(r1[i]);
+          }
         }
-        tc::tmem_st_wait();
-      }
-#pragma unroll
-      for (int c8 = 0; c8 < 8; ++c8) {
-        uint4 u;
-        __half2* hp = reinterpret_cast<__half2*>(&u);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(s[c8 * 8 + 2 * e], s[c8 * 8 + 2 * e + 1]);
-        *reinterpret_cast<uint4*>(prow + ((c8 ^ (row & 7)) << 4)) = u;
-      }
-      tc::fence_proxy_async_smem();
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->p_full[hd]);
-    }
-    // ---------------------------------------------------------------- epilogue
-    double acc = 0.0;
-    if (ok && tc::mbar_wait(&bars->o_full[hd], 0, abort, p.status)) {
-      tc::fence_after_sync();
-      const bool valid = t < p.T;
-      const float inv_l = __fdiv_rn(1.f, l);
-      const int64_t orow = ((int64_t)row0 + (valid ? t : 0)) * (int64_t)(p.Hq * DH) + h * DH;
-      float sq = 0.f, dsum = 0.f;
-#pragma unroll 1
-      for (int ch = 0; ch < DH / 32; ++ch) {
-        uint32_t r[32];
+        tc::fence_before_sync();
         __syncwarp();
-        tc::tmem_ld32(tmem + lane_base + o_col(hd) + ch * 32, r);
-        tc::tmem_ld_wait();
-        float o[32];
+        if (lane == 0) tc::mbar_arrive(&bars->s_empty[sb]);  // S_{g+2} may overwrite the buffer
+        const int k0 = j * SKB + half * 64;
+        if (k0 + 63 > q0 || k0 + 64 > p.T) {  // diagonal or ragged block: mask
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o[i] = __fmul_rn(__uint_as_float(r[i]), inv_l);
-        if (!valid) continue;
-        if (MODE == 0) {
-          float4* dst = reinterpret_cast<float4*>(p.a_out + orow + ch * 32);
+          for (int i = 0; i < 64; ++i)
+            if (k0 + i > t || k0 + i >= p.T) s[i] = -INFINITY;
+        }
+        float mx8[8];
 #pragma unroll
-          for (int v = 0; v < 8; ++v) {
-            dst[v] = make_float4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
-            sq += o[4 * v] * o[4 * v] + o[4 * v + 1] * o[4 * v + 1] + o[4 * v + 2] * o[4 * v + 2] +
-                  o[4 * v + 3] * o[4 * v + 3];
+        for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+        for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
+        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        mx = fmaxf(mx, half_exchange(bars, half, row, seq, mx, abort, p.status));
+        // Scores are raw (unscaled) here; the softmax scale times log2(e) is applied in the exponent.
+        const float m_new = fmaxf(m, mx * p.sl2);
+        const bool resc = m_new > m + kRescaleLog2;
+        const float m_use = resc ? m_new : m;
+        const float alpha = resc ? tc::fast_exp2(m - m_new) : 1.f;
+        float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+          s[i] = tc::fast_exp2(fmaf(s[i], p.sl2, -m_use));
+          rs8[i & 7] += s[i];
+        }
+        l = l * alpha + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
+        m = m_use;
+        // P_{g-1} V_{g-1} (and so every earlier P V) must have completed before P is overwritten
+        // or O is rescaled.
+        if (g > 0 && !tc::mbar_wait(&bars->pv_done, (g - 1) & 1, abort, p.status)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        if (j > 0 && __any_sync(0xffffffffu, resc)) {
+#pragma unroll 1
+          for (int ch = 0; ch < DH / 64; ++ch) {
+            uint32_t r[32];
+            const uint32_t col = L::O_COL + half * (DH / 2) + ch * 32;
+            __syncwarp();
+            tc::tmem_ld32(tmem + lane_base + col, r);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+            tc::tmem_st32(tmem + lane_base + col, r);
           }
-        } else {
-          const float4* ar = reinterpret_cast<const float4*>(p.a_ref + orow + ch * 32);
-          float e[32];
+        }
+        {  // P (fp16 pairs) of keys [64 half, 64 half + 64): P columns [32 half, 32 half + 32)
+          uint32_t pr[32];
 #pragma unroll
-          for (int v = 0; v < 8; ++v) {
-            const float4 a4 = __ldg(ar + v);
-            e[4 * v] = __fsub_rn(o[4 * v], a4.x);
-            e[4 * v + 1] = __fsub_rn(o[4 * v + 1], a4.y);
-            e[4 * v + 2] = __fsub_rn(o[4 * v + 2], a4.z);
-            e[4 * v + 3] = __fsub_rn(o[4 * v + 3], a4.w);
+          for (int i = 0; i < 32; ++i) {
+            const __half2 h2 = __floats2half2_rn(s[2 * i], s[2 * i + 1]);
+            pr[i] = *reinterpret_cast<const uint32_t*>(&h2);
+          }
+          __syncwarp();
+          tc::tmem_st32(tmem + lane_base + L::P_COL + half * 32, pr);
+          tc::tmem_st_wait();
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->p_full);
+      }
+      // ------------------------------------------------------------------ epilogue
+      double acc = 0.0;
+      const bool have = ok && tc::mbar_wait(&bars->o_full, tc_ & 1, abort, p.status);
+      if (have) {
+        tc::fence_after_sync();
+        const float lt = l + half_exchange(bars, half, row, seq, l, abort, p.status);
+        const float inv_l = __fdiv_rn(1.f, lt);
+        // O in 32-column chunks. Coalesced pass: the warp's 32 rows x 32 columns go through shared
+        // memory; lane l then handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte
+        // row segment. In mode 2 the fp16-rounded error goes back through the same slots to the
+        // row's owner, which accumulates D = rowsum(dO * O).
+        const int rbase = quarter * 32;  // first stacked row of this warp
+        const int c4 = lane & 7;
+        float sq = 0.f, dsum = 0.f;
+#pragma unroll 1
+        for (int ch = 0; ch < DH / 64; ++ch) {
+          const int col = h * DH + half * (DH / 2) + ch * 32 + c4 * 4;
+          float4 av[8];
+          if (MODE != 0) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & 63);
+              if (tt < p.T)
+                av[i] = __ldg(reinterpret_cast<const float4*>(
+                    p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col));
+            }
+          }
+          float o[32];
+          {
+            uint32_t r[32];
+            __syncwarp();
+            tc::tmem_ld32(tmem + lane_base + L::O_COL + half * (DH / 2) + ch * 32, r);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __fmul_rn(__uint_as_float(r[i]), inv_l);
           }
 #pragma unroll
-          for (int i = 0; i < 32; ++i) sq += e[i] * e[i];
-          if (MODE == 2) {
-            uint4* dst = reinterpret_cast<uint4*>(p.d_o + orow + ch * 32);
+          for (int v = 0; v < 8; ++v)
+            *reinterpret_cast<float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2)) =
+                make_float4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
+          __syncwarp();
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              uint4 u;
-              __half2* hp = reinterpret_cast<__half2*>(&u);
-#pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                hp[k] = __floats2half2_rn(e[v * 8 + 2 * k], e[v * 8 + 2 * k + 1]);
-                const float2 f = __half22float2(hp[k]);
-                dsum += f.x * o[v * 8 + 2 * k] + f.y * o[v * 8 + 2 * k + 1];
+          for (int i = 0; i < 8; ++i) {
+            const int rr = 4 * i + (lane >> 3);
+            float4* slot = reinterpret_cast<float4*>(stg + rr * 32 + ((c4 ^ (rr & 7)) << 2));
+            const float4 ov = *slot;
+            const int tt = q0 + ((rbase + rr) & 63);
+            if (tt >= p.T) continue;
+            const int64_t off = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
+            if (MODE == 0) {
+              *reinterpret_cast<float4*>(p.a_out + off) = ov;
+              sq += ov.x * ov.x + ov.y * ov.y + ov.z * ov.z + ov.w * ov.w;
+            } else {
+              const float e0 = __fsub_rn(ov.x, av[i].x), e1 = __fsub_rn(ov.y, av[i].y);
+              const float e2 = __fsub_rn(ov.z, av[i].z), e3 = __fsub_rn(ov.w, av[i].w);
+              sq += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+              if (MODE == 2) {
+                const __half2 a01 = __floats2half2_rn(e0, e1), a23 = __floats2half2_rn(e2, e3);
+                uint2 u;
+                u.x = *reinterpret_cast<const uint32_t*>(&a01);
+                u.y = *reinterpret_cast<const uint32_t*>(&a23);
+                *reinterpret_cast<uint2*>(p.d_o + off) = u;
+                const float2 f01 = __half22float2(a01), f23 = __half22float2(a23);
+                *slot = make_float4(f01.x, f01.y, f23.x, f23.y);
               }
-              dst[v] = u;
+            }
+          }
+          __syncwarp();
+          if (MODE == 2) {
+#pragma unroll
+            for (int v = 0; v < 8; ++v) {
+              const float4 e = *reinterpret_cast<const float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2));
+              dsum += e.x * o[4 * v] + e.y * o[4 * v + 1] + e.z * o[4 * v + 2] + e.w * o[4 * v + 3];
             }
           }
         }
-      }
-      if (valid) {
-        if (MODE != 1 && p.lse != nullptr)
-          p.lse[((int64_t)b * p.Hq + h) * p.lse_pitch + t] =
-              MODE == 2 ? m + log2f(l) : (m + log2f(l)) * kLn2;  // mode 2: log2 units
-        if (MODE == 2) p.dvec[((int64_t)b * p.Hq + h) * p.lse_pitch + t] = dsum;
+        // O is no longer needed: the next tile's first P V may overwrite it.
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->o_empty);
+        if (MODE == 2) dsum += half_exchange(bars, half, row, seq, dsum, abort, p.status);
+        if (half == 0 && t < p.T) {
+          const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + t;
+          if (MODE != 1 && p.lse != nullptr)
+            p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
+          if (MODE == 2) p.dvec[li] = dsum;
+        }
         acc = (double)sq;
       }
-    }
-    acc = warp_sum(acc);
-    if (lane == 0) bars->red[warp - 2] = acc;
-    tc::named_bar_sync(1, EW_WARPS * 32);
-    if (quarter == 0 && lane == 0) {  // one thread per head
-      const int w0 = hd * 4;
-      p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb] =
-          bars->red[w0] + bars->red[w0 + 1] + bars->red[w0 + 2] + bars->red[w0 + 3];
+      acc = warp_sum(acc);
+      if (lane == 0) bars->red[warp - 2] = acc;
+      tc::named_bar_sync(1, EW_WARPS * 32);  // every softmax warp reaches this once per tile
+      if (lane == 0 && half == 0 && (quarter & 1) == 0 && have) {
+        // head hd's rows are lane quarters 2 hd and 2 hd + 1, each split over two warps
+        const int wq0 = (2 * hd + 2) & 3;  // warp index - 2 of quarter 2 hd, half 0
+        const double v = bars->red[wq0] + bars->red[(wq0 + 1) & 3] + bars->red[wq0 + 4] +
+                         bars->red[((wq0 + 1) & 3) + 4];
+        p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] = v;
+      }
+      tc::named_bar_sync(1, EW_WARPS * 32);  // red[] is rewritten by the next tile
+      if (!ok || !have) break;
     }
   }
   tc::fence_before_sync();
@@ -754,16 +911,16 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 template <int DH, int MODE>
 cudaError_t launch_fwd_pair(const CUtensorMap& tq, const CUtensorMap& tkv, const FwdParams& p,
-                            dim3 grid, cudaStream_t st) {
+                            int grid, cudaStream_t st) {
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(attn_fwd_pair_kernel<DH, MODE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         PairLayout<DH>::SMEM);
+                                         StackLayout<DH>::SMEM);
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  attn_fwd_pair_kernel<DH, MODE><<<grid, NUM_THREADS, PairLayout<DH>::SMEM, st>>>(tq, tkv, p);
+  attn_fwd_pair_kernel<DH, MODE><<<grid, NUM_THREADS, StackLayout<DH>::SMEM, st>>>(tq, tkv, p);
   return cudaGetLastError();
 }
 
@@ -783,7 +940,7 @@ cudaError_t launch_fwd(const CUtensorMap& tm, const FwdParams& p, dim3 grid, cud
 
 }  // namespace
 
-int attn_fwd_tc_rows() { return BQ; }
+int attn_fwd_tc_rows(int Hq, int Hkv) { return (Hq / Hkv) % 2 == 0 ? SQ : BQ; }
 
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) {
   auto fn = encode_fn();
@@ -815,15 +972,28 @@ cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode) {
   p.d_o = static_cast<half_t*>(L.d_o);
   p.dvec = L.dvec;
   p.status = L.status;
+  p.C = L.C;
   if ((L.Hq / L.Hkv) % 2 == 0) {  // head pairs of one KV group share every K/V tile
-    CUtensorMap tkv;
-    cuuint32_t box64[2] = {64, (cuuint32_t)PBK};
-    if (fn(&tkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(L.qkv), dims, strides, box64,
+    CUtensorMap tq64, tkv;
+    cuuint32_t box_q[2] = {64, (cuuint32_t)SQ};
+    cuuint32_t box_kv[2] = {64, (cuuint32_t)SKB};
+    if (fn(&tq64, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(L.qkv), dims, strides, box_q,
+           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+        fn(&tkv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(L.qkv), dims, strides, box_kv,
            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
-    dim3 pgrid((unsigned)(L.Hq / 2), (unsigned)(L.B * L.C), (unsigned)p.nqb);
-#define JAB_FWD2(DH_, M_) return launch_fwd_pair<DH_, M_>(tm, tkv, p, pgrid, L.stream)
+    static int sms = 0;
+    if (sms == 0) {
+      int dev = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (sms <= 0) sms = 1;
+    }
+    const int64_t ntiles = (int64_t)(L.Hq / 2) * L.B * L.C * ((L.T + SQ - 1) / SQ);
+    const int grid = (int)std::min<int64_t>(ntiles, sms);
+#define JAB_FWD2(DH_, M_) return launch_fwd_pair<DH_, M_>(tq64, tkv, p, grid, L.stream)
     if (L.dh == 128) {
       if (mode == 0) JAB_FWD2(128, 0);
       if (mode == 1) JAB_FWD2(128, 1);

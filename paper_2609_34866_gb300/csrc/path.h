@@ -27,7 +27,7 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, 
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st);
 // attn_tc.cu
-int attn_fwd_tc_rows();  // query rows per CTA (= rows per loss partial)
+int attn_fwd_tc_rows(int Hq, int Hkv);  // query rows per loss partial of the forward kernel
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);
 cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
                                int use_rope, void* dqkvt);
