@@ -410,35 +410,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ============================================================================ head-pair kernel
-// Persistent: one CTA per SM walks a longest-first list of tiles. A tile is 64 query rows of two
-// query heads of one KV group (GQA: both read the same K and V) stacked into the 128 rows of every
-// UMMA: TMEM lane r < 64 is row q0 + r of head h0, lane 64 + r is row q0 + r of head h0 + 1.
-// Keys come in blocks of 128 so that both products are M128 N128 UMMAs with the A operand in tensor
-// memory (TS form), the shape that runs the tensor pipe at full rate on sm_103a:
+// Persistent: one CTA per SM walks a list of tiles. A tile is 64 query rows of two query heads of
+// one KV group (GQA: both read the same K and V) stacked into the 128 rows of every UMMA: TMEM lane
+// r < 64 is row q0 + r of head h0, lane 64 + r is row q0 + r of head h0 + 1. Keys come in blocks of
+// 128 so that both products are M128 N128 UMMAs with the A operand in tensor memory (TS form), the
+// shape that runs the tensor pipe at full rate on sm_103a:
 //   S_j = Q K_j^T     A = Q (TMEM, copied from the TMA-loaded smem tile by tcgen05.cp), B = K_j
 //   O  += P_j V_j     A = P_j (TMEM, fp16 pairs written by the softmax threads), B = V_j (smem,
 //                     MN-major)
 // TMEM columns: S double-buffered at 0 / 128, O at 256 (DH columns), Q (DH / 2 columns) and P
 // (64 columns) after it. S_{j+2} is issued as soon as the softmax has read S_j out of its buffer, so
 // the tensor pipe computes the next scores while the softmax of block j runs.
-//   warp 0      TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages, one
-//               block ahead of V), V ring (2 stages)
+//   warp 0      TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages)
 //   warp 1      TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
-//   warps 2..9  softmax, two warps per TMEM lane quarter: a thread owns one stacked row and one half
-//               (64 keys) of each S block; the halves agree on the row maximum through shared memory.
-//               Lazy rescaling as in the single-head kernel. Epilogue: O is read out of TMEM (and
-//               released to the next tile) at once, then staged through shared memory so that A_ref
-//               loads and dO / A stores are coalesced.
+//   warps 2..9  softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
+//               16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
+//               thread), so row maxima and sums need only warp shuffles. Lazy rescaling as in the
+//               single-head kernel. Epilogue (32x32b shape, one row per thread, half of its
+//               columns): O is staged through shared memory so that A_ref loads and dO / A stores are
+//               coalesced.
+//   warp 10     TMA: V ring (2 stages), so that K loads never queue behind a V stage that is busy.
 constexpr int SQ = 64, SKB = 128, SK_ST = 2, SV_ST = 2;
+constexpr int PAIR_THREADS = 352;
 
 struct StackBars {
   uint64_t q_full, q_empty, k_full[SK_ST], k_empty[SK_ST], v_full[SV_ST], v_empty[SV_ST];
   uint64_t s_full[2], s_empty[2], p_full, pv_done, o_full, o_empty, drain;
   uint32_t tmem_base;
   int abort;
-  double red[EW_WARPS];
-  float xv[2][2][128];  // [sequence parity][half][row]: values exchanged between the two halves
-  int flag[2][128];     // [half][row]: sequence number of the last value posted
+  double red[2][EW_WARPS];  // [tile parity][softmax warp]
+  float row_m[128], row_l[128];  // per stacked row: final running max (log2 units) and sum
+  float xv[2][2][128];           // [sequence parity][half][row]: values exchanged between halves
+  int flag[2][128];              // [half][row]: sequence number of the last value posted
 };
 
 template <int DH>
@@ -461,12 +464,15 @@ struct StackTile {
   int hp, bc, qb, nkb;
 };
 
-// Tile k of the longest-first order: query blocks from the last (most key blocks) to the first.
+// Tile k: (sequence, head pair) major and query blocks minor, from the last query block (most key
+// blocks) to the first. CTAs take tiles k = blockIdx.x + i * gridDim.x, so the tiles running at any
+// time belong to a few (sequence, KV group) pairs whose K and V stay in L2, and every CTA gets a
+// similar mix of long and short tiles.
 __device__ __forceinline__ StackTile stack_tile(int k, int pairs, int BC, int nqb, int T) {
   StackTile t;
-  t.hp = k % pairs;
-  t.bc = (k / pairs) % BC;
-  t.qb = nqb - 1 - k / (pairs * BC);
+  t.qb = nqb - 1 - k % nqb;
+  t.hp = (k / nqb) % pairs;
+  t.bc = k / (nqb * pairs);
   t.nkb = (min((t.qb + 1) * SQ, T) + SKB - 1) / SKB;
   return t;
 }
@@ -498,8 +504,13 @@ __device__ __forceinline__ float half_exchange(StackBars* bars, int half, int ro
   return reinterpret_cast<volatile float*>(&bars->xv[seq & 1][half ^ 1][row])[0];
 }
 
+__device__ __forceinline__ uint32_t pack_half2(float a, float b) {
+  const __half2 h = __floats2half2_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 template <int DH, int MODE>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(PAIR_THREADS, 1)
     attn_fwd_pair_kernel(const __grid_constant__ CUtensorMap tm_q,
                          const __grid_constant__ CUtensorMap tm_kv, const FwdParams p) {
   using L = StackLayout<DH>;
@@ -549,68 +560,54 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
 
-  if (warp == 0) {
-    if (lane == 0) {  // ---------------------------------------------------------------- TMA
-      int gk = 0, gv = 0, tc_ = 0;
-      uint32_t kiss = 0, kpar = 0, viss = 0, vpar = 0, qiss = 0, qpar = 0;
+  if (warp == 0 || warp == 10) {
+    if (lane == 0) {  // ------------------------------------------------ TMA: Q and K (warp 0), V (10)
+      const bool is_v = warp == 10;
+      int gi = 0, tc_ = 0;
+      uint32_t iss = 0, par = 0, qiss = 0, qpar = 0;
       bool ok = true;
-      auto load_k = [&](int kcol, int krow) -> bool {
-        const int st = gk % SK_ST;
-        const uint32_t ph = (gk / SK_ST) & 1;
-        if (!tc::mbar_wait(&bars->k_empty[st], ph ^ 1, abort, p.status)) return false;
-        tc::mbar_expect_tx(&bars->k_full[st], L::TILE);
-        for (int ch = 0; ch < DH / 64; ++ch)
-          tc::tma_load_2d(smem + L::K_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv, &bars->k_full[st],
-                          kcol + ch * 64, krow);
-        kiss |= 1u << st;
-        kpar = (kpar & ~(1u << st)) | (ph << st);
-        ++gk;
-        return true;
-      };
-      auto load_v = [&](int vcol, int vrow) -> bool {
-        const int st = gv % SV_ST;
-        const uint32_t ph = (gv / SV_ST) & 1;
-        if (!tc::mbar_wait(&bars->v_empty[st], ph ^ 1, abort, p.status)) return false;
-        tc::mbar_expect_tx(&bars->v_full[st], L::TILE);
-        for (int ch = 0; ch < DH / 64; ++ch)
-          tc::tma_load_2d(smem + L::V_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv, &bars->v_full[st],
-                          vcol + ch * 64, vrow);
-        viss |= 1u << st;
-        vpar = (vpar & ~(1u << st)) | (ph << st);
-        ++gv;
-        return true;
-      };
+      uint64_t* full = is_v ? bars->v_full : bars->k_full;
+      uint64_t* empty = is_v ? bars->v_empty : bars->k_empty;
+      uint8_t* ring = smem + (is_v ? L::V_OFF : L::K_OFF);
+      constexpr int NST = SK_ST;
+      static_assert(SK_ST == SV_ST, "one ring depth for K and V");
       for (int k = blockIdx.x; ok && k < ntiles; k += gridDim.x, ++tc_) {
         const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
         const int b = tl.bc % p.B, c = tl.bc / p.B, h0 = 2 * tl.hp, g = h0 / ratio;
         const int row0 = b * p.T, q0 = tl.qb * SQ;
-        const int kcol = c * p.D + (p.Hq + g) * DH, vcol = c * p.D + (p.Hq + p.Hkv + g) * DH;
-        if (!tc::mbar_wait(&bars->q_empty, (tc_ & 1) ^ 1, abort, p.status)) break;
-        tc::mbar_expect_tx(&bars->q_full, L::TILE);
-        for (int ch = 0; ch < DH / 64; ++ch)
-          for (int hd = 0; hd < 2; ++hd)
-            tc::tma_load_2d(smem + L::Q_OFF + ch * L::CHUNK + hd * SQ * 128, &tm_q, &bars->q_full,
-                            c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
-        qiss = 1;
-        qpar = tc_ & 1;
-        if (MODE != 0) {  // the epilogue reads these A_ref rows (both heads: 2 DH fp32, contiguous)
-          const int nr = min(SQ, p.T - q0);
-          for (int r = 0; r < nr; ++r)
-            tc::prefetch_l2(p.a_ref + ((int64_t)row0 + q0 + r) * (int64_t)(p.Hq * DH) + h0 * DH,
-                            2 * DH * 4);
+        const int col = c * p.D + (is_v ? p.Hq + p.Hkv + g : p.Hq + g) * DH;
+        if (!is_v) {
+          if (!tc::mbar_wait(&bars->q_empty, (tc_ & 1) ^ 1, abort, p.status)) break;
+          tc::mbar_expect_tx(&bars->q_full, L::TILE);
+          for (int ch = 0; ch < DH / 64; ++ch)
+            for (int hd = 0; hd < 2; ++hd)
+              tc::tma_load_2d(smem + L::Q_OFF + ch * L::CHUNK + hd * SQ * 128, &tm_q, &bars->q_full,
+                              c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
+          qiss = 1;
+          qpar = tc_ & 1;
+          if (MODE != 0) {  // the epilogue reads these A_ref rows (both heads: 2 DH fp32, contiguous)
+            const int nr = min(SQ, p.T - q0);
+            for (int r = 0; r < nr; ++r)
+              tc::prefetch_l2(p.a_ref + ((int64_t)row0 + q0 + r) * (int64_t)(p.Hq * DH) + h0 * DH,
+                              2 * DH * 4);
+          }
         }
-        for (int j = 0; j < tl.nkb; ++j) {  // K runs one block ahead of V
-          if (!load_k(kcol, row0 + j * SKB)) { ok = false; break; }
-          if (j > 0 && !load_v(vcol, row0 + (j - 1) * SKB)) { ok = false; break; }
+        for (int j = 0; j < tl.nkb; ++j, ++gi) {
+          const int st = gi % NST;
+          const uint32_t ph = (gi / NST) & 1;
+          if (!tc::mbar_wait(&empty[st], ph ^ 1, abort, p.status)) { ok = false; break; }
+          tc::mbar_expect_tx(&full[st], L::TILE);
+          for (int ch = 0; ch < DH / 64; ++ch)
+            tc::tma_load_2d(ring + st * L::TILE + ch * L::CHUNK, &tm_kv, &full[st], col + ch * 64,
+                            row0 + j * SKB);
+          iss |= 1u << st;
+          par = (par & ~(1u << st)) | (ph << st);
         }
-        if (ok && !load_v(vcol, row0 + (tl.nkb - 1) * SKB)) ok = false;
       }
       if (*abort) {
         if (qiss) drain_wait(&bars->q_full, qpar);
-        for (int st = 0; st < SK_ST; ++st)
-          if (kiss & (1u << st)) drain_wait(&bars->k_full[st], (kpar >> st) & 1);
-        for (int st = 0; st < SV_ST; ++st)
-          if (viss & (1u << st)) drain_wait(&bars->v_full[st], (vpar >> st) & 1);
+        for (int st = 0; st < NST; ++st)
+          if (iss & (1u << st)) drain_wait(&full[st], (par >> st) & 1);
       }
     }
   } else if (warp == 1) {
@@ -684,8 +681,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {  // ------------------------------------------------------------------------ softmax
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
-    const int row = quarter * 32 + lane;  // stacked row = TMEM lane
-    const int hd = row >> 6;
+    const int cq = lane & 3;                                   // column pair within each 8 columns
+    const int rA = quarter * 32 + half * 16 + (lane >> 2);     // stacked rows of this thread
+    const int rB = rA + 8;
+    const int hd = rA >> 6;                                    // rA and rB belong to the same head
+    const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
+    // epilogue layout (32x32b): one row per thread, half of its columns
+    const int row = quarter * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     float* stg = reinterpret_cast<float*>(smem + L::EPI_OFF + (warp - 2) * 4096);
     int g = 0, tc_ = 0, seq = 0;
@@ -693,11 +695,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (*abort) break;
       const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
       const int b = tl.bc % p.B, c = tl.bc / p.B;
-      const int h = 2 * tl.hp + hd;
       const int q0 = tl.qb * SQ;
-      const int t = q0 + (row & 63);
+      const int tA = q0 + (rA & 63), tB = q0 + (rB & 63);
       const int row0 = b * p.T;
-      float m = -INFINITY, l = 0.f;
+      float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
       bool ok = true;
       for (int j = 0; j < tl.nkb; ++j, ++g) {
         const int sb = g & 1;
@@ -706,49 +707,81 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           break;
         }
         tc::fence_after_sync();
-        float s[64];
+        // x[0]: columns 0..63, x[1]: 64..127; x[h][4n + e] for e < 2 is row A, column
+        // 64 h + 8n + 2 cq + e; e = 2, 3 the same columns of row B.
+        float x[2][32];
         {
           uint32_t r0[32], r1[32];
           __syncwarp();
-          tc::tmem_ld32(tmem + lane_base + L::S_COL + sb * SKB + half * 64, r0);
-          tc::tmem_ld32(tmem + lane_base + L::S_COL + sb * SKB + half * 64 + 32, r1);
+          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + sb * SKB, r0);
+          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + sb * SKB + 64, r1);
           tc::tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            s[i] = __uint_as_float(r0[i]);
-            s[32 + i] = __uint_as_float(r1[i]);
+            x[0][i] = __uint_as_float(r0[i]);
+            x[1][i] = __uint_as_float(r1[i]);
           }
         }
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->s_empty[sb]);  // S_{g+2} may overwrite the buffer
-        const int k0 = j * SKB + half * 64;
-        if (k0 + 63 > q0 || k0 + 64 > p.T) {  // diagonal or ragged block: mask
+        const int k0 = j * SKB + 2 * cq;
+        if (j * SKB + SKB - 1 > q0 || j * SKB + SKB > p.T) {  // diagonal or ragged block: mask
 #pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (k0 + i > t || k0 + i >= p.T) s[i] = -INFINITY;
+          for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+            for (int n = 0; n < 8; ++n)
+#pragma unroll
+              for (int e = 0; e < 2; ++e) {
+                const int key = k0 + 64 * hh + 8 * n + e;
+                if (key > tA || key >= p.T) x[hh][4 * n + e] = -INFINITY;
+                if (key > tB || key >= p.T) x[hh][4 * n + 2 + e] = -INFINITY;
+              }
         }
-        float mx8[8];
+        float mxA = x[0][0], mxB = x[0][2];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+        for (int hh = 0; hh < 2; ++hh)
 #pragma unroll
-        for (int i = 8; i < 64; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], s[i]);
-        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-        mx = fmaxf(mx, half_exchange(bars, half, row, seq, mx, abort, p.status));
+          for (int n = 0; n < 8; ++n) {
+            mxA = tc::fmax3(mxA, x[hh][4 * n], x[hh][4 * n + 1]);
+            mxB = tc::fmax3(mxB, x[hh][4 * n + 2], x[hh][4 * n + 3]);
+          }
+        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
+        mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 1));
+        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 2));
+        mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 2));
         // Scores are raw (unscaled) here; the softmax scale times log2(e) is applied in the exponent.
-        const float m_new = fmaxf(m, mx * p.sl2);
-        const bool resc = m_new > m + kRescaleLog2;
-        const float m_use = resc ? m_new : m;
-        const float alpha = resc ? tc::fast_exp2(m - m_new) : 1.f;
-        float rs8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        const float mnA = fmaxf(mA, mxA * p.sl2), mnB = fmaxf(mB, mxB * p.sl2);
+        const bool rsA = mnA > mA + kRescaleLog2, rsB = mnB > mB + kRescaleLog2;
+        const float muA = rsA ? mnA : mA, muB = rsB ? mnB : mB;
+        const float alA = rsA ? tc::fast_exp2(mA - mnA) : 1.f;
+        const float alB = rsB ? tc::fast_exp2(mB - mnB) : 1.f;
+        float sa0 = 0.f, sa1 = 0.f, sb0 = 0.f, sb1 = 0.f;
 #pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          s[i] = tc::fast_exp2(fmaf(s[i], p.sl2, -m_use));
-          rs8[i & 7] += s[i];
-        }
-        l = l * alpha + (((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7])));
-        m = m_use;
+        for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+          for (int n = 0; n < 8; ++n) {
+            x[hh][4 * n] = tc::fast_exp2(fmaf(x[hh][4 * n], p.sl2, -muA));
+            x[hh][4 * n + 1] = tc::fast_exp2(fmaf(x[hh][4 * n + 1], p.sl2, -muA));
+            x[hh][4 * n + 2] = tc::fast_exp2(fmaf(x[hh][4 * n + 2], p.sl2, -muB));
+            x[hh][4 * n + 3] = tc::fast_exp2(fmaf(x[hh][4 * n + 3], p.sl2, -muB));
+            sa0 += x[hh][4 * n];
+            sa1 += x[hh][4 * n + 1];
+            sb0 += x[hh][4 * n + 2];
+            sb1 += x[hh][4 * n + 3];
+          }
+        lA = lA * alA + (sa0 + sa1);  // this thread's share of row A; summed over the 4 at the end
+        lB = lB * alB + (sb0 + sb1);
+        mA = muA;
+        mB = muB;
+        uint32_t pw[32];  // P words: pw[2n] row A, pw[2n + 1] row B, column 4n + cq of P
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+          for (int n = 0; n < 8; ++n) {
+            pw[2 * (8 * hh + n)] = pack_half2(x[hh][4 * n], x[hh][4 * n + 1]);
+            pw[2 * (8 * hh + n) + 1] = pack_half2(x[hh][4 * n + 2], x[hh][4 * n + 3]);
+          }
         // P_{g-1} V_{g-1} (and so every earlier P V) must have completed before P is overwritten
         // or O is rescaled.
         if (g > 0 && !tc::mbar_wait(&bars->pv_done, (g - 1) & 1, abort, p.status)) {
@@ -756,61 +789,76 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           break;
         }
         tc::fence_after_sync();
-        if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        if (j > 0 && __any_sync(0xffffffffu, rsA || rsB)) {
 #pragma unroll 1
           for (int ch = 0; ch < DH / 64; ++ch) {
             uint32_t r[32];
-            const uint32_t col = L::O_COL + half * (DH / 2) + ch * 32;
+            const uint32_t col = L::O_COL + ch * 64;
             __syncwarp();
-            tc::tmem_ld32(tmem + lane_base + col, r);
+            tc::tmem_ld_16x256b_x8(tmem + lane16 + col, r);
             tc::tmem_ld_wait();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tc::tmem_st32(tmem + lane_base + col, r);
+            for (int n = 0; n < 8; ++n) {
+              r[4 * n] = __float_as_uint(__uint_as_float(r[4 * n]) * alA);
+              r[4 * n + 1] = __float_as_uint(__uint_as_float(r[4 * n + 1]) * alA);
+              r[4 * n + 2] = __float_as_uint(__uint_as_float(r[4 * n + 2]) * alB);
+              r[4 * n + 3] = __float_as_uint(__uint_as_float(r[4 * n + 3]) * alB);
+            }
+            tc::tmem_st_16x256b_x8(tmem + lane16 + col, r);
           }
         }
-        {  // P (fp16 pairs) of keys [64 half, 64 half + 64): P columns [32 half, 32 half + 32)
-          uint32_t pr[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const __half2 h2 = __floats2half2_rn(s[2 * i], s[2 * i + 1]);
-            pr[i] = *reinterpret_cast<const uint32_t*>(&h2);
-          }
-          __syncwarp();
-          tc::tmem_st32(tmem + lane_base + L::P_COL + half * 32, pr);
-          tc::tmem_st_wait();
-        }
+        __syncwarp();
+        tc::tmem_st_16x128b_x16(tmem + lane16 + L::P_COL, pw);
+        tc::tmem_st_wait();
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->p_full);
       }
+      // row statistics for the epilogue, which uses one thread per row
+      lA += __shfl_xor_sync(0xffffffffu, lA, 1);
+      lB += __shfl_xor_sync(0xffffffffu, lB, 1);
+      lA += __shfl_xor_sync(0xffffffffu, lA, 2);
+      lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+      if (cq == 0) {
+        bars->row_m[rA] = mA;
+        bars->row_l[rA] = lA;
+        bars->row_m[rB] = mB;
+        bars->row_l[rB] = lB;
+      }
       // ------------------------------------------------------------------ epilogue
+      // Coalesced pass: the warp's 32 rows x 32 columns of O go through shared memory; lane l then
+      // handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte row segment. The
+      // A_ref loads of every chunk are issued first so that their latency overlaps the wait for O.
+      // In mode 2 the fp16-rounded error goes back through the same slots to the row's owner,
+      // which accumulates D = rowsum(dO * O).
+      const int h = 2 * tl.hp + (row >> 6);
+      const int t = q0 + (row & 63);
+      const int rbase = quarter * 32;  // first stacked row of this warp
+      const int c4 = lane & 7;
+      float4 av[DH / 64][8];
+      if (MODE != 0 && ok) {
+#pragma unroll
+        for (int ch = 0; ch < DH / 64; ++ch)
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & 63);
+            if (tt < p.T)
+              av[ch][i] = __ldg(reinterpret_cast<const float4*>(
+                  p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + h * DH + half * (DH / 2) +
+                  ch * 32 + c4 * 4));
+          }
+      }
+      tc::named_bar_sync(1, EW_WARPS * 32);  // row statistics written
       double acc = 0.0;
       const bool have = ok && tc::mbar_wait(&bars->o_full, tc_ & 1, abort, p.status);
+      const float m = bars->row_m[row], lt = bars->row_l[row];
       if (have) {
         tc::fence_after_sync();
-        const float lt = l + half_exchange(bars, half, row, seq, l, abort, p.status);
         const float inv_l = __fdiv_rn(1.f, lt);
-        // O in 32-column chunks. Coalesced pass: the warp's 32 rows x 32 columns go through shared
-        // memory; lane l then handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte
-        // row segment. In mode 2 the fp16-rounded error goes back through the same slots to the
-        // row's owner, which accumulates D = rowsum(dO * O).
-        const int rbase = quarter * 32;  // first stacked row of this warp
-        const int c4 = lane & 7;
         float sq = 0.f, dsum = 0.f;
-#pragma unroll 1
+#pragma unroll
         for (int ch = 0; ch < DH / 64; ++ch) {
           const int col = h * DH + half * (DH / 2) + ch * 32 + c4 * 4;
-          float4 av[8];
-          if (MODE != 0) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & 63);
-              if (tt < p.T)
-                av[i] = __ldg(reinterpret_cast<const float4*>(
-                    p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col));
-            }
-          }
           float o[32];
           {
             uint32_t r[32];
@@ -837,8 +885,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               *reinterpret_cast<float4*>(p.a_out + off) = ov;
               sq += ov.x * ov.x + ov.y * ov.y + ov.z * ov.z + ov.w * ov.w;
             } else {
-              const float e0 = __fsub_rn(ov.x, av[i].x), e1 = __fsub_rn(ov.y, av[i].y);
-              const float e2 = __fsub_rn(ov.z, av[i].z), e3 = __fsub_rn(ov.w, av[i].w);
+              const float4 a = av[ch][i];
+              const float e0 = __fsub_rn(ov.x, a.x), e1 = __fsub_rn(ov.y, a.y);
+              const float e2 = __fsub_rn(ov.z, a.z), e3 = __fsub_rn(ov.w, a.w);
               sq += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
               if (MODE == 2) {
                 const __half2 a01 = __floats2half2_rn(e0, e1), a23 = __floats2half2_rn(e2, e3);
@@ -858,6 +907,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               const float4 e = *reinterpret_cast<const float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2));
               dsum += e.x * o[4 * v] + e.y * o[4 * v + 1] + e.z * o[4 * v + 2] + e.w * o[4 * v + 3];
             }
+            __syncwarp();
           }
         }
         // O is no longer needed: the next tile's first P V may overwrite it.
@@ -874,16 +924,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         acc = (double)sq;
       }
       acc = warp_sum(acc);
-      if (lane == 0) bars->red[warp - 2] = acc;
-      tc::named_bar_sync(1, EW_WARPS * 32);  // every softmax warp reaches this once per tile
+      double* red = bars->red[tc_ & 1];  // alternate by tile
+      if (lane == 0) red[warp - 2] = acc;
+      // every softmax warp reaches this once per tile; it also keeps row_m / row_l of this tile
+      // until all warps have read them
+      tc::named_bar_sync(1, EW_WARPS * 32);
       if (lane == 0 && half == 0 && (quarter & 1) == 0 && have) {
-        // head hd's rows are lane quarters 2 hd and 2 hd + 1, each split over two warps
-        const int wq0 = (2 * hd + 2) & 3;  // warp index - 2 of quarter 2 hd, half 0
-        const double v = bars->red[wq0] + bars->red[(wq0 + 1) & 3] + bars->red[wq0 + 4] +
-                         bars->red[((wq0 + 1) & 3) + 4];
+        // head (row >> 6)'s rows are lane quarters 2 hd and 2 hd + 1, each split over two warps
+        const int wq0 = (2 * (row >> 6) + 2) & 3;  // warp index - 2 of that quarter, half 0
+        const double v = red[wq0] + red[(wq0 + 1) & 3] + red[wq0 + 4] + red[((wq0 + 1) & 3) + 4];
         p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] = v;
       }
-      tc::named_bar_sync(1, EW_WARPS * 32);  // red[] is rewritten by the next tile
       if (!ok || !have) break;
     }
   }
@@ -920,7 +971,7 @@ cudaError_t launch_fwd_pair(const CUtensorMap& tq, const CUtensorMap& tkv, const
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  attn_fwd_pair_kernel<DH, MODE><<<grid, NUM_THREADS, StackLayout<DH>::SMEM, st>>>(tq, tkv, p);
+  attn_fwd_pair_kernel<DH, MODE><<<grid, PAIR_THREADS, StackLayout<DH>::SMEM, st>>>(tq, tkv, p);
   return cudaGetLastError();
 }
 
