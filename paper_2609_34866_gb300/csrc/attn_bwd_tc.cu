@@ -87,35 +87,54 @@ __device__ __forceinline__ void store_half_row(uint8_t* base, int row, int half,
   }
 }
 
-// Stages this thread's TMEM row of DH gradient columns, times `mul`, optionally through the
-// transpose of RoPE at position `pos`, into tile[dim][row] (bf16, 128 rows per dim). Only the
-// 32-column pairs (pr, pr + DH/64) with pr in [pr0, pr1) are handled by this thread.
+// Stages gradient rows of a TMEM accumulator (DH columns), times `mul`, optionally through the
+// transpose of RoPE, into tile[dim][row] (bf16, 128 rows per dim). The calling warp handles the 16
+// TMEM lanes addressed by `taddr` with the 16x256b shape: thread t holds rows row_a = first + t / 4
+// and row_a + 8 and, in each 8-column group, the column pair 2 (t % 4), so the four threads of a row
+// read 32 contiguous bytes of a cos / sin table row (pos_a, pos_b: table rows of row_a, row_a + 8).
 template <int DH>
-__device__ __forceinline__ void stage_grad_row(uint32_t taddr, float mul, bool rope, int pos,
-                                               const float* cos_t, const float* sin_t,
-                                               bf16_t* tile, int row, int pr0, int pr1) {
+__device__ __forceinline__ void stage_grad_16(uint32_t taddr, float mul, bool rope, int pos_a,
+                                              int pos_b, const float* cos_t, const float* sin_t,
+                                              bf16_t* tile, int row_a) {
   constexpr int HALF = DH / 2;
+  const int cq = threadIdx.x & 3;
 #pragma unroll 1
-  for (int pr = pr0; pr < pr1; ++pr) {
-    const int c1 = pr, c2 = pr + HALF / 32;
-    uint32_t ra[32], rb[32];
+  for (int c = 0; c < HALF / 32; ++c) {
+    uint32_t r1[16], r2[16];
     __syncwarp();
-    tc::tmem_ld32(taddr + c1 * 32, ra);
-    tc::tmem_ld32(taddr + c2 * 32, rb);
+    tc::tmem_ld_16x256b_x4(taddr + c * 32, r1);
+    tc::tmem_ld_16x256b_x4(taddr + HALF + c * 32, r2);
     tc::tmem_ld_wait();
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      float g1 = __uint_as_float(ra[i]) * mul, g2 = __uint_as_float(rb[i]) * mul;
+    for (int n = 0; n < 4; ++n) {
+      const int j0 = c * 32 + 8 * n + 2 * cq;  // columns j0, j0 + 1 of the first half
+      float2 ca = make_float2(1.f, 1.f), sa = make_float2(0.f, 0.f);
+      float2 cb = make_float2(1.f, 1.f), sb = make_float2(0.f, 0.f);
       if (rope) {
-        const int jj = c1 * 32 + i;
-        const float cs = __ldg(cos_t + (int64_t)pos * HALF + jj);
-        const float sn = __ldg(sin_t + (int64_t)pos * HALF + jj);
-        const float x1 = g1, x2 = g2;
-        g1 = x1 * cs + x2 * sn;
-        g2 = x2 * cs - x1 * sn;
+        ca = __ldg(reinterpret_cast<const float2*>(cos_t + (int64_t)pos_a * HALF + j0));
+        sa = __ldg(reinterpret_cast<const float2*>(sin_t + (int64_t)pos_a * HALF + j0));
+        cb = __ldg(reinterpret_cast<const float2*>(cos_t + (int64_t)pos_b * HALF + j0));
+        sb = __ldg(reinterpret_cast<const float2*>(sin_t + (int64_t)pos_b * HALF + j0));
       }
-      tile[(c1 * 32 + i) * 128 + row] = __float2bfloat16_rn(g1);
-      tile[(c2 * 32 + i) * 128 + row] = __float2bfloat16_rn(g2);
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float csa = e ? ca.y : ca.x, sna = e ? sa.y : sa.x;
+        const float csb = e ? cb.y : cb.x, snb = e ? sb.y : sb.x;
+        float a1 = __uint_as_float(r1[4 * n + e]) * mul, a2 = __uint_as_float(r2[4 * n + e]) * mul;
+        float b1 = __uint_as_float(r1[4 * n + 2 + e]) * mul;
+        float b2 = __uint_as_float(r2[4 * n + 2 + e]) * mul;
+        if (rope) {
+          const float x1 = a1, x2 = a2, y1 = b1, y2 = b2;
+          a1 = x1 * csa + x2 * sna;
+          a2 = x2 * csa - x1 * sna;
+          b1 = y1 * csb + y2 * snb;
+          b2 = y2 * csb - y1 * snb;
+        }
+        tile[(j0 + e) * 128 + row_a] = __float2bfloat16_rn(a1);
+        tile[(HALF + j0 + e) * 128 + row_a] = __float2bfloat16_rn(a2);
+        tile[(j0 + e) * 128 + row_a + 8] = __float2bfloat16_rn(b1);
+        tile[(HALF + j0 + e) * 128 + row_a + 8] = __float2bfloat16_rn(b2);
+      }
     }
   }
 }
@@ -362,13 +381,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const bool have = ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status);
     bf16_t* tv = reinterpret_cast<bf16_t*>(smem + L::ST_OFF);
     bf16_t* tk = tv + DH * 128;
-    const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
     if (have) {
       tc::fence_after_sync();
-      stage_grad_row<DH>(tmem + lane_base + DV_COL, 1.f, false, 0, p.cos_t, p.sin_t, tv, row, pr0,
-                         pr1);
-      stage_grad_row<DH>(tmem + lane_base + DK_COL, p.scale, p.use_rope != 0,
-                         key < p.T ? key : 0, p.cos_t, p.sin_t, tk, row, pr0, pr1);
+      const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
+      const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
+      const int ka = kb * BK + ra, kb8 = ka + 8;
+      stage_grad_16<DH>(tmem + lane16 + DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, ra);
+      stage_grad_16<DH>(tmem + lane16 + DK_COL, p.scale, p.use_rope != 0, ka < p.T ? ka : 0,
+                        kb8 < p.T ? kb8 : 0, p.cos_t, p.sin_t, tk, ra);
     }
     tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
     if (have) {
@@ -395,7 +415,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // tiles with 128-key blocks, so every UMMA is M128 N128. TMEM: S = Q K^T (128 columns) and
 // dP = dO V^T (128) single-buffered, and two dQ accumulators (2 x 128) so that the next tile's
 // MMAs run while the elementwise warps finish the previous tile's epilogue. K has a 2-stage ring
-// (read by S and later by dQ), V a single buffer (read only by dP); the next tile's Q and dO load
+// (read by S and later by dQ), V a 2-stage ring (read only by dP); the next tile's Q and dO load
 // as soon as the current tile's last S/dP has completed.
 template <int DH>
 struct DqLayout {
@@ -405,8 +425,8 @@ struct DqLayout {
   static constexpr int Q_OFF = 0;
   static constexpr int DO_OFF = Q_OFF + TILE;
   static constexpr int K_OFF = DO_OFF + TILE;  // 2 stages
-  static constexpr int V_OFF = K_OFF + 2 * TILE;
-  static constexpr int DS_OFF = V_OFF + TILE;  // dS, and the epilogue's staging tile
+  static constexpr int V_OFF = K_OFF + 2 * TILE;  // 2 stages
+  static constexpr int DS_OFF = V_OFF + 2 * TILE;  // dS, and the epilogue's staging tile
   static constexpr int DS_BYTES = BQ * BK * 2;
   static constexpr int BAR_OFF = DS_OFF + DS_BYTES;
   static constexpr int USED = BAR_OFF + 256 + 1024;
@@ -414,7 +434,7 @@ struct DqLayout {
 };
 
 struct DqBars {
-  uint64_t qdo_full, qdo_empty, k_full[2], k_empty[2], v_full, v_empty, s_full, s_empty;
+  uint64_t qdo_full, qdo_empty, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full, s_empty;
   uint64_t p_full, p_empty, o_full[2], o_empty[2], drain;
   uint32_t tmem_base;
   int abort;
@@ -482,9 +502,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::mbar_init(&bars->k_empty[i], 1);
       tc::mbar_init(&bars->o_full[i], 1);
       tc::mbar_init(&bars->o_empty[i], EW_WARPS);
+      tc::mbar_init(&bars->v_full[i], 1);
+      tc::mbar_init(&bars->v_empty[i], 1);
     }
-    tc::mbar_init(&bars->v_full, 1);
-    tc::mbar_init(&bars->v_empty, 1);
     tc::mbar_init(&bars->s_full, 1);
     tc::mbar_init(&bars->s_empty, EW_WARPS);
     tc::mbar_init(&bars->p_full, EW_WARPS);
@@ -511,8 +531,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------------------------- TMA
       uint32_t J = 0;  // key blocks loaded so far (all tiles)
       int n = 0;
-      bool qdo_issued = false, v_issued = false;
-      uint32_t k_issued = 0, k_par = 0, qdo_par = 0, v_par = 0;
+      bool qdo_issued = false;
+      uint32_t k_issued = 0, k_par = 0, qdo_par = 0, v_issued = 0, v_par = 0;
       for (int tile = blockIdx.x; tile < n_tiles && !*abort; tile += gridDim.x, ++n) {
         const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
         const int row0 = tl.b * p.T, g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
@@ -535,20 +555,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             &bars->k_full[st], p.kcol0 + g * DH + ch * 64, row0 + j * BK);
           k_issued |= 1u << st;
           k_par = (k_par & ~(1u << st)) | (((J >> 1) & 1u) << st);
-          if (!tc::mbar_wait(&bars->v_empty, (J & 1) ^ 1, abort, p.status)) break;
-          tc::mbar_expect_tx(&bars->v_full, L::TILE);
+          if (!tc::mbar_wait(&bars->v_empty[st], ((J >> 1) & 1) ^ 1, abort, p.status)) break;
+          tc::mbar_expect_tx(&bars->v_full[st], L::TILE);
           for (int ch = 0; ch < DH / 64; ++ch)
-            tc::tma_load_2d(smem + L::V_OFF + ch * L::CHUNK, &tm_kv, &bars->v_full,
-                            p.vcol0 + g * DH + ch * 64, row0 + j * BK);
-          v_issued = true;
-          v_par = J & 1;
+            tc::tma_load_2d(smem + L::V_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv,
+                            &bars->v_full[st], p.vcol0 + g * DH + ch * 64, row0 + j * BK);
+          v_issued |= 1u << st;
+          v_par = (v_par & ~(1u << st)) | (((J >> 1) & 1u) << st);
         }
       }
       if (*abort) {
         if (qdo_issued) drain_wait(&bars->qdo_full, qdo_par);
         for (int st = 0; st < 2; ++st)
           if (k_issued & (1u << st)) drain_wait(&bars->k_full[st], (k_par >> st) & 1);
-        if (v_issued) drain_wait(&bars->v_full, v_par);
+        for (int st = 0; st < 2; ++st)
+          if (v_issued & (1u << st)) drain_wait(&bars->v_full[st], (v_par >> st) & 1);
       }
     }
   } else if (warp == 1) {
@@ -557,7 +578,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
       const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
       const uint32_t do_base = tc::smem_u32(smem + L::DO_OFF);
-      const uint32_t v_base = tc::smem_u32(smem + L::V_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
       bool ok = true;
       uint32_t Js = 0, Jg = 0;  // S/dP blocks and dQ blocks issued so far (all tiles)
@@ -578,9 +598,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         while (ok && ng < nkb) {
           bool prog = false;
           if (ns < nkb && ns <= ng + 1 && tc::mbar_ready(&bars->k_full[Js & 1], (Js >> 1) & 1) &&
-              tc::mbar_ready(&bars->v_full, Js & 1) && tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
+              tc::mbar_ready(&bars->v_full[Js & 1], (Js >> 1) & 1) &&
+              tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
             tc::fence_after_sync();
             const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Js & 1) * L::TILE);
+            const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + (Js & 1) * L::TILE);
 #pragma unroll
             for (int k = 0; k < DH / 16; ++k) {
               const uint32_t off = (k >> 2) * L::CHUNK + (k & 3) * 32;
@@ -590,7 +612,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                            tc::sdesc_kmajor_sw128(v_base + off), ID_S, k > 0 ? 1u : 0u);
             }
             tc::umma_commit(&bars->s_full);
-            tc::umma_commit(&bars->v_empty);
+            tc::umma_commit(&bars->v_empty[Js & 1]);
             ++ns;
             ++Js;
             if (ns == nkb) tc::umma_commit(&bars->qdo_empty);  // Q, dO free for the next tile
@@ -629,7 +651,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     uint8_t* dsrow = smem + L::DS_OFF + half * (BQ * 128) + row * 128;  // one 64-key swizzle chunk
     bf16_t* stage = reinterpret_cast<bf16_t*>(smem + L::DS_OFF);
-    const int pr0 = half * (DH / 128), pr1 = (half + 1) * (DH / 128) + (DH == 64 && half == 0);
     bool ok = true;
     uint32_t J = 0;
     int n = 0, epoch = 0;
@@ -704,8 +725,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc::fence_after_sync();
-      stage_grad_row<DH>(tmem + lane_base + DQ_COL + (n & 1) * 128, p.scale, p.use_rope != 0,
-                         valid_row ? t : 0, p.cos_t, p.sin_t, stage, row, pr0, pr1);
+      {
+        const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
+        const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
+        const int ta = q0 + ra, tb = ta + 8;
+        stage_grad_16<DH>(tmem + lane16 + DQ_COL + (n & 1) * 128, p.scale, p.use_rope != 0,
+                          ta < p.T ? ta : 0, tb < p.T ? tb : 0, p.cos_t, p.sin_t, stage, ra);
+      }
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->o_empty[n & 1]);  // dQ accumulator reusable
