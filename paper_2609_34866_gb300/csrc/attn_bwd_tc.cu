@@ -411,31 +411,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ================================================================================ dQ
-// Persistent: one CTA per SM walks a longest-first list of (128 query rows, query head, sequence)
-// tiles with 128-key blocks, so every UMMA is M128 N128. TMEM: S = Q K^T (128 columns) and
-// dP = dO V^T (128) single-buffered, and two dQ accumulators (2 x 128) so that the next tile's
-// MMAs run while the elementwise warps finish the previous tile's epilogue. K has a 2-stage ring
-// (read by S and later by dQ), V a 2-stage ring (read only by dP); the next tile's Q and dO load
-// as soon as the current tile's last S/dP has completed.
+// Persistent: one CTA per SM takes (128 query rows, query head, sequence) tiles (sched_tile)
+// with 128-key blocks, so every UMMA is M128 N128. Q and dO live in tensor memory (copied from a 32 KB
+// staging tile by tcgen05.cp), so S = Q K^T and dP = dO V^T are TS-form UMMAs that read only K and V
+// from shared memory, and the shared memory saved holds a third K stage: K is read by S_j and again
+// by dQ_j += dS_j K_j, so it is held for a whole block.
+//   TMEM columns: S 0, dP 128, dQ 256 (DH), Q and dO (DH / 2 each) after it.
+//   warp 0      TMA: Q and dO of each tile through the staging tile, K ring (3 stages)
+//   warp 1      TMEM owner, tcgen05.cp of Q and dO, UMMA issuer (one thread, event-driven)
+//   warps 2..9  elementwise: dS = P (dP - D) with P = exp2(S scale log2(e) - lse), fp16 to shared
+//               memory; the epilogue (transpose of RoPE, dQKV^T columns) while the next tile's Q and
+//               dO are copied in
+//   warp 10     TMA: V ring (2 stages)
+// A tile's Q is copied in once the previous tile's last S has completed and its dO once the last dP
+// has; the staging tile is refilled with the next operand as soon as each copy has completed.
+constexpr int DQ_THREADS = 352;
+
 template <int DH>
 struct DqLayout {
   static constexpr int BQ = 128, BK = 128;
+  static constexpr int KST = 3, VST = 2;
   static constexpr int CHUNK = 128 * 128;  // 64 columns of a 128-row tile
   static constexpr int TILE = 128 * DH * 2;
-  static constexpr int Q_OFF = 0;
-  static constexpr int DO_OFF = Q_OFF + TILE;
-  static constexpr int K_OFF = DO_OFF + TILE;  // 2 stages
-  static constexpr int V_OFF = K_OFF + 2 * TILE;  // 2 stages
-  static constexpr int DS_OFF = V_OFF + 2 * TILE;  // dS, and the epilogue's staging tile
+  static constexpr int STG_OFF = 0;  // Q or dO of a tile, on its way into TMEM
+  static constexpr int K_OFF = STG_OFF + TILE;
+  static constexpr int V_OFF = K_OFF + KST * TILE;
+  static constexpr int DS_OFF = V_OFF + VST * TILE;  // dS, and the epilogue's staging tile
   static constexpr int DS_BYTES = BQ * BK * 2;
   static constexpr int BAR_OFF = DS_OFF + DS_BYTES;
   static constexpr int USED = BAR_OFF + 256 + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+  static constexpr uint32_t S_COL = 0, DP_COL = 128, DQ_COL = 256, Q_COL = 256 + DH,
+                            DO_COL = 256 + DH + DH / 2;
+  static_assert(DO_COL + DH / 2 <= 512, "TMEM budget");
+  static_assert(DS_BYTES >= DH * 128 * 2, "epilogue staging fits the dS buffer");
 };
 
 struct DqBars {
-  uint64_t qdo_full, qdo_empty, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full, s_empty;
-  uint64_t p_full, p_empty, o_full[2], o_empty[2], drain;
+  uint64_t stg_full, stg_empty, k_full[3], k_empty[3], v_full[2], v_empty[2], s_full, s_empty;
+  uint64_t p_full, p_empty, o_full, o_empty, drain;
   uint32_t tmem_base;
   int abort;
   int ew_count;  // arrivals at the elementwise warps' epilogue barrier
@@ -469,7 +483,8 @@ __device__ __forceinline__ void ew_barrier(DqBars* bars, int epoch, volatile int
 struct DqTile {
   int qb, h, b;
 };
-// Tile n of the longest-first order: query blocks from the last (most keys) to the first.
+// Tile n of the most-work-first order: query blocks from the last (most keys) to the first, then
+// query heads and sequences.
 __device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
   const int per_qb = Hq * B;
   const int r = n % per_qb;
@@ -477,12 +492,12 @@ __device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
 }
 
 template <int DH>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(DQ_THREADS, 1)
     attn_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                           const __grid_constant__ CUtensorMap tm_kv,
                           const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
   using L = DqLayout<DH>;
-  constexpr int BQ = L::BQ, BK = L::BK;
+  constexpr int BQ = L::BQ, BK = L::BK, KST = L::KST, VST = L::VST;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -495,13 +510,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   auto n_kb_of = [&](const DqTile& tl) { return (min(tl.qb * BQ + BQ, p.T) + BK - 1) / BK; };
 
   if (threadIdx.x == 0) {
-    tc::mbar_init(&bars->qdo_full, 1);
-    tc::mbar_init(&bars->qdo_empty, 1);
-    for (int i = 0; i < 2; ++i) {
+    tc::mbar_init(&bars->stg_full, 1);
+    tc::mbar_init(&bars->stg_empty, 1);
+    for (int i = 0; i < KST; ++i) {
       tc::mbar_init(&bars->k_full[i], 1);
       tc::mbar_init(&bars->k_empty[i], 1);
-      tc::mbar_init(&bars->o_full[i], 1);
-      tc::mbar_init(&bars->o_empty[i], EW_WARPS);
+    }
+    for (int i = 0; i < VST; ++i) {
       tc::mbar_init(&bars->v_full[i], 1);
       tc::mbar_init(&bars->v_empty[i], 1);
     }
@@ -509,6 +524,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc::mbar_init(&bars->s_empty, EW_WARPS);
     tc::mbar_init(&bars->p_full, EW_WARPS);
     tc::mbar_init(&bars->p_empty, 1);
+    tc::mbar_init(&bars->o_full, 1);
+    tc::mbar_init(&bars->o_empty, EW_WARPS);
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
     bars->ew_count = 0;
@@ -525,113 +542,127 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
-  constexpr uint32_t S_COL = 0, DP_COL = 128, DQ_COL = 256;
 
-  if (warp == 0) {
-    if (lane == 0) {  // ------------------------------------------------------------- TMA
-      uint32_t J = 0;  // key blocks loaded so far (all tiles)
-      int n = 0;
-      bool qdo_issued = false;
-      uint32_t k_issued = 0, k_par = 0, qdo_par = 0, v_issued = 0, v_par = 0;
-      for (int tile = blockIdx.x; tile < n_tiles && !*abort; tile += gridDim.x, ++n) {
+  if (warp == 0 || warp == 10) {
+    if (lane == 0) {  // --------------------------------------- TMA: Q, dO, K (warp 0); V (warp 10)
+      const bool is_v = warp == 10;
+      uint32_t J = 0, U = 0;  // key blocks and staging uses so far (all tiles)
+      const int nst = is_v ? VST : KST;
+      uint64_t* full = is_v ? bars->v_full : bars->k_full;
+      uint64_t* empty = is_v ? bars->v_empty : bars->k_empty;
+      uint8_t* ring = smem + (is_v ? L::V_OFF : L::K_OFF);
+      bool ok = true, stg_issued = false;
+      uint32_t iss = 0, par = 0, stg_par = 0;
+      for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
+           tile = sched_tile(++it, gridDim.x, blockIdx.x)) {
         const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
         const int row0 = tl.b * p.T, g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
-        if (!tc::mbar_wait(&bars->qdo_empty, (n & 1) ^ 1, abort, p.status)) break;
-        tc::mbar_expect_tx(&bars->qdo_full, 2 * L::TILE);
-        for (int ch = 0; ch < DH / 64; ++ch) {
-          tc::tma_load_2d(smem + L::Q_OFF + ch * L::CHUNK, &tm_q, &bars->qdo_full,
-                          p.qcol0 + tl.h * DH + ch * 64, row0 + tl.qb * BQ);
-          tc::tma_load_2d(smem + L::DO_OFF + ch * L::CHUNK, &tm_do, &bars->qdo_full,
-                          tl.h * DH + ch * 64, row0 + tl.qb * BQ);
+        if (!is_v) {
+          for (int u = 0; u < 2; ++u, ++U) {  // Q, then dO
+            if (!tc::mbar_wait(&bars->stg_empty, (U & 1) ^ 1, abort, p.status)) { ok = false; break; }
+            tc::mbar_expect_tx(&bars->stg_full, L::TILE);
+            for (int ch = 0; ch < DH / 64; ++ch) {
+              if (u == 0)
+                tc::tma_load_2d(smem + L::STG_OFF + ch * L::CHUNK, &tm_q, &bars->stg_full,
+                                p.qcol0 + tl.h * DH + ch * 64, row0 + tl.qb * BQ);
+              else
+                tc::tma_load_2d(smem + L::STG_OFF + ch * L::CHUNK, &tm_do, &bars->stg_full,
+                                tl.h * DH + ch * 64, row0 + tl.qb * BQ);
+            }
+            stg_issued = true;
+            stg_par = U & 1;
+          }
+          if (!ok) break;
         }
-        qdo_issued = true;
-        qdo_par = n & 1;
+        const int col = is_v ? p.vcol0 + g * DH : p.kcol0 + g * DH;
         for (int j = 0; j < nkb; ++j, ++J) {
-          const int st = J & 1;
-          if (!tc::mbar_wait(&bars->k_empty[st], ((J >> 1) & 1) ^ 1, abort, p.status)) break;
-          tc::mbar_expect_tx(&bars->k_full[st], L::TILE);
+          const int st = J % nst;
+          const uint32_t ph = (J / nst) & 1;
+          if (!tc::mbar_wait(&empty[st], ph ^ 1, abort, p.status)) { ok = false; break; }
+          tc::mbar_expect_tx(&full[st], L::TILE);
           for (int ch = 0; ch < DH / 64; ++ch)
-            tc::tma_load_2d(smem + L::K_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv,
-                            &bars->k_full[st], p.kcol0 + g * DH + ch * 64, row0 + j * BK);
-          k_issued |= 1u << st;
-          k_par = (k_par & ~(1u << st)) | (((J >> 1) & 1u) << st);
-          if (!tc::mbar_wait(&bars->v_empty[st], ((J >> 1) & 1) ^ 1, abort, p.status)) break;
-          tc::mbar_expect_tx(&bars->v_full[st], L::TILE);
-          for (int ch = 0; ch < DH / 64; ++ch)
-            tc::tma_load_2d(smem + L::V_OFF + st * L::TILE + ch * L::CHUNK, &tm_kv,
-                            &bars->v_full[st], p.vcol0 + g * DH + ch * 64, row0 + j * BK);
-          v_issued |= 1u << st;
-          v_par = (v_par & ~(1u << st)) | (((J >> 1) & 1u) << st);
+            tc::tma_load_2d(ring + st * L::TILE + ch * L::CHUNK, &tm_kv, &full[st], col + ch * 64,
+                            row0 + j * BK);
+          iss |= 1u << st;
+          par = (par & ~(1u << st)) | (ph << st);
         }
       }
       if (*abort) {
-        if (qdo_issued) drain_wait(&bars->qdo_full, qdo_par);
-        for (int st = 0; st < 2; ++st)
-          if (k_issued & (1u << st)) drain_wait(&bars->k_full[st], (k_par >> st) & 1);
-        for (int st = 0; st < 2; ++st)
-          if (v_issued & (1u << st)) drain_wait(&bars->v_full[st], (v_par >> st) & 1);
+        if (stg_issued) drain_wait(&bars->stg_full, stg_par);
+        for (int st = 0; st < nst; ++st)
+          if (iss & (1u << st)) drain_wait(&full[st], (par >> st) & 1);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ------------------------------------------------------------- UMMA
       constexpr uint32_t ID_S = tc::idesc_f16(false, BQ, BK);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
-      const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
-      const uint32_t do_base = tc::smem_u32(smem + L::DO_OFF);
+      const uint32_t stg_base = tc::smem_u32(smem + L::STG_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
       bool ok = true;
-      uint32_t Js = 0, Jg = 0;  // S/dP blocks and dQ blocks issued so far (all tiles)
+      uint32_t Js = 0, Jg = 0, U = 0;  // S/dP blocks, dQ blocks, staging uses so far (all tiles)
       int n = 0;
       tc::Watchdog wd;
-      for (int tile = blockIdx.x; ok && tile < n_tiles; tile += gridDim.x, ++n) {
+      auto copy_in = [&](uint32_t col) -> bool {  // staging tile -> TMEM columns [col, col + DH/2)
+        if (!tc::mbar_wait(&bars->stg_full, U & 1, abort, p.status)) return false;
+        tc::fence_after_sync();
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk)
+          tc::tmem_cp_128x256b(tmem + col + kk * 8,
+                               tc::sdesc_kmajor_sw128(stg_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
+        tc::umma_commit(&bars->stg_empty);
+        ++U;
+        return true;
+      };
+      for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
+           tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
         const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
         const int nkb = n_kb_of(tl);
-        const uint32_t acc = DQ_COL + (n & 1) * 128;
-        if (!tc::mbar_wait(&bars->qdo_full, n & 1, abort, p.status) ||
-            !tc::mbar_wait(&bars->o_empty[n & 1], ((n >> 1) & 1) ^ 1, abort, p.status)) {
-          ok = false;
-          break;
-        }
-        // Event-driven issue: S/dP of block ns as soon as K_ns, V_ns have landed and the
-        // elementwise warps have read the previous S/dP; dQ of block ng once its dS is written.
+        // Q and dO of this tile into TMEM once every S / dP of the previous tile (which read the old
+        // Q and dO) has completed.
+        if (Js > 0 && !tc::mbar_wait(&bars->s_full, (Js - 1) & 1, abort, p.status)) break;
+        if (!copy_in(L::Q_COL) || !copy_in(L::DO_COL)) break;
+        // Event-driven issue: S/dP of block ns once K_ns, V_ns have landed and the elementwise
+        // warps have read the previous S/dP; dQ of block ng once its dS is written (and, for the
+        // tile's first, once the previous tile's dQ has been read out).
         int ns = 0, ng = 0;
         while (ok && ng < nkb) {
           bool prog = false;
-          if (ns < nkb && ns <= ng + 1 && tc::mbar_ready(&bars->k_full[Js & 1], (Js >> 1) & 1) &&
-              tc::mbar_ready(&bars->v_full[Js & 1], (Js >> 1) & 1) &&
+          if (ns < nkb && ns <= ng + 1 && tc::mbar_ready(&bars->k_full[Js % KST], (Js / KST) & 1) &&
+              tc::mbar_ready(&bars->v_full[Js % VST], (Js / VST) & 1) &&
               tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
             tc::fence_after_sync();
-            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Js & 1) * L::TILE);
-            const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + (Js & 1) * L::TILE);
+            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Js % KST) * L::TILE);
+            const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + (Js % VST) * L::TILE);
 #pragma unroll
             for (int k = 0; k < DH / 16; ++k) {
               const uint32_t off = (k >> 2) * L::CHUNK + (k & 3) * 32;
-              tc::umma_f16(tmem + S_COL, tc::sdesc_kmajor_sw128(q_base + off),
-                           tc::sdesc_kmajor_sw128(k_base + off), ID_S, k > 0 ? 1u : 0u);
-              tc::umma_f16(tmem + DP_COL, tc::sdesc_kmajor_sw128(do_base + off),
-                           tc::sdesc_kmajor_sw128(v_base + off), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + k * 8,
+                              tc::sdesc_kmajor_sw128(k_base + off), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::DO_COL + k * 8,
+                              tc::sdesc_kmajor_sw128(v_base + off), ID_S, k > 0 ? 1u : 0u);
             }
             tc::umma_commit(&bars->s_full);
-            tc::umma_commit(&bars->v_empty[Js & 1]);
+            tc::umma_commit(&bars->v_empty[Js % VST]);
             ++ns;
             ++Js;
-            if (ns == nkb) tc::umma_commit(&bars->qdo_empty);  // Q, dO free for the next tile
             prog = true;
           }
-          if (ng < ns && tc::mbar_ready(&bars->p_full, Jg & 1)) {
+          if (ng < ns && tc::mbar_ready(&bars->p_full, Jg & 1) &&
+              (ng > 0 || n == 0 || tc::mbar_ready(&bars->o_empty, (n - 1) & 1))) {
             tc::fence_after_sync();
-            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Jg & 1) * L::TILE);
+            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Jg % KST) * L::TILE);
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k)
-              tc::umma_f16(tmem + acc,
+              tc::umma_f16(tmem + L::DQ_COL,
                            tc::sdesc_kmajor_sw128(ds_base + (k >> 2) * (BQ * 128) + (k & 3) * 32),
                            tc::sdesc_mnmajor_sw128(k_base + k * 16 * 128, L::CHUNK, 1024), ID_G,
                            (ng > 0 || k > 0) ? 1u : 0u);
-            tc::umma_commit(&bars->k_empty[Jg & 1]);
+            tc::umma_commit(&bars->k_empty[Jg % KST]);
             tc::umma_commit(&bars->p_empty);
             ++ng;
             ++Jg;
-            if (ng == nkb) tc::umma_commit(&bars->o_full[n & 1]);
+            if (ng == nkb) tc::umma_commit(&bars->o_full);
             prog = true;
           }
           if (prog)
@@ -654,7 +685,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     bool ok = true;
     uint32_t J = 0;
     int n = 0, epoch = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++n) {
+    for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
+         tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
       const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
       const int nkb = n_kb_of(tl);
       const int q0 = tl.qb * BQ, t = q0 + row, row0 = tl.b * p.T;
@@ -673,8 +705,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int ch = 0; ch < 2; ++ch) {
           uint32_t rs[32], rd[32];
           __syncwarp();
-          tc::tmem_ld32(tmem + lane_base + S_COL + col0 + ch * 32, rs);
-          tc::tmem_ld32(tmem + lane_base + DP_COL + col0 + ch * 32, rd);
+          tc::tmem_ld32(tmem + lane_base + L::S_COL + col0 + ch * 32, rs);
+          tc::tmem_ld32(tmem + lane_base + L::DP_COL + col0 + ch * 32, rd);
           tc::tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
@@ -719,7 +751,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // Epilogue: dQ rows (transpose of RoPE) staged transposed in the dS buffer (free until this
       // tile's successor writes its first dS, which these same warps do next), then stored as
       // dQKV^T columns with coalesced 16-byte stores.
-      if (!tc::mbar_wait(&bars->o_full[n & 1], (n >> 1) & 1, abort, p.status) ||
+      if (!tc::mbar_wait(&bars->o_full, n & 1, abort, p.status) ||
           !tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
         ok = false;
         break;
@@ -729,12 +761,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
         const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
         const int ta = q0 + ra, tb = ta + 8;
-        stage_grad_16<DH>(tmem + lane16 + DQ_COL + (n & 1) * 128, p.scale, p.use_rope != 0,
-                          ta < p.T ? ta : 0, tb < p.T ? tb : 0, p.cos_t, p.sin_t, stage, ra);
+        stage_grad_16<DH>(tmem + lane16 + L::DQ_COL, p.scale, p.use_rope != 0, ta < p.T ? ta : 0,
+                          tb < p.T ? tb : 0, p.cos_t, p.sin_t, stage, ra);
       }
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->o_empty[n & 1]);  // dQ accumulator reusable
+      if (lane == 0) tc::mbar_arrive(&bars->o_empty);  // dQ accumulator reusable
       ew_barrier(bars, ++epoch, abort, p.status);
       store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
                      (int64_t)row0 + q0, min(BQ, p.T - q0), threadIdx.x - 64, EW_WARPS * 32);
@@ -806,7 +838,7 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t dq_tiles = (int64_t)((L.T + 127) / 128) * L.Hq * L.B;
   const unsigned g2 = (unsigned)std::min<int64_t>(dq_tiles, sms > 0 ? sms : 1);
-  attn_bwd_dq_tc_kernel<DH><<<g2, NUM_THREADS, DqLayout<DH>::SMEM, L.stream>>>(kv128, kv128, do128, p);
+  attn_bwd_dq_tc_kernel<DH><<<g2, DQ_THREADS, DqLayout<DH>::SMEM, L.stream>>>(kv128, kv128, do128, p);
   return cudaGetLastError();
 }
 

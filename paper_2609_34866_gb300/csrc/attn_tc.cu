@@ -410,11 +410,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ============================================================================ head-pair kernel
-// Persistent: one CTA per SM walks a list of tiles. A tile is 64 query rows of two query heads of
-// one KV group (GQA: both read the same K and V) stacked into the 128 rows of every UMMA: TMEM lane
-// r < 64 is row q0 + r of head h0, lane 64 + r is row q0 + r of head h0 + 1. Keys come in blocks of
-// 128 so that both products are M128 N128 UMMAs with the A operand in tensor memory (TS form), the
-// shape that runs the tensor pipe at full rate on sm_103a:
+// Persistent: one CTA per SM takes tiles in the order of sched_tile. A tile is 64 query rows of
+// two query heads of one KV group (GQA: both read the same K and V) stacked into the 128 rows of
+// every UMMA: TMEM lane r < 64 is row q0 + r of head h0, lane 64 + r is row q0 + r of head h0 + 1.
+// Keys come in blocks of 128 so that both products are M128 N128 UMMAs with the A operand in
+// tensor memory (TS form), the shape that runs the tensor pipe at full rate on sm_103a:
 //   S_j = Q K_j^T     A = Q (TMEM, copied from the TMA-loaded smem tile by tcgen05.cp), B = K_j
 //   O  += P_j V_j     A = P_j (TMEM, fp16 pairs written by the softmax threads), B = V_j (smem,
 //                     MN-major)
@@ -464,15 +464,13 @@ struct StackTile {
   int hp, bc, qb, nkb;
 };
 
-// Tile k: (sequence, head pair) major and query blocks minor, from the last query block (most key
-// blocks) to the first. CTAs take tiles k = blockIdx.x + i * gridDim.x, so the tiles running at any
-// time belong to a few (sequence, KV group) pairs whose K and V stay in L2, and every CTA gets a
-// similar mix of long and short tiles.
+// Tile k of the most-work-first order: query blocks from the last (most key blocks) to the first,
+// then sequences and head pairs.
 __device__ __forceinline__ StackTile stack_tile(int k, int pairs, int BC, int nqb, int T) {
   StackTile t;
-  t.qb = nqb - 1 - k % nqb;
-  t.hp = (k / nqb) % pairs;
-  t.bc = k / (nqb * pairs);
+  t.hp = k % pairs;
+  t.bc = (k / pairs) % BC;
+  t.qb = nqb - 1 - k / (pairs * BC);
   t.nkb = (min((t.qb + 1) * SQ, T) + SKB - 1) / SKB;
   return t;
 }
@@ -571,7 +569,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       uint8_t* ring = smem + (is_v ? L::V_OFF : L::K_OFF);
       constexpr int NST = SK_ST;
       static_assert(SK_ST == SV_ST, "one ring depth for K and V");
-      for (int k = blockIdx.x; ok && k < ntiles; k += gridDim.x, ++tc_) {
+      for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
+           k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
         const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
         const int b = tl.bc % p.B, c = tl.bc / p.B, h0 = 2 * tl.hp, g = h0 / ratio;
         const int row0 = b * p.T, q0 = tl.qb * SQ;
@@ -649,7 +648,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         tc::umma_commit(&bars->v_empty[vs]);
         return true;
       };
-      for (int k = blockIdx.x; ok && k < ntiles; k += gridDim.x, ++tc_) {
+      for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
+           k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
         const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
         // Q of this tile into TMEM once the previous tile's last S (which read the old Q) is done.
         if (g0 > 0 &&
@@ -684,14 +684,14 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     const int cq = lane & 3;                                   // column pair within each 8 columns
     const int rA = quarter * 32 + half * 16 + (lane >> 2);     // stacked rows of this thread
     const int rB = rA + 8;
-    const int hd = rA >> 6;                                    // rA and rB belong to the same head
     const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
     // epilogue layout (32x32b): one row per thread, half of its columns
     const int row = quarter * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     float* stg = reinterpret_cast<float*>(smem + L::EPI_OFF + (warp - 2) * 4096);
     int g = 0, tc_ = 0, seq = 0;
-    for (int k = blockIdx.x; k < ntiles; k += gridDim.x, ++tc_) {
+    for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
+         k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
       const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
       const int b = tl.bc % p.B, c = tl.bc / p.B;
@@ -930,7 +930,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       // until all warps have read them
       tc::named_bar_sync(1, EW_WARPS * 32);
       if (lane == 0 && half == 0 && (quarter & 1) == 0 && have) {
-        // head (row >> 6)'s rows are lane quarters 2 hd and 2 hd + 1, each split over two warps
+        // the head's rows are lane quarters 2 hd and 2 hd + 1 (hd = row >> 6), each over two warps
         const int wq0 = (2 * (row >> 6) + 2) & 3;  // warp index - 2 of that quarter, half 0
         const double v = red[wq0] + red[(wq0 + 1) & 3] + red[wq0 + 4] + red[((wq0 + 1) & 3) + 4];
         p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] = v;

@@ -61,4 +61,12 @@ __device__ __forceinline__ double block_sum(double x, double* smem /* >= NT/32 *
   return t;
 }
 
+// Static schedule of a persistent kernel: the tile a CTA takes in round i when `ntiles` tiles,
+// ordered from the most work to the least, are dealt to `grid` CTAs. Rounds alternate direction
+// (CTA x takes position x, then grid - 1 - x, ...), so every CTA gets a similar total; the tile
+// index grows with i, so a CTA is done at its first index >= ntiles.
+__device__ __forceinline__ int sched_tile(int i, int grid, int cta) {
+  return i * grid + ((i & 1) ? grid - 1 - cta : cta);
+}
+
 }  // namespace jab
