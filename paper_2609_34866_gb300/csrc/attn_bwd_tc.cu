@@ -24,7 +24,6 @@ namespace {
 
 constexpr int NUM_THREADS = 320;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise (2 per lane quarter)
 constexpr int EW_WARPS = 8;
-constexpr int STAGES = 3;
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct BwdParams {
@@ -41,35 +40,10 @@ struct BwdParams {
   int* status;
 };
 
-struct BwdBars {
-  uint64_t fixed_full, ld_full[STAGES], ld_empty[STAGES], s_full[2], s_empty[2];
-  uint64_t p_full, p_empty, o_full, drain;
-  uint32_t tmem_base;
-  int abort;
-};
-
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   const uint64_t t0 = tc::globaltimer();
   while (!tc::mbar_test(bar, parity))
     if (tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
-}
-
-__device__ __forceinline__ void init_bars(BwdBars* bars) {
-  tc::mbar_init(&bars->fixed_full, 1);
-  for (int i = 0; i < STAGES; ++i) {
-    tc::mbar_init(&bars->ld_full[i], 1);
-    tc::mbar_init(&bars->ld_empty[i], 1);
-  }
-  for (int i = 0; i < 2; ++i) {
-    tc::mbar_init(&bars->s_full[i], 1);
-    tc::mbar_init(&bars->s_empty[i], EW_WARPS);
-  }
-  tc::mbar_init(&bars->p_full, EW_WARPS);
-  tc::mbar_init(&bars->p_empty, 1);
-  tc::mbar_init(&bars->o_full, 1);
-  tc::mbar_init(&bars->drain, 1);
-  bars->abort = 0;
-  tc::fence_mbar_init();
 }
 
 // 32 fp16 values, half of one 128-byte row of a K-major, 128-byte-swizzled operand tile (16-byte
@@ -163,22 +137,41 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
 }
 
 // ================================================================================ dK, dV
+// One CTA per (128-key block, KV head, sequence); it loops over the query heads of the group and over
+// 64-query blocks. K and V live in tensor memory (copied once from shared memory by tcgen05.cp), so
+// S^T = K Q^T and dP^T = V dO^T are TS-form UMMAs that read only Q and dO from shared memory, and the
+// shared memory K and V would take holds a deeper Q / dO ring (5 stages): a stage is released only
+// when dV += P^T dO and dK += dS^T Q of its block have completed, so the ring has to cover a load
+// latency plus a block.
+//   TMEM columns: S^T 0 and dP^T 64 (single-buffered: the elementwise warps read them out at once),
+//   dV 128, dK 128 + DH, K and V (DH / 2 each) after them.
 template <int DH>
 struct DkdvLayout {
-  static constexpr int BK = 128, BQ = 64;
+  static constexpr int BK = 128, BQ = 64, STAGES = 5;
   static constexpr int KCHUNK = BK * 128;  // 64 columns of a 128-row tile
   static constexpr int QCHUNK = BQ * 128;  // 64 columns of a 64-row tile
-  static constexpr int K_OFF = 0;
-  static constexpr int V_OFF = K_OFF + BK * DH * 2;
-  static constexpr int ST_OFF = V_OFF + BK * DH * 2;
+  static constexpr int ST_OFF = 0;
   static constexpr int ST_Q = 0, ST_DO = BQ * DH * 2, ST_LSE = 2 * BQ * DH * 2,
                        ST_D = ST_LSE + BQ * 4, ST_BYTES = ST_D + BQ * 4;
   static constexpr int ST_STRIDE = (ST_BYTES + 1023) / 1024 * 1024;
+  static constexpr int KV_TILE = BK * DH * 2;  // K or V, staged in the last two stage slots
+  static_assert(KV_TILE <= ST_STRIDE, "K / V tile fits a stage slot");
   static constexpr int P_OFF = ST_OFF + STAGES * ST_STRIDE;
   static constexpr int DS_OFF = P_OFF + BK * BQ * 2;
   static constexpr int BAR_OFF = DS_OFF + BK * BQ * 2;
   static constexpr int USED = BAR_OFF + 256 + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+  static constexpr uint32_t S_COL = 0, DP_COL = 64, DV_COL = 128, DK_COL = 128 + DH,
+                            K_COL = 128 + 2 * DH, V_COL = 128 + 2 * DH + DH / 2;
+  static_assert(V_COL + DH / 2 <= 512, "TMEM budget");
+  static_assert(2 * DH * 128 * 2 <= STAGES * ST_STRIDE, "epilogue staging fits the stage ring");
+};
+
+struct DkdvBars {
+  uint64_t kv_full, kv_copied, ld_full[5], ld_empty[5], s_full, s_empty;
+  uint64_t p_full, p_empty, o_full, drain;
+  uint32_t tmem_base;
+  int abort;
 };
 
 template <int DH>
@@ -187,11 +180,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             const __grid_constant__ CUtensorMap tm_q,
                             const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
   using L = DkdvLayout<DH>;
-  constexpr int BK = L::BK, BQ = L::BQ;
+  constexpr int BK = L::BK, BQ = L::BQ, STAGES = L::STAGES;
+  constexpr int KV_A = STAGES - 2, KV_B = STAGES - 1;  // stage slots that first hold K and V
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  BwdBars* bars = reinterpret_cast<BwdBars*>(smem + L::BAR_OFF);
+  DkdvBars* bars = reinterpret_cast<DkdvBars*>(smem + L::BAR_OFF);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
 
@@ -204,7 +198,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int row0 = b * p.T;
 
   if (threadIdx.x == 0) {
-    init_bars(bars);
+    tc::mbar_init(&bars->kv_full, 1);
+    tc::mbar_init(&bars->kv_copied, 1);
+    for (int i = 0; i < STAGES; ++i) {
+      tc::mbar_init(&bars->ld_full[i], 1);
+      tc::mbar_init(&bars->ld_empty[i], 1);
+    }
+    tc::mbar_init(&bars->s_full, 1);
+    tc::mbar_init(&bars->s_empty, EW_WARPS);
+    tc::mbar_init(&bars->p_full, EW_WARPS);
+    tc::mbar_init(&bars->p_empty, 1);
+    tc::mbar_init(&bars->o_full, 1);
+    tc::mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_kv);
     tc::prefetch_tmap(&tm_q);
     tc::prefetch_tmap(&tm_do);
@@ -217,22 +224,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
-  constexpr uint32_t DV_COL = 256, DK_COL = 256 + DH;
 
   if (warp == 0) {
     if (lane == 0) {  // ------------------------------------------------------------- TMA
       uint32_t issued = 0, last_par = 0;
-      tc::mbar_expect_tx(&bars->fixed_full, 2 * BK * DH * 2);
+      tc::mbar_expect_tx(&bars->kv_full, 2 * L::KV_TILE);
       for (int ch = 0; ch < DH / 64; ++ch) {
-        tc::tma_load_2d(smem + L::K_OFF + ch * L::KCHUNK, &tm_kv, &bars->fixed_full,
-                        p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
-        tc::tma_load_2d(smem + L::V_OFF + ch * L::KCHUNK, &tm_kv, &bars->fixed_full,
-                        p.vcol0 + g * DH + ch * 64, row0 + kb * BK);
+        tc::tma_load_2d(smem + L::ST_OFF + KV_A * L::ST_STRIDE + ch * L::KCHUNK, &tm_kv,
+                        &bars->kv_full, p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
+        tc::tma_load_2d(smem + L::ST_OFF + KV_B * L::ST_STRIDE + ch * L::KCHUNK, &tm_kv,
+                        &bars->kv_full, p.vcol0 + g * DH + ch * 64, row0 + kb * BK);
       }
-      for (int it = 0; it < n_it; ++it) {
+      bool ok = true;
+      for (int it = 0; ok && it < n_it; ++it) {
         const int st = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
         const int h = g * r + it / per_head, i = i0 + it % per_head;
+        // The slots that held K and V are free once both have been copied into tensor memory.
+        if (it == KV_A && !tc::mbar_wait(&bars->kv_copied, 0, abort, p.status)) break;
         if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
         uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
         tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
@@ -249,7 +258,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         last_par = (last_par & ~(1u << st)) | (ph << st);
       }
       if (*abort) {
-        drain_wait(&bars->fixed_full, 0);
+        drain_wait(&bars->kv_full, 0);
         for (int st = 0; st < STAGES; ++st)
           if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
       }
@@ -258,34 +267,43 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------------------------- UMMA
       constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
-      const uint32_t k_base = tc::smem_u32(smem + L::K_OFF);
-      const uint32_t v_base = tc::smem_u32(smem + L::V_OFF);
       const uint32_t p_base = tc::smem_u32(smem + L::P_OFF);
       const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
-      // Event-driven issue: S^T / dP^T of block ns go out as soon as their K/V stage has landed and
-      // their TMEM buffer is free (up to two blocks ahead), the gradient MMAs of block ng as soon as
-      // its P^T and dS^T are in shared memory.
-      bool ok = tc::mbar_wait(&bars->fixed_full, 0, abort, p.status);
+      bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
+      if (ok) {  // K and V into tensor memory (A operands of S^T and dP^T)
+        tc::fence_after_sync();
+        const uint32_t ka = tc::smem_u32(smem + L::ST_OFF + KV_A * L::ST_STRIDE);
+        const uint32_t va = tc::smem_u32(smem + L::ST_OFF + KV_B * L::ST_STRIDE);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
+          tc::tmem_cp_128x256b(tmem + L::K_COL + k * 8, tc::sdesc_kmajor_sw128(ka + ko));
+          tc::tmem_cp_128x256b(tmem + L::V_COL + k * 8, tc::sdesc_kmajor_sw128(va + ko));
+        }
+        tc::umma_commit(&bars->kv_copied);
+      }
+      // Event-driven issue: S^T / dP^T of block ns go out as soon as its Q / dO stage has landed
+      // and the elementwise warps have read the previous S^T / dP^T out of tensor memory; the
+      // gradient MMAs of block ng as soon as its P^T and dS^T are in shared memory.
       int ns = 0, ng = 0;
       tc::Watchdog wd;
       while (ok && ng < n_it) {
         bool prog = false;
         if (ns < n_it && ns <= ng + 2) {
-          const int st = ns % STAGES, sbuf = ns & 1;
+          const int st = ns % STAGES;
           if (tc::mbar_ready(&bars->ld_full[st], (ns / STAGES) & 1) &&
-              tc::mbar_ready(&bars->s_empty[sbuf], ((ns >> 1) & 1) ^ 1)) {
+              tc::mbar_ready(&bars->s_empty, (ns & 1) ^ 1)) {
             tc::fence_after_sync();
             const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
 #pragma unroll
             for (int k = 0; k < DH / 16; ++k) {
-              const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
               const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
-              tc::umma_f16(tmem + sbuf * BQ, tc::sdesc_kmajor_sw128(k_base + ko),
-                           tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
-              tc::umma_f16(tmem + 128 + sbuf * BQ, tc::sdesc_kmajor_sw128(v_base + ko),
-                           tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::K_COL + k * 8,
+                              tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::V_COL + k * 8,
+                              tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
             }
-            tc::umma_commit(&bars->s_full[sbuf]);
+            tc::umma_commit(&bars->s_full);
             ++ns;
             prog = true;
           }
@@ -297,10 +315,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k) {
             const uint32_t acc = (ng > 0 || k > 0) ? 1u : 0u;
-            tc::umma_f16(tmem + DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
+            tc::umma_f16(tmem + L::DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
                          tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::QCHUNK, 1024),
                          ID_G, acc);
-            tc::umma_f16(tmem + DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
+            tc::umma_f16(tmem + L::DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
                          tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::QCHUNK, 1024),
                          ID_G, acc);
           }
@@ -328,9 +346,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     bool ok = true;
     for (int it = 0; it < n_it; ++it) {
       const int st = it % STAGES;
-      const int sbuf = it & 1;
       const int i = i0 + it % per_head;
-      if (!tc::mbar_wait(&bars->s_full[sbuf], (it >> 1) & 1, abort, p.status) ||
+      if (!tc::mbar_wait(&bars->s_full, it & 1, abort, p.status) ||
           !tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status)) {
         ok = false;
         break;
@@ -338,12 +355,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::fence_after_sync();
       uint32_t rs[32], rd[32];
       __syncwarp();
-      tc::tmem_ld32(tmem + lane_base + sbuf * BQ + col0, rs);
-      tc::tmem_ld32(tmem + lane_base + 128 + sbuf * BQ + col0, rd);
+      tc::tmem_ld32(tmem + lane_base + L::S_COL + col0, rs);
+      tc::tmem_ld32(tmem + lane_base + L::DP_COL + col0, rd);
       tc::tmem_ld_wait();
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->s_empty[sbuf]);
+      if (lane == 0) tc::mbar_arrive(&bars->s_empty);
       const uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
       const float* lse2 = reinterpret_cast<const float*>(sbase + L::ST_LSE) + col0;
       const float* dd = reinterpret_cast<const float*>(sbase + L::ST_D) + col0;
@@ -386,8 +403,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
       const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
       const int ka = kb * BK + ra, kb8 = ka + 8;
-      stage_grad_16<DH>(tmem + lane16 + DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, ra);
-      stage_grad_16<DH>(tmem + lane16 + DK_COL, p.scale, p.use_rope != 0, ka < p.T ? ka : 0,
+      stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, ra);
+      stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, ka < p.T ? ka : 0,
                         kb8 < p.T ? kb8 : 0, p.cos_t, p.sin_t, tk, ra);
     }
     tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
