@@ -140,14 +140,15 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
 // One CTA per (128-key block, KV head, sequence); it loops over the query heads of the group and over
 // 64-query blocks. K and V live in tensor memory (copied once from shared memory by tcgen05.cp), so
 // S^T = K Q^T and dP^T = V dO^T are TS-form UMMAs that read only Q and dO from shared memory, and the
-// shared memory K and V would take holds a deeper Q / dO ring (5 stages): a stage is released only
+// shared memory K and V would take holds a deeper Q / dO ring (4 stages: a stage is released only
 // when dV += P^T dO and dK += dS^T Q of its block have completed, so the ring has to cover a load
-// latency plus a block.
+// latency plus a block) and double-buffered P^T / dS^T tiles, so the elementwise warps of block j+1
+// do not wait for the gradient MMAs of block j.
 //   TMEM columns: S^T 0 and dP^T 64 (single-buffered: the elementwise warps read them out at once),
 //   dV 128, dK 128 + DH, K and V (DH / 2 each) after them.
 template <int DH>
 struct DkdvLayout {
-  static constexpr int BK = 128, BQ = 64, STAGES = 5;
+  static constexpr int BK = 128, BQ = 64, STAGES = 4;
   static constexpr int KCHUNK = BK * 128;  // 64 columns of a 128-row tile
   static constexpr int QCHUNK = BQ * 128;  // 64 columns of a 64-row tile
   static constexpr int ST_OFF = 0;
@@ -157,8 +158,9 @@ struct DkdvLayout {
   static constexpr int KV_TILE = BK * DH * 2;  // K or V, staged in the last two stage slots
   static_assert(KV_TILE <= ST_STRIDE, "K / V tile fits a stage slot");
   static constexpr int P_OFF = ST_OFF + STAGES * ST_STRIDE;
-  static constexpr int DS_OFF = P_OFF + BK * BQ * 2;
-  static constexpr int BAR_OFF = DS_OFF + BK * BQ * 2;
+  static constexpr int PT = BK * BQ * 2;  // one P^T or dS^T tile
+  static constexpr int DS_OFF = P_OFF + 2 * PT;
+  static constexpr int BAR_OFF = DS_OFF + 2 * PT;
   static constexpr int USED = BAR_OFF + 256 + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
   static constexpr uint32_t S_COL = 0, DP_COL = 64, DV_COL = 128, DK_COL = 128 + DH,
@@ -168,8 +170,8 @@ struct DkdvLayout {
 };
 
 struct DkdvBars {
-  uint64_t kv_full, kv_copied, ld_full[5], ld_empty[5], s_full, s_empty;
-  uint64_t p_full, p_empty, o_full, drain;
+  uint64_t kv_full, kv_copied, ld_full[4], ld_empty[4], s_full, s_empty;
+  uint64_t p_full[2], p_empty[2], o_full, drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -206,8 +208,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     tc::mbar_init(&bars->s_full, 1);
     tc::mbar_init(&bars->s_empty, EW_WARPS);
-    tc::mbar_init(&bars->p_full, EW_WARPS);
-    tc::mbar_init(&bars->p_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&bars->p_full[i], EW_WARPS);
+      tc::mbar_init(&bars->p_empty[i], 1);
+    }
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
@@ -267,8 +271,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------------------------- UMMA
       constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
-      const uint32_t p_base = tc::smem_u32(smem + L::P_OFF);
-      const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
       bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
       if (ok) {  // K and V into tensor memory (A operands of S^T and dP^T)
         tc::fence_after_sync();
@@ -308,10 +310,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             prog = true;
           }
         }
-        if (ng < ns && tc::mbar_ready(&bars->p_full, ng & 1)) {
+        if (ng < ns && tc::mbar_ready(&bars->p_full[ng & 1], (ng >> 1) & 1)) {
           tc::fence_after_sync();
-          const int st = ng % STAGES;
+          const int st = ng % STAGES, pb = ng & 1;
           const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+          const uint32_t p_base = tc::smem_u32(smem + L::P_OFF + pb * L::PT);
+          const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF + pb * L::PT);
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k) {
             const uint32_t acc = (ng > 0 || k > 0) ? 1u : 0u;
@@ -323,7 +327,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                          ID_G, acc);
           }
           tc::umma_commit(&bars->ld_empty[st]);
-          tc::umma_commit(&bars->p_empty);
+          tc::umma_commit(&bars->p_empty[pb]);
           if (ng == n_it - 1) tc::umma_commit(&bars->o_full);
           ++ng;
           prog = true;
@@ -362,8 +366,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->s_empty);
       const uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
-      const float* lse2 = reinterpret_cast<const float*>(sbase + L::ST_LSE) + col0;
-      const float* dd = reinterpret_cast<const float*>(sbase + L::ST_D) + col0;
+      float lse2[32], dd[32];  // per query column (the same for every key row: broadcast reads)
+#pragma unroll
+      for (int v = 0; v < 8; ++v) {
+        const float4 a = reinterpret_cast<const float4*>(sbase + L::ST_LSE)[col0 / 4 + v];
+        const float4 d = reinterpret_cast<const float4*>(sbase + L::ST_D)[col0 / 4 + v];
+        lse2[4 * v] = a.x, lse2[4 * v + 1] = a.y, lse2[4 * v + 2] = a.z, lse2[4 * v + 3] = a.w;
+        dd[4 * v] = d.x, dd[4 * v + 1] = d.y, dd[4 * v + 2] = d.z, dd[4 * v + 3] = d.w;
+      }
       const int q0 = i * BQ + col0;
       float pv[32], dsv[32];
       if (q0 >= kb * BK + BK - 1 && q0 + 31 < p.T) {  // every (key, query) pair is visible
@@ -382,16 +392,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           dsv[c] = valid ? e * (__uint_as_float(rd[c]) - dd[c]) : 0.f;
         }
       }
-      if (!tc::mbar_wait(&bars->p_empty, (it & 1) ^ 1, abort, p.status)) {
+      const int pb = it & 1;  // P^T / dS^T buffer; last read by the gradient MMAs of block it - 2
+      if (!tc::mbar_wait(&bars->p_empty[pb], ((it >> 1) & 1) ^ 1, abort, p.status)) {
         ok = false;
         break;
       }
-      store_half_row(smem + L::P_OFF, row, half, pv);
-      store_half_row(smem + L::DS_OFF, row, half, dsv);
+      store_half_row(smem + L::P_OFF + pb * L::PT, row, half, pv);
+      store_half_row(smem + L::DS_OFF + pb * L::PT, row, half, dsv);
       tc::fence_proxy_async_smem();
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->p_full);
+      if (lane == 0) tc::mbar_arrive(&bars->p_full[pb]);
     }
     // Epilogue: dV and dK rows (transpose of RoPE on dK) staged transposed in the now idle stage
     // buffers, then stored as dQKV^T columns with coalesced 16-byte stores.
