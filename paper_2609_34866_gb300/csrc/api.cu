@@ -251,7 +251,8 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   float* cos_t = reinterpret_cast<float*>(w + wp.rope);
   float* sin_t = cos_t + (int64_t)T * (dh / 2);
   JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
-  JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, wp.ldt, dm, st));
+  if (!use_tc_path())  // the tcgen05 weight-gradient GEMM reads X as stored
+    JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, wp.ldt, dm, st));
   JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_dev, D, dm, G, bits, w + wp.w16, nullptr, nullptr, status,
                           sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
@@ -275,9 +276,8 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   const float coef = (float)(k * 2.0 / n_el);
   JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
   if (use_tc_path())
-    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, w + wp.xt, wp.ldt, W_dev, scales_dev,
-                                                 N, D, dm, G, bits, coef, grad_scales_dev, status,
-                                                 st));
+    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, wp.ldt, X_dev, W_dev, scales_dev, N, D,
+                                                 dm, G, bits, coef, grad_scales_dev, status, st));
   else
     JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_simple(w + wp.dqkvt, w + wp.xt, wp.ldt, W_dev,
                                                      scales_dev, N, D, dm, G, bits, coef,

@@ -1,6 +1,7 @@
 // Tensor-core (tcgen05) GEMMs of the L_JAB path on sm_103a.
 //
-//   C[m, n] = sum_k A[m, k] B[n, k]        A, B K-major 16-bit, fp32 accumulation in TMEM
+//   C[m, n] = sum_k A[m, k] B[n, k]        A K-major 16-bit, fp32 accumulation in TMEM; B K-major
+//                                          (stored [n][k]) or MN-major (stored [k][n])
 //
 // Persistent, warp-specialised kernel, one CTA per SM:
 //   warp 0      TMA producer: 128x64 A tile and 256x64 B tile per stage, 4-stage mbarrier ring
@@ -12,7 +13,9 @@
 //   projection  [Q|K|V] = X w_hat^T: rotate-half RoPE on the Q and K heads (partner column +-d_h/2
 //               lives in the same thread's row), fp16 store.
 //   wgrad       G = dQKV^T X (K = tokens, split-K): ds[o, g] += coef * sum_{i in g} G[o,i] r[o,i]
-//               with the LSQ factor r of Eq. 13 recomputed from w and s; G is never stored.
+//               with the LSQ factor r of Eq. 13 recomputed from w and s; G is never stored. X is
+//               read as it is stored, [tokens, features], as the MN-major B operand (four 64-feature
+//               TMA boxes per stage), so no transposed copy of X is needed.
 #include <cudaTypedefs.h>
 
 #include "path.h"
@@ -181,7 +184,7 @@ __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int
   if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
 }
 
-template <int EPI, bool BF16>
+template <int EPI, bool BF16, bool B_MN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmParams p) {
@@ -231,7 +234,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           uint8_t* sa = smem + stage * STAGE_BYTES;
           tc::mbar_expect_tx(&bars->full[stage], STAGE_BYTES);
           tc::tma_load_2d(sa, &tmA, &bars->full[stage], kb * BK, mb * BM);
-          tc::tma_load_2d(sa + A_BYTES, &tmB, &bars->full[stage], kb * BK, nb * BN);
+          if (B_MN)  // B stored [k][n]: four boxes of BK rows x 64 columns
+            for (int c = 0; c < BN / 64; ++c)
+              tc::tma_load_2d(sa + A_BYTES + c * (BK * 128), &tmB, &bars->full[stage],
+                              nb * BN + c * 64, kb * BK);
+          else
+            tc::tma_load_2d(sa + A_BYTES, &tmB, &bars->full[stage], kb * BK, nb * BN);
           issued |= 1u << stage;
           last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -246,7 +254,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {  // ---------------- UMMA issuer
-      constexpr uint32_t IDESC = tc::idesc_f16(BF16, BM, BN);
+      constexpr uint32_t IDESC = tc::idesc_f16(BF16, BM, BN) | (B_MN ? (1u << 16) : 0u);
       int stage = 0, it = 0;
       uint32_t phase = 0;
       for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x, ++it) {
@@ -270,7 +278,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc::umma_f16(d_tmem, tc::sdesc_kmajor_sw128(a0 + k * 32),
-                         tc::sdesc_kmajor_sw128(b0 + k * 32), IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+                         B_MN ? tc::sdesc_mnmajor_sw128(b0 + k * 16 * 128, BK * 128, 1024)
+                              : tc::sdesc_kmajor_sw128(b0 + k * 32),
+                         IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
@@ -351,19 +361,19 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
-template <int EPI, bool BF16>
+template <int EPI, bool BF16, bool B_MN>
 cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmParams& p,
                         cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI, BF16>,
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI, BF16, B_MN>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   const int total = p.num_m * p.num_n * p.splits;
   const int grid = std::min(total, sm_count());
-  gemm_tc_kernel<EPI, BF16><<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, p);
+  gemm_tc_kernel<EPI, BF16, B_MN><<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, p);
   return cudaGetLastError();
 }
 
@@ -392,14 +402,14 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
   p.T = T;
   p.cos_t = cos_t;
   p.sin_t = sin_t;
-  return launch_gemm<kEpiRope, false>(ta, tb, p, st);
+  return launch_gemm<kEpiRope, false, false>(ta, tb, p, st);
 }
 
-cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
+cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st) {
   CUtensorMap ta, tb;
-  if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, xt, true, N, d, ldt, BN))
+  if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, x, true, d, N, d, BK))
     return cudaErrorInvalidValue;
   GemmParams p{};
   p.M = D;
@@ -422,7 +432,7 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, 
   p.bits = bits;
   p.coef = coef;
   p.ds = ds;
-  return launch_gemm<kEpiLsq, true>(ta, tb, p, st);
+  return launch_gemm<kEpiLsq, true, true>(ta, tb, p, st);
 }
 
 }  // namespace jab

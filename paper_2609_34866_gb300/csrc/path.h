@@ -23,7 +23,8 @@ inline bool use_tc_path() {
 cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
                                 int D, int n_rot, int dh, int T, const float* cos_t,
                                 const float* sin_t, int* status, cudaStream_t st);
-cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
+// x: bf16 [N, d] as the caller stores it (no transposed copy)
+cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st);
 // attn_tc.cu
