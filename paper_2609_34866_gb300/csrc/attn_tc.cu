@@ -418,30 +418,32 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 //   S_j = Q K_j^T     A = Q (TMEM, copied from the TMA-loaded smem tile by tcgen05.cp), B = K_j
 //   O  += P_j V_j     A = P_j (TMEM, fp16 pairs written by the softmax threads), B = V_j (smem,
 //                     MN-major)
-// TMEM columns: S double-buffered at 0 / 128, O at 256 (DH columns), Q (DH / 2 columns) and P
-// (64 columns) after it. S_{j+2} is issued as soon as the softmax has read S_j out of its buffer, so
-// the tensor pipe computes the next scores while the softmax of block j runs.
-//   warp 0      TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages)
-//   warp 1      TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
-//   warps 2..9  softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
-//               16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
-//               thread), so row maxima and sums need only warp shuffles. Lazy rescaling as in the
-//               single-head kernel. Epilogue (32x32b shape, one row per thread, half of its
-//               columns): O is staged through shared memory so that A_ref loads and dO / A stores are
-//               coalesced.
-//   warp 10     TMA: V ring (2 stages), so that K loads never queue behind a V stage that is busy.
+// TMEM columns: S at 0 (128 columns; the softmax reads a block out at once, after which S_{j+1}
+// may overwrite it), O double-buffered by tile parity at 128 / 128 + DH, Q (DH / 2 columns) and P
+// (64 columns) after them. With two O buffers the epilogue of tile i runs on its own warps while the
+// softmax warps already work on tile i + 1.
+//   warp 0       TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages)
+//   warp 1       TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
+//   warps 2..9   softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
+//                16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
+//                thread), so row maxima and sums need only warp shuffles. Lazy rescaling as in the
+//                single-head kernel. At the end of a tile the row statistics go to shared memory.
+//   warp 10      TMA: V ring (2 stages), so that K loads never queue behind a V stage that is busy
+//   warps 11..14 epilogue, one TMEM lane quarter each (32x32b shape, one row per thread, 32 columns
+//                at a time): O is staged through shared memory so that A_ref loads and dO / A
+//                stores are coalesced; per-mode outputs and the SSE partials.
 constexpr int SQ = 64, SKB = 128, SK_ST = 2, SV_ST = 2;
-constexpr int PAIR_THREADS = 352;
+constexpr int PAIR_THREADS = 480;
+constexpr int EPI_WARPS = 4, EPI_WARP0 = 11;
 
 struct StackBars {
   uint64_t q_full, q_empty, k_full[SK_ST], k_empty[SK_ST], v_full[SV_ST], v_empty[SV_ST];
-  uint64_t s_full[2], s_empty[2], p_full, pv_done, o_full, o_empty, drain;
+  uint64_t s_full, s_empty, p_full, pv_done, o_full[2], o_empty[2], st_full[2], st_empty[2];
+  uint64_t drain;
   uint32_t tmem_base;
   int abort;
-  double red[2][EW_WARPS];  // [tile parity][softmax warp]
-  float row_m[128], row_l[128];  // per stacked row: final running max (log2 units) and sum
-  float xv[2][2][128];           // [sequence parity][half][row]: values exchanged between halves
-  int flag[2][128];              // [half][row]: sequence number of the last value posted
+  double red[2][EPI_WARPS];         // [tile parity][epilogue warp]
+  float row_m[2][128], row_l[2][128];  // [tile parity][stacked row]: running max (log2), sum
 };
 
 template <int DH>
@@ -451,12 +453,12 @@ struct StackLayout {
   static constexpr int Q_OFF = 0;
   static constexpr int K_OFF = Q_OFF + TILE;
   static constexpr int V_OFF = K_OFF + SK_ST * TILE;
-  static constexpr int EPI_OFF = V_OFF + SV_ST * TILE;  // per softmax warp: 32 x 32 fp32
-  static constexpr int BAR_OFF = EPI_OFF + EW_WARPS * 4096;
+  static constexpr int EPI_OFF = V_OFF + SV_ST * TILE;  // per epilogue warp: 32 x 32 fp32
+  static constexpr int BAR_OFF = EPI_OFF + EPI_WARPS * 4096;
   static constexpr int USED = BAR_OFF + (int)sizeof(StackBars) + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
-  static constexpr uint32_t S_COL = 0, O_COL = 2 * SKB, Q_COL = 2 * SKB + DH,
-                            P_COL = 2 * SKB + DH + DH / 2;
+  static constexpr uint32_t S_COL = 0, O_COL = SKB, Q_COL = SKB + 2 * DH,
+                            P_COL = SKB + 2 * DH + DH / 2;
   static_assert(P_COL + SKB / 2 <= 512, "TMEM budget");
 };
 
@@ -473,33 +475,6 @@ __device__ __forceinline__ StackTile stack_tile(int k, int pairs, int BC, int nq
   t.qb = nqb - 1 - k / (pairs * BC);
   t.nkb = (min((t.qb + 1) * SQ, T) + SKB - 1) / SKB;
   return t;
-}
-
-// Exchange one float with the thread that owns the other half of the same row. `seq` counts this
-// thread's exchanges; values alternate between two slots, which is enough because neither side can
-// post twice without reading the other's post in between. The wait is time-bounded.
-__device__ __forceinline__ float half_exchange(StackBars* bars, int half, int row, int& seq, float v,
-                                               volatile int* abort, int* status) {
-  ++seq;
-  bars->xv[seq & 1][half][row] = v;
-  __threadfence_block();
-  reinterpret_cast<volatile int*>(&bars->flag[half][row])[0] = seq;
-  volatile int* f = &bars->flag[half ^ 1][row];
-  if (*f < seq) {
-    const uint64_t t0 = tc::globaltimer();
-    for (uint32_t it = 0; *f < seq; ++it) {
-      if ((it & 63u) == 0) {
-        if (*abort) break;
-        if (tc::globaltimer() - t0 > tc::kWaitLimitNs) {
-          *abort = 1;
-          report(status, JAB_ERR_TIMEOUT);
-          break;
-        }
-      }
-    }
-  }
-  __threadfence_block();
-  return reinterpret_cast<volatile float*>(&bars->xv[seq & 1][half ^ 1][row])[0];
 }
 
 __device__ __forceinline__ uint32_t pack_half2(float a, float b) {
@@ -534,21 +509,22 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       tc::mbar_init(&bars->v_full[i], 1);
       tc::mbar_init(&bars->v_empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(&bars->s_full[i], 1);
-      tc::mbar_init(&bars->s_empty[i], EW_WARPS);
-    }
+    tc::mbar_init(&bars->s_full, 1);
+    tc::mbar_init(&bars->s_empty, EW_WARPS);
     tc::mbar_init(&bars->p_full, EW_WARPS);
     tc::mbar_init(&bars->pv_done, 1);
-    tc::mbar_init(&bars->o_full, 1);
-    tc::mbar_init(&bars->o_empty, EW_WARPS);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&bars->o_full[i], 1);
+      tc::mbar_init(&bars->o_empty[i], EPI_WARPS);
+      tc::mbar_init(&bars->st_full[i], EW_WARPS);
+      tc::mbar_init(&bars->st_empty[i], EPI_WARPS);
+    }
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_q);
     tc::prefetch_tmap(&tm_kv);
   }
-  for (int i = threadIdx.x; i < 2 * 128; i += blockDim.x) (&bars->flag[0][0])[i] = 0;
   if (warp == 1) {
     tc::tmem_alloc(&bars->tmem_base, 512);
     tc::tmem_relinquish();
@@ -615,33 +591,36 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       constexpr uint32_t ID_PV = tc::idesc_f16(false, 128, DH) | (1u << 16);  // B = V, MN-major
       int g0 = 0, tc_ = 0;
       bool ok = true;
-      // S of global block gg into buffer gg & 1, once the softmax has read S_{gg-2} out of it.
+      // S of global block gg, once the softmax has read S_{gg-1} out of tensor memory.
       auto issue_s = [&](int gg) -> bool {
-        const int ks = gg % SK_ST, sb = gg & 1;
+        const int ks = gg % SK_ST;
         if (!tc::mbar_wait(&bars->k_full[ks], (gg / SK_ST) & 1, abort, p.status)) return false;
-        if (!tc::mbar_wait(&bars->s_empty[sb], ((gg >> 1) & 1) ^ 1, abort, p.status)) return false;
+        if (!tc::mbar_wait(&bars->s_empty, (gg & 1) ^ 1, abort, p.status)) return false;
         tc::fence_after_sync();
         const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + ks * L::TILE);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk)
-          tc::umma_f16_ts(tmem + L::S_COL + sb * SKB, tmem + L::Q_COL + kk * 8,
+          tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + kk * 8,
                           tc::sdesc_kmajor_sw128(k_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32),
                           ID_S, kk > 0 ? 1u : 0u);
-        tc::umma_commit(&bars->s_full[sb]);
+        tc::umma_commit(&bars->s_full);
         tc::umma_commit(&bars->k_empty[ks]);
         return true;
       };
+      // P V of global block gg into the O buffer of tile tc_; the tile's first one waits until the
+      // epilogue has read that buffer's previous tile out.
       auto issue_pv = [&](int gg, bool first) -> bool {
-        const int vs = gg % SV_ST;
+        const int vs = gg % SV_ST, ob = tc_ & 1;
         if (!tc::mbar_wait(&bars->v_full[vs], (gg / SV_ST) & 1, abort, p.status)) return false;
         if (!tc::mbar_wait(&bars->p_full, gg & 1, abort, p.status)) return false;
-        if (first && tc_ > 0 && !tc::mbar_wait(&bars->o_empty, (tc_ - 1) & 1, abort, p.status))
+        if (first && tc_ >= 2 &&
+            !tc::mbar_wait(&bars->o_empty[ob], ((tc_ >> 1) - 1) & 1, abort, p.status))
           return false;
         tc::fence_after_sync();
         const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + vs * L::TILE);
 #pragma unroll
         for (int k = 0; k < SKB / 16; ++k)
-          tc::umma_f16_ts(tmem + L::O_COL, tmem + L::P_COL + k * 8,
+          tc::umma_f16_ts(tmem + L::O_COL + ob * DH, tmem + L::P_COL + k * 8,
                           tc::sdesc_mnmajor_sw128(v_base + k * 16 * 128, L::CHUNK, 1024), ID_PV,
                           (!first || k > 0) ? 1u : 0u);
         tc::umma_commit(&bars->pv_done);
@@ -652,9 +631,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
            k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
         const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
         // Q of this tile into TMEM once the previous tile's last S (which read the old Q) is done.
-        if (g0 > 0 &&
-            !tc::mbar_wait(&bars->s_full[(g0 - 1) & 1], ((g0 - 1) >> 1) & 1, abort, p.status))
-          break;
+        if (g0 > 0 && !tc::mbar_wait(&bars->s_full, (g0 - 1) & 1, abort, p.status)) break;
         if (!tc::mbar_wait(&bars->q_full, tc_ & 1, abort, p.status)) break;
         tc::fence_after_sync();
         {
@@ -665,44 +642,38 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
                                  tc::sdesc_kmajor_sw128(q_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
           tc::umma_commit(&bars->q_empty);
         }
-        // S runs two blocks ahead of P V.
-        ok = issue_s(g0) && (tl.nkb < 2 || issue_s(g0 + 1));
+        // S runs one block ahead of P V.
+        ok = issue_s(g0);
         for (int j = 0; ok && j < tl.nkb; ++j) {
-          if (j + 2 < tl.nkb && !issue_s(g0 + j + 2)) { ok = false; break; }
+          if (j + 1 < tl.nkb && !issue_s(g0 + j + 1)) { ok = false; break; }
           if (!issue_pv(g0 + j, j == 0)) { ok = false; break; }
         }
         if (!ok) break;
-        tc::umma_commit(&bars->o_full);
+        tc::umma_commit(&bars->o_full[tc_ & 1]);
         g0 += tl.nkb;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else {  // ------------------------------------------------------------------------ softmax
+  } else if (warp < EPI_WARP0) {  // ------------------------------------------------------ softmax
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
     const int cq = lane & 3;                                   // column pair within each 8 columns
     const int rA = quarter * 32 + half * 16 + (lane >> 2);     // stacked rows of this thread
     const int rB = rA + 8;
     const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
-    // epilogue layout (32x32b): one row per thread, half of its columns
-    const int row = quarter * 32 + lane;
-    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    float* stg = reinterpret_cast<float*>(smem + L::EPI_OFF + (warp - 2) * 4096);
-    int g = 0, tc_ = 0, seq = 0;
+    int g = 0, tc_ = 0;
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
       const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
-      const int b = tl.bc % p.B, c = tl.bc / p.B;
       const int q0 = tl.qb * SQ;
       const int tA = q0 + (rA & 63), tB = q0 + (rB & 63);
-      const int row0 = b * p.T;
+      const uint32_t o_col = L::O_COL + (tc_ & 1) * DH;
       float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
       bool ok = true;
       for (int j = 0; j < tl.nkb; ++j, ++g) {
-        const int sb = g & 1;
-        if (!tc::mbar_wait(&bars->s_full[sb], (g >> 1) & 1, abort, p.status)) {
+        if (!tc::mbar_wait(&bars->s_full, g & 1, abort, p.status)) {
           ok = false;
           break;
         }
@@ -713,8 +684,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         {
           uint32_t r0[32], r1[32];
           __syncwarp();
-          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + sb * SKB, r0);
-          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + sb * SKB + 64, r1);
+          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL, r0);
+          tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + 64, r1);
           tc::tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
@@ -724,7 +695,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         }
         tc::fence_before_sync();
         __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->s_empty[sb]);  // S_{g+2} may overwrite the buffer
+        if (lane == 0) tc::mbar_arrive(&bars->s_empty);  // S_{g+1} may overwrite the columns
         const int k0 = j * SKB + 2 * cq;
         if (j * SKB + SKB - 1 > q0 || j * SKB + SKB > p.T) {  // diagonal or ragged block: mask
 #pragma unroll
@@ -793,7 +764,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
 #pragma unroll 1
           for (int ch = 0; ch < DH / 64; ++ch) {
             uint32_t r[32];
-            const uint32_t col = L::O_COL + ch * 64;
+            const uint32_t col = o_col + ch * 64;
             __syncwarp();
             tc::tmem_ld_16x256b_x8(tmem + lane16 + col, r);
             tc::tmem_ld_wait();
@@ -814,59 +785,85 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->p_full);
       }
-      // row statistics for the epilogue, which uses one thread per row
+      // Row statistics for the epilogue warps (the buffer of this tile parity was last read by the
+      // epilogue of tile tc_ - 2).
       lA += __shfl_xor_sync(0xffffffffu, lA, 1);
       lB += __shfl_xor_sync(0xffffffffu, lB, 1);
       lA += __shfl_xor_sync(0xffffffffu, lA, 2);
       lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+      const int sbf = tc_ & 1;
+      if (!ok || (tc_ >= 2 &&
+                  !tc::mbar_wait(&bars->st_empty[sbf], ((tc_ >> 1) - 1) & 1, abort, p.status)))
+        break;
       if (cq == 0) {
-        bars->row_m[rA] = mA;
-        bars->row_l[rA] = lA;
-        bars->row_m[rB] = mB;
-        bars->row_l[rB] = lB;
+        bars->row_m[sbf][rA] = mA;
+        bars->row_l[sbf][rA] = lA;
+        bars->row_m[sbf][rB] = mB;
+        bars->row_l[sbf][rB] = lB;
       }
-      // ------------------------------------------------------------------ epilogue
-      // Coalesced pass: the warp's 32 rows x 32 columns of O go through shared memory; lane l then
-      // handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte row segment. The
-      // A_ref loads of every chunk are issued first so that their latency overlaps the wait for O.
-      // In mode 2 the fp16-rounded error goes back through the same slots to the row's owner,
-      // which accumulates D = rowsum(dO * O).
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->st_full[sbf]);
+    }
+  } else if (warp < EPI_WARP0 + EPI_WARPS) {  // ------------------------------------- epilogue
+    // Coalesced pass: the warp's 32 rows x 32 columns of O go through shared memory; lane l then
+    // handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte row segment. In mode 2
+    // the fp16-rounded error goes back through the same slots to the row's owner, which accumulates
+    // D = rowsum(dO * O).
+    const int quarter = warp & 3;
+    const int ew = warp - EPI_WARP0;
+    const int row = quarter * 32 + lane;  // stacked row = TMEM lane
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    float* stg = reinterpret_cast<float*>(smem + L::EPI_OFF + ew * 4096);
+    const int rbase = quarter * 32;
+    const int c4 = lane & 7;
+    int tc_ = 0;
+    for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
+         k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
+      if (*abort) break;
+      const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
+      const int b = tl.bc % p.B, c = tl.bc / p.B;
       const int h = 2 * tl.hp + (row >> 6);
+      const int q0 = tl.qb * SQ;
       const int t = q0 + (row & 63);
-      const int rbase = quarter * 32;  // first stacked row of this warp
-      const int c4 = lane & 7;
-      float4 av[DH / 64][8];
-      if (MODE != 0 && ok) {
-#pragma unroll
-        for (int ch = 0; ch < DH / 64; ++ch)
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & 63);
-            if (tt < p.T)
-              av[ch][i] = __ldg(reinterpret_cast<const float4*>(
-                  p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + h * DH + half * (DH / 2) +
-                  ch * 32 + c4 * 4));
-          }
-      }
-      tc::named_bar_sync(1, EW_WARPS * 32);  // row statistics written
+      const int row0 = b * p.T;
+      const int ob = tc_ & 1;
+      const uint32_t ph = (tc_ >> 1) & 1;
       double acc = 0.0;
-      const bool have = ok && tc::mbar_wait(&bars->o_full, tc_ & 1, abort, p.status);
-      const float m = bars->row_m[row], lt = bars->row_l[row];
+      const bool have = tc::mbar_wait(&bars->st_full[ob], ph, abort, p.status) &&
+                        tc::mbar_wait(&bars->o_full[ob], ph, abort, p.status);
       if (have) {
+        const float m = bars->row_m[ob][row], lt = bars->row_l[ob][row];
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->st_empty[ob]);
         tc::fence_after_sync();
         const float inv_l = __fdiv_rn(1.f, lt);
         float sq = 0.f, dsum = 0.f;
+#pragma unroll 1
+        for (int ch = 0; ch < DH / 32; ++ch) {
+          const int col = h * DH + ch * 32 + c4 * 4;
+          float4 av[8];
+          if (MODE != 0) {
 #pragma unroll
-        for (int ch = 0; ch < DH / 64; ++ch) {
-          const int col = h * DH + half * (DH / 2) + ch * 32 + c4 * 4;
+            for (int i = 0; i < 8; ++i) {
+              const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & 63);
+              if (tt < p.T)
+                av[i] = __ldg(reinterpret_cast<const float4*>(
+                    p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col));
+            }
+          }
           float o[32];
           {
             uint32_t r[32];
             __syncwarp();
-            tc::tmem_ld32(tmem + lane_base + L::O_COL + half * (DH / 2) + ch * 32, r);
+            tc::tmem_ld32(tmem + lane_base + L::O_COL + ob * DH + ch * 32, r);
             tc::tmem_ld_wait();
 #pragma unroll
             for (int i = 0; i < 32; ++i) o[i] = __fmul_rn(__uint_as_float(r[i]), inv_l);
+          }
+          if (ch == DH / 32 - 1) {  // O of this buffer is read out: the next-but-one tile may use it
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bars->o_empty[ob]);
           }
 #pragma unroll
           for (int v = 0; v < 8; ++v)
@@ -885,7 +882,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
               *reinterpret_cast<float4*>(p.a_out + off) = ov;
               sq += ov.x * ov.x + ov.y * ov.y + ov.z * ov.z + ov.w * ov.w;
             } else {
-              const float4 a = av[ch][i];
+              const float4 a = av[i];
               const float e0 = __fsub_rn(ov.x, a.x), e1 = __fsub_rn(ov.y, a.y);
               const float e2 = __fsub_rn(ov.z, a.z), e3 = __fsub_rn(ov.w, a.w);
               sq += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
@@ -910,12 +907,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             __syncwarp();
           }
         }
-        // O is no longer needed: the next tile's first P V may overwrite it.
-        tc::fence_before_sync();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->o_empty);
-        if (MODE == 2) dsum += half_exchange(bars, half, row, seq, dsum, abort, p.status);
-        if (half == 0 && t < p.T) {
+        if (t < p.T) {
           const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + t;
           if (MODE != 1 && p.lse != nullptr)
             p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
@@ -925,17 +917,15 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       }
       acc = warp_sum(acc);
       double* red = bars->red[tc_ & 1];  // alternate by tile
-      if (lane == 0) red[warp - 2] = acc;
-      // every softmax warp reaches this once per tile; it also keeps row_m / row_l of this tile
-      // until all warps have read them
-      tc::named_bar_sync(1, EW_WARPS * 32);
-      if (lane == 0 && half == 0 && (quarter & 1) == 0 && have) {
-        // the head's rows are lane quarters 2 hd and 2 hd + 1 (hd = row >> 6), each over two warps
-        const int wq0 = (2 * (row >> 6) + 2) & 3;  // warp index - 2 of that quarter, half 0
-        const double v = red[wq0] + red[(wq0 + 1) & 3] + red[wq0 + 4] + red[((wq0 + 1) & 3) + 4];
+      if (lane == 0) red[ew] = acc;
+      tc::named_bar_sync(2, EPI_WARPS * 32);  // every epilogue warp reaches this once per tile
+      if (lane == 0 && (quarter & 1) == 0 && have) {
+        // head hd = row >> 6 has lane quarters 2 hd and 2 hd + 1; quarter q is epilogue warp (q + 1) & 3
+        const int hd = row >> 6;
+        const double v = red[(2 * hd + 1) & 3] + red[(2 * hd + 2) & 3];
         p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] = v;
       }
-      if (!ok || !have) break;
+      if (!have) break;
     }
   }
   tc::fence_before_sync();
