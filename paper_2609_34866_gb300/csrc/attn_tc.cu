@@ -422,7 +422,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // may overwrite it), O double-buffered by tile parity at 128 / 128 + DH, Q (DH / 2 columns) and P
 // (64 columns) after them. With two O buffers the epilogue of tile i runs on its own warps while the
 // softmax warps already work on tile i + 1.
-//   warp 0       TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (2 stages)
+//   warp 0       TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (3 stages: a K
+//                load is issued once S two blocks back has completed and must land before S of
+//                the block after next)
 //   warp 1       TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
 //   warps 2..9   softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
 //                16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
@@ -432,7 +434,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 //   warps 11..14 epilogue, one TMEM lane quarter each (32x32b shape, one row per thread, 32 columns
 //                at a time): O is staged through shared memory so that A_ref loads and dO / A
 //                stores are coalesced; per-mode outputs and the SSE partials.
-constexpr int SQ = 64, SKB = 128, SK_ST = 2, SV_ST = 2;
+constexpr int SQ = 64, SKB = 128, SK_ST = 3, SV_ST = 2;
 constexpr int PAIR_THREADS = 480;
 constexpr int EPI_WARPS = 4, EPI_WARP0 = 11;
 
@@ -543,8 +545,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       uint64_t* full = is_v ? bars->v_full : bars->k_full;
       uint64_t* empty = is_v ? bars->v_empty : bars->k_empty;
       uint8_t* ring = smem + (is_v ? L::V_OFF : L::K_OFF);
-      constexpr int NST = SK_ST;
-      static_assert(SK_ST == SV_ST, "one ring depth for K and V");
+      const int NST = is_v ? SV_ST : SK_ST;
       for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
            k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
         const StackTile tl = stack_tile(k, pairs, BC, nqb, p.T);
