@@ -48,6 +48,10 @@ SMALL_CASES = {
                           shape=BlockShape(512, 4, 2, 128, True, 10000.0)), 1, 257, 64),
     "dh64_gqa4_T65": (replace(WORKLOADS["gpt2_smoke"],
                               shape=BlockShape(256, 4, 1, 64, True, 500.0)), 2, 65, 128),
+    # 512 forward tiles and 512 dQ tiles: several per persistent CTA on a 152-SM GPU (tile
+    # boundaries, both O buffers, the epilogue hand-off), at a cost the oracle still finishes fast
+    "dh64_gqa4_B64_T256": (replace(WORKLOADS["gpt2_smoke"],
+                                   shape=BlockShape(256, 4, 1, 64, True, 500.0)), 64, 256, 128),
     "gpt2_T1": (WORKLOADS["gpt2_smoke"], 3, 1, 128),
 }
 

@@ -85,7 +85,7 @@ def test_teacher_output_parity(name):
 
 # ------------------------------------------------------------------ forward loss over candidates
 @pytest.mark.parametrize("name", ["gpt2_T200", "mistral_T130", "gqa2_T257", "dh64_gqa4_T65",
-                                  "gpt2_T1"])
+                                  "dh64_gqa4_B64_T256", "gpt2_T1"])
 def test_loss_forward_parity(name):
     c = case(name)
     ws = c.workspace(n_cand=5)
@@ -107,7 +107,8 @@ def test_loss_forward_parity(name):
 # ------------------------------------------------------------------ STE / LSQ backward
 @pytest.mark.parametrize("name,bits", [("gpt2_T200", 3), ("mistral_T130", 3),
                                        ("mistral_G64_T70", 2), ("gqa2_T257", 3),
-                                       ("dh64_gqa4_T65", 4), ("gpt2_T1", 3)])
+                                       ("dh64_gqa4_T65", 4), ("dh64_gqa4_B64_T256", 3),
+                                       ("gpt2_T1", 3)])
 def test_backward_parity(name, bits):
     c = case(name)
     ws = c.workspace()
