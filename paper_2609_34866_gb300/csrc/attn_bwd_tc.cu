@@ -7,13 +7,14 @@
 //   dV = P^T dO,  dK = scale * dS^T Q,  dQ = scale * dS K        (summed over the GQA group for K, V)
 // Two kernels, no atomics:
 //   dkdv  one CTA per (128-key block, KV head, sequence); loops over the query heads of the group and
-//         over 64-query blocks: S^T = K Q^T, dP^T = V dO^T into double-buffered TMEM, P^T and dS^T
-//         rows (fp16) to shared memory, dV += P^T dO and dK += dS^T Q accumulated in TMEM.
+//         over 128-query blocks: S^T = K Q^T, dP^T = V dO^T into TMEM, P^T and dS^T (fp16) written
+//         back over them, dV += P^T dO and dK += dS^T Q (A operands in TMEM) accumulated in TMEM.
 //   dq    one CTA per (128 query rows, query head, sequence); loops over 64-key blocks: S = Q K^T,
 //         dP = dO V^T, dS (fp16) to shared memory, dQ += dS K in TMEM.
 // Warp roles: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..9 elementwise: two warps per
-// TMEM lane quarter, each thread owning one row and half of the columns of the S / dP tile. The epilogues apply the transpose of RoPE to dQ and dK and write dQKV^T (bf16, [D, ldt]),
-// the K-major operand of the weight-gradient GEMM.
+// TMEM lane quarter (dkdv: each warp 16 whole rows of S^T / dP^T; dq: each thread one row and half
+// of the columns of S / dP). The epilogues apply the transpose of RoPE to dQ and dK and write
+// dQKV^T (bf16, [D, ldt]), the K-major operand of the weight-gradient GEMM.
 #include <cudaTypedefs.h>
 
 #include "path.h"
@@ -44,21 +45,6 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   const uint64_t t0 = tc::globaltimer();
   while (!tc::mbar_test(bar, parity))
     if (tc::globaltimer() - t0 > tc::kWaitLimitNs) break;
-}
-
-// 32 fp16 values, half of one 128-byte row of a K-major, 128-byte-swizzled operand tile (16-byte
-// chunks 4*half .. 4*half+3), to shared memory.
-__device__ __forceinline__ void store_half_row(uint8_t* base, int row, int half,
-                                               const float (&v)[32]) {
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    uint4 u;
-    __half2* hp = reinterpret_cast<__half2*>(&u);
-#pragma unroll
-    for (int e = 0; e < 4; ++e) hp[e] = __floats2half2_rn(v[k * 8 + 2 * e], v[k * 8 + 2 * e + 1]);
-    const int c8 = half * 4 + k;
-    *reinterpret_cast<uint4*>(base + row * 128 + ((c8 ^ (row & 7)) << 4)) = u;
-  }
 }
 
 // Stages gradient rows of a TMEM accumulator (DH columns), times `mul`, optionally through the
@@ -138,52 +124,48 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
 
 // ================================================================================ dK, dV
 // One CTA per (128-key block, KV head, sequence); it loops over the query heads of the group and over
-// 64-query blocks. K and V live in tensor memory (copied once from shared memory by tcgen05.cp), so
-// S^T = K Q^T and dP^T = V dO^T are TS-form UMMAs that read only Q and dO from shared memory, and the
-// shared memory K and V would take holds a deeper Q / dO ring (4 stages: a stage is released only
-// when dV += P^T dO and dK += dS^T Q of its block have completed, so the ring has to cover a load
-// latency plus a block) and double-buffered P^T / dS^T tiles, so the elementwise warps of block j+1
-// do not wait for the gradient MMAs of block j.
-//   TMEM columns: S^T 0 and dP^T 64 (single-buffered: the elementwise warps read them out at once),
-//   dV 128, dK 128 + DH, K and V (DH / 2 each) after them.
+// 128-query blocks, so that every UMMA runs at N = 128 (an N = 64 UMMA costs the tensor pipe as much
+// time as an N = 128 one). Tensor memory: S^T = K Q^T at column 0 and dP^T = V dO^T at 128 (SS form:
+// K and V stay in shared memory for the whole tile), dV at 256, dK at 256 + DH. The elementwise warps
+// write P^T and dS^T back as packed fp16 over the first 64 columns of S^T and dP^T, where the TS-form
+// gradient UMMAs dV += P^T dO and dK += dS^T Q read them as their A operand. With no room for a second
+// S^T / dP^T buffer, the issuer orders the tensor pipe as
+//   dV(j), S^T(j+1), dK(j), dP^T(j+1), dV(j+1), ...
+// S^T(j+1) going out once dV(j) has completed (it overwrites the P^T(j) columns) and dP^T(j+1) once
+// dK(j) has; the elementwise warps compute P^T(j+1) while dK(j) and dP^T(j+1) run.
 template <int DH>
 struct DkdvLayout {
-  static constexpr int BK = 128, BQ = 64, STAGES = 4;
-  static constexpr int KCHUNK = BK * 128;  // 64 columns of a 128-row tile
-  static constexpr int QCHUNK = BQ * 128;  // 64 columns of a 64-row tile
-  static constexpr int ST_OFF = 0;
-  static constexpr int ST_Q = 0, ST_DO = BQ * DH * 2, ST_LSE = 2 * BQ * DH * 2,
+  static constexpr int BK = 128, BQ = 128, STAGES = 2;
+  static constexpr int PREFETCH = 2;  // blocks beyond the stage ring kept in flight to L2
+  static constexpr int CHUNK = 128 * 128;  // 64 columns of a 128-row fp16 tile
+  static constexpr int NCH = DH / 64;
+  static constexpr int K_OFF = 0, V_OFF = NCH * CHUNK;
+  static constexpr int ST_OFF = 2 * NCH * CHUNK;
+  static constexpr int ST_Q = 0, ST_DO = NCH * CHUNK, ST_LSE = 2 * NCH * CHUNK,
                        ST_D = ST_LSE + BQ * 4, ST_BYTES = ST_D + BQ * 4;
   static constexpr int ST_STRIDE = (ST_BYTES + 1023) / 1024 * 1024;
-  static constexpr int KV_TILE = BK * DH * 2;  // K or V, staged in the last two stage slots
-  static_assert(KV_TILE <= ST_STRIDE, "K / V tile fits a stage slot");
-  static constexpr int P_OFF = ST_OFF + STAGES * ST_STRIDE;
-  static constexpr int PT = BK * BQ * 2;  // one P^T or dS^T tile
-  static constexpr int DS_OFF = P_OFF + 2 * PT;
-  static constexpr int BAR_OFF = DS_OFF + 2 * PT;
+  static constexpr int BAR_OFF = ST_OFF + STAGES * ST_STRIDE;
   static constexpr int USED = BAR_OFF + 256 + 1024;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
-  static constexpr uint32_t S_COL = 0, DP_COL = 64, DV_COL = 128, DK_COL = 128 + DH,
-                            K_COL = 128 + 2 * DH, V_COL = 128 + 2 * DH + DH / 2;
-  static_assert(V_COL + DH / 2 <= 512, "TMEM budget");
+  static constexpr uint32_t S_COL = 0, DP_COL = 128, DV_COL = 256, DK_COL = 256 + DH;
+  static_assert(DK_COL + DH <= 512, "TMEM budget");
   static_assert(2 * DH * 128 * 2 <= STAGES * ST_STRIDE, "epilogue staging fits the stage ring");
+  static_assert(USED <= 227 * 1024, "shared memory budget");
 };
 
 struct DkdvBars {
-  uint64_t kv_full, kv_copied, ld_full[4], ld_empty[4], s_full, s_empty;
-  uint64_t p_full[2], p_empty[2], o_full, drain;
+  uint64_t kv_full, ld_full[2], ld_empty[2], s_full, dp_full, p_full, ds_full, dv_done, dk_done;
+  uint64_t o_full, drain;
   uint32_t tmem_base;
   int abort;
 };
 
 template <int DH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_kv,
-                            const __grid_constant__ CUtensorMap tm_q,
+    attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
                             const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
   using L = DkdvLayout<DH>;
   constexpr int BK = L::BK, BQ = L::BQ, STAGES = L::STAGES;
-  constexpr int KV_A = STAGES - 2, KV_B = STAGES - 1;  // stage slots that first hold K and V
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -194,30 +176,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int kb = blockIdx.z, g = blockIdx.x, b = blockIdx.y;  // key block slowest: longest first
   const int r = p.Hq / p.Hkv;
   const int nq = (p.T + BQ - 1) / BQ;
-  const int i0 = (kb * BK) / BQ;
-  const int per_head = nq - i0;
+  const int per_head = nq - kb;  // query blocks kb .. nq - 1 see keys of block kb
   const int n_it = r * per_head;
   const int row0 = b * p.T;
 
   if (threadIdx.x == 0) {
     tc::mbar_init(&bars->kv_full, 1);
-    tc::mbar_init(&bars->kv_copied, 1);
     for (int i = 0; i < STAGES; ++i) {
       tc::mbar_init(&bars->ld_full[i], 1);
       tc::mbar_init(&bars->ld_empty[i], 1);
     }
     tc::mbar_init(&bars->s_full, 1);
-    tc::mbar_init(&bars->s_empty, EW_WARPS);
-    for (int i = 0; i < 2; ++i) {
-      tc::mbar_init(&bars->p_full[i], EW_WARPS);
-      tc::mbar_init(&bars->p_empty[i], 1);
-    }
+    tc::mbar_init(&bars->dp_full, 1);
+    tc::mbar_init(&bars->p_full, EW_WARPS);
+    tc::mbar_init(&bars->ds_full, EW_WARPS);
+    tc::mbar_init(&bars->dv_done, 1);
+    tc::mbar_init(&bars->dk_done, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
     tc::fence_mbar_init();
-    tc::prefetch_tmap(&tm_kv);
-    tc::prefetch_tmap(&tm_q);
+    tc::prefetch_tmap(&tm_qkv);
     tc::prefetch_tmap(&tm_do);
   }
   if (warp == 1) {
@@ -232,27 +211,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {  // ------------------------------------------------------------- TMA
       uint32_t issued = 0, last_par = 0;
-      tc::mbar_expect_tx(&bars->kv_full, 2 * L::KV_TILE);
-      for (int ch = 0; ch < DH / 64; ++ch) {
-        tc::tma_load_2d(smem + L::ST_OFF + KV_A * L::ST_STRIDE + ch * L::KCHUNK, &tm_kv,
-                        &bars->kv_full, p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
-        tc::tma_load_2d(smem + L::ST_OFF + KV_B * L::ST_STRIDE + ch * L::KCHUNK, &tm_kv,
-                        &bars->kv_full, p.vcol0 + g * DH + ch * 64, row0 + kb * BK);
+      tc::mbar_expect_tx(&bars->kv_full, 2 * BK * DH * 2);
+      for (int ch = 0; ch < L::NCH; ++ch) {
+        tc::tma_load_2d(smem + L::K_OFF + ch * L::CHUNK, &tm_qkv, &bars->kv_full,
+                        p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
+        tc::tma_load_2d(smem + L::V_OFF + ch * L::CHUNK, &tm_qkv, &bars->kv_full,
+                        p.vcol0 + g * DH + ch * 64, row0 + kb * BK);
       }
-      bool ok = true;
-      for (int it = 0; ok && it < n_it; ++it) {
+      // The stage ring holds two blocks; blocks further ahead are prefetched into L2 so that a
+      // stage load, which can start only when dK of the block two back has completed, hits L2.
+      auto prefetch = [&](int j) {
+        const int hj = g * r + j / per_head, ij = kb + j % per_head;
+        for (int ch = 0; ch < L::NCH; ++ch) {
+          tc::tma_prefetch_2d(&tm_qkv, p.qcol0 + hj * DH + ch * 64, row0 + ij * BQ);
+          tc::tma_prefetch_2d(&tm_do, hj * DH + ch * 64, row0 + ij * BQ);
+        }
+        const int64_t lrow = ((int64_t)b * p.Hq + hj) * p.lse_pitch + ij * BQ;
+        tc::prefetch_l2(p.lse + lrow, BQ * 4);
+        tc::prefetch_l2(p.dvec + lrow, BQ * 4);
+      };
+      for (int j = STAGES; j < STAGES + L::PREFETCH - 1 && j < n_it; ++j) prefetch(j);
+      for (int it = 0; it < n_it; ++it) {
         const int st = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
-        const int h = g * r + it / per_head, i = i0 + it % per_head;
-        // The slots that held K and V are free once both have been copied into tensor memory.
-        if (it == KV_A && !tc::mbar_wait(&bars->kv_copied, 0, abort, p.status)) break;
+        const int h = g * r + it / per_head, i = kb + it % per_head;
+        if (it + STAGES + L::PREFETCH - 1 < n_it) prefetch(it + STAGES + L::PREFETCH - 1);
         if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
         uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
         tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
-        for (int ch = 0; ch < DH / 64; ++ch) {
-          tc::tma_load_2d(sbase + L::ST_Q + ch * L::QCHUNK, &tm_q, &bars->ld_full[st],
+        for (int ch = 0; ch < L::NCH; ++ch) {
+          tc::tma_load_2d(sbase + L::ST_Q + ch * L::CHUNK, &tm_qkv, &bars->ld_full[st],
                           p.qcol0 + h * DH + ch * 64, row0 + i * BQ);
-          tc::tma_load_2d(sbase + L::ST_DO + ch * L::QCHUNK, &tm_do, &bars->ld_full[st],
+          tc::tma_load_2d(sbase + L::ST_DO + ch * L::CHUNK, &tm_do, &bars->ld_full[st],
                           h * DH + ch * 64, row0 + i * BQ);
         }
         const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + i * BQ;
@@ -271,65 +261,70 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------------------------- UMMA
       constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
+      const uint32_t ka = tc::smem_u32(smem + L::K_OFF), va = tc::smem_u32(smem + L::V_OFF);
       bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
-      if (ok) {  // K and V into tensor memory (A operands of S^T and dP^T)
-        tc::fence_after_sync();
-        const uint32_t ka = tc::smem_u32(smem + L::ST_OFF + KV_A * L::ST_STRIDE);
-        const uint32_t va = tc::smem_u32(smem + L::ST_OFF + KV_B * L::ST_STRIDE);
-#pragma unroll
-        for (int k = 0; k < DH / 16; ++k) {
-          const uint32_t ko = (k >> 2) * L::KCHUNK + (k & 3) * 32;
-          tc::tmem_cp_128x256b(tmem + L::K_COL + k * 8, tc::sdesc_kmajor_sw128(ka + ko));
-          tc::tmem_cp_128x256b(tmem + L::V_COL + k * 8, tc::sdesc_kmajor_sw128(va + ko));
-        }
-        tc::umma_commit(&bars->kv_copied);
-      }
-      // Event-driven issue: S^T / dP^T of block ns go out as soon as its Q / dO stage has landed
-      // and the elementwise warps have read the previous S^T / dP^T out of tensor memory; the
-      // gradient MMAs of block ng as soon as its P^T and dS^T are in shared memory.
-      int ns = 0, ng = 0;
+      // Event-driven issue in the order dV(j), S^T(j+1), dK(j), dP^T(j+1): ns, nd, nv, nk count
+      // the S^T, dP^T, dV and dK UMMA groups issued so far.
+      int ns = 0, nd = 0, nv = 0, nk = 0;
       tc::Watchdog wd;
-      while (ok && ng < n_it) {
+      while (ok && nk < n_it) {
         bool prog = false;
-        if (ns < n_it && ns <= ng + 2) {
-          const int st = ns % STAGES;
-          if (tc::mbar_ready(&bars->ld_full[st], (ns / STAGES) & 1) &&
-              tc::mbar_ready(&bars->s_empty, (ns & 1) ^ 1)) {
-            tc::fence_after_sync();
-            const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
-#pragma unroll
-            for (int k = 0; k < DH / 16; ++k) {
-              const uint32_t qo = (k >> 2) * L::QCHUNK + (k & 3) * 32;
-              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::K_COL + k * 8,
-                              tc::sdesc_kmajor_sw128(sb + L::ST_Q + qo), ID_S, k > 0 ? 1u : 0u);
-              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::V_COL + k * 8,
-                              tc::sdesc_kmajor_sw128(sb + L::ST_DO + qo), ID_S, k > 0 ? 1u : 0u);
-            }
-            tc::umma_commit(&bars->s_full);
-            ++ns;
-            prog = true;
-          }
-        }
-        if (ng < ns && tc::mbar_ready(&bars->p_full[ng & 1], (ng >> 1) & 1)) {
+        // S^T(ns): its Q has landed and dV(ns - 1) has read P^T(ns - 1) out of the S^T columns.
+        if (ns < n_it && nv == ns && tc::mbar_ready(&bars->ld_full[ns % STAGES], (ns / STAGES) & 1) &&
+            (ns == 0 || tc::mbar_ready(&bars->dv_done, (ns - 1) & 1))) {
           tc::fence_after_sync();
-          const int st = ng % STAGES, pb = ng & 1;
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
-          const uint32_t p_base = tc::smem_u32(smem + L::P_OFF + pb * L::PT);
-          const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF + pb * L::PT);
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (ns % STAGES) * L::ST_STRIDE);
 #pragma unroll
-          for (int k = 0; k < BQ / 16; ++k) {
-            const uint32_t acc = (ng > 0 || k > 0) ? 1u : 0u;
-            tc::umma_f16(tmem + L::DV_COL, tc::sdesc_kmajor_sw128(p_base + k * 32),
-                         tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::QCHUNK, 1024),
-                         ID_G, acc);
-            tc::umma_f16(tmem + L::DK_COL, tc::sdesc_kmajor_sw128(ds_base + k * 32),
-                         tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::QCHUNK, 1024),
-                         ID_G, acc);
+          for (int k = 0; k < DH / 16; ++k) {
+            const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
+            tc::umma_f16(tmem + L::S_COL, tc::sdesc_kmajor_sw128(ka + o),
+                         tc::sdesc_kmajor_sw128(sb + L::ST_Q + o), ID_S, k > 0 ? 1u : 0u);
           }
-          tc::umma_commit(&bars->ld_empty[st]);
-          tc::umma_commit(&bars->p_empty[pb]);
-          if (ng == n_it - 1) tc::umma_commit(&bars->o_full);
-          ++ng;
+          tc::umma_commit(&bars->s_full);
+          ++ns;
+          prog = true;
+        }
+        // dP^T(nd): after S^T(nd) (same stage) and once dK(nd - 1) has read dS^T(nd - 1).
+        if (nd < ns && nk == nd && (nd == 0 || tc::mbar_ready(&bars->dk_done, (nd - 1) & 1))) {
+          tc::fence_after_sync();
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (nd % STAGES) * L::ST_STRIDE);
+#pragma unroll
+          for (int k = 0; k < DH / 16; ++k) {
+            const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
+            tc::umma_f16(tmem + L::DP_COL, tc::sdesc_kmajor_sw128(va + o),
+                         tc::sdesc_kmajor_sw128(sb + L::ST_DO + o), ID_S, k > 0 ? 1u : 0u);
+          }
+          tc::umma_commit(&bars->dp_full);
+          ++nd;
+          prog = true;
+        }
+        // dV(nv) += P^T(nv) dO(nv) once the elementwise warps have written P^T(nv).
+        if (nv < ns && tc::mbar_ready(&bars->p_full, nv & 1)) {
+          tc::fence_after_sync();
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (nv % STAGES) * L::ST_STRIDE);
+#pragma unroll
+          for (int k = 0; k < BQ / 16; ++k)
+            tc::umma_f16_ts(tmem + L::DV_COL, tmem + L::S_COL + k * 8,
+                            tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::CHUNK, 1024),
+                            ID_G, (nv > 0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&bars->dv_done);
+          ++nv;
+          prog = true;
+        }
+        // dK(nk) += dS^T(nk) Q(nk) once dS^T(nk) is written, behind S^T(nk + 1) in the pipe.
+        if (nk < nd && (ns > nk + 1 || ns == n_it) && tc::mbar_ready(&bars->ds_full, nk & 1)) {
+          tc::fence_after_sync();
+          const int st = nk % STAGES;
+          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+#pragma unroll
+          for (int k = 0; k < BQ / 16; ++k)
+            tc::umma_f16_ts(tmem + L::DK_COL, tmem + L::DP_COL + k * 8,
+                            tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::CHUNK, 1024),
+                            ID_G, (nk > 0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&bars->dk_done);
+          tc::umma_commit(&bars->ld_empty[st]);  // dV(nk) and dK(nk) were the stage's last readers
+          if (nk == n_it - 1) tc::umma_commit(&bars->o_full);
+          ++nk;
           prog = true;
         }
         if (prog)
@@ -340,69 +335,111 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else {  // ------------------------------------------------ elementwise: row = key, 32 queries
+  } else {  // ------------------------------------ elementwise: 16 key rows x 128 queries per warp
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
-    const int row = quarter * 32 + lane;
-    const int key = kb * BK + row;
-    const int col0 = half * 32;
-    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const int cq = lane & 3;
+    const int rA = quarter * 32 + half * 16 + (lane >> 2);  // key rows rA and rA + 8 of the block
+    const int keyA = kb * BK + rA, keyB = keyA + 8;
+    const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
     bool ok = true;
     for (int it = 0; it < n_it; ++it) {
       const int st = it % STAGES;
-      const int i = i0 + it % per_head;
-      if (!tc::mbar_wait(&bars->s_full, it & 1, abort, p.status) ||
-          !tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status)) {
+      const int i = kb + it % per_head;
+      const float* lse_s = reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_LSE);
+      const float* d_s = reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_D);
+      if (!tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status) ||
+          !tc::mbar_wait(&bars->s_full, it & 1, abort, p.status)) {
         ok = false;
         break;
       }
       tc::fence_after_sync();
-      uint32_t rs[32], rd[32];
-      __syncwarp();
-      tc::tmem_ld32(tmem + lane_base + L::S_COL + col0, rs);
-      tc::tmem_ld32(tmem + lane_base + L::DP_COL + col0, rd);
-      tc::tmem_ld_wait();
+      // x[hh][4n + e] (e < 2): row A, query column 64 hh + 8n + 2 cq + e; e = 2, 3: row B.
+      float x[2][32];
+      {
+        uint32_t r0[32], r1[32];
+        __syncwarp();
+        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL, r0);
+        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + 64, r1);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          x[0][c] = __uint_as_float(r0[c]);
+          x[1][c] = __uint_as_float(r1[c]);
+        }
+      }
+      const int qc0 = i * BQ + 2 * cq;  // query of x[0][0]
+      const bool full = i > kb && i * BQ + BQ <= p.T;
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+          const float2 l2 = *reinterpret_cast<const float2*>(lse_s + 64 * hh + 8 * n + 2 * cq);
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const float le = e ? l2.y : l2.x;
+            float pa = tc::fast_exp2(fmaf(x[hh][4 * n + e], p.sl2, -le));
+            float pb = tc::fast_exp2(fmaf(x[hh][4 * n + 2 + e], p.sl2, -le));
+            if (!full) {
+              const int q = qc0 + 64 * hh + 8 * n + e;
+              if (q >= p.T || q < keyA) pa = 0.f;
+              if (q >= p.T || q < keyB) pb = 0.f;
+            }
+            x[hh][4 * n + e] = pa;
+            x[hh][4 * n + 2 + e] = pb;
+          }
+        }
+      {
+        uint32_t pw[32];  // pw[2m] row A, pw[2m + 1] row B, packed column 4m + cq
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+          for (int n = 0; n < 8; ++n) {
+            pw[2 * (8 * hh + n)] = tc::pack_half2(x[hh][4 * n], x[hh][4 * n + 1]);
+            pw[2 * (8 * hh + n) + 1] = tc::pack_half2(x[hh][4 * n + 2], x[hh][4 * n + 3]);
+          }
+        __syncwarp();
+        tc::tmem_st_16x128b_x16(tmem + lane16 + L::S_COL, pw);
+        tc::tmem_st_wait();
+      }
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->s_empty);
-      const uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
-      float lse2[32], dd[32];  // per query column (the same for every key row: broadcast reads)
-#pragma unroll
-      for (int v = 0; v < 8; ++v) {
-        const float4 a = reinterpret_cast<const float4*>(sbase + L::ST_LSE)[col0 / 4 + v];
-        const float4 d = reinterpret_cast<const float4*>(sbase + L::ST_D)[col0 / 4 + v];
-        lse2[4 * v] = a.x, lse2[4 * v + 1] = a.y, lse2[4 * v + 2] = a.z, lse2[4 * v + 3] = a.w;
-        dd[4 * v] = d.x, dd[4 * v + 1] = d.y, dd[4 * v + 2] = d.z, dd[4 * v + 3] = d.w;
-      }
-      const int q0 = i * BQ + col0;
-      float pv[32], dsv[32];
-      if (q0 >= kb * BK + BK - 1 && q0 + 31 < p.T) {  // every (key, query) pair is visible
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          pv[c] = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2[c]));
-          dsv[c] = pv[c] * (__uint_as_float(rd[c]) - dd[c]);
-        }
-      } else {
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const int q = q0 + c;
-          const bool valid = q < p.T && q >= key;
-          const float e = tc::fast_exp2(fmaf(__uint_as_float(rs[c]), p.sl2, -lse2[c]));
-          pv[c] = valid ? e : 0.f;
-          dsv[c] = valid ? e * (__uint_as_float(rd[c]) - dd[c]) : 0.f;
-        }
-      }
-      const int pb = it & 1;  // P^T / dS^T buffer; last read by the gradient MMAs of block it - 2
-      if (!tc::mbar_wait(&bars->p_empty[pb], ((it >> 1) & 1) ^ 1, abort, p.status)) {
+      if (lane == 0) tc::mbar_arrive(&bars->p_full);
+      if (!tc::mbar_wait(&bars->dp_full, it & 1, abort, p.status)) {
         ok = false;
         break;
       }
-      store_half_row(smem + L::P_OFF + pb * L::PT, row, half, pv);
-      store_half_row(smem + L::DS_OFF + pb * L::PT, row, half, dsv);
-      tc::fence_proxy_async_smem();
+      tc::fence_after_sync();
+      uint32_t dw[32];
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        uint32_t rd[32];
+        __syncwarp();
+        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::DP_COL + 64 * hh, rd);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+          const float2 d2 = *reinterpret_cast<const float2*>(d_s + 64 * hh + 8 * n + 2 * cq);
+          float a0 = x[hh][4 * n] * (__uint_as_float(rd[4 * n]) - d2.x);
+          float a1 = x[hh][4 * n + 1] * (__uint_as_float(rd[4 * n + 1]) - d2.y);
+          float b0 = x[hh][4 * n + 2] * (__uint_as_float(rd[4 * n + 2]) - d2.x);
+          float b1 = x[hh][4 * n + 3] * (__uint_as_float(rd[4 * n + 3]) - d2.y);
+          if (!full) {  // masked entries (P = 0; D past T is not written): dS = 0
+            if (x[hh][4 * n] == 0.f) a0 = 0.f;
+            if (x[hh][4 * n + 1] == 0.f) a1 = 0.f;
+            if (x[hh][4 * n + 2] == 0.f) b0 = 0.f;
+            if (x[hh][4 * n + 3] == 0.f) b1 = 0.f;
+          }
+          dw[2 * (8 * hh + n)] = tc::pack_half2(a0, a1);
+          dw[2 * (8 * hh + n) + 1] = tc::pack_half2(b0, b1);
+        }
+      }
+      __syncwarp();
+      tc::tmem_st_16x128b_x16(tmem + lane16 + L::DP_COL, dw);
+      tc::tmem_st_wait();
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->p_full[pb]);
+      if (lane == 0) tc::mbar_arrive(&bars->ds_full);
     }
     // Epilogue: dV and dK rows (transpose of RoPE on dK) staged transposed in the now idle stage
     // buffers, then stored as dQKV^T columns with coalesced 16-byte stores.
@@ -411,12 +448,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     bf16_t* tk = tv + DH * 128;
     if (have) {
       tc::fence_after_sync();
-      const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
-      const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
-      const int ka = kb * BK + ra, kb8 = ka + 8;
-      stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, ra);
-      stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, ka < p.T ? ka : 0,
-                        kb8 < p.T ? kb8 : 0, p.cos_t, p.sin_t, tk, ra);
+      const int kA = keyA < p.T ? keyA : 0, kB = keyB < p.T ? keyB : 0;
+      stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, rA);
+      stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, kA, kB, p.cos_t,
+                        p.sin_t, tk, rA);
     }
     tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
     if (have) {
@@ -847,9 +882,8 @@ cudaError_t set_smem(K kernel, int bytes, bool& done) {
 template <int DH>
 cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   const int64_t N = (int64_t)L.B * L.T;
-  CUtensorMap kv128, q64, do64, do128;
-  if (!tmap_rows(&kv128, L.qkv, L.ldq, N, 128) || !tmap_rows(&q64, L.qkv, L.ldq, N, 64) ||
-      !tmap_rows(&do64, L.d_o, (uint64_t)L.Hq * DH, N, 64) ||
+  CUtensorMap kv128, do128;
+  if (!tmap_rows(&kv128, L.qkv, L.ldq, N, 128) ||
       !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128))
     return cudaErrorInvalidValue;
   static bool a1 = false, a2 = false;
@@ -858,7 +892,7 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   e = set_smem(attn_bwd_dq_tc_kernel<DH>, DqLayout<DH>::SMEM, a2);
   if (e != cudaSuccess) return e;
   dim3 g1((unsigned)L.Hkv, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
-  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, q64, do64, p);
+  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -894,7 +928,7 @@ cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const fl
   p.dqkvt = static_cast<bf16_t*>(dqkvt);
   p.status = L.status;
   if ((reinterpret_cast<uintptr_t>(L.lse) & 15u) || (reinterpret_cast<uintptr_t>(L.dvec) & 15u) ||
-      (L.lse_pitch % 64) != 0)
+      (L.lse_pitch % 128) != 0)
     return cudaErrorInvalidValue;
   return L.dh == 128 ? launch_bwd<128>(L, p) : launch_bwd<64>(L, p);
 }

@@ -479,11 +479,6 @@ __device__ __forceinline__ StackTile stack_tile(int k, int pairs, int BC, int nq
   return t;
 }
 
-__device__ __forceinline__ uint32_t pack_half2(float a, float b) {
-  const __half2 h = __floats2half2_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&h);
-}
-
 template <int DH, int MODE>
 __global__ void __launch_bounds__(PAIR_THREADS, 1)
     attn_fwd_pair_kernel(const __grid_constant__ CUtensorMap tm_q,
@@ -751,8 +746,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         for (int hh = 0; hh < 2; ++hh)
 #pragma unroll
           for (int n = 0; n < 8; ++n) {
-            pw[2 * (8 * hh + n)] = pack_half2(x[hh][4 * n], x[hh][4 * n + 1]);
-            pw[2 * (8 * hh + n) + 1] = pack_half2(x[hh][4 * n + 2], x[hh][4 * n + 3]);
+            pw[2 * (8 * hh + n)] = tc::pack_half2(x[hh][4 * n], x[hh][4 * n + 1]);
+            pw[2 * (8 * hh + n) + 1] = tc::pack_half2(x[hh][4 * n + 2], x[hh][4 * n + 3]);
           }
         // P_{g-1} V_{g-1} (and so every earlier P V) must have completed before P is overwritten
         // or O is rescaled.

@@ -21,11 +21,11 @@ struct Workspace {
   // backward only
   size_t xt;       // bf16 [d, ldt]          X transposed (K-major operand of the weight gradient)
   size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
-  size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 64)
+  size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 128)
   size_t dvec;     // fp32 [B, Hq, Tp]       rowsum(dO * O)
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
   int64_t ldt;     // row pitch (elements) of xt and dqkvt: N rounded up to 64
-  int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 64
+  int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 128
   size_t total;
 };
 
@@ -41,7 +41,7 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
   const int64_t N = B * T, D = block_rows(d), dm = d->d_model, dh = d->head_dim;
   const int64_t nP = (T + kPartRows - 1) / kPartRows;
   w.ldt = (N + 63) / 64 * 64;
-  w.tp = (T + 63) / 64 * 64;
+  w.tp = (T + 127) / 128 * 128;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     size_t o = off;
