@@ -370,24 +370,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       const int qc0 = i * BQ + 2 * cq;  // query of x[0][0]
       const bool full = i > kb && i * BQ + BQ <= p.T;
+      const float2 sl2 = make_float2(p.sl2, p.sl2);
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh)
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
           const float2 l2 = *reinterpret_cast<const float2*>(lse_s + 64 * hh + 8 * n + 2 * cq);
+          const float2 nl = make_float2(tc::neg_bits(l2.x), tc::neg_bits(l2.y));
+          const float2 ea = tc::fma2(make_float2(x[hh][4 * n], x[hh][4 * n + 1]), sl2, nl);
+          const float2 eb = tc::fma2(make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]), sl2, nl);
+          float pa[2] = {tc::fast_exp2(ea.x), tc::fast_exp2(ea.y)};
+          float pb[2] = {tc::fast_exp2(eb.x), tc::fast_exp2(eb.y)};
+          if (!full) {
 #pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const float le = e ? l2.y : l2.x;
-            float pa = tc::fast_exp2(fmaf(x[hh][4 * n + e], p.sl2, -le));
-            float pb = tc::fast_exp2(fmaf(x[hh][4 * n + 2 + e], p.sl2, -le));
-            if (!full) {
+            for (int e = 0; e < 2; ++e) {
               const int q = qc0 + 64 * hh + 8 * n + e;
-              if (q >= p.T || q < keyA) pa = 0.f;
-              if (q >= p.T || q < keyB) pb = 0.f;
+              if (q >= p.T || q < keyA) pa[e] = 0.f;
+              if (q >= p.T || q < keyB) pb[e] = 0.f;
             }
-            x[hh][4 * n + e] = pa;
-            x[hh][4 * n + 2 + e] = pb;
           }
+          x[hh][4 * n] = pa[0];
+          x[hh][4 * n + 1] = pa[1];
+          x[hh][4 * n + 2] = pb[0];
+          x[hh][4 * n + 3] = pb[1];
         }
       {
         uint32_t pw[32];  // pw[2m] row A, pw[2m + 1] row B, packed column 4m + cq
@@ -420,18 +425,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
           const float2 d2 = *reinterpret_cast<const float2*>(d_s + 64 * hh + 8 * n + 2 * cq);
-          float a0 = x[hh][4 * n] * (__uint_as_float(rd[4 * n]) - d2.x);
-          float a1 = x[hh][4 * n + 1] * (__uint_as_float(rd[4 * n + 1]) - d2.y);
-          float b0 = x[hh][4 * n + 2] * (__uint_as_float(rd[4 * n + 2]) - d2.x);
-          float b1 = x[hh][4 * n + 3] * (__uint_as_float(rd[4 * n + 3]) - d2.y);
+          const float2 ta = tc::sub2(make_float2(__uint_as_float(rd[4 * n]), __uint_as_float(rd[4 * n + 1])), d2);
+          const float2 tb = tc::sub2(make_float2(__uint_as_float(rd[4 * n + 2]), __uint_as_float(rd[4 * n + 3])), d2);
+          float2 da = tc::mul2(make_float2(x[hh][4 * n], x[hh][4 * n + 1]), ta);
+          float2 db = tc::mul2(make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]), tb);
           if (!full) {  // masked entries (P = 0; D past T is not written): dS = 0
-            if (x[hh][4 * n] == 0.f) a0 = 0.f;
-            if (x[hh][4 * n + 1] == 0.f) a1 = 0.f;
-            if (x[hh][4 * n + 2] == 0.f) b0 = 0.f;
-            if (x[hh][4 * n + 3] == 0.f) b1 = 0.f;
+            if (x[hh][4 * n] == 0.f) da.x = 0.f;
+            if (x[hh][4 * n + 1] == 0.f) da.y = 0.f;
+            if (x[hh][4 * n + 2] == 0.f) db.x = 0.f;
+            if (x[hh][4 * n + 3] == 0.f) db.y = 0.f;
           }
-          dw[2 * (8 * hh + n)] = tc::pack_half2(a0, a1);
-          dw[2 * (8 * hh + n) + 1] = tc::pack_half2(b0, b1);
+          dw[2 * (8 * hh + n)] = tc::pack_half2(da.x, da.y);
+          dw[2 * (8 * hh + n) + 1] = tc::pack_half2(db.x, db.y);
         }
       }
       __syncwarp();
@@ -781,15 +786,22 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->s_empty);
         const int k0 = j * BK + col0;
-        if (k0 + 63 <= q0) {  // every key of this slice is visible to every row of the tile
+        {  // packed FP32 pairs: the tensor pipe keeps its speed while these run
+          const float2 sl2 = make_float2(p.sl2, p.sl2);
+          const float2 nl = make_float2(tc::neg_bits(lse2), tc::neg_bits(lse2));
+          const float2 d2 = make_float2(drow, drow);
+          const bool all_visible = k0 + 63 <= q0;  // every key of this slice, every row of the tile
 #pragma unroll
-          for (int c = 0; c < 64; ++c)
-            dp[c] = tc::fast_exp2(fmaf(sv[c], p.sl2, -lse2)) * (dp[c] - drow);
-        } else {
-#pragma unroll
-          for (int c = 0; c < 64; ++c) {
-            const float e = tc::fast_exp2(fmaf(sv[c], p.sl2, -lse2));
-            dp[c] = (k0 + c <= t) ? e * (dp[c] - drow) : 0.f;
+          for (int c = 0; c < 64; c += 2) {
+            const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
+            const float2 pe = make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y));
+            float2 ds = tc::mul2(pe, tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
+            if (!all_visible) {
+              if (k0 + c > t) ds.x = 0.f;
+              if (k0 + c + 1 > t) ds.y = 0.f;
+            }
+            dp[c] = ds.x;
+            dp[c + 1] = ds.y;
           }
         }
         if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {

@@ -723,22 +723,26 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         const float muA = rsA ? mnA : mA, muB = rsB ? mnB : mB;
         const float alA = rsA ? tc::fast_exp2(mA - mnA) : 1.f;
         const float alB = rsB ? tc::fast_exp2(mB - mnB) : 1.f;
-        float sa0 = 0.f, sa1 = 0.f, sb0 = 0.f, sb1 = 0.f;
+        // Packed FP32 pairs (two columns of one row) keep the tensor pipe at speed meanwhile.
+        const float2 sl2 = make_float2(p.sl2, p.sl2);
+        const float2 nmA = make_float2(tc::neg_bits(muA), tc::neg_bits(muA));
+        const float2 nmB = make_float2(tc::neg_bits(muB), tc::neg_bits(muB));
+        float2 sA = make_float2(0.f, 0.f), sB = make_float2(0.f, 0.f);
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh)
 #pragma unroll
           for (int n = 0; n < 8; ++n) {
-            x[hh][4 * n] = tc::fast_exp2(fmaf(x[hh][4 * n], p.sl2, -muA));
-            x[hh][4 * n + 1] = tc::fast_exp2(fmaf(x[hh][4 * n + 1], p.sl2, -muA));
-            x[hh][4 * n + 2] = tc::fast_exp2(fmaf(x[hh][4 * n + 2], p.sl2, -muB));
-            x[hh][4 * n + 3] = tc::fast_exp2(fmaf(x[hh][4 * n + 3], p.sl2, -muB));
-            sa0 += x[hh][4 * n];
-            sa1 += x[hh][4 * n + 1];
-            sb0 += x[hh][4 * n + 2];
-            sb1 += x[hh][4 * n + 3];
+            const float2 ea = tc::fma2(make_float2(x[hh][4 * n], x[hh][4 * n + 1]), sl2, nmA);
+            const float2 eb = tc::fma2(make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]), sl2, nmB);
+            x[hh][4 * n] = tc::fast_exp2(ea.x);
+            x[hh][4 * n + 1] = tc::fast_exp2(ea.y);
+            x[hh][4 * n + 2] = tc::fast_exp2(eb.x);
+            x[hh][4 * n + 3] = tc::fast_exp2(eb.y);
+            sA = tc::add2(sA, make_float2(x[hh][4 * n], x[hh][4 * n + 1]));
+            sB = tc::add2(sB, make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]));
           }
-        lA = lA * alA + (sa0 + sa1);  // this thread's share of row A; summed over the 4 at the end
-        lB = lB * alB + (sb0 + sb1);
+        lA = lA * alA + (sA.x + sA.y);  // this thread's share of row A; summed over the 4 at the end
+        lB = lB * alB + (sB.x + sB.y);
         mA = muA;
         mB = muB;
         uint32_t pw[32];  // P words: pw[2n] row A, pw[2n + 1] row B, column 4n + cq of P
@@ -764,12 +768,15 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             __syncwarp();
             tc::tmem_ld_16x256b_x8(tmem + lane16 + col, r);
             tc::tmem_ld_wait();
+            const float2 a2 = make_float2(alA, alA), b2 = make_float2(alB, alB);
 #pragma unroll
             for (int n = 0; n < 8; ++n) {
-              r[4 * n] = __float_as_uint(__uint_as_float(r[4 * n]) * alA);
-              r[4 * n + 1] = __float_as_uint(__uint_as_float(r[4 * n + 1]) * alA);
-              r[4 * n + 2] = __float_as_uint(__uint_as_float(r[4 * n + 2]) * alB);
-              r[4 * n + 3] = __float_as_uint(__uint_as_float(r[4 * n + 3]) * alB);
+              const float2 ra = tc::mul2(make_float2(__uint_as_float(r[4 * n]), __uint_as_float(r[4 * n + 1])), a2);
+              const float2 rb = tc::mul2(make_float2(__uint_as_float(r[4 * n + 2]), __uint_as_float(r[4 * n + 3])), b2);
+              r[4 * n] = __float_as_uint(ra.x);
+              r[4 * n + 1] = __float_as_uint(ra.y);
+              r[4 * n + 2] = __float_as_uint(rb.x);
+              r[4 * n + 3] = __float_as_uint(rb.y);
             }
             tc::tmem_st_16x256b_x8(tmem + lane16 + col, r);
           }
@@ -833,7 +840,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         if (lane == 0) tc::mbar_arrive(&bars->st_empty[ob]);
         tc::fence_after_sync();
         const float inv_l = __fdiv_rn(1.f, lt);
-        float sq = 0.f, dsum = 0.f;
+        float2 sq = make_float2(0.f, 0.f), dsum = make_float2(0.f, 0.f);  // packed partial sums
+        const float2 il2 = make_float2(inv_l, inv_l);
 #pragma unroll 1
         for (int ch = 0; ch < DH / 32; ++ch) {
           const int col = h * DH + ch * 32 + c4 * 4;
@@ -854,7 +862,11 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             tc::tmem_ld32(tmem + lane_base + L::O_COL + ob * DH + ch * 32, r);
             tc::tmem_ld_wait();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __fmul_rn(__uint_as_float(r[i]), inv_l);
+            for (int i = 0; i < 32; i += 2) {
+              const float2 v = tc::mul2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), il2);
+              o[i] = v.x;
+              o[i + 1] = v.y;
+            }
           }
           if (ch == DH / 32 - 1) {  // O of this buffer is read out: the next-but-one tile may use it
             tc::fence_before_sync();
@@ -876,12 +888,14 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             const int64_t off = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
             if (MODE == 0) {
               *reinterpret_cast<float4*>(p.a_out + off) = ov;
-              sq += ov.x * ov.x + ov.y * ov.y + ov.z * ov.z + ov.w * ov.w;
+              const float2 v01 = make_float2(ov.x, ov.y), v23 = make_float2(ov.z, ov.w);
+              sq = tc::fma2(v23, v23, tc::fma2(v01, v01, sq));
             } else {
               const float4 a = av[i];
-              const float e0 = __fsub_rn(ov.x, a.x), e1 = __fsub_rn(ov.y, a.y);
-              const float e2 = __fsub_rn(ov.z, a.z), e3 = __fsub_rn(ov.w, a.w);
-              sq += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+              const float2 e01 = tc::sub2(make_float2(ov.x, ov.y), make_float2(a.x, a.y));
+              const float2 e23 = tc::sub2(make_float2(ov.z, ov.w), make_float2(a.z, a.w));
+              const float e0 = e01.x, e1 = e01.y, e2 = e23.x, e3 = e23.y;
+              sq = tc::fma2(e23, e23, tc::fma2(e01, e01, sq));
               if (MODE == 2) {
                 const __half2 a01 = __floats2half2_rn(e0, e1), a23 = __floats2half2_rn(e2, e3);
                 uint2 u;
@@ -898,7 +912,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
 #pragma unroll
             for (int v = 0; v < 8; ++v) {
               const float4 e = *reinterpret_cast<const float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2));
-              dsum += e.x * o[4 * v] + e.y * o[4 * v + 1] + e.z * o[4 * v + 2] + e.w * o[4 * v + 3];
+              dsum = tc::fma2(make_float2(e.x, e.y), make_float2(o[4 * v], o[4 * v + 1]), dsum);
+              dsum = tc::fma2(make_float2(e.z, e.w), make_float2(o[4 * v + 2], o[4 * v + 3]), dsum);
             }
             __syncwarp();
           }
@@ -907,9 +922,9 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
           const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + t;
           if (MODE != 1 && p.lse != nullptr)
             p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
-          if (MODE == 2) p.dvec[li] = dsum;
+          if (MODE == 2) p.dvec[li] = dsum.x + dsum.y;
         }
-        acc = (double)sq;
+        acc = (double)sq.x + (double)sq.y;
       }
       acc = warp_sum(acc);
       double* red = bars->red[tc_ & 1];  // alternate by tile
