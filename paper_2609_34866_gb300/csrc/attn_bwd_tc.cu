@@ -9,8 +9,8 @@
 //   dkdv  one CTA per (128-key block, KV head, sequence); loops over the query heads of the group and
 //         over 128-query blocks: S^T = K Q^T, dP^T = V dO^T into TMEM, P^T and dS^T (fp16) written
 //         back over them, dV += P^T dO and dK += dS^T Q (A operands in TMEM) accumulated in TMEM.
-//   dq    one CTA per (128 query rows, query head, sequence); loops over 64-key blocks: S = Q K^T,
-//         dP = dO V^T, dS (fp16) to shared memory, dQ += dS K in TMEM.
+//   dq    persistent, (128 query rows, query head, sequence) tiles; loops over 128-key blocks:
+//         S = Q K^T, dP = dO V^T (Q, dO in TMEM), dS (fp16) to shared memory, dQ += dS K in TMEM.
 // Warp roles: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..9 elementwise: two warps per
 // TMEM lane quarter (dkdv: each warp 16 whole rows of S^T / dP^T; dq: each thread one row and half
 // of the columns of S / dP). The epilogues apply the transpose of RoPE to dQ and dK and write
@@ -786,22 +786,28 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&bars->s_empty);
         const int k0 = j * BK + col0;
-        {  // packed FP32 pairs: the tensor pipe keeps its speed while these run
+        {  // packed FP32 pairs; one loop per mask case keeps the per-element work minimal
           const float2 sl2 = make_float2(p.sl2, p.sl2);
           const float2 nl = make_float2(tc::neg_bits(lse2), tc::neg_bits(lse2));
           const float2 d2 = make_float2(drow, drow);
-          const bool all_visible = k0 + 63 <= q0;  // every key of this slice, every row of the tile
+          if (k0 + 63 <= q0) {  // every key of this slice is visible to every row of the tile
 #pragma unroll
-          for (int c = 0; c < 64; c += 2) {
-            const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
-            const float2 pe = make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y));
-            float2 ds = tc::mul2(pe, tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
-            if (!all_visible) {
-              if (k0 + c > t) ds.x = 0.f;
-              if (k0 + c + 1 > t) ds.y = 0.f;
+            for (int c = 0; c < 64; c += 2) {
+              const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
+              const float2 ds = tc::mul2(make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y)),
+                                         tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
+              dp[c] = ds.x;
+              dp[c + 1] = ds.y;
             }
-            dp[c] = ds.x;
-            dp[c + 1] = ds.y;
+          } else {
+#pragma unroll
+            for (int c = 0; c < 64; c += 2) {
+              const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
+              const float2 ds = tc::mul2(make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y)),
+                                         tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
+              dp[c] = (k0 + c <= t) ? ds.x : 0.f;
+              dp[c + 1] = (k0 + c + 1 <= t) ? ds.y : 0.f;
+            }
           }
         }
         if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
