@@ -261,7 +261,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------------------------- UMMA
       constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
-      const uint32_t ka = tc::smem_u32(smem + L::K_OFF), va = tc::smem_u32(smem + L::V_OFF);
+      const uint64_t ka = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF));
+      const uint64_t va = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::V_OFF));
       bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
       // Event-driven issue in the order dV(j), S^T(j+1), dK(j), dP^T(j+1): ns, nd, nv, nk count
       // the S^T, dP^T, dV and dK UMMA groups issued so far.
@@ -273,12 +274,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (ns < n_it && nv == ns && tc::mbar_ready(&bars->ld_full[ns % STAGES], (ns / STAGES) & 1) &&
             (ns == 0 || tc::mbar_ready(&bars->dv_done, (ns - 1) & 1))) {
           tc::fence_after_sync();
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (ns % STAGES) * L::ST_STRIDE);
+          const uint64_t bq = tc::sdesc_kmajor_sw128(
+              tc::smem_u32(smem + L::ST_OFF + (ns % STAGES) * L::ST_STRIDE + L::ST_Q));
 #pragma unroll
           for (int k = 0; k < DH / 16; ++k) {
             const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
-            tc::umma_f16(tmem + L::S_COL, tc::sdesc_kmajor_sw128(ka + o),
-                         tc::sdesc_kmajor_sw128(sb + L::ST_Q + o), ID_S, k > 0 ? 1u : 0u);
+            tc::umma_f16(tmem + L::S_COL, tc::sdesc_advance(ka, o), tc::sdesc_advance(bq, o), ID_S,
+                         k > 0 ? 1u : 0u);
           }
           tc::umma_commit(&bars->s_full);
           ++ns;
@@ -287,12 +289,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // dP^T(nd): after S^T(nd) (same stage) and once dK(nd - 1) has read dS^T(nd - 1).
         if (nd < ns && nk == nd && (nd == 0 || tc::mbar_ready(&bars->dk_done, (nd - 1) & 1))) {
           tc::fence_after_sync();
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (nd % STAGES) * L::ST_STRIDE);
+          const uint64_t bd = tc::sdesc_kmajor_sw128(
+              tc::smem_u32(smem + L::ST_OFF + (nd % STAGES) * L::ST_STRIDE + L::ST_DO));
 #pragma unroll
           for (int k = 0; k < DH / 16; ++k) {
             const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
-            tc::umma_f16(tmem + L::DP_COL, tc::sdesc_kmajor_sw128(va + o),
-                         tc::sdesc_kmajor_sw128(sb + L::ST_DO + o), ID_S, k > 0 ? 1u : 0u);
+            tc::umma_f16(tmem + L::DP_COL, tc::sdesc_advance(va, o), tc::sdesc_advance(bd, o), ID_S,
+                         k > 0 ? 1u : 0u);
           }
           tc::umma_commit(&bars->dp_full);
           ++nd;
@@ -301,11 +304,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // dV(nv) += P^T(nv) dO(nv) once the elementwise warps have written P^T(nv).
         if (nv < ns && tc::mbar_ready(&bars->p_full, nv & 1)) {
           tc::fence_after_sync();
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + (nv % STAGES) * L::ST_STRIDE);
+          const uint64_t bd = tc::sdesc_mnmajor_sw128(
+              tc::smem_u32(smem + L::ST_OFF + (nv % STAGES) * L::ST_STRIDE + L::ST_DO), L::CHUNK, 1024);
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k)
-            tc::umma_f16_ts(tmem + L::DV_COL, tmem + L::S_COL + k * 8,
-                            tc::sdesc_mnmajor_sw128(sb + L::ST_DO + k * 16 * 128, L::CHUNK, 1024),
+            tc::umma_f16_ts(tmem + L::DV_COL, tmem + L::S_COL + k * 8, tc::sdesc_advance(bd, k * 16 * 128),
                             ID_G, (nv > 0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->dv_done);
           ++nv;
@@ -315,11 +318,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (nk < nd && (ns > nk + 1 || ns == n_it) && tc::mbar_ready(&bars->ds_full, nk & 1)) {
           tc::fence_after_sync();
           const int st = nk % STAGES;
-          const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+          const uint64_t bq = tc::sdesc_mnmajor_sw128(
+              tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_Q), L::CHUNK, 1024);
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k)
-            tc::umma_f16_ts(tmem + L::DK_COL, tmem + L::DP_COL + k * 8,
-                            tc::sdesc_mnmajor_sw128(sb + L::ST_Q + k * 16 * 128, L::CHUNK, 1024),
+            tc::umma_f16_ts(tmem + L::DK_COL, tmem + L::DP_COL + k * 8, tc::sdesc_advance(bq, k * 16 * 128),
                             ID_G, (nk > 0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->dk_done);
           tc::umma_commit(&bars->ld_empty[st]);  // dV(nk) and dK(nk) were the stage's last readers

@@ -172,6 +172,13 @@ __device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t saddr) {
 
 // Instruction descriptor of tcgen05.mma.kind::f16: fp32 accumulator, A and B of the same 16-bit
 // type (fp16 or bf16), both K-major, M x N tile.
+// A descriptor for the tile `bytes` further on (a multiple of 16, within the same shared memory
+// window): the start-address field is addr >> 4 in the low bits, so the step is a plain add. Cheaper
+// to issue than rebuilding the descriptor per UMMA.
+__device__ __forceinline__ uint64_t sdesc_advance(uint64_t desc, uint32_t bytes) {
+  return desc + (uint64_t)(bytes >> 4);
+}
+
 __host__ __device__ constexpr uint32_t idesc_f16(bool bf16, int M, int N) {
   return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) |
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
