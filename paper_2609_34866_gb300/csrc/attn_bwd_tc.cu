@@ -669,7 +669,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       constexpr uint32_t ID_S = tc::idesc_f16(false, BQ, BK);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
       const uint32_t stg_base = tc::smem_u32(smem + L::STG_OFF);
-      const uint32_t ds_base = tc::smem_u32(smem + L::DS_OFF);
+      const uint64_t dsd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::DS_OFF));
       bool ok = true;
       uint32_t Js = 0, Jg = 0, U = 0;  // S/dP blocks, dQ blocks, staging uses so far (all tiles)
       int n = 0;
@@ -703,15 +703,15 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
               tc::mbar_ready(&bars->v_full[Js % VST], (Js / VST) & 1) &&
               tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
             tc::fence_after_sync();
-            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Js % KST) * L::TILE);
-            const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + (Js % VST) * L::TILE);
+            const uint64_t kd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF + (Js % KST) * L::TILE));
+            const uint64_t vd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::V_OFF + (Js % VST) * L::TILE));
 #pragma unroll
             for (int k = 0; k < DH / 16; ++k) {
               const uint32_t off = (k >> 2) * L::CHUNK + (k & 3) * 32;
-              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + k * 8,
-                              tc::sdesc_kmajor_sw128(k_base + off), ID_S, k > 0 ? 1u : 0u);
-              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::DO_COL + k * 8,
-                              tc::sdesc_kmajor_sw128(v_base + off), ID_S, k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + k * 8, tc::sdesc_advance(kd, off), ID_S,
+                              k > 0 ? 1u : 0u);
+              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::DO_COL + k * 8, tc::sdesc_advance(vd, off), ID_S,
+                              k > 0 ? 1u : 0u);
             }
             tc::umma_commit(&bars->s_full);
             tc::umma_commit(&bars->v_empty[Js % VST]);
@@ -722,13 +722,12 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
           if (ng < ns && tc::mbar_ready(&bars->p_full, Jg & 1) &&
               (ng > 0 || n == 0 || tc::mbar_ready(&bars->o_empty, (n - 1) & 1))) {
             tc::fence_after_sync();
-            const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + (Jg % KST) * L::TILE);
+            const uint64_t kd = tc::sdesc_mnmajor_sw128(
+                tc::smem_u32(smem + L::K_OFF + (Jg % KST) * L::TILE), L::CHUNK, 1024);
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k)
-              tc::umma_f16(tmem + L::DQ_COL,
-                           tc::sdesc_kmajor_sw128(ds_base + (k >> 2) * (BQ * 128) + (k & 3) * 32),
-                           tc::sdesc_mnmajor_sw128(k_base + k * 16 * 128, L::CHUNK, 1024), ID_G,
-                           (ng > 0 || k > 0) ? 1u : 0u);
+              tc::umma_f16(tmem + L::DQ_COL, tc::sdesc_advance(dsd, (k >> 2) * (BQ * 128) + (k & 3) * 32),
+                           tc::sdesc_advance(kd, k * 16 * 128), ID_G, (ng > 0 || k > 0) ? 1u : 0u);
             tc::umma_commit(&bars->k_empty[Jg % KST]);
             tc::umma_commit(&bars->p_empty);
             ++ng;

@@ -593,12 +593,12 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         if (!tc::mbar_wait(&bars->k_full[ks], (gg / SK_ST) & 1, abort, p.status)) return false;
         if (!tc::mbar_wait(&bars->s_empty, (gg & 1) ^ 1, abort, p.status)) return false;
         tc::fence_after_sync();
-        const uint32_t k_base = tc::smem_u32(smem + L::K_OFF + ks * L::TILE);
+        const uint64_t kd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF + ks * L::TILE));
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk)
           tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + kk * 8,
-                          tc::sdesc_kmajor_sw128(k_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32),
-                          ID_S, kk > 0 ? 1u : 0u);
+                          tc::sdesc_advance(kd, (kk >> 2) * L::CHUNK + (kk & 3) * 32), ID_S,
+                          kk > 0 ? 1u : 0u);
         tc::umma_commit(&bars->s_full);
         tc::umma_commit(&bars->k_empty[ks]);
         return true;
@@ -613,12 +613,12 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             !tc::mbar_wait(&bars->o_empty[ob], ((tc_ >> 1) - 1) & 1, abort, p.status))
           return false;
         tc::fence_after_sync();
-        const uint32_t v_base = tc::smem_u32(smem + L::V_OFF + vs * L::TILE);
+        const uint64_t vd =
+            tc::sdesc_mnmajor_sw128(tc::smem_u32(smem + L::V_OFF + vs * L::TILE), L::CHUNK, 1024);
 #pragma unroll
         for (int k = 0; k < SKB / 16; ++k)
           tc::umma_f16_ts(tmem + L::O_COL + ob * DH, tmem + L::P_COL + k * 8,
-                          tc::sdesc_mnmajor_sw128(v_base + k * 16 * 128, L::CHUNK, 1024), ID_PV,
-                          (!first || k > 0) ? 1u : 0u);
+                          tc::sdesc_advance(vd, k * 16 * 128), ID_PV, (!first || k > 0) ? 1u : 0u);
         tc::umma_commit(&bars->pv_done);
         tc::umma_commit(&bars->v_empty[vs]);
         return true;
