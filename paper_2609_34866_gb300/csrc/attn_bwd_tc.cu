@@ -646,9 +646,16 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
           if (!ok) break;
         }
         const int col = is_v ? p.vcol0 + g * DH : p.kcol0 + g * DH;
+        // A ring slot frees only when the block it holds has been used by the last UMMA that reads
+        // it, so blocks are also prefetched into L2 a ring's depth ahead of their load.
+        auto prefetch = [&](int j) {
+          for (int ch = 0; ch < DH / 64; ++ch) tc::tma_prefetch_2d(&tm_kv, col + ch * 64, row0 + j * BK);
+        };
+        for (int j = 0; j < nst && j < nkb; ++j) prefetch(j);
         for (int j = 0; j < nkb; ++j, ++J) {
           const int st = J % nst;
           const uint32_t ph = (J / nst) & 1;
+          if (j + nst < nkb) prefetch(j + nst);
           if (!tc::mbar_wait(&empty[st], ph ^ 1, abort, p.status)) { ok = false; break; }
           tc::mbar_expect_tx(&full[st], L::TILE);
           for (int ch = 0; ch < DH / 64; ++ch)

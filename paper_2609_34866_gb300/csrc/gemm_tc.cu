@@ -113,16 +113,24 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
       const int jj0 = o % p.dh;
       const float4* cp = reinterpret_cast<const float4*>(p.cos_t + (int64_t)t * half + jj0);
       const float4* sp = reinterpret_cast<const float4*>(p.sin_t + (int64_t)t * half + jj0);
+      // Packed FP32 pairs: this epilogue overlaps the next tile's UMMAs, which scalar FP32
+      // instructions at a high rate slow down.
 #pragma unroll
       for (int v = 0; v < 8; ++v) {
         const float4 c4 = __ldg(cp + v), s4 = __ldg(sp + v);
-        const float cs[4] = {c4.x, c4.y, c4.z, c4.w}, sn[4] = {s4.x, s4.y, s4.z, s4.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
+        for (int e = 0; e < 4; e += 2) {
           const int i = v * 4 + e;
-          const float x1 = a[i], x2 = b[i];
-          a[i] = x1 * cs[e] - x2 * sn[e];
-          b[i] = x2 * cs[e] + x1 * sn[e];
+          const float2 cs = e ? make_float2(c4.z, c4.w) : make_float2(c4.x, c4.y);
+          const float2 sn = e ? make_float2(s4.z, s4.w) : make_float2(s4.x, s4.y);
+          const float2 nsn = make_float2(tc::neg_bits(sn.x), tc::neg_bits(sn.y));
+          const float2 x1 = make_float2(a[i], a[i + 1]), x2 = make_float2(b[i], b[i + 1]);
+          const float2 ra = tc::fma2(x2, nsn, tc::mul2(x1, cs));  // x1 cos - x2 sin
+          const float2 rb = tc::fma2(x1, sn, tc::mul2(x2, cs));   // x2 cos + x1 sin
+          a[i] = ra.x;
+          a[i + 1] = ra.y;
+          b[i] = rb.x;
+          b[i + 1] = rb.y;
         }
       }
     }
