@@ -10,7 +10,7 @@ import torch
 from oracle import jab_oracle as O
 from workloads import BlockShape, Workload, WORKLOADS, make_x, make_block_weights
 
-# Tolerances (stated in the spec bars): attention-output error <= 1e-2 of its RMS, L_JAB
+# Tolerances: attention-output error <= 1e-2 of its RMS, L_JAB
 # relative error <= 1e-2, scale-gradient cosine >= 0.999; integer codes bit-exact.
 A_TOL = 1e-2
 L_TOL = 1e-2
