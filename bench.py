@@ -5,8 +5,9 @@ One step = one forward L_JAB + STE/LSQ scale-gradient evaluation (jab_loss_backw
 Mistral-7B-shaped attention block (d_model 4096, 32 query / 8 KV heads of 128, RoPE theta 1e4),
 X = 128 sequences x 2048 tokens of Student-t(4) unit-variance activations, 3-bit groups of 128.
 The teacher output A(X; W) is computed once before the timed region (it is shared by every
-evaluation of the block, like the STE fitting loop's 200 steps). The forward-only rate
-(jab_loss_forward, one candidate) is reported beside it.
+evaluation of the block, like the STE fitting loop's 200 steps). Reported beside it: the
+forward-only rate (jab_loss_forward, one candidate) and the Fisher-coupling probe (loss and squared
+STE weight-gradient norm at 2 bits, jab_loss_backward_weights).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 
@@ -307,6 +308,29 @@ def run_ours(args, wl):
     fwd_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     fwd_value = world * args.steps / (fwd_ms / 1e3)
 
+    # ---- Fisher-coupling probe (App. B): the loss and ||dL/dw_hat||^2 at 2 bits with round-to-
+    # nearest (absmax) scales, one fwd + bwd per evaluation; reported beside the main metric
+    s2 = torch.empty_like(scales)
+    J.jab_init_scales(desc, 2, 0, W, s2)
+    sq = torch.empty(1, dtype=torch.float64, device=dev)
+
+    def fisher_step():
+        J.jab_loss_backward_weights(desc, B, T, X, W, A, 2, s2, loss, grad_sqnorm=sq, ws=ws)
+
+    n_fis = max(1, min(args.steps, 3))
+    for _ in range(max(1, min(args.warmup, 2))):
+        fisher_step()
+    barrier()
+    torch.cuda.synchronize()
+    e0.record(st)
+    for _ in range(n_fis):
+        fisher_step()
+    e1.record(st)
+    torch.cuda.synchronize()
+    fis_ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    if J.jab_get_device_status() != 0:
+        raise RuntimeError("device status set during the Fisher-coupling probe")
+
     # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed region.
     # Every step copies its own inputs (X, W, A_ref, scales) host -> device and reads its result
     # (loss, scale gradient) back. As in a fitting loop, step i + 1's inputs are copied on a second
@@ -391,6 +415,9 @@ def run_ours(args, wl):
         "algorithmic_tflop_per_step": {"fwd": fwd_f / 1e12, "bwd": bwd_f / 1e12},
         "fwd_only": {"value": fwd_value, "unit": "evals/s", "ms_per_eval": fwd_ms / args.steps,
                      "achieved_tflops": fwd_f / (fwd_ms / args.steps / 1e3) / 1e12},
+        "fisher_probe": {"value": world * n_fis / (fis_ms / 1e3), "unit": "evals/s", "bits": 2,
+                         "ms_per_eval": fis_ms / n_fis,
+                         "achieved_tflops": (fwd_f + bwd_f) / (fis_ms / n_fis / 1e3) / 1e12},
         "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": gpu_launches, "clocks": clk.summary(),
         "path": "tcgen05" if tc else "cuda-core",

@@ -108,6 +108,22 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
                                     double* loss_dev, float* grad_scales_dev, void* ws,
                                     size_t ws_bytes, jab_stream_t stream);
 
+/* Forward L_JAB and the STE weight gradient for one candidate (App. B "Joint STE fine-tuning":
+ * d w_hat / d w = 1, so dL/dW = dL/dw_hat), and its squared Frobenius norm: the Fisher-coupling score
+ * of App. B "Fisher-coupling" when called with bits = 2 and round-to-nearest scales
+ * (jab_init_scales mode 0).
+ *   grad_w_dev      out fp32 [(Hq+2Hkv)*d_h, d_model] or NULL   dL/dw_hat = (2/n) dQKV^T X, n = B*T*Hq*d_h
+ *   grad_sqnorm_dev out fp64 [1] or NULL                        ||dL/dw_hat||_F^2 (fp64 atomics: the
+ *                                                               last bits may differ between calls)
+ *   loss_dev        out fp64 [1]
+ * At least one of grad_w_dev and grad_sqnorm_dev must be non-NULL. Uses the with_bwd workspace of
+ * jab_workspace_size. Returns JAB_ERR_UNSUPPORTED on the CUDA-core path (JAB_PATH=simple). */
+jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int32_t T,
+                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                     int32_t bits, const float* scales_dev, double* loss_dev,
+                                     float* grad_w_dev, double* grad_sqnorm_dev, void* ws,
+                                     size_t ws_bytes, jab_stream_t stream);
+
 /* Quantiser alone (Section 2.1, Eq. 2): v = fl32(w / s), q = clip(round-half-even(v), -qmax, qmax).
  *   codes_dev      out int8 [(Hq+2Hkv)*d_h, d_model] or NULL
  *   w_hat_dev      out fp32 [(Hq+2Hkv)*d_h, d_model] or NULL   fl32(q * s) */

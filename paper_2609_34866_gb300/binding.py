@@ -74,6 +74,7 @@ def lib() -> ctypes.CDLL:
     L.jab_loss_forward_noalloc.argtypes = [D, i32, i32, _P, _P, _P, i32, ctypes.POINTER(i32),
                                            ctypes.POINTER(_P), _P, _P, _P]
     L.jab_loss_backward_scales.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P, _P, sz, _P]
+    L.jab_loss_backward_weights.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, _P, _P, _P, _P, sz, _P]
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
     L.jab_get_device_status.argtypes = [_P]
@@ -88,7 +89,7 @@ def lib() -> ctypes.CDLL:
                                  ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
     L.jab_timing_reset.argtypes = []
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
-               "jab_loss_backward_scales",
+               "jab_loss_backward_scales", "jab_loss_backward_weights",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
                "jab_selftest_wait_timeout",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
@@ -197,6 +198,17 @@ def jab_loss_backward_scales(desc, B, T, X, W, A_ref, bits: int, scales, kappa: 
         float(kappa), _ptr(loss, torch.float64, "loss"),
         _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "jab_loss_backward_scales")
+
+
+def jab_loss_backward_weights(desc, B, T, X, W, A_ref, bits: int, scales, loss, grad_w=None,
+                              grad_sqnorm=None, ws: Workspace = None, stream=None):
+    """Loss and the STE weight gradient dL/dw_hat (fp32 [D, d]) and/or its squared norm (fp64 [1])."""
+    st = lib().jab_loss_backward_weights(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), int(bits), _ptr(scales, torch.float32, "scales"),
+        _ptr(loss, torch.float64, "loss"), _ptr(grad_w, torch.float32, "grad_w"),
+        _ptr(grad_sqnorm, torch.float64, "grad_sqnorm"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_loss_backward_weights")
 
 
 def jab_quantize(desc, bits, W, scales, codes=None, w_hat=None, stream=None):

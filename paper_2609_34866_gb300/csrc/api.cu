@@ -224,26 +224,27 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
   return JAB_OK;
 }
 
-jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+// Steps shared by the backward entry points (App. B, STE): quantise, project (+ RoPE), attention
+// forward in mode 2 (loss partials, dO = A_hat - A_ref, lse, D), the loss, and the attention backward
+// into dQKV^T (bf16 [D, ldt]) in the workspace. Checks the arguments common to both.
+static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32_t T,
                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
-                                    int32_t bits, const float* scales_dev, float kappa,
-                                    double* loss_dev, float* grad_scales_dev, void* ws,
-                                    size_t ws_bytes, jab_stream_t stream) {
+                                    int32_t bits, const float* scales_dev, double* loss_dev,
+                                    void* ws, size_t ws_bytes, cudaStream_t st, Workspace* wp_out,
+                                    int** status_out) {
   jab_status s = check_desc(desc);
   if (s != JAB_OK) return s;
   if ((s = check_bt(B, T)) != JAB_OK) return s;
-  if (bits < 2 || bits > 8 || !X_dev || !W_dev || !A_ref_dev || !scales_dev || !loss_dev ||
-      !grad_scales_dev || !ws)
+  if (bits < 2 || bits > 8 || !X_dev || !W_dev || !A_ref_dev || !scales_dev || !loss_dev || !ws)
     return JAB_ERR_INVALID_ARG;
   if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) || !aligned16(scales_dev) ||
-      !aligned16(grad_scales_dev) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+      (reinterpret_cast<uintptr_t>(ws) & 255u))
     return JAB_ERR_INVALID_ARG;
   const Workspace wp = plan_workspace(desc, B, T, 1, true);
   if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
   int* status;
   int sms;
   if ((s = device_info(&status, &sms)) != JAB_OK) return s;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   const int64_t N = (int64_t)B * T;
   const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
@@ -272,6 +273,30 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
                              st));
   JAB_SITE("attn_bwd", 2, use_tc_path() ? launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt)
                         : launch_attn_bwd_simple(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt));
+  *wp_out = wp;
+  *status_out = status;
+  return JAB_OK;
+}
+
+jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                    int32_t bits, const float* scales_dev, float kappa,
+                                    double* loss_dev, float* grad_scales_dev, void* ws,
+                                    size_t ws_bytes, jab_stream_t stream) {
+  if (!grad_scales_dev || !aligned16(grad_scales_dev)) {
+    const jab_status s = check_desc(desc);
+    return s != JAB_OK ? s : JAB_ERR_INVALID_ARG;
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  Workspace wp;
+  int* status;
+  jab_status s = backward_to_dqkvt(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, loss_dev,
+                                   ws, ws_bytes, st, &wp, &status);
+  if (s != JAB_OK) return s;
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, G = desc->group_size;
+  const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
   const double k = kappa > 0.f ? (double)kappa : 1.0 / sqrt((double)G * qmax_of(bits));
   const float coef = (float)(k * 2.0 / n_el);
   JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
@@ -283,6 +308,35 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
                                                      scales_dev, N, D, dm, G, bits, coef,
                                                      grad_scales_dev, st));
   JAB_SITE("check_finite", 1, launch_check_finite(grad_scales_dev, (int64_t)D * (dm / G), status, st));
+  return JAB_OK;
+}
+
+jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int32_t T,
+                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                     int32_t bits, const float* scales_dev, double* loss_dev,
+                                     float* grad_w_dev, double* grad_sqnorm_dev, void* ws,
+                                     size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((!grad_w_dev && !grad_sqnorm_dev) || (grad_w_dev && !aligned16(grad_w_dev)))
+    return JAB_ERR_INVALID_ARG;
+  if (!use_tc_path()) return JAB_ERR_UNSUPPORTED;  // the store epilogue exists on the tcgen05 path
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  Workspace wp;
+  int* status;
+  s = backward_to_dqkvt(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, loss_dev, ws,
+                        ws_bytes, st, &wp, &status);
+  if (s != JAB_OK) return s;
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model;
+  const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
+  if (grad_sqnorm_dev) JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_sqnorm_dev, 0, sizeof(double), st));
+  JAB_SITE("wgrad_store", 1, launch_wgrad_store_tc(w + wp.dqkvt, wp.ldt, X_dev, N, D, dm,
+                                                   (float)(2.0 / n_el), grad_w_dev, grad_sqnorm_dev,
+                                                   status, st));
+  if (grad_w_dev)
+    JAB_SITE("check_finite", 1, launch_check_finite(grad_w_dev, (int64_t)D * dm, status, st));
   return JAB_OK;
 }
 

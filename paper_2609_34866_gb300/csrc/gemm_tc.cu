@@ -32,7 +32,7 @@ constexpr int NUM_THREADS = 192;
 constexpr uint32_t TMEM_COLS = 2 * BN;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
 
-enum EpiKind { kEpiRope = 0, kEpiLsq = 1 };
+enum EpiKind { kEpiRope = 0, kEpiLsq = 1, kEpiStore = 2 };
 
 struct GemmParams {
   int64_t M;
@@ -50,6 +50,9 @@ struct GemmParams {
   int d, G, bits;
   float coef;
   float* ds;
+  // weight-gradient store epilogue (one unit covers the whole K range)
+  float* dw;
+  double* sqnorm;
 };
 
 struct Bars {
@@ -151,6 +154,43 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
         d2[v] = u2;
       }
     }
+  }
+}
+
+// STE weight gradient (App. B: d w_hat / d w = 1, so dL/dW = dL/dw_hat = coef * dQKV^T X): the
+// tile times coef stored as fp32 rows of dw (when set) and its squared Frobenius norm added to
+// *sqnorm (when set; fp64 atomics, one per warp and tile). Packed FP32 pairs, as this runs beside
+// the next tile's UMMAs.
+__device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, int mb, int nb,
+                                          int row) {
+  const int64_t o = (int64_t)mb * BM + row;  // M = D is a multiple of 128: every row is valid
+  const float2 c2 = make_float2(p.coef, p.coef);
+  float2 sq = make_float2(0.f, 0.f);
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    const int i0 = nb * BN + c * 32;
+    if (i0 >= p.Nn) break;  // uniform over the warp
+    uint32_t r[32];
+    __syncwarp();
+    tc::tmem_ld32(taddr + c * 32, r);
+    tc::tmem_ld_wait();
+    float g[32];
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      const float2 v = tc::mul2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), c2);
+      g[i] = v.x;
+      g[i + 1] = v.y;
+      sq = tc::fma2(v, v, sq);
+    }
+    if (p.dw != nullptr) {
+      float4* d = reinterpret_cast<float4*>(p.dw + o * p.Nn + i0);
+#pragma unroll
+      for (int v = 0; v < 8; ++v) d[v] = make_float4(g[4 * v], g[4 * v + 1], g[4 * v + 2], g[4 * v + 3]);
+    }
+  }
+  if (p.sqnorm != nullptr) {
+    const double t = warp_sum((double)sq.x + (double)sq.y);
+    if ((threadIdx.x & 31) == 0) atomicAdd(p.sqnorm, t);
   }
 }
 
@@ -315,8 +355,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + acc * BN;
       if (EPI == kEpiRope)
         epi_rope(p, taddr, mb, nb, row);
-      else
+      else if (EPI == kEpiLsq)
         epi_lsq(p, taddr, mb, nb, row);
+      else
+        epi_store(p, taddr, mb, nb, row);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->tempty[acc]);
@@ -441,6 +483,28 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.coef = coef;
   p.ds = ds;
   return launch_gemm<kEpiLsq, true, true>(ta, tb, p, st);
+}
+
+cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
+                                  int d, float coef, float* dw, double* sqnorm, int* status,
+                                  cudaStream_t st) {
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, x, true, d, N, d, BK))
+    return cudaErrorInvalidValue;
+  GemmParams p{};
+  p.M = D;
+  p.Nn = d;
+  p.K = (int)std::min<int64_t>(N, INT32_MAX);
+  p.num_m = D / BM;
+  p.num_n = (d + BN - 1) / BN;
+  p.k_blocks = (int)((N + BK - 1) / BK);
+  p.splits = 1;  // the stored tile and its squared norm need the whole sum over tokens
+  p.group_m = 8;
+  p.status = status;
+  p.coef = coef;
+  p.dw = dw;
+  p.sqnorm = sqnorm;
+  return launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
 }
 
 }  // namespace jab

@@ -27,6 +27,11 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
 cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st);
+// coef * dQKV^T X stored fp32 [D, d] (dw may be NULL) and its squared norm added to *sqnorm (may be
+// NULL; the caller zeroes it)
+cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
+                                  int d, float coef, float* dw, double* sqnorm, int* status,
+                                  cudaStream_t st);
 // attn_tc.cu
 int attn_fwd_tc_rows(int Hq, int Hkv);  // query rows per loss partial of the forward kernel
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);

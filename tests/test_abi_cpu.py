@@ -27,6 +27,7 @@ def libjab():
 def test_header_declares_the_boundary():
     syms = _declared_symbols()
     for name in ("jab_reference_forward", "jab_loss_forward", "jab_loss_backward_scales",
+                 "jab_loss_backward_weights",
                  "jab_workspace_size", "jab_quantize", "jab_init_scales", "jab_get_device_status",
                  "jab_status_string"):
         assert name in syms
@@ -53,6 +54,10 @@ def test_host_side_checks_without_gpu(libjab):
     # NULL pointers are rejected on the host before any CUDA call
     st = L.jab_loss_backward_scales(ctypes.byref(good), 2, 130, None, None, None, 3, None, 1.0,
                                     None, None, None, 0, None)
+    assert st == 1
+    # neither a gradient nor its norm requested
+    st = L.jab_loss_backward_weights(ctypes.byref(good), 2, 130, None, None, None, 2, None, None,
+                                     None, None, None, 0, None)
     assert st == 1
     st = L.jab_quantize(ctypes.byref(bad_dh), 3, None, None, None, None, None)
     assert st == 2

@@ -135,6 +135,55 @@ def test_backward_parity(name, bits):
     assert J().jab_get_device_status() == 0
 
 
+# ------------------------------------------------------------------ STE weight gradient, Fisher score
+@pytest.mark.parametrize("name,bits", [("gpt2_T200", 2), ("mistral_T130", 2), ("gqa2_T257", 3),
+                                       ("dh64_gqa4_B64_T256", 2)])
+def test_weight_gradient_and_fisher_coupling_score(name, bits):
+    """dL/dw_hat (App. B, STE) against the oracle's finite-difference-pinned gradient, and its squared
+    norm: with bits = 2 and absmax (round-to-nearest) scales, the Fisher-coupling score (App. B)."""
+    c = case(name)
+    ws = c.workspace()
+    A, _, _ = c.gpu_teacher(ws)
+    s = c.gpu_scales(bits, mode=0)
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    gw = torch.empty(c.W.shape, dtype=torch.float32, device="cuda")
+    sq = torch.empty(1, dtype=torch.float64, device="cuda")
+    J().jab_loss_backward_weights(c.desc, c.B, c.T, c.X, c.W, A, bits, s, loss, grad_w=gw,
+                                  grad_sqnorm=sq, ws=ws)
+    r = O.jab_loss_and_grad(c.x64, c.w64, s.cpu().numpy(), bits, c.odesc, a_ref=c.oracle_teacher(),
+                            kappa=1.0)
+    assert abs(loss.item() - r["loss"]) <= L_TOL * r["loss"]
+    g, go = np64(gw), r["grad_w_hat"]
+    assert cosine(g, go) >= COS_MIN, cosine(g, go)
+    # the norm matches the stored gradient's own (fp64 sum of the same fp32 values, other order) ...
+    np.testing.assert_allclose(sq.item(), (g ** 2).sum(), rtol=1e-5)
+    # ... and the oracle's within the gradient's error (|g|^2 = |go|^2 (1 + O(err^2)))
+    np.testing.assert_allclose(sq.item(), (go ** 2).sum(), rtol=2e-2)
+    # the score alone, without storing the gradient
+    sq2 = torch.empty(1, dtype=torch.float64, device="cuda")
+    J().jab_loss_backward_weights(c.desc, c.B, c.T, c.X, c.W, A, bits, s, loss, grad_sqnorm=sq2, ws=ws)
+    np.testing.assert_allclose(sq2.item(), sq.item(), rtol=1e-6)
+    assert J().jab_get_device_status() == 0
+
+
+def test_weight_gradient_vanishes_on_grid():
+    """Weights on the grid: student = teacher, so L = 0, dL/dw_hat = 0 and the score is 0 exactly."""
+    c = case("mistral_T130")
+    rng = np.random.default_rng(1)
+    q = rng.integers(-1, 2, size=c.W.shape)
+    W = torch.tensor(q * 2.0 ** -6, dtype=torch.bfloat16, device="cuda")
+    s = torch.full((c.D, c.shape.d_model // c.G), 2.0 ** -6, dtype=torch.float32, device="cuda")
+    ws = c.workspace()
+    A = torch.empty((c.B, c.T, c.Hq * c.dh), dtype=torch.float32, device="cuda")
+    J().jab_reference_forward(c.desc, c.B, c.T, c.X, W, A, ws)
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    gw = torch.full(W.shape, 7.0, dtype=torch.float32, device="cuda")
+    sq = torch.full((1,), 7.0, dtype=torch.float64, device="cuda")
+    J().jab_loss_backward_weights(c.desc, c.B, c.T, c.X, W, A, 2, s, loss, grad_w=gw, grad_sqnorm=sq,
+                                  ws=ws)
+    assert loss.item() == 0.0 and sq.item() == 0.0 and not gw.any()
+
+
 # ------------------------------------------------------------------ exact special cases
 def test_loss_exactly_zero_on_grid():
     """Weights on the grid: the student is the teacher bit for bit, so L = 0 and grad = 0."""
