@@ -259,6 +259,9 @@ def test_loss_zero_when_weights_on_grid():
     assert r["loss"] == 0.0 and r["sse"] == 0.0
     g = O.jab_loss_and_grad(x, w, s, 3, desc)
     assert g["loss"] == 0.0 and not g["grad_s"].any()
+    # the STE weight gradient vanishes identically at the float point (App. B, Fisher-coupling:
+    # why a gradient score needs an off-grid probe)
+    assert not g["grad_w_hat"].any()
 
 
 def test_single_token_closed_form():
