@@ -28,6 +28,10 @@ Readings of points the paper leaves open (each is stated where it is used):
   R7  RoPE is the rotate-half convention with inv_freq_j = theta^(-2j/d_h).
   R8  GQA: query head h reads key/value head floor(h / (Hq / Hkv)).
   R9  an all-zero group gets scale 1 at absmax init (any positive scale gives code 0).
+  R10 the KL term of Eq. 3 (not on the GPU path yet) is D_KL(P || Q(w)) with the implemented
+      batchmean convention: the sum over sequences, query heads, query rows and keys of
+      P log(P / Q), divided by B; P is the teacher's post-softmax map, Q the student's; masked
+      entries have P = Q = 0 and contribute nothing; lambda_KL defaults to 0.1 (Section 3).
 """
 from __future__ import annotations
 
@@ -37,7 +41,7 @@ __all__ = [
     "qmax_of", "expand_groups", "fp32_quotient", "quantize", "init_scales_absmax",
     "init_scales_minmse", "project", "rope_tables", "apply_rope", "apply_rope_transpose",
     "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
-    "jab_loss_and_grad", "lsq_factor", "default_kappa",
+    "jab_loss_and_grad", "lsq_factor", "default_kappa", "kl_attention_term", "jab_loss_joint",
 ]
 
 
@@ -246,6 +250,31 @@ def jab_loss(x, w, s, bits: int, desc: dict, a_ref=None):
     sse = float(sse_parts.sum())
     return dict(loss=sse / (B * T * Hq * dh), sse=sse, sse_parts=sse_parts, codes=codes,
                 w_hat=w_hat, a_ref=a_ref, a_hat=a_hat)
+
+
+def kl_attention_term(x, w, s, bits: int, desc: dict):
+    """D_KL(P || Q(w)), the second term of Eq. 3, batchmean as implemented (reading R10; App. B
+    "Effective weight of the KL term"). P and Q are the post-softmax maps of the block with the
+    float and with the quantized weights. Returns dict(kl, kl_rows [B, Hq, T], P, Q).
+    """
+    G = desc["group_size"]
+    _, w_hat, _ = quantize(w, s, bits, G)
+    _, teacher = block_forward(x, w, desc, return_parts=True)
+    _, student = block_forward(x, w_hat, desc, return_parts=True)
+    P, Q = teacher["P"], student["P"]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        terms = np.where(P > 0, P * (np.log(P) - np.log(Q)), 0.0)   # 0 log 0 = 0 on masked keys
+    kl_rows = terms.sum(axis=3)
+    B = x.shape[0]
+    return dict(kl=float(kl_rows.sum()) / B, kl_rows=kl_rows, P=P, Q=Q)
+
+
+def jab_loss_joint(x, w, s, bits: int, desc: dict, lam_kl: float = 0.1):
+    """Eq. 3 with both terms as implemented: the MSE mean (reading R3) plus lam_kl times the KL
+    batchmean (reading R10). Returns dict(loss, mse, kl)."""
+    mse = jab_loss(x, w, s, bits, desc)["loss"]
+    kl = kl_attention_term(x, w, s, bits, desc)["kl"]
+    return dict(loss=mse + lam_kl * kl, mse=mse, kl=kl)
 
 
 # --------------------------------------------------------------------------------------------

@@ -366,3 +366,75 @@ def test_kappa_is_a_pure_multiplier_and_default():
     g2 = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=0.0)
     np.testing.assert_allclose(g2["grad_s"], g1["grad_s"] / np.sqrt(4 * 3), rtol=1e-14)
     assert O.default_kappa(3, 128) == 1 / np.sqrt(128 * 3)
+
+
+# ------------------------------------------------------------------ KL term of Eq. 3 (reading R10)
+
+def _kl_case(seed=0, rope=True, bits=2, B=2, T=6):
+    desc, x, w = _tiny(seed=seed, rope=rope, B=B, T=T)
+    s = O.init_scales_absmax(w, bits, 4)
+    return desc, x, w, s
+
+
+@pytest.mark.parametrize("rope", [False, True])
+def test_kl_term_matches_library_relative_entropy(rope):
+    """sum(rel_entr(P, Q)) / B from scipy's elementwise relative entropy, per row and in total."""
+    special = pytest.importorskip("scipy.special")
+    desc, x, w, s = _kl_case(rope=rope)
+    r = O.kl_attention_term(x, w, s, 2, desc)
+    rows = special.rel_entr(r["P"], r["Q"]).sum(axis=3)
+    np.testing.assert_allclose(r["kl_rows"], rows, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(r["kl"], rows.sum() / x.shape[0], rtol=1e-12)
+    assert r["kl"] > 0.0
+
+
+def test_kl_row_logit_identity():
+    """With log P = s^T - lse^T and log Q = s^S - lse^S on the visible keys, and rows of P summing to
+    one: KL_row = sum_j P_j (s^T_j - s^S_j) + lse^S - lse^T (scores and lse taken from the teacher's
+    and the student's own forward passes)."""
+    desc, x, w, s = _kl_case(seed=3)
+    r = O.kl_attention_term(x, w, s, 2, desc)
+    _, w_hat, _ = O.quantize(w, s, 2, 4)
+    _, tp = O.block_forward(x, w, desc, return_parts=True)
+    _, sp = O.block_forward(x, w_hat, desc, return_parts=True)
+    scale = 1.0 / np.sqrt(desc["head_dim"])
+    B, T, Hq, _ = tp["q"].shape
+    for b in range(B):
+        for h in range(Hq):
+            g = h // (Hq // desc["n_kv_heads"])
+            st = tp["q"][b, :, h] @ tp["k"][b, :, g].T * scale
+            ss = sp["q"][b, :, h] @ sp["k"][b, :, g].T * scale
+            for t in range(T):
+                p = tp["P"][b, h, t, : t + 1]
+                kl = float(p @ (st[t, : t + 1] - ss[t, : t + 1])) + sp["lse"][b, h, t] - tp["lse"][b, h, t]
+                np.testing.assert_allclose(r["kl_rows"][b, h, t], kl, rtol=1e-9, atol=1e-14)
+
+
+def test_kl_zero_on_grid_and_for_a_single_token():
+    desc, x, _ = _tiny(rope=True)
+    rng = np.random.default_rng(5)
+    w = rng.integers(-3, 4, size=(16, 8)) * 2.0 ** -4
+    s = np.full((16, 2), 2.0 ** -4, dtype=np.float32)
+    assert O.kl_attention_term(x, w, s, 3, desc)["kl"] == 0.0           # student = teacher
+    desc1, x1, w1, s1 = _kl_case(T=1)
+    r = O.kl_attention_term(x1, w1, s1, 2, desc1)                          # one key: P = Q = 1
+    assert r["kl"] == 0.0 and not r["kl_rows"].any()
+
+
+def test_kl_nonnegative_rows_and_batchmean():
+    """Gibbs' inequality row by row; batchmean: repeating the batch leaves the value unchanged."""
+    for seed in range(4):
+        desc, x, w, s = _kl_case(seed=seed)
+        r = O.kl_attention_term(x, w, s, 2, desc)
+        assert (r["kl_rows"] >= -1e-15).all()
+        r2 = O.kl_attention_term(np.concatenate([x, x]), w, s, 2, desc)
+        np.testing.assert_allclose(r2["kl"], r["kl"], rtol=1e-12)
+        np.testing.assert_allclose(r2["kl_rows"].sum(), 2 * r["kl_rows"].sum(), rtol=1e-12)
+
+
+def test_joint_loss_is_mse_plus_weighted_kl():
+    desc, x, w, s = _kl_case(seed=2)
+    j0 = O.jab_loss_joint(x, w, s, 2, desc, lam_kl=0.0)
+    assert j0["loss"] == O.jab_loss(x, w, s, 2, desc)["loss"]
+    j = O.jab_loss_joint(x, w, s, 2, desc)                      # lambda_KL = 0.1 (Section 3)
+    np.testing.assert_allclose(j["loss"], j["mse"] + 0.1 * j["kl"], rtol=1e-15)
