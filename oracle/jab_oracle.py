@@ -28,10 +28,13 @@ Readings of points the paper leaves open (each is stated where it is used):
   R7  RoPE is the rotate-half convention with inv_freq_j = theta^(-2j/d_h).
   R8  GQA: query head h reads key/value head floor(h / (Hq / Hkv)).
   R9  an all-zero group gets scale 1 at absmax init (any positive scale gives code 0).
-  R10 the KL term of Eq. 3 (not on the GPU path yet) is D_KL(P || Q(w)) with the implemented
+  R18 the KL term of Eq. 3 (not on the GPU path yet) is D_KL(P || Q(w)) with the implemented
       batchmean convention: the sum over sequences, query heads, query rows and keys of
       P log(P / Q), divided by B; P is the teacher's post-softmax map, Q the student's; masked
       entries have P = Q = 0 and contribute nothing; lambda_KL defaults to 0.1 (Section 3).
+  R19 the sensitivity criterion (Section 2.4, Eq. 5-6, not on the GPU path yet) is taken for the
+      MSE term as normalised in R3 (lambda_KL = 0): at the float point H = 2 J_A^T J_A / n with
+      n = B*T*Hq*d_h, so v^T H v = 2 ||J_A v||^2 / n; the Rademacher probes are inputs.
 """
 from __future__ import annotations
 
@@ -42,6 +45,7 @@ __all__ = [
     "init_scales_minmse", "project", "rope_tables", "apply_rope", "apply_rope_transpose",
     "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
     "jab_loss_and_grad", "lsq_factor", "default_kappa", "kl_attention_term", "jab_loss_joint",
+    "attention_jvp", "block_jvp", "gn_quadratic_form", "hutchinson_trace", "omega_scores",
 ]
 
 
@@ -253,7 +257,7 @@ def jab_loss(x, w, s, bits: int, desc: dict, a_ref=None):
 
 
 def kl_attention_term(x, w, s, bits: int, desc: dict):
-    """D_KL(P || Q(w)), the second term of Eq. 3, batchmean as implemented (reading R10; App. B
+    """D_KL(P || Q(w)), the second term of Eq. 3, batchmean as implemented (reading R18; App. B
     "Effective weight of the KL term"). P and Q are the post-softmax maps of the block with the
     float and with the quantized weights. Returns dict(kl, kl_rows [B, Hq, T], P, Q).
     """
@@ -271,7 +275,7 @@ def kl_attention_term(x, w, s, bits: int, desc: dict):
 
 def jab_loss_joint(x, w, s, bits: int, desc: dict, lam_kl: float = 0.1):
     """Eq. 3 with both terms as implemented: the MSE mean (reading R3) plus lam_kl times the KL
-    batchmean (reading R10). Returns dict(loss, mse, kl)."""
+    batchmean (reading R18). Returns dict(loss, mse, kl)."""
     mse = jab_loss(x, w, s, bits, desc)["loss"]
     kl = kl_attention_term(x, w, s, bits, desc)["kl"]
     return dict(loss=mse + lam_kl * kl, mse=mse, kl=kl)
@@ -352,3 +356,64 @@ def jab_loss_and_grad(x, w, s, bits: int, desc: dict, a_ref=None, kappa: float =
     grad_s = kappa * (grad_w_hat * r).reshape(D, d // G, G).sum(axis=2)
     return dict(loss=sse / n_el, sse=sse, grad_s=grad_s, grad_w_hat=grad_w_hat, codes=codes,
                 w_hat=w_hat, a_ref=a_ref, a_hat=a_hat, lse=parts["lse"])
+
+
+# --------------------------------------------------------------------------------------------
+# 7. Sensitivity (Section 2.4, Eq. 5-6; reading R19): forward-mode products and Hutchinson
+# --------------------------------------------------------------------------------------------
+
+def attention_jvp(q, k, v, P, dq, dk, dv, scale: float):
+    """Jacobian-vector product of causal GQA attention (forward mode): with S = Q K^T * scale,
+    dS = (dQ K^T + Q dK^T) * scale on the visible keys, dP = P * (dS - rowsum(P * dS)) (softmax),
+    dO = dP V + P dV. Inputs as for attention_vjp, tangents dq [B,T,Hq,d_h], dk/dv [B,T,Hkv,d_h]."""
+    B, T, Hq, dh = q.shape
+    Hkv = k.shape[2]
+    mask = np.triu(np.ones((T, T), dtype=bool), k=1)
+    dO = np.empty_like(q)
+    for b in range(B):
+        for h in range(Hq):
+            g = _kv_head(h, Hq, Hkv)
+            Ph = P[b, h]
+            dS = (dq[b, :, h, :] @ k[b, :, g, :].T + q[b, :, h, :] @ dk[b, :, g, :].T) * scale
+            dS = np.where(mask, 0.0, dS)
+            dP = Ph * (dS - (Ph * dS).sum(axis=1, keepdims=True))
+            dO[b, :, h, :] = dP @ v[b, :, g, :] + Ph @ dv[b, :, g, :]
+    return dO
+
+
+def block_jvp(x: np.ndarray, w: np.ndarray, V: np.ndarray, desc: dict) -> np.ndarray:
+    """J_A V: the derivative of A(X; w) [B, T, Hq*d_h] along the weight direction V (shaped like w):
+    projection X V^T, the same RoPE rotation (linear), then the attention JVP."""
+    B, T, _ = x.shape
+    Hq, Hkv, dh = desc["n_q_heads"], desc["n_kv_heads"], desc["head_dim"]
+    _, parts = block_forward(x, w, desc, return_parts=True)
+    dq, dk, dv = split_heads(project(x, V), Hq, Hkv, dh)
+    if desc.get("use_rope", False):
+        cos, sin = rope_tables(T, dh, float(desc.get("rope_theta", 10000.0)))
+        dq = apply_rope(dq, cos, sin)
+        dk = apply_rope(dk, cos, sin)
+    dO = attention_jvp(parts["q"], parts["k"], parts["v"], parts["P"], dq, dk, dv,
+                       _softmax_scale(desc))
+    return dO.reshape(B, T, Hq * dh)
+
+
+def gn_quadratic_form(x, w, V, desc) -> float:
+    """v^T H v at the float point (Eq. 5, lambda_KL = 0): 2 ||J_A v||^2 / n (reading R19)."""
+    jv = block_jvp(x, w, V, desc)
+    return 2.0 * float((jv ** 2).sum()) / jv.size
+
+
+def hutchinson_trace(x, w, desc, probes) -> float:
+    """Tr(H) ~ (1/m) sum_i v_i^T H v_i over the given Rademacher probes [m, *w.shape] (Hutchinson
+    estimator, Section 2.4)."""
+    return float(np.mean([gn_quadratic_form(x, w, v, desc) for v in probes]))
+
+
+def omega_scores(trace: float, w: np.ndarray, s: np.ndarray, bits: int, group_size: int,
+                 layers_after: int = 0):
+    """Eq. 6: C1 Omega(b) = Tr(H) ||Q_b(W) - W||_F^2 and C2 = (L - i) Omega(b), with
+    layers_after = L - i. Returns (c1, c2)."""
+    _, w_hat, _ = quantize(w, s, bits, group_size)
+    c1 = trace * float(((w_hat - w) ** 2).sum())
+    return c1, layers_after * c1
+

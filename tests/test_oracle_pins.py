@@ -368,7 +368,7 @@ def test_kappa_is_a_pure_multiplier_and_default():
     assert O.default_kappa(3, 128) == 1 / np.sqrt(128 * 3)
 
 
-# ------------------------------------------------------------------ KL term of Eq. 3 (reading R10)
+# ------------------------------------------------------------------ KL term of Eq. 3 (reading R18)
 
 def _kl_case(seed=0, rope=True, bits=2, B=2, T=6):
     desc, x, w = _tiny(seed=seed, rope=rope, B=B, T=T)
@@ -438,3 +438,80 @@ def test_joint_loss_is_mse_plus_weighted_kl():
     assert j0["loss"] == O.jab_loss(x, w, s, 2, desc)["loss"]
     j = O.jab_loss_joint(x, w, s, 2, desc)                      # lambda_KL = 0.1 (Section 3)
     np.testing.assert_allclose(j["loss"], j["mse"] + 0.1 * j["kl"], rtol=1e-15)
+
+
+# ------------------------------------------------------------------ sensitivity (Section 2.4, R19)
+
+@pytest.mark.parametrize("rope,Hq,Hkv", [(False, 2, 1), (True, 2, 2), (True, 4, 2)])
+def test_block_jvp_matches_central_differences(rope, Hq, Hkv):
+    desc, x, w = _tiny(seed=7, rope=rope, Hq=Hq, Hkv=Hkv)
+    V = np.random.default_rng(8).standard_normal(w.shape)
+    h = 1e-6
+    fd = (O.block_forward(x, w + h * V, desc) - O.block_forward(x, w - h * V, desc)) / (2 * h)
+    np.testing.assert_allclose(O.block_jvp(x, w, V, desc), fd, rtol=1e-6, atol=1e-9)
+
+
+def test_gn_quadratic_form_is_the_second_difference_of_the_loss():
+    """At the float point L(w* + eps v) = eps^2 v^T H v / 2 + O(eps^3) (L and its gradient vanish
+    there), so the symmetric second difference (L(eps) + L(-eps)) / eps^2 gives v^T H v."""
+    desc, x, w = _tiny(seed=9, rope=True)
+    a_ref = O.block_forward(x, w, desc)
+    V = np.random.default_rng(10).standard_normal(w.shape)
+
+    def loss(e):
+        return float(((O.block_forward(x, w + e * V, desc) - a_ref) ** 2).mean())
+
+    eps = 1e-3
+    np.testing.assert_allclose((loss(eps) + loss(-eps)) / eps ** 2, O.gn_quadratic_form(x, w, V, desc),
+                               rtol=1e-4)
+
+
+def test_hutchinson_trace_matches_the_exact_trace():
+    """Exact Tr(H) = 2 sum_k ||J e_k||^2 / n from a central-difference Jacobian; the estimator over
+    m Rademacher probes lies within 5 standard errors, sqrt(2 sum_{i != j} H_ij^2 / m)."""
+    desc = _desc(4, 1, 1, 2, 4, rope=True)
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((1, 6, 4))
+    w = rng.standard_normal((6, 4)) * 0.6
+    n_w = w.size
+    J = np.empty((6 * 2, n_w))
+    h = 1e-6
+    for i in range(n_w):
+        e = np.zeros(n_w)
+        e[i] = h
+        J[:, i] = ((O.block_forward(x, w + e.reshape(w.shape), desc) -
+                    O.block_forward(x, w - e.reshape(w.shape), desc)) / (2 * h)).ravel()
+    H = 2.0 * J.T @ J / J.shape[0]
+    m = 3000
+    probes = rng.choice([-1.0, 1.0], size=(m,) + w.shape)
+    est = O.hutchinson_trace(x, w, desc, probes)
+    off = H - np.diag(np.diag(H))
+    se = np.sqrt(2.0 * (off ** 2).sum() / m)
+    assert abs(est - np.trace(H)) <= 5 * se, (est, np.trace(H), se)
+    # one probe direction against the explicit quadratic form
+    np.testing.assert_allclose(O.gn_quadratic_form(x, w, probes[0], desc),
+                               probes[0].ravel() @ H @ probes[0].ravel(), rtol=1e-6)
+
+
+def test_gn_quadratic_form_vanishes_on_the_query_key_scaling_direction():
+    """W_Q (1 + e), W_K / (1 + e) leaves A unchanged (RoPE commutes with the scalar), so its tangent
+    (W_Q, -W_K, 0) is in the null space of J_A and of H (Section 2.3)."""
+    desc, x, w = _tiny(seed=13, rope=True)
+    nq = desc["n_q_heads"] * desc["head_dim"]
+    nk = desc["n_kv_heads"] * desc["head_dim"]
+    V = np.zeros_like(w)
+    V[:nq] = w[:nq]
+    V[nq:nq + nk] = -w[nq:nq + nk]
+    ref = O.gn_quadratic_form(x, w, np.random.default_rng(14).standard_normal(w.shape), desc)
+    assert O.gn_quadratic_form(x, w, V, desc) <= 1e-12 * ref
+
+
+def test_omega_scores_vanish_on_the_grid_and_scale_with_depth():
+    desc, _, _ = _tiny()
+    rng = np.random.default_rng(15)
+    w = rng.integers(-3, 4, size=(16, 8)) * 2.0 ** -4
+    s = np.full((16, 2), 2.0 ** -4, dtype=np.float32)
+    assert O.omega_scores(2.5, w, s, 3, 4, layers_after=3) == (0.0, 0.0)
+    w2 = w + rng.standard_normal(w.shape) * 2.0 ** -7
+    c1, c2 = O.omega_scores(2.5, w2, s, 3, 4, layers_after=3)
+    assert c1 > 0 and c2 == 3 * c1
