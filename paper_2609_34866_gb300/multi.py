@@ -52,3 +52,16 @@ def combine_shards(loss: torch.Tensor, grad: torch.Tensor, n_local: int, n_total
         dist.all_reduce(loss)
         dist.all_reduce(grad)
     return loss, grad
+
+
+def fisher_score_from_shards(grad_w: torch.Tensor, n_local: int, n_total: int) -> float:
+    """Fisher-coupling score of one evaluation whose sequences are sharded over the ranks: the weight
+    gradient dL/dw_hat (jab_loss_backward_weights' grad_w of this rank's shard) is additive over
+    sequences like the scale gradient, but its squared norm is not, so the shards' gradients are
+    combined first (one all-reduce of D x d floats, in place) and the norm is taken of the sum."""
+    import torch.distributed as dist
+    grad_w.mul_(float(n_local) / float(n_total))
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(grad_w)
+    return float((grad_w.double() ** 2).sum())
+

@@ -1,6 +1,7 @@
 """Multi-process host logic on CPU with the gloo backend, world size 2: sequence sharding of one
 evaluation (size-weighted all-reduce equals the full batch, computed here with the oracle on each
-shard) and the max-over-ranks timing reduction used by bench.py."""
+shard), the Fisher-coupling score of a sharded evaluation (norm of the combined weight gradient),
+and the max-over-ranks timing reduction used by bench.py."""
 import os
 import socket
 
@@ -25,7 +26,8 @@ def _worker(rank, world, port, out):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
         from oracle import jab_oracle as O
-        from paper_2609_34866_gb300.multi import (combine_shards, dist_env, max_over_ranks,
+        from paper_2609_34866_gb300.multi import (combine_shards, dist_env,
+                                                  fisher_score_from_shards, max_over_ranks,
                                                   shard_sequences)
         assert dist_env() == (world, rank, rank)
         rng = np.random.default_rng(0)
@@ -40,6 +42,8 @@ def _worker(rank, world, port, out):
         loss = torch.tensor([r["loss"]], dtype=torch.float64)
         grad = torch.tensor(r["grad_s"], dtype=torch.float64)
         combine_shards(loss, grad, b - a, B)
+        gw = torch.tensor(r["grad_w_hat"], dtype=torch.float64)
+        score = fisher_score_from_shards(gw, b - a, B)
         t = max_over_ranks(10.0 + rank)
         if rank == 0:
             full = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=1.0)
@@ -47,6 +51,7 @@ def _worker(rank, world, port, out):
             out["grad"] = float(np.abs(grad.numpy() - full["grad_s"]).max() /
                                 np.abs(full["grad_s"]).max())
             out["tmax"] = t
+            out["score"] = (score, float((full["grad_w_hat"] ** 2).sum()))
     finally:
         dist.destroy_process_group()
 
@@ -71,3 +76,5 @@ def test_sharded_evaluation_matches_full_batch_gloo_world2():
         np.testing.assert_allclose(loss_sharded, loss_full, rtol=1e-12)
         assert out["grad"] < 1e-12
         assert out["tmax"] == 11.0
+        score_sharded, score_full = out["score"]
+        np.testing.assert_allclose(score_sharded, score_full, rtol=1e-12)
