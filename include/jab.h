@@ -124,6 +124,29 @@ jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int3
                                      float* grad_w_dev, double* grad_sqnorm_dev, void* ws,
                                      size_t ws_bytes, jab_stream_t stream);
 
+/* Bit-width allocation over L layers (Section 2.4, Eq. 7; App. B "Allocators"). Host code only: no
+ * device memory, no CUDA call, synchronous.
+ * Minimises sum_i omega[i, b_i] subject to sum_i n_i b_i <= avg_bits * sum_i n_i.
+ * The walk (App. B "Allocators"):
+ *   - every layer starts at its highest width;
+ *   - while over budget, apply the one-step downgrade with the least score increase per bit saved;
+ *   - then, while one fits and lowers the total, apply the one-step upgrade with the largest score
+ *     decrease per bit.
+ * Ties go to the lowest layer index.
+ *   omega_host      fp64 [L, n_widths]  finite score of layer i at widths_host[k]: direct L_JAB
+ *                                       (jab_loss_forward), or Omega C1 / C2 of Eq. 6
+ *   widths_host     int32 [n_widths]    strictly increasing bit widths, e.g. {2, 3, 4, 8, 16}
+ *   n_weights_host  int64 [L]           weights of each layer: a layer at width b costs n_i * b bits
+ *   avg_bits        average bits per weight allowed
+ *   method          0: walk over every width (greedy); 1: walk over each layer's Pareto-efficient
+ *                   points only (a point is dropped when a cheaper one scores no worse)
+ *   bits_out_host   out int32 [L]
+ * Returns JAB_ERR_INVALID_ARG for NULL pointers, sizes < 1, non-increasing widths, non-finite
+ * scores, or a budget below the cost of every layer at its lowest width. */
+jab_status jab_allocate_bits(const double* omega_host, const int32_t* widths_host,
+                             const int64_t* n_weights_host, int32_t L, int32_t n_widths,
+                             double avg_bits, int32_t method, int32_t* bits_out_host);
+
 /* Quantiser alone (Section 2.1, Eq. 2): v = fl32(w / s), q = clip(round-half-even(v), -qmax, qmax).
  *   codes_dev      out int8 [(Hq+2Hkv)*d_h, d_model] or NULL
  *   w_hat_dev      out fp32 [(Hq+2Hkv)*d_h, d_model] or NULL   fl32(q * s) */

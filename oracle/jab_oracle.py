@@ -35,6 +35,11 @@ Readings of points the paper leaves open (each is stated where it is used):
   R19 the sensitivity criterion (Section 2.4, Eq. 5-6, not on the GPU path yet) is taken for the
       MSE term as normalised in R3 (lambda_KL = 0): at the float point H = 2 J_A^T J_A / n with
       n = B*T*Hq*d_h, so v^T H v = 2 ||J_A v||^2 / n; the Rademacher probes are inputs.
+  R20 allocation (Section 2.4, Eq. 7; App. B "Allocators"): layer i at width b costs n_i * b bits and
+      the budget is avg_bits * sum_i n_i; each greedy step moves one layer to the adjacent width of
+      its candidate list; the step ratio is dOmega / dcost in float64; ties go to the lowest layer
+      index; after the budget is met, upgrades are applied while one fits and lowers sum Omega
+      (best gain per bit first). The Pareto variant walks each layer's non-dominated points only.
 """
 from __future__ import annotations
 
@@ -46,6 +51,7 @@ __all__ = [
     "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
     "jab_loss_and_grad", "lsq_factor", "default_kappa", "kl_attention_term", "jab_loss_joint",
     "attention_jvp", "block_jvp", "gn_quadratic_form", "hutchinson_trace", "omega_scores",
+    "pareto_frontier", "allocate_bits",
 ]
 
 
@@ -416,4 +422,75 @@ def omega_scores(trace: float, w: np.ndarray, s: np.ndarray, bits: int, group_si
     _, w_hat, _ = quantize(w, s, bits, group_size)
     c1 = trace * float(((w_hat - w) ** 2).sum())
     return c1, layers_after * c1
+
+
+# --------------------------------------------------------------------------------------------
+# 8. Allocation (Section 2.4, Eq. 7; App. B "Allocators"; reading R20)
+# --------------------------------------------------------------------------------------------
+
+def pareto_frontier(costs, omegas):
+    """Indices of the non-dominated points of one layer, given in increasing cost: point k is kept
+    when every cheaper point has a strictly larger Omega."""
+    keep, best = [], None
+    for k, om in enumerate(omegas):
+        if best is None or om < best:
+            keep.append(k)
+            best = om
+    return keep
+
+
+def allocate_bits(omega, widths, n_weights, avg_bits: float, method: str = "greedy"):
+    """min sum_i Omega_i(b_i) s.t. sum_i n_i b_i <= avg_bits * sum_i n_i (Eq. 7), by the greedy walk
+    (method "greedy") or the same walk on each layer's Pareto frontier ("pareto"). omega [L, K] for
+    the increasing widths [K]. Returns the chosen width of every layer."""
+    omega = [[float(v) for v in row] for row in omega]
+    widths = [int(b) for b in widths]
+    n = [int(v) for v in n_weights]
+    L = len(omega)
+    budget = float(avg_bits) * float(sum(n))
+    if method == "greedy":
+        cand = [list(range(len(widths))) for _ in range(L)]
+    elif method == "pareto":
+        cand = [pareto_frontier([n[i] * b for b in widths], omega[i]) for i in range(L)]
+    else:
+        raise ValueError(method)
+    if sum(n[i] * widths[cand[i][0]] for i in range(L)) > budget:
+        raise ValueError("budget below the cheapest allocation")
+    pos = [len(c) - 1 for c in cand]                       # start at the highest width
+    cost = sum(n[i] * widths[cand[i][pos[i]]] for i in range(L))
+
+    def width(i, p):
+        return widths[cand[i][p]]
+
+    def om(i, p):
+        return omega[i][cand[i][p]]
+
+    while cost > budget:                                   # downgrades: least damage per bit saved
+        best, pick = None, None
+        for i in range(L):
+            if pos[i] == 0:
+                continue
+            dc = n[i] * (width(i, pos[i]) - width(i, pos[i] - 1))
+            r = (om(i, pos[i] - 1) - om(i, pos[i])) / dc
+            if best is None or r < best:
+                best, pick = r, i
+        cost -= n[pick] * (width(pick, pos[pick]) - width(pick, pos[pick] - 1))
+        pos[pick] -= 1
+    while True:                                            # leftovers: best gain per bit that fits
+        best, pick = None, None
+        for i in range(L):
+            if pos[i] + 1 == len(cand[i]):
+                continue
+            dc = n[i] * (width(i, pos[i] + 1) - width(i, pos[i]))
+            gain = om(i, pos[i]) - om(i, pos[i] + 1)
+            if cost + dc > budget or not gain > 0:
+                continue
+            r = gain / dc
+            if best is None or r > best:
+                best, pick = r, i
+        if pick is None:
+            break
+        cost += n[pick] * (width(pick, pos[pick] + 1) - width(pick, pos[pick]))
+        pos[pick] += 1
+    return [width(i, pos[i]) for i in range(L)]
 

@@ -9,7 +9,7 @@ Python or CPU fallback.
 from .binding import (  # noqa: F401
     BlockDesc, JabError, JAB_OK, desc_from_shape, lib, lib_path, jab_workspace_size,
     jab_reference_forward, jab_loss_forward, jab_loss_forward_noalloc, jab_loss_backward_scales,
-    jab_loss_backward_weights, jab_quantize,
+    jab_loss_backward_weights, jab_allocate_bits, jab_quantize,
     jab_init_scales, jab_get_device_status, jab_status_string, Workspace, jab_timing_enable,
     jab_timing_reset, jab_timing_read, jab_selftest_wait_timeout,
 )

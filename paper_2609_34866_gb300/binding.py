@@ -76,6 +76,7 @@ def lib() -> ctypes.CDLL:
     L.jab_loss_backward_scales.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P, _P, sz, _P]
     L.jab_loss_backward_weights.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, _P, _P, _P, _P, sz, _P]
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
+    L.jab_allocate_bits.argtypes = [_P, _P, _P, i32, i32, ctypes.c_double, i32, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
     L.jab_get_device_status.argtypes = [_P]
     L.jab_selftest_wait_timeout.argtypes = [_P]
@@ -89,7 +90,7 @@ def lib() -> ctypes.CDLL:
                                  ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
     L.jab_timing_reset.argtypes = []
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
-               "jab_loss_backward_scales", "jab_loss_backward_weights",
+               "jab_loss_backward_scales", "jab_loss_backward_weights", "jab_allocate_bits",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
                "jab_selftest_wait_timeout",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
@@ -209,6 +210,25 @@ def jab_loss_backward_weights(desc, B, T, X, W, A_ref, bits: int, scales, loss, 
         _ptr(loss, torch.float64, "loss"), _ptr(grad_w, torch.float32, "grad_w"),
         _ptr(grad_sqnorm, torch.float64, "grad_sqnorm"), ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "jab_loss_backward_weights")
+
+
+def jab_allocate_bits(omega, widths, n_weights, avg_bits: float, method: str = "greedy"):
+    """Width per layer minimising the summed score within avg_bits per weight (Eq. 7). Host only.
+
+    omega: [L, K] scores (any array-like of floats); widths: K increasing ints; n_weights: L ints.
+    method: "greedy" or "pareto". Returns a list of L widths."""
+    import numpy as np
+    om = np.ascontiguousarray(np.asarray(omega, dtype=np.float64))
+    w = np.ascontiguousarray(np.asarray(widths, dtype=np.int32))
+    n = np.ascontiguousarray(np.asarray(n_weights, dtype=np.int64))
+    if om.ndim != 2 or om.shape != (n.size, w.size):
+        raise ValueError("omega must be [len(n_weights), len(widths)]")
+    out = np.zeros(n.size, dtype=np.int32)
+    st = lib().jab_allocate_bits(om.ctypes.data, w.ctypes.data, n.ctypes.data, int(n.size),
+                                 int(w.size), float(avg_bits), {"greedy": 0, "pareto": 1}[method],
+                                 out.ctypes.data)
+    _check(st, "jab_allocate_bits")
+    return [int(b) for b in out]
 
 
 def jab_quantize(desc, bits, W, scales, codes=None, w_hat=None, stream=None):

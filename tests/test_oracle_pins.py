@@ -515,3 +515,79 @@ def test_omega_scores_vanish_on_the_grid_and_scale_with_depth():
     w2 = w + rng.standard_normal(w.shape) * 2.0 ** -7
     c1, c2 = O.omega_scores(2.5, w2, s, 3, 4, layers_after=3)
     assert c1 > 0 and c2 == 3 * c1
+
+
+# ------------------------------------------------------------------ allocation (Eq. 7, App. B, R20)
+
+def test_allocation_hand_worked_example():
+    """Widths (2, 4, 8), 10 weights per layer, 4 bits on average (80 bits). From (8, 8), 160 bits:
+    layer 0 8 -> 4 costs (2 - 1) / 40 = 0.025 per bit against (3 - 0.5) / 40 = 0.0625 for layer 1,
+    then layer 1 8 -> 4 (0.0625 < (5 - 2) / 20 = 0.15) meets 80 bits; no upgrade fits."""
+    om = [[5.0, 2.0, 1.0], [9.0, 3.0, 0.5]]
+    for method in ("greedy", "pareto"):
+        assert O.allocate_bits(om, [2, 4, 8], [10, 10], 4.0, method) == [4, 4]
+    # 5 bits on average (100 bits): the leftover 20 bits cannot buy an 8-bit layer (+40)
+    assert O.allocate_bits(om, [2, 4, 8], [10, 10], 5.0) == [4, 4]
+    # 6 bits (120): after layer 0's first step the budget holds at (4, 8)
+    assert O.allocate_bits(om, [2, 4, 8], [10, 10], 6.0) == [4, 8]
+
+
+def test_allocation_extremes_and_infeasible_budget():
+    rng = np.random.default_rng(20)
+    om = np.sort(rng.random((5, 4)), axis=1)[:, ::-1]
+    n = rng.integers(1, 100, size=5)
+    assert O.allocate_bits(om, [2, 3, 4, 8], n, 8.0) == [8] * 5
+    assert O.allocate_bits(om, [2, 3, 4, 8], n, 2.0) == [2] * 5
+    with pytest.raises(ValueError):
+        O.allocate_bits(om, [2, 3, 4, 8], n, 1.99)
+
+
+def test_greedy_is_optimal_for_convex_scores_with_unit_steps():
+    """Marginal analysis: for separable convex, decreasing scores and equal cost steps (widths one
+    bit apart, one weight per layer), the greedy walk reaches the exhaustive-search optimum."""
+    import itertools
+    rng = np.random.default_rng(21)
+    widths = [2, 3, 4, 5, 6]
+    for _ in range(40):
+        L = int(rng.integers(2, 5))
+        steps = np.sort(rng.random((L, len(widths) - 1)), axis=1)[:, ::-1]   # shrinking decrements
+        om = np.concatenate([np.zeros((L, 1)), -np.cumsum(steps, axis=1)], axis=1) + 10.0
+        budget = int(rng.integers(2 * L, 6 * L + 1))
+        got = O.allocate_bits(om, widths, [1] * L, budget / L)
+        best = min(sum(om[i][widths.index(b)] for i, b in enumerate(c))
+                   for c in itertools.product(widths, repeat=L) if sum(c) <= budget)
+        assert sum(got) <= budget
+        np.testing.assert_allclose(sum(om[i][widths.index(b)] for i, b in enumerate(got)), best,
+                                   rtol=1e-12)
+
+
+def test_greedy_result_is_feasible_and_admits_no_improving_upgrade():
+    rng = np.random.default_rng(22)
+    widths = [2, 3, 4, 8, 16]
+    for _ in range(50):
+        L = int(rng.integers(1, 7))
+        om = rng.random((L, len(widths))) * rng.random()
+        n = rng.integers(1, 50, size=L)
+        avg = float(rng.uniform(2.0, 16.0))
+        for method in ("greedy", "pareto"):
+            got = O.allocate_bits(om, widths, n, avg, method)
+            cost = sum(int(n[i]) * b for i, b in enumerate(got))
+            assert cost <= avg * n.sum()
+            if method == "greedy":
+                for i, b in enumerate(got):      # every single upgrade either does not fit or does not help
+                    k = widths.index(b)
+                    if k + 1 < len(widths):
+                        fits = cost + int(n[i]) * (widths[k + 1] - b) <= avg * n.sum()
+                        assert not (fits and om[i][k + 1] < om[i][k])
+
+
+def test_pareto_frontier_keeps_exactly_the_non_dominated_points():
+    rng = np.random.default_rng(23)
+    for _ in range(100):
+        K = int(rng.integers(1, 7))
+        costs = np.sort(rng.choice(100, size=K, replace=False))
+        oms = rng.integers(0, 5, size=K).astype(float)                 # ties on purpose
+        kept = O.pareto_frontier(costs, oms)
+        brute = [k for k in range(K)
+                 if not any(j != k and costs[j] <= costs[k] and oms[j] <= oms[k] for j in range(K))]
+        assert kept == brute
