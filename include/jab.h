@@ -126,7 +126,8 @@ jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int3
 
 /* Bit-width allocation over L layers (Section 2.4, Eq. 7; App. B "Allocators"). Host code only: no
  * device memory, no CUDA call, synchronous.
- * Minimises sum_i omega[i, b_i] subject to sum_i n_i b_i <= avg_bits * sum_i n_i.
+ * Minimises sum_i omega[i, b_i] subject to sum_i n_i b_i <= avg_bits * sum_i n_i (the parameter-
+ * weighted budget of Eq. 8: c(b_i) = n_i b_i).
  * The walk (App. B "Allocators"):
  *   - every layer starts at its highest width;
  *   - while over budget, apply the one-step downgrade with the least score increase per bit saved;

@@ -36,7 +36,7 @@ Readings of points the paper leaves open (each is stated where it is used):
       MSE term as normalised in R3 (lambda_KL = 0): at the float point H = 2 J_A^T J_A / n with
       n = B*T*Hq*d_h, so v^T H v = 2 ||J_A v||^2 / n; the Rademacher probes are inputs.
   R20 allocation (Section 2.4, Eq. 7; App. B "Allocators"): layer i at width b costs n_i * b bits and
-      the budget is avg_bits * sum_i n_i; each greedy step moves one layer to the adjacent width of
+      the budget is avg_bits * sum_i n_i (the parameter-weighted budget of Eq. 8); each greedy step moves one layer to the adjacent width of
       its candidate list; the step ratio is dOmega / dcost in float64; ties go to the lowest layer
       index; after the budget is met, upgrades are applied while one fits and lowers sum Omega
       (best gain per bit first). The Pareto variant walks each layer's non-dominated points only.

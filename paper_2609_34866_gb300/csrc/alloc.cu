@@ -1,7 +1,7 @@
 // Bit-width allocation over layers (Section 2.4, Eq. 7; App. B "Allocators"): host code only, no
 // device memory and no CUDA call. It consumes a score table Omega[layer][width] (direct L_JAB from
 // jab_loss_forward, or the C1 / C2 scores of Eq. 6) and solves
-//   min sum_i Omega_i(b_i)   s.t.   sum_i n_i b_i <= avg_bits * sum_i n_i
+//   min sum_i Omega_i(b_i)   s.t.   sum_i n_i b_i <= avg_bits * sum_i n_i   (cost of Eq. 8)
 // by the greedy walk of App. B: every layer starts at its highest width; while over budget, the
 // one-step downgrade with the least score increase per bit saved is applied; then, while one fits,
 // the one-step upgrade with the largest score decrease per bit is applied. The Pareto variant runs
