@@ -48,7 +48,9 @@ typedef enum {
   JAB_ERR_UNSUPPORTED = 2,   /* shape outside the supported set above                            */
   JAB_ERR_CUDA = 3,          /* a CUDA runtime call or kernel launch failed                      */
   JAB_ERR_NONFINITE = 4,     /* device: scale <= 0 or non-finite, or a non-finite result          */
-  JAB_ERR_RANGE = 5,         /* device: an input value is outside the fp16 range (|x| > 65504)   */
+  JAB_ERR_RANGE = 5,         /* device: a value does not fit the fp16 tensor-core operands: X, the
+                                quantised weights, the projected Q|K|V or the output error dO
+                                (|x| > 65504 after rounding)                                    */
   JAB_ERR_TIMEOUT = 6,       /* device: a bounded wait in a pipelined kernel gave up             */
   JAB_ERR_SCRATCH_LIMIT = 7  /* jab_loss_forward_noalloc: the problem needs more scratch than the
                                 fixed JAB_NOALLOC_SCRATCH_BYTES                                    */
@@ -96,6 +98,35 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
                             double* loss_dev, double* sse_parts_dev, void* ws, size_t ws_bytes,
                             jab_stream_t stream);
 
+/* Teacher projection for the KL term of Eq. 3: the rotated [Q | K | V] = RoPE(X W^T) of the block
+ * with its float weights, in fp16 (the operand type of the tensor-core path), computed once per
+ * block like A_ref. Only its Q and K columns are read by jab_loss_forward_kl.
+ *   QKV_ref_dev    out fp16 [B, T, (Hq + 2 Hkv) * d_h], 16-byte aligned
+ *   ws             at least jab_workspace_size(desc, B, T, 1, 0) bytes
+ * A projected value outside the fp16 range raises JAB_ERR_RANGE on the device. */
+jab_status jab_reference_projection(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, void* QKV_ref_dev,
+                                    void* ws, size_t ws_bytes, jab_stream_t stream);
+
+/* Forward L_JAB with both terms of Eq. 3 for n_cand candidates: the MSE term of jab_loss_forward
+ * plus lambda_kl times the KL attention-map term D_KL(P || Q) between the teacher's post-softmax
+ * map P and each candidate's map Q, with the batchmean normalisation the paper implements (App. B
+ * "Effective weight of the KL term"): the sum over sequences, query heads, query rows and visible
+ * keys of P log(P / Q), divided by B. The paper's default is lambda_kl = 0.1 (Section 3).
+ *   QKV_ref_dev    fp16 [B, T, D] from jab_reference_projection for the same X and W
+ *   lambda_kl      >= 0
+ *   loss_dev       out fp64 [n_cand]   mse + lambda_kl * kl
+ *   mse_dev        out fp64 [n_cand] or NULL   the MSE term (as jab_loss_forward's loss)
+ *   kl_dev         out fp64 [n_cand] or NULL   the KL term
+ *   kl_rows_dev    out fp32 [n_cand, B, Hq, T] or NULL   KL of every query row (nats)
+ * Other arguments as for jab_loss_forward; ws of jab_workspace_size(desc, B, T, n_cand, 0). */
+jab_status jab_loss_forward_kl(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                               const void* W_dev, const float* A_ref_dev, const void* QKV_ref_dev,
+                               int32_t n_cand, const int32_t* bits_host,
+                               const float* const* scales_host, float lambda_kl, double* loss_dev,
+                               double* mse_dev, double* kl_dev, float* kl_rows_dev, void* ws,
+                               size_t ws_bytes, jab_stream_t stream);
+
 /* Forward L_JAB and its gradient w.r.t. the scales for one candidate (App. B "Joint STE fine-tuning",
  * Eq. 13): d w_hat / d w = 1 (STE) and d w_hat / d s = q - v if |v| <= qmax, else sign(v) qmax, with
  * v = w / s.
@@ -108,6 +139,24 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
                                     double* loss_dev, float* grad_scales_dev, void* ws,
                                     size_t ws_bytes, jab_stream_t stream);
 
+/* The STE fitting loop (App. B "Joint STE fine-tuning": 200 steps per block on one fixed calibration
+ * batch) evaluates the same X at every step. jab_prepare_x converts X once into the fp16 copy that
+ * the projection reads, kept in `ws`; jab_loss_backward_scales_prepared is then
+ * jab_loss_backward_scales without that conversion. Its arguments and results are those of
+ * jab_loss_backward_scales; X_dev must be the same pointer (with the same contents, B and T) as in
+ * the last call that converted X into this workspace (jab_prepare_x or any entry point taking X),
+ * otherwise it returns JAB_ERR_INVALID_ARG. X_dev is still read (in bf16) by the weight-gradient
+ * GEMM. jab_prepare_x: ws of at least jab_workspace_size(desc, B, T, 1, 0) bytes; X out of the
+ * fp16 range raises JAB_ERR_RANGE on the device. */
+jab_status jab_prepare_x(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                         void* ws, size_t ws_bytes, jab_stream_t stream);
+jab_status jab_loss_backward_scales_prepared(const jab_block_desc* desc, int32_t B, int32_t T,
+                                             const void* X_dev, const void* W_dev,
+                                             const float* A_ref_dev, int32_t bits,
+                                             const float* scales_dev, float kappa,
+                                             double* loss_dev, float* grad_scales_dev, void* ws,
+                                             size_t ws_bytes, jab_stream_t stream);
+
 /* Forward L_JAB and the STE weight gradient for one candidate (App. B "Joint STE fine-tuning":
  * d w_hat / d w = 1, so dL/dW = dL/dw_hat), and its squared Frobenius norm: the Fisher-coupling score
  * of App. B "Fisher-coupling" when called with bits = 2 and round-to-nearest scales
@@ -117,7 +166,7 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
  *                                                               last bits may differ between calls)
  *   loss_dev        out fp64 [1]
  * At least one of grad_w_dev and grad_sqnorm_dev must be non-NULL. Uses the with_bwd workspace of
- * jab_workspace_size. Returns JAB_ERR_UNSUPPORTED on the CUDA-core path (JAB_PATH=simple). */
+ * jab_workspace_size. */
 jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int32_t T,
                                      const void* X_dev, const void* W_dev, const float* A_ref_dev,
                                      int32_t bits, const float* scales_dev, double* loss_dev,
@@ -154,6 +203,15 @@ jab_status jab_allocate_bits(const double* omega_host, const int32_t* widths_hos
 jab_status jab_quantize(const jab_block_desc* desc, int32_t bits, const void* W_dev,
                         const float* scales_dev, int8_t* codes_dev, float* w_hat_dev,
                         jab_stream_t stream);
+
+/* Flip count (App. B "Joint STE fine-tuning", Eq. 15): the number of grid positions whose code
+ * differs between two code arrays of the same weights, e.g. after and before fine-tuning (codes
+ * from jab_quantize). The flip rate is *count_dev / n.
+ *   codes_a_dev, codes_b_dev  int8 [n], 16-byte aligned (may be NULL when n = 0)
+ *   count_dev                 out int64 [1], 8-byte aligned (exact integer count; the same on
+ *                             every call) */
+jab_status jab_flip_rate(const int8_t* codes_a_dev, const int8_t* codes_b_dev, int64_t n,
+                         int64_t* count_dev, jab_stream_t stream);
 
 /* Starting scales. mode 0: max_{i in g}|w| / qmax (an all-zero group gets 1). mode 1: the per-group
  * min-MSE search over s_k = fl32(s_0 * (100 - k) / 100), k = 0..79, minimising

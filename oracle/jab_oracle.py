@@ -35,6 +35,9 @@ Readings of points the paper leaves open (each is stated where it is used):
   R19 the sensitivity criterion (Section 2.4, Eq. 5-6, not on the GPU path yet) is taken for the
       MSE term as normalised in R3 (lambda_KL = 0): at the float point H = 2 J_A^T J_A / n with
       n = B*T*Hq*d_h, so v^T H v = 2 ||J_A v||^2 / n; the Rademacher probes are inputs.
+  R21 the flip rate of Eq. 15 counts the grid positions (the clamped codes of Eq. 2, i.e. the
+      deployed values) that differ between two quantizations of the same weights, over d' = the
+      number of weights compared.
   R20 allocation (Section 2.4, Eq. 7; App. B "Allocators"): layer i at width b costs n_i * b bits and
       the budget is avg_bits * sum_i n_i (the parameter-weighted budget of Eq. 8); each greedy step moves one layer to the adjacent width of
       its candidate list; the step ratio is dOmega / dcost in float64; ties go to the lowest layer
@@ -51,7 +54,7 @@ __all__ = [
     "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
     "jab_loss_and_grad", "lsq_factor", "default_kappa", "kl_attention_term", "jab_loss_joint",
     "attention_jvp", "block_jvp", "gn_quadratic_form", "hutchinson_trace", "omega_scores",
-    "pareto_frontier", "allocate_bits",
+    "pareto_frontier", "allocate_bits", "flip_count",
 ]
 
 
@@ -97,6 +100,16 @@ def quantize(w: np.ndarray, s: np.ndarray, bits: int, group_size: int):
     q = np.clip(np.rint(v), -qm, qm)          # np.rint rounds half to even
     w_hat = q * s_full
     return q.astype(np.int8), w_hat, v
+
+
+def flip_count(codes_a: np.ndarray, codes_b: np.ndarray) -> int:
+    """Eq. 15 numerator: the number of positions whose grid position differs between two code
+    arrays of the same weights (reading R21); the flip rate is this count over their size."""
+    a = np.asarray(codes_a).ravel()
+    b = np.asarray(codes_b).ravel()
+    if a.shape != b.shape:
+        raise ValueError("code arrays differ in size")
+    return int(np.count_nonzero(a != b))
 
 
 def init_scales_absmax(w: np.ndarray, bits: int, group_size: int) -> np.ndarray:

@@ -11,5 +11,7 @@ from .binding import (  # noqa: F401
     jab_reference_forward, jab_loss_forward, jab_loss_forward_noalloc, jab_loss_backward_scales,
     jab_loss_backward_weights, jab_allocate_bits, jab_quantize,
     jab_init_scales, jab_get_device_status, jab_status_string, Workspace, jab_timing_enable,
-    jab_timing_reset, jab_timing_read, jab_selftest_wait_timeout,
+    jab_timing_reset, jab_timing_read, jab_selftest_wait_timeout, jab_prepare_x,
+    jab_loss_backward_scales_prepared, jab_flip_rate, jab_reference_projection,
+    jab_loss_forward_kl,
 )

@@ -75,6 +75,13 @@ def lib() -> ctypes.CDLL:
                                            ctypes.POINTER(_P), _P, _P, _P]
     L.jab_loss_backward_scales.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P, _P, sz, _P]
     L.jab_loss_backward_weights.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, _P, _P, _P, _P, sz, _P]
+    L.jab_prepare_x.argtypes = [D, i32, i32, _P, _P, sz, _P]
+    L.jab_loss_backward_scales_prepared.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P,
+                                                    _P, sz, _P]
+    L.jab_flip_rate.argtypes = [_P, _P, ctypes.c_int64, _P, _P]
+    L.jab_reference_projection.argtypes = [D, i32, i32, _P, _P, _P, _P, sz, _P]
+    L.jab_loss_forward_kl.argtypes = [D, i32, i32, _P, _P, _P, _P, i32, ctypes.POINTER(i32),
+                                      ctypes.POINTER(_P), f32, _P, _P, _P, _P, _P, sz, _P]
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
     L.jab_allocate_bits.argtypes = [_P, _P, _P, i32, i32, ctypes.c_double, i32, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
@@ -91,6 +98,8 @@ def lib() -> ctypes.CDLL:
     L.jab_timing_reset.argtypes = []
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
                "jab_loss_backward_scales", "jab_loss_backward_weights", "jab_allocate_bits",
+               "jab_prepare_x", "jab_loss_backward_scales_prepared", "jab_flip_rate",
+               "jab_reference_projection", "jab_loss_forward_kl",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
                "jab_selftest_wait_timeout",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
@@ -173,6 +182,32 @@ def jab_loss_forward(desc, B, T, X, W, A_ref, bits: Sequence[int], scales: Seque
     _check(st, "jab_loss_forward")
 
 
+def jab_reference_projection(desc, B, T, X, W, QKV_ref, ws: Workspace, stream=None):
+    """Teacher [Q|K|V] (rotated, fp16 [B, T, D]) for the KL term."""
+    st = lib().jab_reference_projection(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(QKV_ref, torch.float16, "QKV_ref"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_reference_projection")
+
+
+def jab_loss_forward_kl(desc, B, T, X, W, A_ref, QKV_ref, bits: Sequence[int],
+                        scales: Sequence[torch.Tensor], lambda_kl: float, loss, ws: Workspace,
+                        mse=None, kl=None, kl_rows=None, stream=None):
+    """Both terms of Eq. 3 per candidate: loss = mse + lambda_kl * kl (fp64 [n_cand] each)."""
+    n = len(bits)
+    if len(scales) != n:
+        raise ValueError("bits and scales must have the same length")
+    bits_arr = (ctypes.c_int32 * n)(*[int(b) for b in bits])
+    sc_arr = (ctypes.c_void_p * n)(*[_ptr(s, torch.float32, "scales") for s in scales])
+    st = lib().jab_loss_forward_kl(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), _ptr(QKV_ref, torch.float16, "QKV_ref"), n, bits_arr,
+        sc_arr, float(lambda_kl), _ptr(loss, torch.float64, "loss"), _ptr(mse, torch.float64, "mse"),
+        _ptr(kl, torch.float64, "kl"), _ptr(kl_rows, torch.float32, "kl_rows"), ws.ptr, ws.nbytes,
+        _stream(stream))
+    _check(st, "jab_loss_forward_kl")
+
+
 def jab_loss_forward_noalloc(desc, B, T, X, W, A_ref, bits: Sequence[int],
                              scales: Sequence[torch.Tensor], loss, sse_parts=None, stream=None):
     """jab_loss_forward on the library's fixed device scratch (no workspace argument): for callers
@@ -199,6 +234,36 @@ def jab_loss_backward_scales(desc, B, T, X, W, A_ref, bits: int, scales, kappa: 
         float(kappa), _ptr(loss, torch.float64, "loss"),
         _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "jab_loss_backward_scales")
+
+
+def jab_prepare_x(desc, B, T, X, ws: Workspace, stream=None):
+    """Converts X into the workspace's fp16 copy for jab_loss_backward_scales_prepared."""
+    st = lib().jab_prepare_x(ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), ws.ptr,
+                             ws.nbytes, _stream(stream))
+    _check(st, "jab_prepare_x")
+
+
+def jab_loss_backward_scales_prepared(desc, B, T, X, W, A_ref, bits: int, scales, kappa: float,
+                                      loss, grad_scales, ws: Workspace, stream=None):
+    """jab_loss_backward_scales on the fp16 X that jab_prepare_x left in `ws`."""
+    st = lib().jab_loss_backward_scales_prepared(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), int(bits), _ptr(scales, torch.float32, "scales"),
+        float(kappa), _ptr(loss, torch.float64, "loss"),
+        _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_loss_backward_scales_prepared")
+
+
+def jab_flip_rate(codes_a, codes_b, count, stream=None):
+    """Number of positions where two int8 code tensors differ (Eq. 15), into count (int64 [1])."""
+    if codes_a.numel() != codes_b.numel():
+        raise ValueError("code arrays differ in size")
+    if codes_a.numel() == 0:
+        codes_a = codes_b = None
+    n = 0 if codes_a is None else int(codes_a.numel())
+    st = lib().jab_flip_rate(_ptr(codes_a, torch.int8, "codes_a"), _ptr(codes_b, torch.int8, "codes_b"),
+                             n, _ptr(count, torch.int64, "count"), _stream(stream))
+    _check(st, "jab_flip_rate")
 
 
 def jab_loss_backward_weights(desc, B, T, X, W, A_ref, bits: int, scales, loss, grad_w=None,

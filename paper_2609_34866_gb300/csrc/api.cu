@@ -6,9 +6,10 @@
 
 #include <mutex>
 
+#include <vector>
+
 #include "common.cuh"
 #include "kernels.h"
-#include "path.h"
 #include "timing.h"
 #include "workspace.h"
 
@@ -95,12 +96,8 @@ jab_status run_projection(const jab_block_desc* d, int64_t N, int T, int C, cons
                           int* status, cudaStream_t st) {
   const int D = (int)block_rows(d);
   const int n_rot = d->use_rope ? (d->n_q_heads + d->n_kv_heads) * d->head_dim : 0;
-  if (use_tc_path())
-    JAB_SITE("proj_gemm", 1, launch_proj_gemm_tc(x16, w16, qkv, N, C * D, d->d_model, D, n_rot,
-                                                 d->head_dim, T, cos_t, sin_t, status, st));
-  else
-    JAB_SITE("proj_gemm", 1, launch_proj_gemm_simple(x16, w16, qkv, N, C * D, d->d_model, D, n_rot, d->head_dim, T,
-                                    cos_t, sin_t, st));
+  JAB_SITE("proj_gemm", 1, launch_proj_gemm_tc(x16, w16, qkv, N, C * D, d->d_model, D, n_rot,
+                                               d->head_dim, T, cos_t, sin_t, status, st));
   return JAB_OK;
 }
 
@@ -117,13 +114,50 @@ AttnLaunch attn_launch(const jab_block_desc* d, int B, int T, int C, char* ws,
   L.dh = d->head_dim;
   L.C = C;
   L.scale = softmax_scale(d);
-  const int rows = use_tc_path() ? attn_fwd_tc_rows(d->n_q_heads, d->n_kv_heads) : kPartRows;
+  const int rows = attn_fwd_tc_rows(d->n_q_heads, d->n_kv_heads);
   L.nP = (T + rows - 1) / rows;
   L.lse_pitch = T;
   L.part = reinterpret_cast<double*>(ws + wp.part);
   L.status = status;
   L.stream = st;
   return L;
+}
+
+// Which X each workspace holds in fp16 (its x16 slot): written by every call that converts X into
+// a workspace, read by the *_prepared entry points, which skip the conversion.
+struct PreparedX {
+  const void* ws;
+  const void* x;
+  int32_t B, T, d;
+};
+std::mutex g_prep_mu;
+std::vector<PreparedX> g_prep;
+
+void note_prepared(const void* ws, const void* x, int32_t B, int32_t T, int32_t d) {
+  std::lock_guard<std::mutex> lk(g_prep_mu);
+  for (auto& e : g_prep)
+    if (e.ws == ws) {
+      e = PreparedX{ws, x, B, T, d};
+      return;
+    }
+  g_prep.push_back(PreparedX{ws, x, B, T, d});
+}
+
+bool is_prepared(const void* ws, const void* x, int32_t B, int32_t T, int32_t d) {
+  std::lock_guard<std::mutex> lk(g_prep_mu);
+  for (const auto& e : g_prep)
+    if (e.ws == ws) return e.x == x && e.B == B && e.T == T && e.d == d;
+  return false;
+}
+
+// X (bf16) -> the workspace's fp16 copy, with the fp16 range check; records it for *_prepared.
+jab_status convert_x_into(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                          void* ws, const Workspace& wp, int* status, int sms, cudaStream_t st) {
+  const int64_t N = (int64_t)B * T;
+  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, static_cast<char*>(ws) + wp.x16,
+                                            N * desc->d_model, status, sms, st));
+  note_prepared(ws, X_dev, B, T, desc->d_model);
+  return JAB_OK;
 }
 
 }  // namespace
@@ -161,7 +195,7 @@ jab_status jab_reference_forward(const jab_block_desc* desc, int32_t B, int32_t 
   const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
   float* cos_t = reinterpret_cast<float*>(w + wp.rope);
   float* sin_t = cos_t + (int64_t)T * (dh / 2);
-  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
+  if ((s = convert_x_into(desc, B, T, X_dev, ws, wp, status, sms, st)) != JAB_OK) return s;
   JAB_SITE("quantize", 1, launch_quantize(W_dev, nullptr, D, dm, desc->group_size, 0, w + wp.w16, nullptr, nullptr,
                           status, sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
@@ -171,21 +205,28 @@ jab_status jab_reference_forward(const jab_block_desc* desc, int32_t B, int32_t 
   AttnLaunch L = attn_launch(desc, B, T, 1, w, wp, status, st);
   L.a_out = A_ref_dev;
   L.lse = lse_dev;
-  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 0) : launch_attn_fwd_simple(L, 0));
+  JAB_SITE("attn_fwd", 1, launch_attn_fwd_tc(L, 0));
   if (a_sqnorm_dev)
-    JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0, a_sqnorm_dev, nullptr, st));
+    JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0,
+                                                  a_sqnorm_dev, nullptr, status, st));
   return JAB_OK;
 }
 
-jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
-                            const void* W_dev, const float* A_ref_dev, int32_t n_cand,
-                            const int32_t* bits_host, const float* const* scales_host,
-                            double* loss_dev, double* sse_parts_dev, void* ws, size_t ws_bytes,
-                            jab_stream_t stream) {
+}  // extern "C"
+
+// The candidate forward of jab_loss_forward: quantise every candidate, one projection GEMM over all
+// of them (+ RoPE), the attention forward with the MSE epilogue, the loss per candidate into
+// mse_dev. On success *wp_out / *status_out describe the workspace and the status word.
+static jab_status forward_candidates(const jab_block_desc* desc, int32_t B, int32_t T,
+                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                     int32_t n_cand, const int32_t* bits_host,
+                                     const float* const* scales_host, double* mse_dev,
+                                     double* sse_parts_dev, void* ws, size_t ws_bytes,
+                                     cudaStream_t st, Workspace* wp_out, int** status_out) {
   jab_status s = check_desc(desc);
   if (s != JAB_OK) return s;
   if ((s = check_bt(B, T)) != JAB_OK) return s;
-  if (n_cand < 1 || !bits_host || !scales_host || !X_dev || !W_dev || !A_ref_dev || !loss_dev ||
+  if (n_cand < 1 || !bits_host || !scales_host || !X_dev || !W_dev || !A_ref_dev || !mse_dev ||
       !ws)
     return JAB_ERR_INVALID_ARG;
   if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) ||
@@ -201,13 +242,12 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
   int* status;
   int sms;
   if ((s = device_info(&status, &sms)) != JAB_OK) return s;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   const int64_t N = (int64_t)B * T;
   const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
   float* cos_t = reinterpret_cast<float*>(w + wp.rope);
   float* sin_t = cos_t + (int64_t)T * (dh / 2);
-  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
+  if ((s = convert_x_into(desc, B, T, X_dev, ws, wp, status, sms, st)) != JAB_OK) return s;
   for (int c = 0; c < n_cand; ++c)
     JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_host[c], D, dm, desc->group_size, bits_host[c],
                             w + wp.w16 + (size_t)c * D * dm * 2, nullptr, nullptr, status, sms, st));
@@ -217,10 +257,93 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
     return s;
   AttnLaunch L = attn_launch(desc, B, T, n_cand, w, wp, status, st);
   L.a_ref = A_ref_dev;
-  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 1) : launch_attn_fwd_simple(L, 1));
+  JAB_SITE("attn_fwd", 1, launch_attn_fwd_tc(L, 1));
   const double inv_n = 1.0 / ((double)N * desc->n_q_heads * dh);
-  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, n_cand, B, desc->n_q_heads, L.nP, inv_n, loss_dev,
-                             sse_parts_dev, st));
+  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, n_cand, B, desc->n_q_heads, L.nP, inv_n,
+                                                mse_dev, sse_parts_dev, status, st));
+  *wp_out = wp;
+  *status_out = status;
+  return JAB_OK;
+}
+
+extern "C" {
+
+jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                            const void* W_dev, const float* A_ref_dev, int32_t n_cand,
+                            const int32_t* bits_host, const float* const* scales_host,
+                            double* loss_dev, double* sse_parts_dev, void* ws, size_t ws_bytes,
+                            jab_stream_t stream) {
+  Workspace wp;
+  int* status;
+  return forward_candidates(desc, B, T, X_dev, W_dev, A_ref_dev, n_cand, bits_host, scales_host,
+                            loss_dev, sse_parts_dev, ws, ws_bytes,
+                            reinterpret_cast<cudaStream_t>(stream), &wp, &status);
+}
+
+jab_status jab_reference_projection(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, void* QKV_ref_dev,
+                                    void* ws, size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (!X_dev || !W_dev || !QKV_ref_dev || !ws) return JAB_ERR_INVALID_ARG;
+  if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(QKV_ref_dev) ||
+      (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, B, T, 1, false);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
+  float* cos_t = reinterpret_cast<float*>(w + wp.rope);
+  float* sin_t = cos_t + (int64_t)T * (dh / 2);
+  if ((s = convert_x_into(desc, B, T, X_dev, ws, wp, status, sms, st)) != JAB_OK) return s;
+  JAB_SITE("quantize", 1, launch_quantize(W_dev, nullptr, D, dm, desc->group_size, 0, w + wp.w16,
+                                          nullptr, nullptr, status, sms, st));
+  if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
+  return run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, QKV_ref_dev, cos_t, sin_t, status,
+                        st);
+}
+
+jab_status jab_loss_forward_kl(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                               const void* W_dev, const float* A_ref_dev, const void* QKV_ref_dev,
+                               int32_t n_cand, const int32_t* bits_host,
+                               const float* const* scales_host, float lambda_kl, double* loss_dev,
+                               double* mse_dev, double* kl_dev, float* kl_rows_dev, void* ws,
+                               size_t ws_bytes, jab_stream_t stream) {
+  if (!QKV_ref_dev || !aligned16(QKV_ref_dev) || !loss_dev || !(lambda_kl >= 0.f) ||
+      !isfinite(lambda_kl)) {
+    const jab_status s = check_desc(desc);
+    return s != JAB_OK ? s : JAB_ERR_INVALID_ARG;
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (n_cand >= 1 && desc != nullptr && check_desc(desc) == JAB_OK && check_bt(B, T) == JAB_OK) {
+    const Workspace wp0 = plan_workspace(desc, B, T, n_cand, false);
+    if (ws != nullptr && ws_bytes >= wp0.total && !mse_dev)
+      mse_dev = reinterpret_cast<double*>(static_cast<char*>(ws) + wp0.scal);
+  }
+  Workspace wp;
+  int* status;
+  jab_status s = forward_candidates(desc, B, T, X_dev, W_dev, A_ref_dev, n_cand, bits_host,
+                                    scales_host, mse_dev, nullptr, ws, ws_bytes, st, &wp, &status);
+  if (s != JAB_OK) return s;
+  char* w = static_cast<char*>(ws);
+  double* kl = kl_dev ? kl_dev : reinterpret_cast<double*>(w + wp.scal) + n_cand;
+  double* part = reinterpret_cast<double*>(w + wp.part);
+  const int nP = (T + attn_kl_tc_rows() - 1) / attn_kl_tc_rows();
+  JAB_SITE("attn_kl", 1, launch_attn_kl_tc(w + wp.qkv, (int64_t)n_cand * block_rows(desc),
+                                           QKV_ref_dev, B, T, n_cand, desc->n_q_heads,
+                                           desc->n_kv_heads, desc->head_dim, softmax_scale(desc),
+                                           part, nP, kl_rows_dev, status, st));
+  // batchmean (App. B "Effective weight of the KL term"): the sum over rows divided by B
+  JAB_SITE("loss_reduce", 1, launch_loss_reduce(part, n_cand, B, desc->n_q_heads, nP, 1.0 / B, kl,
+                                                nullptr, status, st));
+  JAB_SITE("loss_combine", 1, launch_loss_combine(mse_dev, kl, (double)lambda_kl, n_cand, loss_dev,
+                                                  st));
   return JAB_OK;
 }
 
@@ -230,8 +353,8 @@ jab_status jab_loss_forward(const jab_block_desc* desc, int32_t B, int32_t T, co
 static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32_t T,
                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
                                     int32_t bits, const float* scales_dev, double* loss_dev,
-                                    void* ws, size_t ws_bytes, cudaStream_t st, Workspace* wp_out,
-                                    int** status_out) {
+                                    void* ws, size_t ws_bytes, bool x_prepared, cudaStream_t st,
+                                    Workspace* wp_out, int** status_out) {
   jab_status s = check_desc(desc);
   if (s != JAB_OK) return s;
   if ((s = check_bt(B, T)) != JAB_OK) return s;
@@ -251,9 +374,11 @@ static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32
   const int G = desc->group_size;
   float* cos_t = reinterpret_cast<float*>(w + wp.rope);
   float* sin_t = cos_t + (int64_t)T * (dh / 2);
-  JAB_SITE("convert_x", 1, launch_convert_x(X_dev, w + wp.x16, N * dm, status, sms, st));
-  if (!use_tc_path())  // the tcgen05 weight-gradient GEMM reads X as stored
-    JAB_SITE("transpose_x", 1, launch_transpose_x(X_dev, w + wp.xt, N, wp.ldt, dm, st));
+  if (x_prepared) {  // the workspace already holds this X in fp16 (jab_prepare_x)
+    if (!is_prepared(ws, X_dev, B, T, dm)) return JAB_ERR_INVALID_ARG;
+  } else if ((s = convert_x_into(desc, B, T, X_dev, ws, wp, status, sms, st)) != JAB_OK) {
+    return s;
+  }
   JAB_SITE("quantize", 1, launch_quantize(W_dev, scales_dev, D, dm, G, bits, w + wp.w16, nullptr, nullptr, status,
                           sms, st));
   if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
@@ -267,22 +392,25 @@ static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32
   L.dvec = reinterpret_cast<float*>(w + wp.dvec);
   L.ldt = wp.ldt;
   L.lse_pitch = (int)wp.tp;
-  JAB_SITE("attn_fwd", 1, use_tc_path() ? launch_attn_fwd_tc(L, 2) : launch_attn_fwd_simple(L, 2));
+  JAB_SITE("attn_fwd", 1, launch_attn_fwd_tc(L, 2));
   const double n_el = (double)N * desc->n_q_heads * dh;
-  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el, loss_dev, nullptr,
-                             st));
-  JAB_SITE("attn_bwd", 2, use_tc_path() ? launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt)
-                        : launch_attn_bwd_simple(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt));
+  JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el,
+                                                loss_dev, nullptr, status, st));
+  JAB_SITE("attn_bwd", 2, launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt));
   *wp_out = wp;
   *status_out = status;
   return JAB_OK;
 }
 
-jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
-                                    const void* X_dev, const void* W_dev, const float* A_ref_dev,
-                                    int32_t bits, const float* scales_dev, float kappa,
-                                    double* loss_dev, float* grad_scales_dev, void* ws,
-                                    size_t ws_bytes, jab_stream_t stream) {
+}  // extern "C"
+
+// jab_loss_backward_scales with the fp16 conversion of X either done here or taken from the
+// workspace (x_prepared).
+static jab_status backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+                                  const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                  int32_t bits, const float* scales_dev, float kappa,
+                                  double* loss_dev, float* grad_scales_dev, void* ws,
+                                  size_t ws_bytes, bool x_prepared, jab_stream_t stream) {
   if (!grad_scales_dev || !aligned16(grad_scales_dev)) {
     const jab_status s = check_desc(desc);
     return s != JAB_OK ? s : JAB_ERR_INVALID_ARG;
@@ -291,7 +419,7 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   Workspace wp;
   int* status;
   jab_status s = backward_to_dqkvt(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, loss_dev,
-                                   ws, ws_bytes, st, &wp, &status);
+                                   ws, ws_bytes, x_prepared, st, &wp, &status);
   if (s != JAB_OK) return s;
   char* w = static_cast<char*>(ws);
   const int64_t N = (int64_t)B * T;
@@ -300,14 +428,61 @@ jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32
   const double k = kappa > 0.f ? (double)kappa : 1.0 / sqrt((double)G * qmax_of(bits));
   const float coef = (float)(k * 2.0 / n_el);
   JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
-  if (use_tc_path())
-    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, wp.ldt, X_dev, W_dev, scales_dev, N, D,
-                                                 dm, G, bits, coef, grad_scales_dev, status, st));
-  else
-    JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_simple(w + wp.dqkvt, w + wp.xt, wp.ldt, W_dev,
-                                                     scales_dev, N, D, dm, G, bits, coef,
-                                                     grad_scales_dev, st));
+  JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, wp.ldt, X_dev, W_dev, scales_dev, N, D,
+                                               dm, G, bits, coef, grad_scales_dev, status, st));
   JAB_SITE("check_finite", 1, launch_check_finite(grad_scales_dev, (int64_t)D * (dm / G), status, st));
+  return JAB_OK;
+}
+
+extern "C" {
+
+jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
+                                    const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                    int32_t bits, const float* scales_dev, float kappa,
+                                    double* loss_dev, float* grad_scales_dev, void* ws,
+                                    size_t ws_bytes, jab_stream_t stream) {
+  return backward_scales(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, kappa, loss_dev,
+                         grad_scales_dev, ws, ws_bytes, false, stream);
+}
+
+jab_status jab_prepare_x(const jab_block_desc* desc, int32_t B, int32_t T, const void* X_dev,
+                         void* ws, size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (!X_dev || !ws || !aligned16(X_dev) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, B, T, 1, false);
+  if (ws_bytes < wp.x16 + (size_t)B * T * desc->d_model * 2) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  return convert_x_into(desc, B, T, X_dev, ws, wp, status, sms,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+jab_status jab_loss_backward_scales_prepared(const jab_block_desc* desc, int32_t B, int32_t T,
+                                             const void* X_dev, const void* W_dev,
+                                             const float* A_ref_dev, int32_t bits,
+                                             const float* scales_dev, float kappa,
+                                             double* loss_dev, float* grad_scales_dev, void* ws,
+                                             size_t ws_bytes, jab_stream_t stream) {
+  return backward_scales(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, kappa, loss_dev,
+                         grad_scales_dev, ws, ws_bytes, true, stream);
+}
+
+jab_status jab_flip_rate(const int8_t* codes_a_dev, const int8_t* codes_b_dev, int64_t n,
+                         int64_t* count_dev, jab_stream_t stream) {
+  if (!count_dev || n < 0 || (reinterpret_cast<uintptr_t>(count_dev) & 7u))
+    return JAB_ERR_INVALID_ARG;
+  if (n > 0 && (!codes_a_dev || !codes_b_dev || !aligned16(codes_a_dev) || !aligned16(codes_b_dev)))
+    return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  const jab_status s = device_info(&status, &sms);
+  if (s != JAB_OK) return s;
+  JAB_TRY(launch_flip_count(codes_a_dev, codes_b_dev, n, count_dev, sms,
+                            reinterpret_cast<cudaStream_t>(stream)));
   return JAB_OK;
 }
 
@@ -320,12 +495,11 @@ jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int3
   if (s != JAB_OK) return s;
   if ((!grad_w_dev && !grad_sqnorm_dev) || (grad_w_dev && !aligned16(grad_w_dev)))
     return JAB_ERR_INVALID_ARG;
-  if (!use_tc_path()) return JAB_ERR_UNSUPPORTED;  // the store epilogue exists on the tcgen05 path
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   Workspace wp;
   int* status;
   s = backward_to_dqkvt(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, loss_dev, ws,
-                        ws_bytes, st, &wp, &status);
+                        ws_bytes, false, st, &wp, &status);
   if (s != JAB_OK) return s;
   char* w = static_cast<char*>(ws);
   const int64_t N = (int64_t)B * T;

@@ -17,7 +17,7 @@
 // dQKV^T (bf16, [D, ldt]), the K-major operand of the weight-gradient GEMM.
 #include <cudaTypedefs.h>
 
-#include "path.h"
+#include "kernels.h"
 #include "tc.cuh"
 
 namespace jab {

@@ -20,7 +20,7 @@
 
 #include <algorithm>
 
-#include "path.h"
+#include "kernels.h"
 #include "tc.cuh"
 
 namespace jab {
@@ -372,6 +372,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const float2 f = __half22float2(hp[k]);
                 dsum += f.x * o[v * 8 + 2 * k] + f.y * o[v * 8 + 2 * k + 1];
               }
+              if (half2_exp_all_ones(u.x) | half2_exp_all_ones(u.y) | half2_exp_all_ones(u.z) |
+                  half2_exp_all_ones(u.w))
+                report(p.status, JAB_ERR_RANGE);  // dO out of the fp16 range (or NaN)
               dst[v] = u;
             }
           }
@@ -820,6 +823,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     const int rbase = quarter * 32;
     const int c4 = lane & 7;
     int tc_ = 0;
+    uint32_t range_bits = 0;  // mode 2: an fp16 dO value out of range (inf) or NaN
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
@@ -902,6 +906,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
                 u.x = *reinterpret_cast<const uint32_t*>(&a01);
                 u.y = *reinterpret_cast<const uint32_t*>(&a23);
                 *reinterpret_cast<uint2*>(p.d_o + off) = u;
+                range_bits |= half2_exp_all_ones(u.x) | half2_exp_all_ones(u.y);
                 const float2 f01 = __half22float2(a01), f23 = __half22float2(a23);
                 *slot = make_float4(f01.x, f01.y, f23.x, f23.y);
               }
@@ -938,6 +943,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       }
       if (!have) break;
     }
+    if (MODE == 2 && range_bits) report(p.status, JAB_ERR_RANGE);
   }
   tc::fence_before_sync();
   __syncthreads();

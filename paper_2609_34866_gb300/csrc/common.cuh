@@ -18,6 +18,12 @@ __device__ __forceinline__ void report(int* status, int code) {
   if (status != nullptr) atomicCAS(status, 0, code);
 }
 
+// Non-zero when either half of a packed fp16 pair has every exponent bit set: an infinity (the
+// rounded value was outside the fp16 range) or a NaN. Integer SIMD compare, no FP instructions.
+__device__ __forceinline__ uint32_t half2_exp_all_ones(uint32_t h2) {
+  return __vcmpeq2(h2 & 0x7C007C00u, 0x7C007C00u);
+}
+
 __host__ __device__ __forceinline__ int qmax_of(int bits) { return (1 << (bits - 1)) - 1; }
 
 // Eq. 2 with reading R1: v = fl32(w / s) (IEEE round-to-nearest division), q = clip(rint(v)).

@@ -18,7 +18,7 @@
 //               TMA boxes per stage), so no transposed copy of X is needed.
 #include <cudaTypedefs.h>
 
-#include "path.h"
+#include "kernels.h"
 #include "tc.cuh"
 
 namespace jab {
@@ -140,6 +140,7 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
     if (row_ok) {
       uint4* d1 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1);
       uint4* d2 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1 + half);
+      uint32_t inf_bits = 0;  // a half with all exponent bits set: inf (out of fp16 range) or NaN
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
         uint4 u1, u2;
@@ -150,9 +151,14 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
           h1[e] = __floats2half2_rn(a[v * 8 + 2 * e], a[v * 8 + 2 * e + 1]);
           h2[e] = __floats2half2_rn(b[v * 8 + 2 * e], b[v * 8 + 2 * e + 1]);
         }
+        inf_bits |= half2_exp_all_ones(u1.x) | half2_exp_all_ones(u1.y) |
+                    half2_exp_all_ones(u1.z) | half2_exp_all_ones(u1.w) |
+                    half2_exp_all_ones(u2.x) | half2_exp_all_ones(u2.y) |
+                    half2_exp_all_ones(u2.z) | half2_exp_all_ones(u2.w);
         d1[v] = u1;
         d2[v] = u2;
       }
+      if (inf_bits) report(p.status, JAB_ERR_RANGE);
     }
   }
 }

@@ -26,29 +26,49 @@ struct AttnLaunch {
 
 // prep.cu
 cudaError_t launch_convert_x(const void* x, void* xh, int64_t n, int* status, int sms, cudaStream_t st);
-cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int64_t ldt, int d, cudaStream_t st);
 cudaError_t launch_quantize(const void* w, const float* s, int D, int d, int G, int bits, void* w16,
                             int8_t* codes, float* w_hat32, int* status, int sms, cudaStream_t st);
+// codes a, b: int8 [n], 16-byte aligned; *count (int64, device) = #{i : a[i] != b[i]}
+cudaError_t launch_flip_count(const int8_t* a, const int8_t* b, int64_t n, int64_t* count,
+                              int sms, cudaStream_t st);
 cudaError_t launch_init_scales(const void* w, int D, int d, int G, int bits, int mode, float* s_out,
                                cudaStream_t st);
 cudaError_t launch_rope_table(int T, int dh, double theta, float* cos_t, float* sin_t, cudaStream_t st);
 
-// gemm_simple.cu
-cudaError_t launch_proj_gemm_simple(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
-                                    int D, int n_rot, int dh, int T, const float* cos_t,
-                                    const float* sin_t, cudaStream_t st);
-cudaError_t launch_wgrad_lsq_simple(const void* dqkvt, const void* xt, int64_t ldt, const void* w,
-                                    const float* s, int64_t N, int D, int d, int G, int bits,
-                                    float coef, float* ds, cudaStream_t st);
+// gemm_tc.cu
+cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t M, int Nn, int K,
+                                int D, int n_rot, int dh, int T, const float* cos_t,
+                                const float* sin_t, int* status, cudaStream_t st);
+// x: bf16 [N, d] as the caller stores it (no transposed copy)
+cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
+                                const float* s, int64_t N, int D, int d, int G, int bits,
+                                float coef, float* ds, int* status, cudaStream_t st);
+// coef * dQKV^T X stored fp32 [D, d] (dw may be NULL) and its squared norm added to *sqnorm (may be
+// NULL; the caller zeroes it)
+cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
+                                  int d, float coef, float* dw, double* sqnorm, int* status,
+                                  cudaStream_t st);
+// attn_tc.cu
+int attn_fwd_tc_rows(int Hq, int Hkv);  // query rows per loss partial of the forward kernel
+cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);
+cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
+                               int use_rope, void* dqkvt);
 
-// attn_simple.cu
-cudaError_t launch_attn_fwd_simple(const AttnLaunch& L, int mode);
-cudaError_t launch_attn_bwd_simple(const AttnLaunch& L, const float* cos_t, const float* sin_t,
-                                   int use_rope, void* dqkvt);
+// attn_kl_tc.cu: KL attention-map term (Eq. 3). qkv_s: student fp16 [B*T, ldq] (candidate c at
+// column c * D); qkv_t: teacher fp16 [B*T, D]. part [C, B, Hq, nP] (nP >= ceil(T / rows)), kl_rows
+// fp32 [C, B, Hq, T] or null.
+int attn_kl_tc_rows();
+cudaError_t launch_attn_kl_tc(const void* qkv_s, int64_t ldq, const void* qkv_t, int B, int T,
+                              int C, int Hq, int Hkv, int dh, float scale, double* part, int nP,
+                              float* kl_rows, int* status, cudaStream_t st);
 
 // reduce.cu
+// A non-finite total raises JAB_ERR_NONFINITE in *status.
 cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
-                               double* out, double* parts_out, cudaStream_t st);
+                               double* out, double* parts_out, int* status, cudaStream_t st);
+// out[c] = a[c] + lam * b[c] for c < C
+cudaError_t launch_loss_combine(const double* a, const double* b, double lam, int C, double* out,
+                                cudaStream_t st);
 cudaError_t launch_check_finite(const float* x, int64_t n, int* status, cudaStream_t st);
 
 }  // namespace jab

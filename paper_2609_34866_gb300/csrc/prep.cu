@@ -29,25 +29,6 @@ __global__ void convert_x_kernel(const uint4* __restrict__ x, uint4* __restrict_
   else if (bad & 1) report(status, JAB_ERR_RANGE);
 }
 
-// X [N, d] bf16 -> X^T [d, N] bf16 through a 64x64 shared-memory tile.
-__global__ void transpose_bf16_kernel(const bf16_t* __restrict__ x, bf16_t* __restrict__ xt,
-                                      int64_t N, int64_t ldt, int d) {
-  __shared__ bf16_t tile[64][65];
-  const int64_t n0 = (int64_t)blockIdx.x * 64;
-  const int c0 = blockIdx.y * 64;
-  for (int r = threadIdx.y; r < 64; r += blockDim.y) {
-    const int64_t n = n0 + r;
-    const int c = c0 + threadIdx.x;
-    tile[r][threadIdx.x] = (n < N && c < d) ? x[n * d + c] : __float2bfloat16(0.f);
-  }
-  __syncthreads();
-  for (int r = threadIdx.y; r < 64; r += blockDim.y) {
-    const int c = c0 + r;
-    const int64_t n = n0 + threadIdx.x;
-    if (n < N && c < d) xt[(int64_t)c * ldt + n] = tile[threadIdx.x][r];
-  }
-}
-
 // ---------------------------------------------------------------- quantiser (Section 2.1, Eq. 2)
 // bits == 0: plain bf16 -> fp16 conversion of W (the teacher's weights).
 __global__ void quantize_kernel(const uint4* __restrict__ w, const float* __restrict__ s, int D,
@@ -92,11 +73,46 @@ __global__ void quantize_kernel(const uint4* __restrict__ w, const float* __rest
       uint4 o;
       half_t* h = reinterpret_cast<half_t*>(&o);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) h[k] = __float2half_rn(out[k]);
+      for (int k = 0; k < 8; ++k) {
+        h[k] = __float2half_rn(out[k]);
+        if (__hisinf(h[k]) || __hisnan(h[k])) bad |= 2;  // not representable as an fp16 operand
+      }
       w16[i] = o;
     }
   }
-  if (bad) report(status, JAB_ERR_NONFINITE);
+  if (bad & 1) report(status, JAB_ERR_NONFINITE);
+  else if (bad & 2) report(status, JAB_ERR_RANGE);
+}
+
+// ---------------------------------------------------------------- flip count (App. B, Eq. 15)
+// Number of positions where two int8 code arrays differ; 16 bytes per thread and step, one 64-bit
+// atomic per block (integer sums: the result does not depend on the order).
+__global__ void __launch_bounds__(256) flip_count_kernel(const uint4* __restrict__ a,
+                                                         const uint4* __restrict__ b, int64_t n16,
+                                                         const int8_t* __restrict__ a_tail,
+                                                         const int8_t* __restrict__ b_tail,
+                                                         int tail,
+                                                         unsigned long long* __restrict__ count) {
+  __shared__ unsigned long long red[8];
+  unsigned long long c = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const uint4 x = __ldg(a + i), y = __ldg(b + i);
+    // __vcmpne4: 0xff in each byte that differs
+    c += __popc(__vcmpne4(x.x, y.x)) + __popc(__vcmpne4(x.y, y.y)) + __popc(__vcmpne4(x.z, y.z)) +
+         __popc(__vcmpne4(x.w, y.w));
+  }
+  c >>= 3;  // eight set bits per differing byte
+  if (blockIdx.x == 0 && (int)threadIdx.x < tail) c += a_tail[threadIdx.x] != b_tail[threadIdx.x];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long t = 0;
+    for (int w = 0; w < 8; ++w) t += red[w];
+    atomicAdd(count, t);
+  }
 }
 
 // ---------------------------------------------------------------- starting scales
@@ -167,19 +183,24 @@ cudaError_t launch_convert_x(const void* x, void* xh, int64_t n, int* status, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_transpose_x(const void* x, void* xt, int64_t N, int64_t ldt, int d,
-                               cudaStream_t st) {
-  dim3 grid((unsigned)((N + 63) / 64), (unsigned)((d + 63) / 64));
-  transpose_bf16_kernel<<<grid, dim3(64, 8), 0, st>>>((const bf16_t*)x, (bf16_t*)xt, N, ldt, d);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_quantize(const void* w, const float* s, int D, int d, int G, int bits,
                             void* w16, int8_t* codes, float* w_hat32, int* status, int sms,
                             cudaStream_t st) {
   const int64_t n8 = (int64_t)D * d / 8;
   quantize_kernel<<<grid_for(n8, 256, sms), 256, 0, st>>>(
       (const uint4*)w, s, D, d, G, bits, (uint4*)w16, codes, w_hat32, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_flip_count(const int8_t* a, const int8_t* b, int64_t n, int64_t* count,
+                              int sms, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int64_t), st);
+  if (e != cudaSuccess) return e;
+  const int64_t n16 = n / 16;
+  const int tail = (int)(n - n16 * 16);
+  flip_count_kernel<<<grid_for(n16 > 0 ? n16 : 1, 256, sms), 256, 0, st>>>(
+      (const uint4*)a, (const uint4*)b, n16, a + n16 * 16, b + n16 * 16, tail,
+      reinterpret_cast<unsigned long long*>(count));
   return cudaGetLastError();
 }
 

@@ -8,7 +8,8 @@ namespace jab {
 __global__ void __launch_bounds__(256) loss_reduce_kernel(const double* __restrict__ part, int B,
                                                           int Hq, int nP, double inv_n,
                                                           double* __restrict__ out,
-                                                          double* __restrict__ parts_out) {
+                                                          double* __restrict__ parts_out,
+                                                          int* status) {
   __shared__ double red[8];
   const int c = blockIdx.x;
   const int nbh = B * Hq;
@@ -21,7 +22,15 @@ __global__ void __launch_bounds__(256) loss_reduce_kernel(const double* __restri
     acc += s;
   }
   const double tot = block_sum<256>(acc, red);
-  if (threadIdx.x == 0) out[c] = tot * inv_n;
+  if (threadIdx.x == 0) {
+    out[c] = tot * inv_n;
+    if (!isfinite(tot)) report(status, JAB_ERR_NONFINITE);
+  }
+}
+
+__global__ void loss_combine_kernel(const double* __restrict__ a, const double* __restrict__ b,
+                                    double lam, int C, double* __restrict__ out) {
+  for (int c = threadIdx.x; c < C; c += blockDim.x) out[c] = a[c] + lam * b[c];
 }
 
 __global__ void check_finite_kernel(const float* __restrict__ x, int64_t n, int* status) {
@@ -33,8 +42,14 @@ __global__ void check_finite_kernel(const float* __restrict__ x, int64_t n, int*
 }
 
 cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
-                               double* out, double* parts_out, cudaStream_t st) {
-  loss_reduce_kernel<<<C, 256, 0, st>>>(part, B, Hq, nP, inv_n, out, parts_out);
+                               double* out, double* parts_out, int* status, cudaStream_t st) {
+  loss_reduce_kernel<<<C, 256, 0, st>>>(part, B, Hq, nP, inv_n, out, parts_out, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_combine(const double* a, const double* b, double lam, int C, double* out,
+                                cudaStream_t st) {
+  loss_combine_kernel<<<1, 128, 0, st>>>(a, b, lam, C, out);
   return cudaGetLastError();
 }
 

@@ -18,13 +18,13 @@ struct Workspace {
   size_t rope;     // fp32 [2, T, d_h/2]     cos then sin
   size_t part;     // fp64 [C, B, Hq, nP]    per-tile partial sums (SSE or ||A||^2)
   size_t status;   // int32 [4]              reserved
+  size_t scal;     // fp64 [2, C]            per-candidate scalars (MSE and KL terms)
   // backward only
-  size_t xt;       // bf16 [d, ldt]          X transposed (K-major operand of the weight gradient)
   size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
   size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 128)
   size_t dvec;     // fp32 [B, Hq, Tp]       rowsum(dO * O)
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
-  int64_t ldt;     // row pitch (elements) of xt and dqkvt: N rounded up to 64
+  int64_t ldt;     // row pitch (elements) of dqkvt: N rounded up to 64
   int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 128
   size_t total;
 };
@@ -54,14 +54,14 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
   w.qkv = take((size_t)N * C * D * 2);
   w.rope = take((size_t)2 * T * (dh / 2) * 4);
   w.part = take((size_t)C * B * d->n_q_heads * nP * 8);
+  w.scal = take((size_t)2 * C * 8);
   if (bwd) {
-    w.xt = take((size_t)w.ldt * dm * 2);
     w.d_o = take((size_t)N * d->n_q_heads * dh * 2);
     w.lse = take((size_t)B * d->n_q_heads * w.tp * 4);
     w.dvec = take((size_t)B * d->n_q_heads * w.tp * 4);
     w.dqkvt = take((size_t)D * w.ldt * 2);
   } else {
-    w.xt = w.d_o = w.lse = w.dvec = w.dqkvt = SIZE_MAX;
+    w.d_o = w.lse = w.dvec = w.dqkvt = SIZE_MAX;
   }
   w.total = off;
   return w;

@@ -59,6 +59,11 @@ def test_host_side_checks_without_gpu(libjab):
     st = L.jab_loss_backward_weights(ctypes.byref(good), 2, 130, None, None, None, 2, None, None,
                                      None, None, None, 0, None)
     assert st == 1
+    st = L.jab_loss_backward_scales_prepared(ctypes.byref(good), 2, 130, None, None, None, 3, None,
+                                             1.0, None, None, None, 0, None)
+    assert st == 1
+    assert L.jab_prepare_x(ctypes.byref(good), 2, 130, None, None, 0, None) == 1
+    assert L.jab_flip_rate(None, None, 16, None, None) == 1
     st = L.jab_quantize(ctypes.byref(bad_dh), 3, None, None, None, None, None)
     assert st == 2
     assert L.jab_status_string(4).decode() == "non-finite or non-positive value"

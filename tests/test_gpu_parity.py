@@ -8,7 +8,9 @@ import pytest
 import torch
 
 from oracle import jab_oracle as O
-from tests.harness import A_TOL, COS_MIN, L_TOL, SMALL_CASES, Case, J, cosine, np64
+from tests.harness import (A_TOL, COS_MIN, HEAVY_TAILED, KL_ROW_ATOL, KL_ROW_TOL, KL_TOL, L_TOL,
+                           LSE_ATOL, PARTS_RTOL, SMALL_CASES,
+                           Case, J, cosine, np64)
 
 pytestmark = pytest.mark.gpu
 
@@ -76,11 +78,17 @@ def test_teacher_output_parity(name):
     a_o, parts = O.block_forward(c.x64, c.w64, c.odesc, return_parts=True)
     A = np64(A)
     rms = np.sqrt((a_o ** 2).mean())
-    err_rms = np.sqrt(((A - a_o) ** 2).mean())
-    assert err_rms <= A_TOL * rms, (err_rms, rms)                    # the bar: error RMS / RMS
-    assert np.abs(A - a_o).max() <= A_TOL * np.abs(a_o).max()       # and element-wise vs. max
-    np.testing.assert_allclose(np64(lse), parts["lse"], rtol=1e-3, atol=1e-2)  # fp16 Q, K scores
-    np.testing.assert_allclose(sq.item(), (a_o ** 2).sum(), rtol=2e-3)
+    err = np.abs(A - a_o)
+    assert np.sqrt((err ** 2).mean()) <= A_TOL * rms, (np.sqrt((err ** 2).mean()), rms)  # the bar
+    if name in HEAVY_TAILED:
+        # element-wise against the larger of the RMS and the element's own size (fp16 operands
+        # round large entries relatively); the strict form max|err| <= 1e-2 RMS measures 1.5e-2 here
+        assert (err / (rms + np.abs(a_o))).max() <= A_TOL, (err / (rms + np.abs(a_o))).max()
+    else:
+        assert err.max() <= A_TOL * rms, err.max() / rms                # element-wise, strict
+    lse_err = np.abs(np64(lse) - parts["lse"]).max()
+    assert lse_err <= LSE_ATOL.get(name, 2e-3), lse_err                 # fp16 Q, K scores
+    np.testing.assert_allclose(sq.item(), (a_o ** 2).sum(), rtol=2e-4)
 
 
 # ------------------------------------------------------------------ forward loss over candidates
@@ -99,9 +107,47 @@ def test_loss_forward_parity(name):
     for i, b in enumerate(bits):
         r = O.jab_loss(c.x64, c.w64, scales[i].cpu().numpy(), b, c.odesc, a_ref=a_ref)
         assert abs(loss[i].item() - r["loss"]) <= L_TOL * r["loss"], (b, loss[i].item(), r["loss"])
-        np.testing.assert_allclose(parts[i].cpu().numpy(), r["sse_parts"], rtol=5e-2)
+        np.testing.assert_allclose(parts[i].cpu().numpy(), r["sse_parts"], rtol=PARTS_RTOL[b])
         np.testing.assert_allclose(parts[i].sum().item(), r["sse"], rtol=L_TOL)
     assert J().jab_get_device_status() == 0
+
+
+# ------------------------------------------------------------------ KL attention-map term (Eq. 3)
+@pytest.mark.parametrize("name", ["gpt2_T200", "mistral_T130", "mistral_G64_T70", "gqa2_T257",
+                                  "dh64_gqa4_T65", "gpt2_T1"])
+def test_kl_forward_parity(name):
+    """Both terms of Eq. 3 per candidate against the oracle's kl_attention_term / jab_loss_joint:
+    the KL batchmean, every row's KL, the MSE term and their sum with lambda_KL = 0.1."""
+    c = case(name)
+    bits = [2, 3, 4, 8]
+    ws = c.workspace(n_cand=len(bits), with_bwd=False)
+    A, _, _ = c.gpu_teacher(ws)
+    qkv_ref = torch.empty((c.B, c.T, c.D), dtype=torch.float16, device="cuda")
+    J().jab_reference_projection(c.desc, c.B, c.T, c.X, c.W, qkv_ref, ws)
+    scales = [c.gpu_scales(b) for b in bits]
+    loss, mse, kl = (torch.empty(len(bits), dtype=torch.float64, device="cuda") for _ in range(3))
+    rows = torch.empty((len(bits), c.B, c.Hq, c.T), dtype=torch.float32, device="cuda")
+    J().jab_loss_forward_kl(c.desc, c.B, c.T, c.X, c.W, A, qkv_ref, bits, scales, 0.1, loss, ws,
+                            mse=mse, kl=kl, kl_rows=rows)
+    assert J().jab_get_device_status() == 0
+    a_ref = c.oracle_teacher()
+    for i, b in enumerate(bits):
+        s = scales[i].cpu().numpy()
+        r = O.kl_attention_term(c.x64, c.w64, s, b, c.odesc)
+        ro = r["kl_rows"]
+        floor = KL_ROW_ATOL * c.Hq * c.T                  # per-row floor, summed as the batchmean
+        assert abs(kl[i].item() - r["kl"]) <= KL_TOL[b] * r["kl"] + floor, (b, kl[i].item(), r["kl"])
+        if b in KL_ROW_TOL:
+            err = np.abs(np64(rows[i]) - ro)
+            # each row within KL_ROW_TOL of itself plus the mean row (t = 0: one visible key, KL 0)
+            bound = KL_ROW_TOL[b] * (ro + ro.mean()) + KL_ROW_ATOL
+            assert (err <= bound).all(), (b, (err / bound).max())
+        m = O.jab_loss(c.x64, c.w64, s, b, c.odesc, a_ref=a_ref)["loss"]
+        assert abs(mse[i].item() - m) <= L_TOL * m
+        j = O.jab_loss_joint(c.x64, c.w64, s, b, c.odesc, lam_kl=0.1)["loss"]
+        assert abs(loss[i].item() - j) <= L_TOL * j, (b, loss[i].item(), j)
+        lam = float(np.float32(0.1))                      # lambda_kl crosses the ABI as a float
+        np.testing.assert_allclose(loss[i].item(), mse[i].item() + lam * kl[i].item(), rtol=1e-12)
 
 
 # ------------------------------------------------------------------ STE / LSQ backward
@@ -213,6 +259,116 @@ def test_repeated_calls_are_bit_identical():
     J().jab_loss_forward(c.desc, c.B, c.T, c.X, c.W, A, [2, 4], s, l1, ws)
     J().jab_loss_forward(c.desc, c.B, c.T, c.X, c.W, A, [2, 4], s, l2, ws)
     assert torch.equal(l1, l2)
+
+
+# ------------------------------------------------------------------ fitting loop (App. B, Eq. 14, 15)
+def test_prepared_x_backward_matches_the_plain_call():
+    """jab_loss_backward_scales_prepared (X converted once by jab_prepare_x) computes what
+    jab_loss_backward_scales computes; another X than the prepared one is refused."""
+    c = case("mistral_G64_T70")
+    ws = c.workspace()
+    A, _, _ = c.gpu_teacher(ws)
+    s = c.gpu_scales(2, mode=1)
+    l1 = torch.empty(1, dtype=torch.float64, device="cuda")
+    l2 = torch.empty_like(l1)
+    g1, g2 = torch.empty_like(s), torch.empty_like(s)
+    J().jab_loss_backward_scales(c.desc, c.B, c.T, c.X, c.W, A, 2, s, 0.0, l1, g1, ws)
+    J().jab_prepare_x(c.desc, c.B, c.T, c.X, ws)
+    J().jab_loss_backward_scales_prepared(c.desc, c.B, c.T, c.X, c.W, A, 2, s, 0.0, l2, g2, ws)
+    assert l1.item() == l2.item()                      # same kernels, fixed-order loss reduction
+    # (the scale gradient sums with fp32 atomics: the order differs between calls)
+    np.testing.assert_allclose(np64(g2), np64(g1), rtol=1e-4, atol=1e-5 * np.abs(np64(g1)).max())
+    with pytest.raises(J().JabError) as e:
+        J().jab_loss_backward_scales_prepared(c.desc, c.B, c.T, c.X.clone(), c.W, A, 2, s, 0.0, l2,
+                                              g2, ws)
+    assert e.value.status == 1
+    assert J().jab_get_device_status() == 0
+
+
+def test_ste_scale_fitting_loop_lowers_the_loss():
+    """Ten steps of the scale fit of App. B "Joint STE fine-tuning" on a long-context-workload case
+    (2 bits, G 64, min-MSE warm start): Adam with the grid-relative rate eta_s = alpha_s * mean grid
+    step (Eq. 14, alpha_s = 0.02, cosine-annealed), the optimizer caller-side in torch, gradients
+    from jab_loss_backward_scales_prepared. The first loss matches the oracle; the loss falls; the
+    flip count of Eq. 15 against the warm start is what jab_flip_rate reports."""
+    c = case("mistral_G64_T70")
+    ws = c.workspace()
+    A, _, _ = c.gpu_teacher(ws)
+    s0 = c.gpu_scales(2, mode=1)
+    s = torch.nn.Parameter(s0.clone())
+    steps = 10
+    opt = torch.optim.Adam([s], lr=0.02 * s0.mean().item())
+    sched = torch.optim.lr_scheduler.CosineAnnealingLR(opt, T_max=steps)
+    J().jab_prepare_x(c.desc, c.B, c.T, c.X, ws)
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    grad = torch.empty_like(s0)
+    losses = []
+    for _ in range(steps):
+        J().jab_loss_backward_scales_prepared(c.desc, c.B, c.T, c.X, c.W, A, 2, s.data, 0.0, loss,
+                                              grad, ws)
+        losses.append(loss.item())
+        s.grad = grad.clone()
+        opt.step()
+        sched.step()
+    assert J().jab_get_device_status() == 0
+    r = O.jab_loss(c.x64, c.w64, s0.cpu().numpy(), 2, c.odesc, a_ref=c.oracle_teacher())
+    assert abs(losses[0] - r["loss"]) <= L_TOL * r["loss"]
+    assert losses[-1] < losses[0], losses
+    codes0 = torch.empty(c.W.shape, dtype=torch.int8, device="cuda")
+    codes1 = torch.empty_like(codes0)
+    J().jab_quantize(c.desc, 2, c.W, s0, codes=codes0)
+    J().jab_quantize(c.desc, 2, c.W, s.data.contiguous(), codes=codes1)
+    count = torch.empty(1, dtype=torch.int64, device="cuda")
+    J().jab_flip_rate(codes1, codes0, count)
+    assert count.item() == O.flip_count(codes1.cpu().numpy(), codes0.cpu().numpy()) > 0
+
+
+def test_flip_rate_is_an_exact_count():
+    """Eq. 15: the number of changed grid positions, bit-exact against the oracle's count, on a
+    length with a ragged tail (not a multiple of 16 bytes) and on an empty range."""
+    c = case("gpt2_T200")
+    s1 = c.gpu_scales(3)
+    s2 = s1 * 0.93
+    ca = torch.empty(c.W.shape, dtype=torch.int8, device="cuda")
+    cb = torch.empty_like(ca)
+    J().jab_quantize(c.desc, 3, c.W, s1, codes=ca)
+    J().jab_quantize(c.desc, 3, c.W, s2, codes=cb)
+    count = torch.empty(1, dtype=torch.int64, device="cuda")
+    fa, fb = ca.view(-1), cb.view(-1)
+    for n in (fa.numel(), fa.numel() - 5, 37, 0):
+        J().jab_flip_rate(fa[:n], fb[:n], count)
+        assert count.item() == O.flip_count(fa[:n].cpu().numpy(), fb[:n].cpu().numpy()), n
+    assert count.item() == 0
+
+
+# ------------------------------------------------------------------ fp16 operand range
+def test_fp16_range_guards():
+    """Values the fp16 tensor-core operands cannot hold are reported with JAB_ERR_RANGE rather than
+    carried on as inf: the projected Q|K|V, and the output error dO of the backward; a non-finite
+    forward loss is reported as JAB_ERR_NONFINITE. No GPU fault: the kernels run to completion."""
+    c = case("gpt2_T200")
+    ws = c.workspace()
+    A = torch.empty((c.B, c.T, c.Hq * c.dh), dtype=torch.float32, device="cuda")
+    X = c.X.clone()
+    X[0, 3, :] = 1000.0                      # in the fp16 range, as is the weight row below ...
+    W = c.W.clone()
+    W[5, :] = 200.0                          # ... but Q[0, 3, 5] = 768 * 2e5 is not
+    J().jab_get_device_status()
+    J().jab_reference_forward(c.desc, c.B, c.T, X, W, A, ws)
+    assert J().jab_get_device_status() == 5
+    A, _, _ = c.gpu_teacher(ws)
+    s = c.gpu_scales(3)
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    grad = torch.empty_like(s)
+    A2 = A.clone()
+    A2[1, 7, 9] = 1.0e6                      # dO = A_hat - A_ref leaves the fp16 range
+    J().jab_loss_backward_scales(c.desc, c.B, c.T, c.X, c.W, A2, 3, s, 1.0, loss, grad, ws)
+    assert J().jab_get_device_status() == 5
+    A2[1, 7, 9] = float("inf")               # the forward-only loss checks its total
+    J().jab_loss_forward(c.desc, c.B, c.T, c.X, c.W, A2, [3], [s], loss, ws)
+    assert J().jab_get_device_status() == 4
+    J().jab_loss_forward(c.desc, c.B, c.T, c.X, c.W, A, [3], [s], loss, ws)
+    assert J().jab_get_device_status() == 0
 
 
 # ------------------------------------------------------------------ error paths (no GPU fault)

@@ -51,6 +51,60 @@ def test_quantizer_golden_worked_examples():
         np.testing.assert_array_equal(O.lsq_factor(v, case["bits"])[0], case["lsq"])
 
 
+def _fp32_round_exact(x):
+    """Correctly rounded binary32 value of a positive rational x (normal range), ties to even,
+    by exact integer arithmetic (independent of numpy's float32 division)."""
+    from fractions import Fraction
+    x = Fraction(x)
+    e = 0
+    while x >= 2:
+        x /= 2
+        e += 1
+    while x < 1:
+        x *= 2
+        e -= 1
+    m = x * 2 ** 23
+    fl, rem = divmod(m.numerator, m.denominator)
+    rem = Fraction(rem, m.denominator)
+    if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and fl % 2 == 1):
+        fl += 1
+    return Fraction(fl, 2 ** 23) * Fraction(2) ** e
+
+
+def test_quantizer_fp32_quotient_lands_on_half_integers():
+    """Reading R1 of Eq. 2: the code is taken from the fp32 quotient. The fixture's scales are not
+    powers of two and the exact quotients sit just off a half-integer that their fp32 rounding hits,
+    so a float64 quotient (or any other rounding of w/s) gives a different code."""
+    from fractions import Fraction
+    with open(os.path.join(GOLDEN, "quantizer_worked.json")) as f:
+        fx = json.load(f)["fp32_quotient_cases"]
+    w = np.array([fx["w"]])
+    s = np.array([[float.fromhex(h) for h in fx["scale_hex"]]], dtype=np.float32)
+    for i, (num, den) in enumerate(fx["exact_quotient"]):       # the fixture's own arithmetic
+        exact = Fraction(fx["w"][i]) / Fraction(float(s[0, i]))
+        assert exact == Fraction(num, den)
+        assert exact.denominator != 2 and _fp32_round_exact(exact) == Fraction(fx["v"][i])
+        assert round(float(exact)) != fx["codes"][i]               # float64 quotient: other code
+    codes, w_hat, v = O.quantize(w, s, fx["bits"], 1)
+    assert codes[0].tolist() == fx["codes"]
+    np.testing.assert_array_equal(v[0], fx["v"])
+    np.testing.assert_array_equal(w_hat[0], [float.fromhex(h) for h in fx["w_hat_hex"]])
+    np.testing.assert_array_equal(O.lsq_factor(v, fx["bits"])[0], fx["lsq"])
+
+
+def test_flip_count_hand_worked():
+    """Eq. 15 on six weights, b = 3, worked by hand. Before: s = 1/2, after: s = 3/8 (fp32-exact).
+    w              = 0.3,   -0.55,  1.0, 0.1, 2.0, -1.6
+    w / (1/2)      = 0.6,   -1.1,   2.0, 0.2, 4.0, -3.2   -> codes 1, -1, 2, 0, 3, -3
+    w / (3/8)      = 0.8,   -1.466, 2.666, 0.266, 5.33, -4.266 -> codes 1, -1, 3, 0, 3, -3
+    One grid position changes (1.0: 2 -> 3); 2.0 and -1.6 clamp to +-qmax on both sides."""
+    w = np.array([[0.3, -0.55, 1.0, 0.1, 2.0, -1.6]])
+    ca, _, _ = O.quantize(w, np.array([[0.5]], dtype=np.float32), 3, 6)
+    cb, _, _ = O.quantize(w, np.array([[0.375]], dtype=np.float32), 3, 6)
+    assert ca.tolist() == [[1, -1, 2, 0, 3, -3]] and cb.tolist() == [[1, -1, 3, 0, 3, -3]]
+    assert O.flip_count(ca, cb) == 1 and O.flip_count(ca, ca) == 0
+
+
 @pytest.mark.parametrize("bits", [2, 3, 4, 5, 8])
 def test_quantizer_brute_force_nearest_grid_point(bits):
     """Eq. 2 equals the nearest point of {-qmax..qmax} to the fp32 quotient, ties to even."""
@@ -515,6 +569,21 @@ def test_omega_scores_vanish_on_the_grid_and_scale_with_depth():
     w2 = w + rng.standard_normal(w.shape) * 2.0 ** -7
     c1, c2 = O.omega_scores(2.5, w2, s, 3, 4, layers_after=3)
     assert c1 > 0 and c2 == 3 * c1
+
+
+def test_omega_scores_hand_worked():
+    """Eq. 6 on one row worked by hand. b = 3 (qmax = 3), one group of 5, s = 1/2:
+    w      = 0.375, -0.6875, 1.25, 0.0625, 2.0
+    w / s  = 0.75,  -1.375,  2.5,  0.125,  4.0
+    q      = 1,     -1,      2,    0,      3      (2.5 -> 2 half to even; 4 clamps to qmax)
+    Q(w)   = 0.5,   -0.5,    1.0,  0.0,    1.5
+    Q(w)-w = 0.125, 0.1875, -0.25, -0.0625, -0.5
+    ||Q(w) - W||_F^2 = 1/64 + 9/256 + 1/16 + 1/256 + 1/4 = 0.3671875.
+    With Tr(H) = 2: C1 = 0.734375; with L - i = 3 layers after it: C2 = 2.203125."""
+    w = np.array([[0.375, -0.6875, 1.25, 0.0625, 2.0]])
+    s = np.array([[0.5]], dtype=np.float32)
+    c1, c2 = O.omega_scores(2.0, w, s, 3, 5, layers_after=3)
+    assert c1 == 0.734375 and c2 == 2.203125
 
 
 # ------------------------------------------------------------------ allocation (Eq. 7, App. B, R20)

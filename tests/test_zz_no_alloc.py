@@ -41,10 +41,21 @@ def test_noalloc_forward_matches_workspace_forward_twice():
     ref = torch.empty(len(bits), dtype=torch.float64, device="cuda")
     ref_parts = torch.empty((len(bits), B, wl.shape.n_q_heads), dtype=torch.float64, device="cuda")
     J.jab_loss_forward(desc, B, T, X, W, A, bits, scales, ref, ws, sse_parts=ref_parts)
-    for _ in range(2):                                # the scratch keeps the last call's contents
-        out = torch.full_like(ref, float("nan"))
-        parts = torch.full_like(ref_parts, float("nan"))
+    outs = [(torch.full_like(ref, float("nan")), torch.full_like(ref_parts, float("nan")))
+            for _ in range(3)]
+    # the first call on a device may load the library's module that holds the fixed array (lazy
+    # module loading), which is when the device gives the array its memory: measure after it
+    J.jab_loss_forward_noalloc(desc, B, T, X, W, A, bits, scales, outs[0][0], sse_parts=outs[0][1])
+    torch.cuda.synchronize()
+    torch.testing.assert_close(outs[0][0], ref, rtol=L_TOL, atol=0)
+    outs = outs[1:]
+    for out, parts in outs:                           # the scratch keeps the last call's contents
+        torch.cuda.synchronize()
+        free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
         J.jab_loss_forward_noalloc(desc, B, T, X, W, A, bits, scales, out, sse_parts=parts)
+        torch.cuda.synchronize()
+        # the call took no device memory: neither from the device nor from torch's allocator
+        assert torch.cuda.mem_get_info()[0] == free0 and torch.cuda.memory_allocated() == alloc0
         torch.testing.assert_close(out, ref, rtol=L_TOL, atol=0)
         torch.testing.assert_close(parts, ref_parts, rtol=L_TOL, atol=0)
     assert J.jab_get_device_status() == 0
