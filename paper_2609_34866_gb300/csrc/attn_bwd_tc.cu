@@ -491,12 +491,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 //   warp 0      TMA: Q and dO of each tile through the staging tile, K ring (3 stages)
 //   warp 1      TMEM owner, tcgen05.cp of Q and dO, UMMA issuer (one thread, event-driven)
 //   warps 2..9  elementwise: dS = P (dP - D) with P = exp2(S scale log2(e) - lse), fp16 to shared
-//               memory; the epilogue (transpose of RoPE, dQKV^T columns) while the next tile's Q and
-//               dO are copied in
+//               memory; at the end of a tile they read dQ out of TMEM, apply the transpose of RoPE
+//               and stage the tile transposed (bf16) in the dS buffer, then go on with the next tile
 //   warp 10     TMA: V ring (2 stages)
+//   warp 11     stores the staged tile as dQKV^T columns (coalesced 16-byte stores) while the
+//               elementwise warps work on the next tile's first block
 // A tile's Q is copied in once the previous tile's last S has completed and its dO once the last dP
 // has; the staging tile is refilled with the next operand as soon as each copy has completed.
-constexpr int DQ_THREADS = 352;
+constexpr int DQ_THREADS = 384;  // 12 warps: 65536 / 384 leaves 168 registers per thread
+constexpr int DQ_STORE_WARP = 11;
 
 template <int DH>
 struct DqLayout {
@@ -520,36 +523,10 @@ struct DqLayout {
 
 struct DqBars {
   uint64_t stg_full, stg_empty, k_full[3], k_empty[3], v_full[2], v_empty[2], s_full, s_empty;
-  uint64_t p_full, p_empty, o_full, o_empty, drain;
+  uint64_t p_full, p_empty, o_full, o_empty, out_full, out_free, drain;
   uint32_t tmem_base;
   int abort;
-  int ew_count;  // arrivals at the elementwise warps' epilogue barrier
 };
-
-// Time-bounded barrier of the 8 elementwise warps (epoch-numbered; no hardware barrier that could
-// hang if a warp left early).
-__device__ __forceinline__ void ew_barrier(DqBars* bars, int epoch, volatile int* abort,
-                                           int* status) {
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) {
-    __threadfence_block();
-    atomicAdd(&bars->ew_count, 1);
-    volatile int* c = &bars->ew_count;
-    const uint64_t t0 = tc::globaltimer();
-    for (uint32_t it = 0; *c < EW_WARPS * epoch; ++it) {
-      if ((it & 63u) == 0) {
-        if (*abort) break;
-        if (tc::globaltimer() - t0 > tc::kWaitLimitNs) {
-          *abort = 1;
-          report(status, JAB_ERR_TIMEOUT);
-          break;
-        }
-      }
-    }
-    __threadfence_block();
-  }
-  __syncwarp();
-}
 
 struct DqTile {
   int qb, h, b;
@@ -597,9 +574,10 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
     tc::mbar_init(&bars->p_empty, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->o_empty, EW_WARPS);
+    tc::mbar_init(&bars->out_full, EW_WARPS);  // the tile's dQ is staged in the dS buffer
+    tc::mbar_init(&bars->out_free, 1);         // the store warp has read the staged tile
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
-    bars->ew_count = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_q);
     tc::prefetch_tmap(&tm_kv);
@@ -751,6 +729,21 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
+  } else if (warp == DQ_STORE_WARP) {  // ------------------------------------- dQKV^T stores
+    // The staged tile of each tile in turn, once the elementwise warps have written it; the buffer
+    // is handed back before the same warps write the next tile's first dS into it.
+    const bf16_t* stage = reinterpret_cast<const bf16_t*>(smem + L::DS_OFF);
+    int n = 0;
+    for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
+         tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
+      const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+      const int q0 = tl.qb * BQ;
+      if (!tc::mbar_wait(&bars->out_full, n & 1, abort, p.status)) break;
+      store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
+                     (int64_t)tl.b * p.T + q0, min(BQ, p.T - q0), lane, 32);
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->out_free);
+    }
   } else {  // ------------------------------------------------ elementwise: row = query, 64 keys
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
@@ -761,12 +754,12 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
     bf16_t* stage = reinterpret_cast<bf16_t*>(smem + L::DS_OFF);
     bool ok = true;
     uint32_t J = 0;
-    int n = 0, epoch = 0;
+    int n = 0;
     for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
          tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
       const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
       const int nkb = n_kb_of(tl);
-      const int q0 = tl.qb * BQ, t = q0 + row, row0 = tl.b * p.T;
+      const int q0 = tl.qb * BQ, t = q0 + row;
       const bool valid_row = t < p.T;
       const int64_t lrow = ((int64_t)tl.b * p.Hq + tl.h) * p.lse_pitch + (valid_row ? t : 0);
       const float lse2 = valid_row ? p.lse[lrow] : INFINITY;  // P = 0 on rows past T
@@ -819,8 +812,9 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
             }
           }
         }
-        if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
-          ok = false;
+        if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status) ||
+            (j == 0 && n > 0 && !tc::mbar_wait(&bars->out_free, (n - 1) & 1, abort, p.status))) {
+          ok = false;  // (the first dS of a tile waits until the previous tile's dQ is stored)
           break;
         }
 #pragma unroll
@@ -839,8 +833,8 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       }
       if (!ok) break;
       // Epilogue: dQ rows (transpose of RoPE) staged transposed in the dS buffer (free until this
-      // tile's successor writes its first dS, which these same warps do next), then stored as
-      // dQKV^T columns with coalesced 16-byte stores.
+      // tile's successor writes its first dS, which waits for the store warp), stored by the store
+      // warp as dQKV^T columns.
       if (!tc::mbar_wait(&bars->o_full, n & 1, abort, p.status) ||
           !tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
         ok = false;
@@ -856,11 +850,10 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       }
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->o_empty);  // dQ accumulator reusable
-      ew_barrier(bars, ++epoch, abort, p.status);
-      store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
-                     (int64_t)row0 + q0, min(BQ, p.T - q0), threadIdx.x - 64, EW_WARPS * 32);
-      ew_barrier(bars, ++epoch, abort, p.status);
+      if (lane == 0) {
+        tc::mbar_arrive(&bars->o_empty);   // dQ accumulator reusable
+        tc::mbar_arrive(&bars->out_full);  // this warp's share of the staged tile is written
+      }
     }
   }
   tc::fence_before_sync();
