@@ -127,6 +127,42 @@ jab_status jab_loss_forward_kl(const jab_block_desc* desc, int32_t B, int32_t T,
                                double* mse_dev, double* kl_dev, float* kl_rows_dev, void* ws,
                                size_t ws_bytes, jab_stream_t stream);
 
+/* Hutchinson estimate of Tr(H), the trace of the Hessian of L_JAB (MSE term) w.r.t. the joint
+ * weights at the float point (Section 2.4, Eq. 5): Tr(H) ~ (1/m) sum_i v_i^T H v_i over m
+ * Rademacher probes v_i. At the float weights H = 2 J_A^T J_A / n (n = B T Hq d_h), so each probe
+ * costs one forward-mode (JVP) pass: v^T H v = 2 ||J_A v||^2 / n, with J_A v the derivative of the
+ * block output along v (the tangent projection X v^T through the same RoPE, then the attention
+ * JVP), no second backward pass.
+ * Probe i, entry e (row-major over [(Hq+2Hkv) d_h, d_model]) is -1 when the top bit of the
+ * (i * (Hq+2Hkv) d_h d_model + e + 1)-th output of SplitMix64 (Steele, Lea and Flood, 2014)
+ * seeded with `seed` is set, else +1.
+ *   A_ref_dev, lse_ref_dev  the teacher pass of jab_reference_forward (lse_ref required)
+ *   trace_dev      out fp64 [1]            the estimate
+ *   vhv_dev        out fp64 [n_probes] or NULL   v_i^T H v_i of each probe
+ *   ws             at least jab_workspace_size(desc, B, T, 2, 0) bytes */
+jab_status jab_hutchinson_trace(const jab_block_desc* desc, int32_t B, int32_t T,
+                                const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                const float* lse_ref_dev, int32_t n_probes, uint64_t seed,
+                                double* trace_dev, double* vhv_dev, void* ws, size_t ws_bytes,
+                                jab_stream_t stream);
+
+/* The probe entries of jab_hutchinson_trace: entries first .. first + n - 1 of the probe sequence
+ * of `seed` (probe i, entry e is number i * (Hq+2Hkv) d_h d_model + e) as fp16 -1 / +1.
+ *   out_dev        out fp16 [n], 16-byte aligned; n a multiple of 8 */
+jab_status jab_rademacher_probes(uint64_t seed, int64_t first, int64_t n, void* out_dev,
+                                 jab_stream_t stream);
+
+/* Sensitivity scores of Eq. 6 for n_cand candidate (bits, scales) quantisations of the block:
+ *   C1: Omega(b) = Tr(H) ||Q_b(W) - W||_F^2,   C2: (L - i) Omega(b) with layers_after = L - i.
+ *   trace_dev      fp64 [1] on the device (e.g. from jab_hutchinson_trace)
+ *   c1_dev         out fp64 [n_cand];  c2_dev  out fp64 [n_cand] or NULL
+ *   ws             at least jab_workspace_size(desc, 1, 1, n_cand, 0) bytes
+ * The squared error is summed in fp64 in a fixed order (repeated calls give identical bits). */
+jab_status jab_omega_scores(const jab_block_desc* desc, const void* W_dev, int32_t n_cand,
+                            const int32_t* bits_host, const float* const* scales_host,
+                            const double* trace_dev, int32_t layers_after, double* c1_dev,
+                            double* c2_dev, void* ws, size_t ws_bytes, jab_stream_t stream);
+
 /* Forward L_JAB and its gradient w.r.t. the scales for one candidate (App. B "Joint STE fine-tuning",
  * Eq. 13): d w_hat / d w = 1 (STE) and d w_hat / d s = q - v if |v| <= qmax, else sign(v) qmax, with
  * v = w / s.

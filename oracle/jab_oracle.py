@@ -54,7 +54,7 @@ __all__ = [
     "split_heads", "causal_gqa_attention", "block_forward", "jab_loss", "attention_vjp",
     "jab_loss_and_grad", "lsq_factor", "default_kappa", "kl_attention_term", "jab_loss_joint",
     "attention_jvp", "block_jvp", "gn_quadratic_form", "hutchinson_trace", "omega_scores",
-    "pareto_frontier", "allocate_bits", "flip_count",
+    "pareto_frontier", "allocate_bits", "flip_count", "splitmix64", "rademacher_probe",
 ]
 
 
@@ -420,6 +420,31 @@ def gn_quadratic_form(x, w, V, desc) -> float:
     """v^T H v at the float point (Eq. 5, lambda_KL = 0): 2 ||J_A v||^2 / n (reading R19)."""
     jv = block_jvp(x, w, V, desc)
     return 2.0 * float((jv ** 2).sum()) / jv.size
+
+
+_SM64_GAMMA = np.uint64(0x9E3779B97F4A7C15)
+_SM64_M1 = np.uint64(0xBF58476D1CE4E5B9)
+_SM64_M2 = np.uint64(0x94D049BB133111EB)
+
+
+def splitmix64(seed: int, counters) -> np.ndarray:
+    """Outputs number n + 1 (n = counters) of the SplitMix64 generator seeded with `seed` (Steele,
+    Lea and Flood, "Fast splittable pseudorandom number generators", 2014): the state after n + 1
+    steps is seed + (n + 1) * gamma (mod 2^64), passed through the generator's mixing function."""
+    n = np.asarray(counters, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = np.uint64(seed) + (n + np.uint64(1)) * _SM64_GAMMA
+        z = (z ^ (z >> np.uint64(30))) * _SM64_M1
+        z = (z ^ (z >> np.uint64(27))) * _SM64_M2
+        return z ^ (z >> np.uint64(31))
+
+
+def rademacher_probe(seed: int, probe: int, shape) -> np.ndarray:
+    """Rademacher probe number `probe` (entries +-1) of the Hutchinson estimate: entry e (row-major)
+    takes output probe * size + e + 1 of splitmix64(seed); -1 when its top bit is set, else +1."""
+    size = int(np.prod(shape))
+    z = splitmix64(seed, np.arange(size, dtype=np.uint64) + np.uint64(probe * size))
+    return np.where((z >> np.uint64(63)) == 1, -1.0, 1.0).reshape(shape)
 
 
 def hutchinson_trace(x, w, desc, probes) -> float:

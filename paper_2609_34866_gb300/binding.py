@@ -80,6 +80,11 @@ def lib() -> ctypes.CDLL:
                                                     _P, sz, _P]
     L.jab_flip_rate.argtypes = [_P, _P, ctypes.c_int64, _P, _P]
     L.jab_reference_projection.argtypes = [D, i32, i32, _P, _P, _P, _P, sz, _P]
+    L.jab_hutchinson_trace.argtypes = [D, i32, i32, _P, _P, _P, _P, i32, ctypes.c_uint64, _P, _P,
+                                       _P, sz, _P]
+    L.jab_rademacher_probes.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, _P, _P]
+    L.jab_omega_scores.argtypes = [D, _P, i32, ctypes.POINTER(i32), ctypes.POINTER(_P), _P, i32,
+                                   _P, _P, _P, sz, _P]
     L.jab_loss_forward_kl.argtypes = [D, i32, i32, _P, _P, _P, _P, i32, ctypes.POINTER(i32),
                                       ctypes.POINTER(_P), f32, _P, _P, _P, _P, _P, sz, _P]
     L.jab_quantize.argtypes = [D, i32, _P, _P, _P, _P, _P]
@@ -99,7 +104,8 @@ def lib() -> ctypes.CDLL:
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
                "jab_loss_backward_scales", "jab_loss_backward_weights", "jab_allocate_bits",
                "jab_prepare_x", "jab_loss_backward_scales_prepared", "jab_flip_rate",
-               "jab_reference_projection", "jab_loss_forward_kl",
+               "jab_reference_projection", "jab_loss_forward_kl", "jab_hutchinson_trace",
+               "jab_omega_scores", "jab_rademacher_probes",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
                "jab_selftest_wait_timeout",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
@@ -206,6 +212,39 @@ def jab_loss_forward_kl(desc, B, T, X, W, A_ref, QKV_ref, bits: Sequence[int],
         _ptr(kl, torch.float64, "kl"), _ptr(kl_rows, torch.float32, "kl_rows"), ws.ptr, ws.nbytes,
         _stream(stream))
     _check(st, "jab_loss_forward_kl")
+
+
+def jab_hutchinson_trace(desc, B, T, X, W, A_ref, lse_ref, n_probes: int, seed: int, trace,
+                         ws: Workspace, vhv=None, stream=None):
+    """Tr(H) of L_JAB at the float weights from n_probes Rademacher probes (Section 2.4, Eq. 5)."""
+    st = lib().jab_hutchinson_trace(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), _ptr(lse_ref, torch.float32, "lse_ref"), int(n_probes),
+        int(seed) & ((1 << 64) - 1), _ptr(trace, torch.float64, "trace"),
+        _ptr(vhv, torch.float64, "vhv"), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_hutchinson_trace")
+
+
+def jab_rademacher_probes(seed: int, first: int, out, stream=None):
+    """Probe entries first .. first + out.numel() - 1 of jab_hutchinson_trace's sequence (fp16 +-1)."""
+    st = lib().jab_rademacher_probes(int(seed) & ((1 << 64) - 1), int(first), int(out.numel()),
+                                     _ptr(out, torch.float16, "out"), _stream(stream))
+    _check(st, "jab_rademacher_probes")
+
+
+def jab_omega_scores(desc, W, bits: Sequence[int], scales: Sequence[torch.Tensor], trace,
+                     layers_after: int, c1, ws: Workspace, c2=None, stream=None):
+    """Eq. 6: C1 = Tr(H) ||Q_b(W) - W||^2 per candidate (and C2 = layers_after * C1)."""
+    n = len(bits)
+    if len(scales) != n:
+        raise ValueError("bits and scales must have the same length")
+    bits_arr = (ctypes.c_int32 * n)(*[int(b) for b in bits])
+    sc_arr = (ctypes.c_void_p * n)(*[_ptr(s, torch.float32, "scales") for s in scales])
+    st = lib().jab_omega_scores(ctypes.byref(desc), _ptr(W, torch.bfloat16, "W"), n, bits_arr,
+                                sc_arr, _ptr(trace, torch.float64, "trace"), int(layers_after),
+                                _ptr(c1, torch.float64, "c1"), _ptr(c2, torch.float64, "c2"),
+                                ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "jab_omega_scores")
 
 
 def jab_loss_forward_noalloc(desc, B, T, X, W, A_ref, bits: Sequence[int],

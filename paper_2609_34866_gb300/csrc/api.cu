@@ -347,6 +347,106 @@ jab_status jab_loss_forward_kl(const jab_block_desc* desc, int32_t B, int32_t T,
   return JAB_OK;
 }
 
+jab_status jab_hutchinson_trace(const jab_block_desc* desc, int32_t B, int32_t T,
+                                const void* X_dev, const void* W_dev, const float* A_ref_dev,
+                                const float* lse_ref_dev, int32_t n_probes, uint64_t seed,
+                                double* trace_dev, double* vhv_dev, void* ws, size_t ws_bytes,
+                                jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (n_probes < 1 || !X_dev || !W_dev || !A_ref_dev || !lse_ref_dev || !trace_dev || !ws)
+    return JAB_ERR_INVALID_ARG;
+  if (!aligned16(X_dev) || !aligned16(W_dev) || !aligned16(A_ref_dev) ||
+      (reinterpret_cast<uintptr_t>(lse_ref_dev) & 3u) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, B, T, 2, false);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  const int64_t N = (int64_t)B * T;
+  const int D = (int)block_rows(desc), dm = desc->d_model, dh = desc->head_dim;
+  float* cos_t = reinterpret_cast<float*>(w + wp.rope);
+  float* sin_t = cos_t + (int64_t)T * (dh / 2);
+  char* qkv = w + wp.qkv;                      // primal [N, D]
+  char* tqkv = qkv + (size_t)N * D * 2;        // tangent [N, D]
+  double* part = reinterpret_cast<double*>(w + wp.part);
+  double* tmp = reinterpret_cast<double*>(w + wp.scal);
+  const int nP = (T + attn_jvp_tc_rows() - 1) / attn_jvp_tc_rows();
+  const double n_el = (double)N * desc->n_q_heads * dh;
+  if ((s = convert_x_into(desc, B, T, X_dev, ws, wp, status, sms, st)) != JAB_OK) return s;
+  JAB_SITE("quantize", 1, launch_quantize(W_dev, nullptr, D, dm, desc->group_size, 0, w + wp.w16,
+                                          nullptr, nullptr, status, sms, st));
+  if (desc->use_rope) JAB_SITE("rope_table", 1, launch_rope_table(T, dh, desc->rope_theta, cos_t, sin_t, st));
+  if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, qkv, cos_t, sin_t, status, st)) !=
+      JAB_OK)
+    return s;
+  JAB_SITE("memset_grad", 0, cudaMemsetAsync(trace_dev, 0, sizeof(double), st));
+  for (int pr = 0; pr < n_probes; ++pr) {
+    // probe pr: entries pr * D * d .. of the seed's sequence, the tangent projection X V^T + RoPE
+    JAB_SITE("probe", 1, launch_rademacher_probe(seed, (uint64_t)pr * D * dm, (int64_t)D * dm,
+                                                 w + wp.w16, sms, st));
+    if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, tqkv, cos_t, sin_t, status,
+                            st)) != JAB_OK)
+      return s;
+    JAB_SITE("attn_jvp", 1, launch_attn_jvp_tc(qkv, tqkv, lse_ref_dev, T, A_ref_dev, B, T,
+                                               desc->n_q_heads, desc->n_kv_heads, dh,
+                                               softmax_scale(desc), part, nP, status, st));
+    double* vhv = vhv_dev ? vhv_dev + pr : tmp;
+    // v^T H v = 2 ||J_A v||^2 / n (Eq. 5 at the float weights, MSE term)
+    JAB_SITE("loss_reduce", 1, launch_loss_reduce(part, 1, B, desc->n_q_heads, nP, 2.0 / n_el,
+                                                  vhv, nullptr, status, st));
+    JAB_SITE("loss_combine", 1, launch_loss_combine(trace_dev, vhv, 1.0 / n_probes, 1, trace_dev,
+                                                    st));
+  }
+  return JAB_OK;
+}
+
+jab_status jab_rademacher_probes(uint64_t seed, int64_t first, int64_t n, void* out_dev,
+                                 jab_stream_t stream) {
+  if (!out_dev || n < 0 || first < 0 || (n & 7) || !aligned16(out_dev)) return JAB_ERR_INVALID_ARG;
+  if (n == 0) return JAB_OK;
+  int* status;
+  int sms;
+  const jab_status s = device_info(&status, &sms);
+  if (s != JAB_OK) return s;
+  JAB_TRY(launch_rademacher_probe(seed, (uint64_t)first, n, out_dev, sms,
+                                  reinterpret_cast<cudaStream_t>(stream)));
+  return JAB_OK;
+}
+
+jab_status jab_omega_scores(const jab_block_desc* desc, const void* W_dev, int32_t n_cand,
+                            const int32_t* bits_host, const float* const* scales_host,
+                            const double* trace_dev, int32_t layers_after, double* c1_dev,
+                            double* c2_dev, void* ws, size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if (n_cand < 1 || !W_dev || !bits_host || !scales_host || !trace_dev || !c1_dev || !ws ||
+      layers_after < 0 || !aligned16(W_dev) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return JAB_ERR_INVALID_ARG;
+  for (int c = 0; c < n_cand; ++c)
+    if (bits_host[c] < 2 || bits_host[c] > 8 || scales_host[c] == nullptr)
+      return JAB_ERR_INVALID_ARG;
+  const Workspace wp = plan_workspace(desc, 1, 1, n_cand, false);
+  if (ws_bytes < wp.total) return JAB_ERR_INVALID_ARG;
+  int* status;
+  int sms;
+  if ((s = device_info(&status, &sms)) != JAB_OK) return s;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  double* red = reinterpret_cast<double*>(static_cast<char*>(ws) + wp.red);
+  const int D = (int)block_rows(desc), dm = desc->d_model;
+  for (int c = 0; c < n_cand; ++c)
+    JAB_SITE("qerr", 1, launch_qerr_partial(W_dev, scales_host[c], D, dm, desc->group_size,
+                                            bits_host[c], red + (size_t)c * kRedBlocks, kRedBlocks,
+                                            status, st));
+  JAB_SITE("omega", 1, launch_omega_finish(red, kRedBlocks, n_cand, trace_dev,
+                                           (double)layers_after, c1_dev, c2_dev, st));
+  return JAB_OK;
+}
+
 // Steps shared by the backward entry points (App. B, STE): quantise, project (+ RoPE), attention
 // forward in mode 2 (loss partials, dO = A_hat - A_ref, lse, D), the loss, and the attention backward
 // into dQKV^T (bf16 [D, ldt]) in the workspace. Checks the arguments common to both.

@@ -62,6 +62,21 @@ cudaError_t launch_attn_kl_tc(const void* qkv_s, int64_t ldq, const void* qkv_t,
                               int C, int Hq, int Hkv, int dh, float scale, double* part, int nP,
                               float* kl_rows, int* status, cudaStream_t st);
 
+// attn_jvp_tc.cu: ||J_A v||^2 partials of the forward-mode attention product (Section 2.4). qkv and
+// tqkv: primal and tangent projections, fp16 [B*T, D]; lse: teacher log-sum-exp (natural log)
+// [B, Hq, lse_pitch]; a_ref: teacher output fp32 [B*T, Hq*dh]; part [B, Hq, nP].
+int attn_jvp_tc_rows();
+cudaError_t launch_attn_jvp_tc(const void* qkv, const void* tqkv, const float* lse, int lse_pitch,
+                               const float* a_ref, int B, int T, int Hq, int Hkv, int dh,
+                               float scale, double* part, int nP, int* status, cudaStream_t st);
+
+// prep.cu: Rademacher probe entries first .. first + n - 1 of the SplitMix64 sequence of `seed` as
+// fp16 +-1 (n a multiple of 8); partial sums of the squared quantisation error, one per block.
+cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, void* out, int sms,
+                                    cudaStream_t st);
+cudaError_t launch_qerr_partial(const void* w, const float* s, int D, int d, int G, int bits,
+                                double* part, int nblocks, int* status, cudaStream_t st);
+
 // reduce.cu
 // A non-finite total raises JAB_ERR_NONFINITE in *status.
 cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
@@ -69,6 +84,9 @@ cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP,
 // out[c] = a[c] + lam * b[c] for c < C
 cudaError_t launch_loss_combine(const double* a, const double* b, double lam, int C, double* out,
                                 cudaStream_t st);
+cudaError_t launch_omega_finish(const double* part, int nblocks, int C, const double* trace,
+                                double layers_after, double* c1, double* c2, cudaStream_t st);
+cudaError_t launch_mean(const double* x, int n, double* out, cudaStream_t st);
 cudaError_t launch_check_finite(const float* x, int64_t n, int* status, cudaStream_t st);
 
 }  // namespace jab

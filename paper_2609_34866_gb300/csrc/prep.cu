@@ -84,6 +84,67 @@ __global__ void quantize_kernel(const uint4* __restrict__ w, const float* __rest
   else if (bad & 2) report(status, JAB_ERR_RANGE);
 }
 
+// ---------------------------------------------------------------- Rademacher probes (Section 2.4)
+// SplitMix64 (Steele, Lea and Flood, "Fast splittable pseudorandom number generators", 2014) used as
+// a counter-based generator: entry n of the probe sequence (n = probe * D * d + flat index) takes
+// the (n + 1)-th output of the stream seeded with `seed`; its top bit selects -1, else +1.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t n) {
+  uint64_t z = seed + (n + 1) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void rademacher_probe_kernel(uint64_t seed, uint64_t first, int64_t n8,
+                                        uint4* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    uint4 o;
+    uint16_t* h = reinterpret_cast<uint16_t*>(&o);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      h[k] = (splitmix64_at(seed, first + (uint64_t)(i * 8 + k)) >> 63) ? 0xBC00u : 0x3C00u;  // -1, +1
+    out[i] = o;
+  }
+}
+
+// ---------------------------------------------------------------- quantisation error (Eq. 6)
+// Partial sums of (Q_b(w) - w)^2 over a grid-stride range, one per block (fp64, each term exact as
+// the oracle forms it: q s - w in double); reduced in fixed order by omega_finish_kernel.
+__global__ void __launch_bounds__(256) qerr_partial_kernel(const uint4* __restrict__ w,
+                                                           const float* __restrict__ s, int D,
+                                                           int d, int G, int bits,
+                                                           double* __restrict__ part, int* status) {
+  __shared__ double red[8];
+  const int64_t n8 = (int64_t)D * d / 8;
+  const int qmax = qmax_of(bits);
+  const int ng = d / G;
+  double acc = 0.0;
+  int bad = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    uint4 v = __ldg(w + i);
+    const bf16_t* b = reinterpret_cast<const bf16_t*>(&v);
+    const int64_t e0 = i * 8;
+    const int64_t row = e0 / d;
+    const int col = (int)(e0 - row * d);
+    float sc = __ldg(s + row * ng + col / G);
+    if (!(sc > 0.f) || !isfinite(sc)) {
+      bad = 1;
+      sc = 1.f;
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float wv = __bfloat162float(b[k]);
+      const double e = (double)quant_code(wv, sc, qmax, nullptr) * (double)sc - (double)wv;
+      acc += e * e;
+    }
+  }
+  const double t = block_sum<256>(acc, red);
+  if (threadIdx.x == 0) part[blockIdx.x] = t;
+  if (bad) report(status, JAB_ERR_NONFINITE);
+}
+
 // ---------------------------------------------------------------- flip count (App. B, Eq. 15)
 // Number of positions where two int8 code arrays differ; 16 bytes per thread and step, one 64-bit
 // atomic per block (integer sums: the result does not depend on the order).
@@ -201,6 +262,19 @@ cudaError_t launch_flip_count(const int8_t* a, const int8_t* b, int64_t n, int64
   flip_count_kernel<<<grid_for(n16 > 0 ? n16 : 1, 256, sms), 256, 0, st>>>(
       (const uint4*)a, (const uint4*)b, n16, a + n16 * 16, b + n16 * 16, tail,
       reinterpret_cast<unsigned long long*>(count));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, void* out, int sms,
+                                    cudaStream_t st) {
+  const int64_t n8 = n / 8;
+  rademacher_probe_kernel<<<grid_for(n8, 256, sms), 256, 0, st>>>(seed, first, n8, (uint4*)out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_qerr_partial(const void* w, const float* s, int D, int d, int G, int bits,
+                                double* part, int nblocks, int* status, cudaStream_t st) {
+  qerr_partial_kernel<<<nblocks, 256, 0, st>>>((const uint4*)w, s, D, d, G, bits, part, status);
   return cudaGetLastError();
 }
 

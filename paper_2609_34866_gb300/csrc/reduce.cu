@@ -33,6 +33,29 @@ __global__ void loss_combine_kernel(const double* __restrict__ a, const double* 
   for (int c = threadIdx.x; c < C; c += blockDim.x) out[c] = a[c] + lam * b[c];
 }
 
+// Omega of Eq. 6 per candidate: c1[c] = Tr(H) * sum of the candidate's quantisation-error partials
+// (fixed order), c2[c] = layers_after * c1[c].
+__global__ void omega_finish_kernel(const double* __restrict__ part, int nblocks, int C,
+                                    const double* __restrict__ trace, double layers_after,
+                                    double* __restrict__ c1, double* __restrict__ c2) {
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    double e = 0.0;
+    for (int k = 0; k < nblocks; ++k) e += part[(int64_t)c * nblocks + k];
+    const double v = *trace * e;
+    c1[c] = v;
+    if (c2) c2[c] = layers_after * v;
+  }
+}
+
+// mean over n of a fp64 array (the Hutchinson estimate over its probes), fixed order
+__global__ void mean_kernel(const double* __restrict__ x, int n, double* __restrict__ out) {
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int i = 0; i < n; ++i) t += x[i];
+    *out = t / n;
+  }
+}
+
 __global__ void check_finite_kernel(const float* __restrict__ x, int64_t n, int* status) {
   bool bad = false;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
@@ -50,6 +73,17 @@ cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP,
 cudaError_t launch_loss_combine(const double* a, const double* b, double lam, int C, double* out,
                                 cudaStream_t st) {
   loss_combine_kernel<<<1, 128, 0, st>>>(a, b, lam, C, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_omega_finish(const double* part, int nblocks, int C, const double* trace,
+                                double layers_after, double* c1, double* c2, cudaStream_t st) {
+  omega_finish_kernel<<<1, 128, 0, st>>>(part, nblocks, C, trace, layers_after, c1, c2);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mean(const double* x, int n, double* out, cudaStream_t st) {
+  mean_kernel<<<1, 32, 0, st>>>(x, n, out);
   return cudaGetLastError();
 }
 

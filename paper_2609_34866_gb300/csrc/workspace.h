@@ -9,6 +9,7 @@
 namespace jab {
 
 constexpr int kPartRows = 64;  // query rows per loss partial (one partial per (c, b, h, 64 rows))
+constexpr int kRedBlocks = 1024;  // blocks of a grid-stride reduction over the weights
 
 struct Workspace {
   // byte offsets into ws; SIZE_MAX when absent
@@ -19,6 +20,7 @@ struct Workspace {
   size_t part;     // fp64 [C, B, Hq, nP]    per-tile partial sums (SSE or ||A||^2)
   size_t status;   // int32 [4]              reserved
   size_t scal;     // fp64 [2, C]            per-candidate scalars (MSE and KL terms)
+  size_t red;      // fp64 [C, kRedBlocks]   per-block partial sums of the quantisation error
   // backward only
   size_t d_o;      // fp16 [N, Hq*d_h]       e = A_hat - A_ref (dL/dA_hat up to 2/n)
   size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 128)
@@ -55,6 +57,7 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
   w.rope = take((size_t)2 * T * (dh / 2) * 4);
   w.part = take((size_t)C * B * d->n_q_heads * nP * 8);
   w.scal = take((size_t)2 * C * 8);
+  w.red = take((size_t)C * kRedBlocks * 8);
   if (bwd) {
     w.d_o = take((size_t)N * d->n_q_heads * dh * 2);
     w.lse = take((size_t)B * d->n_q_heads * w.tp * 4);

@@ -41,6 +41,9 @@ KL_TOL = {2: 1e-2, 3: 1e-2, 4: 1e-2, 5: 1e-2, 8: 3e-2}
 # of per cent of noise (0.31 on the small cases, 0.56 on the scoring batch) that averages out over
 # rows; b = 8 is checked through its totals only.
 KL_ROW_TOL = {2: 1e-2, 3: 2e-2, 4: 3e-2, 5: 7e-2}
+# Hutchinson quadratic forms v^T H v = 2 ||J_A v||^2 / n (Section 2.4), relative: the forward-mode
+# product rounds its fp16 operands (tangent projections, P, P o dS) like the forward does.
+JVP_TOL = 1e-2
 # Absolute floor per row (nats): the difference form of the row KL rounds to ~1e-7 of the scores.
 KL_ROW_ATOL = 1e-6
 

@@ -8,8 +8,8 @@ import pytest
 import torch
 
 from oracle import jab_oracle as O
-from tests.harness import (A_TOL, COS_MIN, HEAVY_TAILED, KL_ROW_ATOL, KL_ROW_TOL, KL_TOL, L_TOL,
-                           LSE_ATOL, PARTS_RTOL, SMALL_CASES,
+from tests.harness import (A_TOL, COS_MIN, HEAVY_TAILED, JVP_TOL, KL_ROW_ATOL, KL_ROW_TOL, KL_TOL,
+                           L_TOL, LSE_ATOL, PARTS_RTOL, SMALL_CASES,
                            Case, J, cosine, np64)
 
 pytestmark = pytest.mark.gpu
@@ -148,6 +148,57 @@ def test_kl_forward_parity(name):
         assert abs(loss[i].item() - j) <= L_TOL * j, (b, loss[i].item(), j)
         lam = float(np.float32(0.1))                      # lambda_kl crosses the ABI as a float
         np.testing.assert_allclose(loss[i].item(), mse[i].item() + lam * kl[i].item(), rtol=1e-12)
+
+
+# ------------------------------------------------------------------ sensitivity (Section 2.4, Eq. 5-6)
+def test_rademacher_probes_bit_exact():
+    """The probe entries are the oracle's SplitMix64 signs, including at an offset into the
+    sequence (probe 3 of a 24 x 40 weight)."""
+    out = torch.empty(24 * 40, dtype=torch.float16, device="cuda")
+    J().jab_rademacher_probes(99, 3 * 24 * 40, out)
+    np.testing.assert_array_equal(out.float().cpu().numpy(),
+                                  O.rademacher_probe(99, 3, (24, 40)).ravel())
+
+
+@pytest.mark.parametrize("name", ["gpt2_T200", "mistral_T130", "gqa2_T257", "dh64_gqa4_T65",
+                                  "mistral_G64_T70", "gpt2_T1"])
+def test_hutchinson_trace_parity(name):
+    """Per probe, v^T H v = 2 ||J_A v||^2 / n from the forward-mode attention kernel against the
+    oracle's quadratic form on the same probe; the trace is their mean (Eq. 5, reading R19)."""
+    c = case(name)
+    ws = c.workspace(n_cand=2, with_bwd=False)
+    A, lse, _ = c.gpu_teacher(ws)
+    m, seed = 3, 1234
+    trace = torch.empty(1, dtype=torch.float64, device="cuda")
+    vhv = torch.empty(m, dtype=torch.float64, device="cuda")
+    J().jab_hutchinson_trace(c.desc, c.B, c.T, c.X, c.W, A, lse, m, seed, trace, ws, vhv=vhv)
+    assert J().jab_get_device_status() == 0
+    probes = [O.rademacher_probe(seed, i, c.W.shape) for i in range(m)]
+    for i, v in enumerate(probes):
+        want = O.gn_quadratic_form(c.x64, c.w64, v, c.odesc)
+        assert abs(vhv[i].item() - want) <= JVP_TOL * want, (i, vhv[i].item(), want)
+    np.testing.assert_allclose(trace.item(), vhv.cpu().numpy().sum() / m, rtol=1e-12)
+    want = O.hutchinson_trace(c.x64, c.w64, c.odesc, probes)
+    assert abs(trace.item() - want) <= JVP_TOL * want
+
+
+def test_omega_scores_parity():
+    """Eq. 6: C1 = Tr(H) ||Q_b(W) - W||^2 and C2 = (L - i) C1 for five widths against the oracle
+    (both sum the same exact fp64 terms), bit-identical on a repeated call."""
+    c = case("mistral_G64_T70")
+    bits = [2, 3, 4, 5, 8]
+    scales = [c.gpu_scales(b, mode=1) for b in bits]
+    trace = torch.tensor([2.5], dtype=torch.float64, device="cuda")
+    ws = J().Workspace(c.desc, 1, 1, len(bits), False)
+    c1, c2, c1b = (torch.empty(len(bits), dtype=torch.float64, device="cuda") for _ in range(3))
+    J().jab_omega_scores(c.desc, c.W, bits, scales, trace, 3, c1, ws, c2=c2)
+    J().jab_omega_scores(c.desc, c.W, bits, scales, trace, 3, c1b, ws)
+    assert torch.equal(c1, c1b)
+    for i, b in enumerate(bits):
+        e1, e2 = O.omega_scores(2.5, c.w64, scales[i].cpu().numpy(), b, c.G, layers_after=3)
+        np.testing.assert_allclose([c1[i].item(), c2[i].item()], [e1, e2], rtol=1e-10)
+    assert (np.diff(c1.cpu().numpy()) < 0).all()      # more bits, smaller quantisation error
+    assert J().jab_get_device_status() == 0
 
 
 # ------------------------------------------------------------------ STE / LSQ backward

@@ -138,6 +138,25 @@ def test_mistral_scoring_kl_full_size():
             assert (np.abs(got - ro) <= bound).all(), (bits, (np.abs(got - ro) / bound).max())
 
 
+def test_mistral_scoring_hutchinson_full_sequence():
+    """The Hutchinson quadratic form on one full-length sequence of the scoring workload's block
+    (T = 2048, d_model 4096, GQA 32/8, RoPE), one probe, against the oracle on that sequence."""
+    from tests.harness import JVP_TOL
+    wl, desc, X, W = _setup("mistral_scoring")
+    x1 = X[:1].contiguous()
+    ws = J().Workspace(desc, 1, wl.seq_len, 2, False)
+    A = torch.empty((1, wl.seq_len, wl.shape.n_q_heads * wl.shape.head_dim), dtype=torch.float32,
+                    device="cuda")
+    lse = torch.empty((1, wl.shape.n_q_heads, wl.seq_len), dtype=torch.float32, device="cuda")
+    J().jab_reference_forward(desc, 1, wl.seq_len, x1, W, A, ws, lse=lse)
+    trace = torch.empty(1, dtype=torch.float64, device="cuda")
+    J().jab_hutchinson_trace(desc, 1, wl.seq_len, x1, W, A, lse, 1, 77, trace, ws)
+    assert J().jab_get_device_status() == 0
+    v = O.rademacher_probe(77, 0, tuple(W.shape))
+    want = O.gn_quadratic_form(np64(x1), np64(W), v, oracle_desc(wl.shape, wl.group_size))
+    assert abs(trace.item() - want) <= JVP_TOL * want, (trace.item(), want)
+
+
 def _backward(wl, desc, X, W, A, s, bits, B):
     ws = J().Workspace(desc, B, wl.seq_len, 1, True)
     loss = torch.empty(1, dtype=torch.float64, device="cuda")

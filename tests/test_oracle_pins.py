@@ -571,6 +571,20 @@ def test_omega_scores_vanish_on_the_grid_and_scale_with_depth():
     assert c1 > 0 and c2 == 3 * c1
 
 
+def test_splitmix64_published_outputs_and_probe_signs():
+    """The probes' generator reproduces SplitMix64's published first outputs; probe entries take
+    their sign from the top bit, probe i starting at counter i * size; the signs are balanced."""
+    with open(os.path.join(GOLDEN, "splitmix64.json")) as f:
+        fx = json.load(f)
+    want = [int(h, 16) for h in fx["outputs_hex"]]
+    assert [int(v) for v in O.splitmix64(fx["seed"], [0, 1, 2])] == want
+    assert O.rademacher_probe(0, 0, (1, 3)).tolist() == [[-1.0 if v >> 63 else 1.0 for v in want]]
+    p1 = O.rademacher_probe(0, 1, (1, 3))            # probe 1 starts at counter 3
+    assert p1[0, 0] == (-1.0 if int(O.splitmix64(0, [3])[0]) >> 63 else 1.0)
+    big = O.rademacher_probe(7, 2, (200, 500))
+    assert set(np.unique(big)) == {-1.0, 1.0} and abs(big.mean()) < 5 / np.sqrt(big.size)
+
+
 def test_omega_scores_hand_worked():
     """Eq. 6 on one row worked by hand. b = 3 (qmax = 3), one group of 5, s = 1/2:
     w      = 0.375, -0.6875, 1.25, 0.0625, 2.0
