@@ -68,8 +68,10 @@ def work_of(wl, C=1):
         "attn_bwd": ("flop", 2.5 * attn),
         "wgrad_lsq": ("flop", 2.0 * N * D * d),
         "wgrad_store": ("flop", 2.0 * N * D * d),
+        "attn_jvp": ("flop", 2.5 * attn * C),
         "convert_x": ("byte", 4.0 * N * d),
         "quantize": ("byte", 4.0 * D * d * C),
+        "probe": ("byte", 2.0 * D * d * C),
     }
 
 
@@ -412,6 +414,42 @@ def wl_table(J, wl, args, dev, pk, st, with_cpu):
                                "cores": os.cpu_count(), "kind": "oracle",
                                "sample": f"block 0, 1 of {wl.batch} sequences, teacher + all "
                                          f"{C} widths; extrapolated linearly in sequences"}
+
+    # The paper's own sensitivity score on the same blocks (Section 2.4, Eq. 5-6): the teacher pass
+    # (A_ref and its log-sum-exp), a 10-probe Hutchinson trace through the forward-mode attention
+    # kernel, and Omega C1 / C2 for every width.
+    m, nbh = 10, 2
+    lse = torch.empty((B, wl.shape.n_q_heads, T), dtype=torch.float32, device=dev)
+    ws2 = J.Workspace(desc, B, T, 2, False, device=dev)
+    wso = J.Workspace(desc, 1, 1, C, False, device=dev)
+    trace = torch.empty(1, dtype=torch.float64, device=dev)
+    c1, c2 = (torch.empty((nb, C), dtype=torch.float64, device=dev) for _ in range(2))
+
+    def hutch():
+        for i in range(nbh):
+            J.jab_reference_forward(desc, B, T, X, Ws[i], A, ws2, lse=lse)
+            J.jab_hutchinson_trace(desc, B, T, X, Ws[i], A, lse, m, 1000 + i, trace, ws2)
+            for k, b in enumerate(wl.bits):
+                J.jab_init_scales(desc, b, 0, Ws[i], scales[k])
+            J.jab_omega_scores(desc, Ws[i], list(wl.bits), scales, trace, nb - 1 - i, c1[i], wso,
+                               c2=c2[i])
+
+    hms, _ = timed(J, hutch, 1, 1, st, sites=False)
+    _, hsites = timed(J, hutch, 1, 0, st)
+    w1 = work_of(wl, 1)   # per block: teacher (projection, attention), primal projection, m probes
+    hw = {"proj_gemm": ("flop", w1["proj_gemm"][1] * nbh * (2 + m)),
+          "attn_fwd": ("flop", w1["attn_fwd"][1] * nbh),
+          "attn_jvp": ("flop", w1["attn_jvp"][1] * nbh * m),
+          "convert_x": ("byte", w1["convert_x"][1] * nbh * 2),
+          "quantize": ("byte", w1["quantize"][1] * nbh * 2),
+          "probe": ("byte", w1["probe"][1] * nbh * m)}
+    hflops = hw["proj_gemm"][1] + hw["attn_fwd"][1] + hw["attn_jvp"][1]
+    out["hutchinson"] = {
+        "metric": "blocks/s scored by the Hutchinson trace (10 probes) and Omega C1/C2 for every "
+                  "width, teacher pass included", "value": nbh / (hms / 1e3), "unit": "blocks/s",
+        "probe_evals_per_s": nbh * m / (hms / 1e3), "ms_per_block": hms / nbh,
+        **rates(hflops / nbh, hms / nbh, pk), "roofline": roofline_of(hsites, hw, pk),
+        "blocks_timed": nbh, "probes_per_block": m}
     return out
 
 
@@ -533,6 +571,18 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
     fwd_ms = max_over_ranks(fwd_ms, dev)
     fwd_value = world * args.steps / (fwd_ms / 1e3)
 
+    # ---- forward with both terms of Eq. 3 (MSE + 0.1 KL, one candidate; teacher projection once)
+    qkv_ref = torch.empty((B, T, s.d_out), dtype=torch.float16, device=dev)
+    J.jab_reference_projection(desc, B, T, X, W, qkv_ref, ws)
+
+    def kl_step():
+        J.jab_loss_forward_kl(desc, B, T, X, W, A, qkv_ref, [bits], [scales], 0.1, loss, ws)
+
+    kl_ms, _ = timed(J, kl_step, args.steps, max(1, args.warmup), st, barrier, sites=False)
+    kl_ms = max_over_ranks(kl_ms, dev)
+    del qkv_ref
+    kl_f = fwd_f + work_of(wl)["attn_kl"][1]
+
     # ---- Fisher-coupling probe (App. B): the loss and ||dL/dw_hat||^2 at 2 bits with round-to-
     # nearest (absmax) scales, one fwd + bwd per evaluation; reported beside the main metric
     s2 = scales_for(J, desc, wl, W, 2, dev, mode=0)
@@ -625,6 +675,9 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
         "algorithmic_tflop_per_step": {"fwd": fwd_f / 1e12, "bwd": bwd_f / 1e12},
         "fwd_only": {"value": fwd_value, "unit": "evals/s", "ms_per_eval": fwd_ms / args.steps,
                      "achieved_tflops": fwd_f / (fwd_ms / args.steps / 1e3) / 1e12},
+        "fwd_kl": {"value": world * args.steps / (kl_ms / 1e3), "unit": "evals/s",
+                   "ms_per_eval": kl_ms / args.steps, "lambda_kl": 0.1,
+                   "achieved_tflops": kl_f / (kl_ms / args.steps / 1e3) / 1e12},
         "fisher_probe": {"value": world * n_fis / (fis_ms / 1e3), "unit": "evals/s", "bits": 2,
                          "ms_per_eval": fis_ms / n_fis,
                          "achieved_tflops": (fwd_f + bwd_f) / (fis_ms / n_fis / 1e3) / 1e12},

@@ -135,7 +135,10 @@ jab_status jab_loss_forward_kl(const jab_block_desc* desc, int32_t B, int32_t T,
  * JVP), no second backward pass.
  * Probe i, entry e (row-major over [(Hq+2Hkv) d_h, d_model]) is -1 when the top bit of the
  * (i * (Hq+2Hkv) d_h d_model + e + 1)-th output of SplitMix64 (Steele, Lea and Flood, 2014)
- * seeded with `seed` is set, else +1.
+ * seeded with `seed` is set, else +1. The probe enters the tensor-core path scaled by the exact
+ * power of two 2^-k, k = floor(log2(sqrt(d_model))), so that the tangent projections stay in the
+ * fp16 range; the quadratic form is rescaled by 4^k (exactly). A tangent value that still leaves
+ * the fp16 range raises JAB_ERR_RANGE on the device.
  *   A_ref_dev, lse_ref_dev  the teacher pass of jab_reference_forward (lse_ref required)
  *   trace_dev      out fp64 [1]            the estimate
  *   vhv_dev        out fp64 [n_probes] or NULL   v_i^T H v_i of each probe

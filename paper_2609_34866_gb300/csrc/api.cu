@@ -1,6 +1,8 @@
 // C ABI of libjab (include/jab.h): argument validation, workspace carving and kernel sequencing.
 // Every step of the computation runs in the kernels of this library; there is no host fallback.
 #include <math.h>
+
+#include <cmath>
 #include <stdlib.h>
 #include <string.h>
 
@@ -384,10 +386,16 @@ jab_status jab_hutchinson_trace(const jab_block_desc* desc, int32_t B, int32_t T
   if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, qkv, cos_t, sin_t, status, st)) !=
       JAB_OK)
     return s;
+  // The probe enters scaled by c = 2^-k, k = floor(log2(sqrt(d_model))): the tangent projections
+  // X (c v)^T are then of the order of the activations, inside the fp16 range of the tensor-core
+  // operands; v^T H v = ||J_A (c v)||^2 * 2 / (n c^2) is rescaled exactly (a power of two).
+  int k2 = 0;
+  while ((1 << (2 * (k2 + 1))) <= dm && k2 < 14) ++k2;
+  const double rescale = std::ldexp(1.0, 2 * k2);
   JAB_SITE("memset_grad", 0, cudaMemsetAsync(trace_dev, 0, sizeof(double), st));
   for (int pr = 0; pr < n_probes; ++pr) {
     // probe pr: entries pr * D * d .. of the seed's sequence, the tangent projection X V^T + RoPE
-    JAB_SITE("probe", 1, launch_rademacher_probe(seed, (uint64_t)pr * D * dm, (int64_t)D * dm,
+    JAB_SITE("probe", 1, launch_rademacher_probe(seed, (uint64_t)pr * D * dm, (int64_t)D * dm, k2,
                                                  w + wp.w16, sms, st));
     if ((s = run_projection(desc, N, T, 1, w + wp.x16, w + wp.w16, tqkv, cos_t, sin_t, status,
                             st)) != JAB_OK)
@@ -397,8 +405,8 @@ jab_status jab_hutchinson_trace(const jab_block_desc* desc, int32_t B, int32_t T
                                                softmax_scale(desc), part, nP, status, st));
     double* vhv = vhv_dev ? vhv_dev + pr : tmp;
     // v^T H v = 2 ||J_A v||^2 / n (Eq. 5 at the float weights, MSE term)
-    JAB_SITE("loss_reduce", 1, launch_loss_reduce(part, 1, B, desc->n_q_heads, nP, 2.0 / n_el,
-                                                  vhv, nullptr, status, st));
+    JAB_SITE("loss_reduce", 1, launch_loss_reduce(part, 1, B, desc->n_q_heads, nP,
+                                                  2.0 * rescale / n_el, vhv, nullptr, status, st));
     JAB_SITE("loss_combine", 1, launch_loss_combine(trace_dev, vhv, 1.0 / n_probes, 1, trace_dev,
                                                     st));
   }
@@ -413,7 +421,7 @@ jab_status jab_rademacher_probes(uint64_t seed, int64_t first, int64_t n, void* 
   int sms;
   const jab_status s = device_info(&status, &sms);
   if (s != JAB_OK) return s;
-  JAB_TRY(launch_rademacher_probe(seed, (uint64_t)first, n, out_dev, sms,
+  JAB_TRY(launch_rademacher_probe(seed, (uint64_t)first, n, 0, out_dev, sms,
                                   reinterpret_cast<cudaStream_t>(stream)));
   return JAB_OK;
 }

@@ -287,6 +287,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int k0 = j * BK + 2 * cq;
       const bool masked = j * BK + BK - 1 > q0 || j * BK + BK > p.T;  // diagonal or ragged block
       float2 uA = make_float2(0.f, 0.f), uB = uA;
+      uint32_t inf_bits = 0;
       uint32_t pw[32], uw[32];  // packed P and U: [2m] row A, [2m + 1] row B, packed column 4m + cq
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh)
@@ -314,9 +315,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           pw[2 * m + 1] = tc::pack_half2(pb.x, pb.y);
           uw[2 * m] = tc::pack_half2(ua.x, ua.y);
           uw[2 * m + 1] = tc::pack_half2(ub.x, ub.y);
+          inf_bits |= half2_exp_all_ones(uw[2 * m]) | half2_exp_all_ones(uw[2 * m + 1]);
         }
       rsA += uA.x + uA.y;
       rsB += uB.x + uB.y;
+      if (inf_bits) report(p.status, JAB_ERR_RANGE);  // U out of the fp16 range (or NaN)
       __syncwarp();
       tc::tmem_st_16x128b_x16(tmem + lane16 + L::S_COL, pw);
       tc::tmem_st_16x128b_x16(tmem + lane16 + L::T_COL, uw);

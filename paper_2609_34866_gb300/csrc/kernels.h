@@ -71,9 +71,10 @@ cudaError_t launch_attn_jvp_tc(const void* qkv, const void* tqkv, const float* l
                                float scale, double* part, int nP, int* status, cudaStream_t st);
 
 // prep.cu: Rademacher probe entries first .. first + n - 1 of the SplitMix64 sequence of `seed` as
-// fp16 +-1 (n a multiple of 8); partial sums of the squared quantisation error, one per block.
-cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, void* out, int sms,
-                                    cudaStream_t st);
+// fp16 +-2^-log2_scale (n a multiple of 8, 0 <= log2_scale <= 14); partial sums of the squared
+// quantisation error, one per block.
+cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, int log2_scale,
+                                    void* out, int sms, cudaStream_t st);
 cudaError_t launch_qerr_partial(const void* w, const float* s, int D, int d, int G, int bits,
                                 double* part, int nblocks, int* status, cudaStream_t st);
 

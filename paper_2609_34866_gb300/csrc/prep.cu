@@ -95,15 +95,17 @@ __device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t n) {
   return z ^ (z >> 31);
 }
 
-__global__ void rademacher_probe_kernel(uint64_t seed, uint64_t first, int64_t n8,
+// Entries are written as +-2^-k (fp16: exponent field 15 - k, zero mantissa), an exact scaling.
+__global__ void rademacher_probe_kernel(uint64_t seed, uint64_t first, int64_t n8, int k2,
                                         uint4* __restrict__ out) {
+  const uint16_t pos = (uint16_t)((15 - k2) << 10), neg = (uint16_t)(0x8000u | pos);
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
        i += (int64_t)gridDim.x * blockDim.x) {
     uint4 o;
     uint16_t* h = reinterpret_cast<uint16_t*>(&o);
 #pragma unroll
     for (int k = 0; k < 8; ++k)
-      h[k] = (splitmix64_at(seed, first + (uint64_t)(i * 8 + k)) >> 63) ? 0xBC00u : 0x3C00u;  // -1, +1
+      h[k] = (splitmix64_at(seed, first + (uint64_t)(i * 8 + k)) >> 63) ? neg : pos;
     out[i] = o;
   }
 }
@@ -265,10 +267,12 @@ cudaError_t launch_flip_count(const int8_t* a, const int8_t* b, int64_t n, int64
   return cudaGetLastError();
 }
 
-cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, void* out, int sms,
-                                    cudaStream_t st) {
+cudaError_t launch_rademacher_probe(uint64_t seed, uint64_t first, int64_t n, int log2_scale,
+                                    void* out, int sms, cudaStream_t st) {
   const int64_t n8 = n / 8;
-  rademacher_probe_kernel<<<grid_for(n8, 256, sms), 256, 0, st>>>(seed, first, n8, (uint4*)out);
+  if (log2_scale < 0 || log2_scale > 14) return cudaErrorInvalidValue;
+  rademacher_probe_kernel<<<grid_for(n8, 256, sms), 256, 0, st>>>(seed, first, n8, log2_scale,
+                                                                 (uint4*)out);
   return cudaGetLastError();
 }
 
