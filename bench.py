@@ -15,8 +15,10 @@ oracle baseline.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 
-Under torchrun each rank evaluates its own seeded batch on its own GPU (independent units, no
-collective on the data path): weak scaling, value = all ranks' evaluations / max rank time.
+Under torchrun the ranks evaluate one batch sharded by sequence: rank r holds its own seeded shard of
+the workload's size, and every step combines the shards' loss and scale gradient with one
+all-reduce of 1 + D d/G fp64 values (weak scaling; value = shards evaluated by all ranks / max rank
+time).
 `--impl reference` times the float64 CPU oracle on a bounded sample of the same workload.
 """
 from __future__ import annotations
@@ -36,7 +38,7 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-from paper_2609_34866_gb300.multi import dist_env, max_over_ranks  # noqa: E402
+from paper_2609_34866_gb300.multi import combine_shards, dist_env, max_over_ranks  # noqa: E402
 from workloads import WORKLOADS, make_block_weights, make_x  # noqa: E402
 
 METRIC = "JAB candidate-loss evals/s (fwd+STE bwd), Mistral-7B-shaped attention block"
@@ -512,8 +514,13 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
     loss = torch.empty(1, dtype=torch.float64, device=dev)
     grad = torch.empty_like(scales)
 
+    # Under torchrun the ranks evaluate one global batch of B * world sequences, sharded by
+    # sequence (rank r holds its own seeded B sequences): every step combines the shards' loss and
+    # scale gradient into the global ones with one all-reduce (multi.combine_shards).
     def step():
         J.jab_loss_backward_scales_prepared(desc, B, T, X, W, A, bits, scales, 0.0, loss, grad, ws)
+        if world > 1:
+            combine_shards(loss, grad, B, B * world)
 
     for _ in range(args.warmup):
         step()
@@ -625,6 +632,8 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
             st.wait_event(copied[b])
             dX, dW, dA, dS = dbuf[b]
             J.jab_loss_backward_scales(desc, B, T, dX, dW, dA, bits, dS, 0.0, loss, grad, ws, stream=st)
+            if world > 1:
+                combine_shards(loss, grad, B, B * world)
             ev = torch.cuda.Event()
             ev.record(st)
             freed[b] = ev
@@ -670,7 +679,11 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {**config_of(wl), "x_f16": "converted once per calibration batch (jab_prepare_x): "
-                                              "the scale fit's X is fixed across its steps"},
+                                              "the scale fit's X is fixed across its steps",
+                   "parallelism": ("single GPU" if world == 1 else
+                                   f"sequence-sharded over {world} ranks: each rank a {B}-sequence "
+                                   f"shard of a {B * world}-sequence batch, loss and scale gradient "
+                                   "combined by one all-reduce per step")},
         **rates(fwd_f + bwd_f, ms_step, pk),
         "algorithmic_tflop_per_step": {"fwd": fwd_f / 1e12, "bwd": bwd_f / 1e12},
         "fwd_only": {"value": fwd_value, "unit": "evals/s", "ms_per_eval": fwd_ms / args.steps,

@@ -43,14 +43,18 @@ def shard_sequences(batch: int, world: int, rank: int) -> Tuple[int, int]:
 def combine_shards(loss: torch.Tensor, grad: torch.Tensor, n_local: int, n_total: int):
     """Full-batch L_JAB and scale gradient from per-shard values computed on n_local of n_total
     sequences: each shard's mean-normalised values are weighted by n_local / n_total and summed over
-    ranks with one all-reduce (in place on `loss` and `grad`)."""
+    ranks with one all-reduce of a single fp64 buffer holding the loss and the gradient (1 + D d/G
+    values), written back in place into `loss` and `grad`."""
     import torch.distributed as dist
     w = float(n_local) / float(n_total)
-    loss.mul_(w)
-    grad.mul_(w)
     if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
-        dist.all_reduce(loss)
-        dist.all_reduce(grad)
+        buf = torch.cat([loss.reshape(-1).double(), grad.reshape(-1).double()]).mul_(w)
+        dist.all_reduce(buf)
+        loss.copy_(buf[:loss.numel()].view_as(loss))
+        grad.copy_(buf[loss.numel():].view_as(grad))
+    else:
+        loss.mul_(w)
+        grad.mul_(w)
     return loss, grad
 
 
