@@ -28,11 +28,11 @@ Readings of points the paper leaves open (each is stated where it is used):
   R7  RoPE is the rotate-half convention with inv_freq_j = theta^(-2j/d_h).
   R8  GQA: query head h reads key/value head floor(h / (Hq / Hkv)).
   R9  an all-zero group gets scale 1 at absmax init (any positive scale gives code 0).
-  R18 the KL term of Eq. 3 (not on the GPU path yet) is D_KL(P || Q(w)) with the implemented
+  R18 the KL term of Eq. 3 is D_KL(P || Q(w)) with the implemented
       batchmean convention: the sum over sequences, query heads, query rows and keys of
       P log(P / Q), divided by B; P is the teacher's post-softmax map, Q the student's; masked
       entries have P = Q = 0 and contribute nothing; lambda_KL defaults to 0.1 (Section 3).
-  R19 the sensitivity criterion (Section 2.4, Eq. 5-6, not on the GPU path yet) is taken for the
+  R19 the sensitivity criterion (Section 2.4, Eq. 5-6) is taken for the
       MSE term as normalised in R3 (lambda_KL = 0): at the float point H = 2 J_A^T J_A / n with
       n = B*T*Hq*d_h, so v^T H v = 2 ||J_A v||^2 / n; the Rademacher probes are inputs.
   R21 the flip rate of Eq. 15 counts the grid positions (the clamped codes of Eq. 2, i.e. the
