@@ -52,8 +52,10 @@ typedef enum {
                                 quantised weights, the projected Q|K|V or the output error dO
                                 (|x| > 65504 after rounding)                                    */
   JAB_ERR_TIMEOUT = 6,       /* device: a bounded wait in a pipelined kernel gave up             */
-  JAB_ERR_SCRATCH_LIMIT = 7  /* jab_loss_forward_noalloc: the problem needs more scratch than the
+  JAB_ERR_SCRATCH_LIMIT = 7, /* jab_loss_forward_noalloc: the problem needs more scratch than the
                                 fixed JAB_NOALLOC_SCRATCH_BYTES                                    */
+  JAB_ERR_INTERNAL = 8       /* device: an internal invariant did not hold (e.g. the alignment of
+                                a kernel's shared memory); the kernel returned without work     */
 } jab_status;
 
 /* One attention block. Section 2.1 (d, d_head), App. C (Mistral-7B: GQA, RoPE theta = 1e4). */

@@ -16,7 +16,7 @@ import torch
 JAB_OK = 0
 _STATUS_NAMES = {0: "JAB_OK", 1: "JAB_ERR_INVALID_ARG", 2: "JAB_ERR_UNSUPPORTED", 3: "JAB_ERR_CUDA",
                  4: "JAB_ERR_NONFINITE", 5: "JAB_ERR_RANGE", 6: "JAB_ERR_TIMEOUT",
-                 7: "JAB_ERR_SCRATCH_LIMIT"}
+                 7: "JAB_ERR_SCRATCH_LIMIT", 8: "JAB_ERR_INTERNAL"}
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 

@@ -500,6 +500,7 @@ static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32
   L.dvec = reinterpret_cast<float*>(w + wp.dvec);
   L.ldt = wp.ldt;
   L.lse_pitch = (int)wp.tp;
+  L.ds = w + wp.ds;
   JAB_SITE("attn_fwd", 1, launch_attn_fwd_tc(L, 2));
   const double n_el = (double)N * desc->n_q_heads * dh;
   JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el,
@@ -675,6 +676,7 @@ const char* jab_status_string(jab_status status) {
     case JAB_ERR_RANGE: return "input outside the fp16 range";
     case JAB_ERR_TIMEOUT: return "device wait timed out";
     case JAB_ERR_SCRATCH_LIMIT: return "problem larger than the fixed no-allocation scratch";
+    case JAB_ERR_INTERNAL: return "internal device invariant failed";
   }
   return "unknown status";
 }

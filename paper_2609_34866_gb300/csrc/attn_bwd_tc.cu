@@ -9,12 +9,13 @@
 //   dkdv  one CTA per (128-key block, KV head, sequence); loops over the query heads of the group and
 //         over 128-query blocks: S^T = K Q^T, dP^T = V dO^T into TMEM, P^T and dS^T (fp16) written
 //         back over them, dV += P^T dO and dK += dS^T Q (A operands in TMEM) accumulated in TMEM.
-//   dq    persistent, (128 query rows, query head, sequence) tiles; loops over 128-key blocks:
-//         S = Q K^T, dP = dO V^T (Q, dO in TMEM), dS (fp16) to shared memory, dQ += dS K in TMEM.
-// Warp roles: warp 0 TMA, warp 1 TMEM owner + UMMA issuer, warps 2..9 elementwise: two warps per
-// TMEM lane quarter (dkdv: each warp 16 whole rows of S^T / dP^T; dq: each thread one row and half
-// of the columns of S / dP). The epilogues apply the transpose of RoPE to dQ and dK and write
-// dQKV^T (bf16, [D, ldt]), the K-major operand of the weight-gradient GEMM.
+//         Each dS^T tile is also staged in shared memory and stored to HBM by TMA (a store warp).
+//   dq    persistent, (128 query rows, query head, sequence) tiles: dQ = scale * sum_kb dS K from the
+//         stored dS^T tiles, a plain tensor-core product per key block (no recomputation of S, P or
+//         dP: two of the three products and all elementwise work of a recomputing dq are saved, for
+//         one HBM write and one read of the fp16 dS tiles).
+// Both epilogues apply the transpose of RoPE to dQ and dK and write dQKV^T (bf16, [D, ldt]), the
+// K-major operand of the weight-gradient GEMM.
 #include <cudaTypedefs.h>
 
 #include "kernels.h"
@@ -23,7 +24,7 @@
 namespace jab {
 namespace {
 
-constexpr int NUM_THREADS = 320;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise (2 per lane quarter)
+constexpr int NUM_THREADS = 352;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise, warp 10 dS^T stores
 constexpr int EW_WARPS = 8;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -31,6 +32,7 @@ struct BwdParams {
   int T, B, Hq, Hkv, lse_pitch;
   int qcol0, kcol0, vcol0;  // column offsets of Q, K, V heads in the QKV matrix
   int64_t ldt;
+  int npairs;  // (query block, key block) pairs of one (sequence, head): nq (nq + 1) / 2
   float scale, sl2;
   const float* lse;
   const float* dvec;
@@ -144,8 +146,11 @@ struct DkdvLayout {
   static constexpr int ST_Q = 0, ST_DO = NCH * CHUNK, ST_LSE = 2 * NCH * CHUNK,
                        ST_D = ST_LSE + BQ * 4, ST_BYTES = ST_D + BQ * 4;
   static constexpr int ST_STRIDE = (ST_BYTES + 1023) / 1024 * 1024;
-  static constexpr int BAR_OFF = ST_OFF + STAGES * ST_STRIDE;
-  static constexpr int USED = BAR_OFF + 256 + 1024;
+  static constexpr int DSS_OFF = ST_OFF + STAGES * ST_STRIDE;  // dS^T staging: two 64-query halves
+  static constexpr int BAR_OFF = DSS_OFF + 2 * CHUNK;
+  // No slack for aligning the base: the kernel checks that it is 1024-byte aligned (it is, after the
+  // per-CTA reserved shared memory) and returns with JAB_ERR_INTERNAL otherwise.
+  static constexpr int USED = BAR_OFF + 256;
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
   static constexpr uint32_t S_COL = 0, DP_COL = 128, DV_COL = 256, DK_COL = 256 + DH;
   static_assert(DK_COL + DH <= 512, "TMEM budget");
@@ -155,7 +160,7 @@ struct DkdvLayout {
 
 struct DkdvBars {
   uint64_t kv_full, ld_full[2], ld_empty[2], s_full, dp_full, p_full, ds_full, dv_done, dk_done;
-  uint64_t o_full, drain;
+  uint64_t o_full, drain, dss_full, dss_free;
   uint32_t tmem_base;
   int abort;
 };
@@ -163,12 +168,16 @@ struct DkdvBars {
 template <int DH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
-                            const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
+                            const __grid_constant__ CUtensorMap tm_do,
+                            const __grid_constant__ CUtensorMap tm_ds, const BwdParams p) {
   using L = DkdvLayout<DH>;
   constexpr int BK = L::BK, BQ = L::BQ, STAGES = L::STAGES;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (tc::smem_u32(smem_raw) & 1023u) {  // the swizzled TMA tiles need a 1024-byte aligned base
+    if (threadIdx.x == 0) report(p.status, JAB_ERR_INTERNAL);
+    return;
+  }
+  uint8_t* smem = smem_raw;
   DkdvBars* bars = reinterpret_cast<DkdvBars*>(smem + L::BAR_OFF);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
@@ -194,10 +203,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc::mbar_init(&bars->dk_done, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
+    tc::mbar_init(&bars->dss_full, EW_WARPS);  // the block's dS^T is in the staging tile
+    tc::mbar_init(&bars->dss_free, 1);         // the store warp's TMA stores have read it
     bars->abort = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_qkv);
     tc::prefetch_tmap(&tm_do);
+    tc::prefetch_tmap(&tm_ds);
   }
   if (warp == 1) {
     tc::tmem_alloc(&bars->tmem_base, 512);
@@ -338,6 +350,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
+  } else if (warp == 10) {
+    if (lane == 0) {  // ------------------------------------------ dS^T tiles to global memory
+      // Tile (sequence b, head h, query block i, key block kb) is row block
+      // (b Hq + h) npairs + i (i + 1) / 2 + kb of the dS^T buffer: 128 key rows of 128 queries.
+      for (int it = 0; it < n_it; ++it) {
+        if (!tc::mbar_wait(&bars->dss_full, it & 1, abort, p.status)) break;
+        const int h = g * r + it / per_head, i = kb + it % per_head;
+        const int64_t tile = ((int64_t)b * p.Hq + h) * p.npairs + (int64_t)i * (i + 1) / 2 + kb;
+        tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF, 0, (int32_t)(tile * BK));
+        tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF + L::CHUNK, 64, (int32_t)(tile * BK));
+        tc::bulk_commit_group();
+        tc::bulk_wait_group_read<0>();  // the staging tile may be rewritten
+        tc::mbar_arrive(&bars->dss_free);
+      }
+      tc::bulk_wait_group<0>();
+    }
   } else {  // ------------------------------------ elementwise: 16 key rows x 128 queries per warp
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
@@ -448,6 +476,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->ds_full);
+      // The same dS^T words into the staging tile (two 64-query halves, 128-byte swizzle) for the
+      // store warp, once it has stored the previous block's: packed column c = 4m + cq (queries
+      // 2c, 2c + 1) is 16-byte unit m % 8 of half m / 8 of its key row.
+      if (it > 0 && !tc::mbar_wait(&bars->dss_free, (it - 1) & 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        uint8_t* hb = smem + L::DSS_OFF + (m >> 3) * L::CHUNK;
+        *reinterpret_cast<uint32_t*>(hb + rA * 128 + (((m & 7) ^ (rA & 7)) << 4) + cq * 4) = dw[2 * m];
+        *reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + (((m & 7) ^ ((rA + 8) & 7)) << 4) + cq * 4) =
+            dw[2 * m + 1];
+      }
+      tc::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->dss_full);
     }
     // Epilogue: dV and dK rows (transpose of RoPE on dK) staged transposed in the now idle stage
     // buffers, then stored as dQKV^T columns with coalesced 16-byte stores.
@@ -482,57 +527,44 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // ================================================================================ dQ
-// Persistent: one CTA per SM takes (128 query rows, query head, sequence) tiles (sched_tile)
-// with 128-key blocks, so every UMMA is M128 N128. Q and dO live in tensor memory (copied from a 32 KB
-// staging tile by tcgen05.cp), so S = Q K^T and dP = dO V^T are TS-form UMMAs that read only K and V
-// from shared memory, and the shared memory saved holds a third K stage: K is read by S_j and again
-// by dQ_j += dS_j K_j, so it is held for a whole block.
-//   TMEM columns: S 0, dP 128, dQ 256 (DH), Q and dO (DH / 2 each) after it.
-//   warp 0      TMA: Q and dO of each tile through the staging tile, K ring (3 stages)
-//   warp 1      TMEM owner, tcgen05.cp of Q and dO, UMMA issuer (one thread, event-driven)
-//   warps 2..9  elementwise: dS = P (dP - D) with P = exp2(S scale log2(e) - lse), fp16 to shared
-//               memory; at the end of a tile they read dQ out of TMEM, apply the transpose of RoPE
-//               and stage the tile transposed (bf16) in the dS buffer, then go on with the next tile
-//   warp 10     TMA: V ring (2 stages)
-//   warp 11     stores the staged tile as dQKV^T columns (coalesced 16-byte stores) while the
-//               elementwise warps work on the next tile's first block
-// A tile's Q is copied in once the previous tile's last S has completed and its dO once the last dP
-// has; the staging tile is refilled with the next operand as soon as each copy has completed.
-constexpr int DQ_THREADS = 384;  // 12 warps: 65536 / 384 leaves 168 registers per thread
-constexpr int DQ_STORE_WARP = 11;
+// dQ = scale * dS K from the dS^T tiles the dK/dV kernel stored: no recomputation of S, P or dP.
+// Persistent: one CTA per SM takes (128 query rows, query head, sequence) tiles (sched_tile,
+// most key blocks first); for each key block kb <= qb one stage holds the dS^T tile (128 keys x 128
+// queries: the MN-major A operand of dS K) and K_kb (128 keys x d_h: the MN-major B operand), and
+// eight M128 N = d_h K16 UMMAs accumulate into one of two dQ buffers in TMEM.
+//   warp 0      TMA: dS^T and K tiles, 3-stage ring
+//   warp 1      TMEM owner, UMMA issuer (one thread)
+//   warps 2..9  epilogue of the previous tile (its dQ buffer): transpose of RoPE, staged transposed
+//               in shared memory, stored as dQKV^T columns with coalesced 16-byte stores
+constexpr int DQ_THREADS = 320;
 
 template <int DH>
 struct DqLayout {
-  static constexpr int BQ = 128, BK = 128;
-  static constexpr int KST = 3, VST = 2;
-  static constexpr int CHUNK = 128 * 128;  // 64 columns of a 128-row tile
-  static constexpr int TILE = 128 * DH * 2;
-  static constexpr int STG_OFF = 0;  // Q or dO of a tile, on its way into TMEM
-  static constexpr int K_OFF = STG_OFF + TILE;
-  static constexpr int V_OFF = K_OFF + KST * TILE;
-  static constexpr int DS_OFF = V_OFF + VST * TILE;  // dS, and the epilogue's staging tile
-  static constexpr int DS_BYTES = BQ * BK * 2;
-  static constexpr int BAR_OFF = DS_OFF + DS_BYTES;
-  static constexpr int USED = BAR_OFF + 256 + 1024;
+  static constexpr int BQ = 128, BK = 128, STAGES = 3;
+  static constexpr int CHUNK = 128 * 128;       // 64 columns of a 128-row fp16 tile
+  static constexpr int DS_TILE = 128 * 128 * 2;  // dS^T: 128 keys x 128 queries
+  static constexpr int K_TILE = 128 * DH * 2;    // 128 keys x d_h
+  static constexpr int STAGE = DS_TILE + K_TILE;
+  static constexpr int STG_OFF = STAGES * STAGE;  // epilogue staging: d_h x 128 bf16
+  static constexpr int BAR_OFF = STG_OFF + DH * 128 * 2;
+  static constexpr int USED = BAR_OFF + 256;      // base alignment checked in the kernel
   static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
-  static constexpr uint32_t S_COL = 0, DP_COL = 128, DQ_COL = 256, Q_COL = 256 + DH,
-                            DO_COL = 256 + DH + DH / 2;
-  static_assert(DO_COL + DH / 2 <= 512, "TMEM budget");
-  static_assert(DS_BYTES >= DH * 128 * 2, "epilogue staging fits the dS buffer");
+  static constexpr uint32_t DQ_STRIDE = 128;      // TMEM columns between the two dQ buffers
+  static_assert(USED <= 227 * 1024, "shared memory budget");
 };
 
 struct DqBars {
-  uint64_t stg_full, stg_empty, k_full[3], k_empty[3], v_full[2], v_empty[2], s_full, s_empty;
-  uint64_t p_full, p_empty, o_full, o_empty, out_full, out_free, drain;
+  uint64_t full[3], empty[3], o_full[2], o_empty[2], drain;
   uint32_t tmem_base;
   int abort;
+  int stop;  // the epilogue warps' common decision to leave (a snapshot of abort)
 };
 
 struct DqTile {
   int qb, h, b;
 };
 // Tile n of the most-work-first order: query blocks from the last (most keys) to the first, then
-// query heads and sequences.
+// query heads (the heads of a KV group next to each other: K tiles shared in L2) and sequences.
 __device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
   const int per_qb = Hq * B;
   const int r = n % per_qb;
@@ -541,14 +573,16 @@ __device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
 
 template <int DH>
 __global__ void __launch_bounds__(DQ_THREADS, 1)
-    attn_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
-                          const __grid_constant__ CUtensorMap tm_kv,
-                          const __grid_constant__ CUtensorMap tm_do, const BwdParams p) {
+    attn_bwd_dq_tc_kernel(const __grid_constant__ CUtensorMap tm_ds,
+                          const __grid_constant__ CUtensorMap tm_kv, const BwdParams p) {
   using L = DqLayout<DH>;
-  constexpr int BQ = L::BQ, BK = L::BK, KST = L::KST, VST = L::VST;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
+  constexpr int BQ = L::BQ, BK = L::BK, NST = L::STAGES;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (tc::smem_u32(smem_raw) & 1023u) {  // the swizzled TMA tiles need a 1024-byte aligned base
+    if (threadIdx.x == 0) report(p.status, JAB_ERR_INTERNAL);
+    return;
+  }
+  uint8_t* smem = smem_raw;
   DqBars* bars = reinterpret_cast<DqBars*>(smem + L::BAR_OFF);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
@@ -558,33 +592,23 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
   auto n_kb_of = [&](const DqTile& tl) { return (min(tl.qb * BQ + BQ, p.T) + BK - 1) / BK; };
 
   if (threadIdx.x == 0) {
-    tc::mbar_init(&bars->stg_full, 1);
-    tc::mbar_init(&bars->stg_empty, 1);
-    for (int i = 0; i < KST; ++i) {
-      tc::mbar_init(&bars->k_full[i], 1);
-      tc::mbar_init(&bars->k_empty[i], 1);
+    for (int i = 0; i < NST; ++i) {
+      tc::mbar_init(&bars->full[i], 1);
+      tc::mbar_init(&bars->empty[i], 1);
     }
-    for (int i = 0; i < VST; ++i) {
-      tc::mbar_init(&bars->v_full[i], 1);
-      tc::mbar_init(&bars->v_empty[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&bars->o_full[i], 1);
+      tc::mbar_init(&bars->o_empty[i], EW_WARPS);
     }
-    tc::mbar_init(&bars->s_full, 1);
-    tc::mbar_init(&bars->s_empty, EW_WARPS);
-    tc::mbar_init(&bars->p_full, EW_WARPS);
-    tc::mbar_init(&bars->p_empty, 1);
-    tc::mbar_init(&bars->o_full, 1);
-    tc::mbar_init(&bars->o_empty, EW_WARPS);
-    tc::mbar_init(&bars->out_full, EW_WARPS);  // the tile's dQ is staged in the dS buffer
-    tc::mbar_init(&bars->out_free, 1);         // the store warp has read the staged tile
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
+    bars->stop = 0;
     tc::fence_mbar_init();
-    tc::prefetch_tmap(&tm_q);
+    tc::prefetch_tmap(&tm_ds);
     tc::prefetch_tmap(&tm_kv);
-    tc::prefetch_tmap(&tm_do);
   }
   if (warp == 1) {
-    tc::tmem_alloc(&bars->tmem_base, 512);
+    tc::tmem_alloc(&bars->tmem_base, 256);
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
@@ -592,268 +616,98 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
   tc::fence_after_sync();
   const uint32_t tmem = bars->tmem_base;
 
-  if (warp == 0 || warp == 10) {
-    if (lane == 0) {  // --------------------------------------- TMA: Q, dO, K (warp 0); V (warp 10)
-      const bool is_v = warp == 10;
-      uint32_t J = 0, U = 0;  // key blocks and staging uses so far (all tiles)
-      const int nst = is_v ? VST : KST;
-      uint64_t* full = is_v ? bars->v_full : bars->k_full;
-      uint64_t* empty = is_v ? bars->v_empty : bars->k_empty;
-      uint8_t* ring = smem + (is_v ? L::V_OFF : L::K_OFF);
-      bool ok = true, stg_issued = false;
-      uint32_t iss = 0, par = 0, stg_par = 0;
+  if (warp == 0) {
+    if (lane == 0) {  // ---------------------------------------------------------------- TMA
+      uint32_t J = 0, iss = 0, par = 0;
+      bool ok = true;
       for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
            tile = sched_tile(++it, gridDim.x, blockIdx.x)) {
         const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
-        const int row0 = tl.b * p.T, g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
-        if (!is_v) {
-          for (int u = 0; u < 2; ++u, ++U) {  // Q, then dO
-            if (!tc::mbar_wait(&bars->stg_empty, (U & 1) ^ 1, abort, p.status)) { ok = false; break; }
-            tc::mbar_expect_tx(&bars->stg_full, L::TILE);
-            for (int ch = 0; ch < DH / 64; ++ch) {
-              if (u == 0)
-                tc::tma_load_2d(smem + L::STG_OFF + ch * L::CHUNK, &tm_q, &bars->stg_full,
-                                p.qcol0 + tl.h * DH + ch * 64, row0 + tl.qb * BQ);
-              else
-                tc::tma_load_2d(smem + L::STG_OFF + ch * L::CHUNK, &tm_do, &bars->stg_full,
-                                tl.h * DH + ch * 64, row0 + tl.qb * BQ);
-            }
-            stg_issued = true;
-            stg_par = U & 1;
-          }
-          if (!ok) break;
-        }
-        const int col = is_v ? p.vcol0 + g * DH : p.kcol0 + g * DH;
-        // A ring slot frees only when the block it holds has been used by the last UMMA that reads
-        // it, so blocks are also prefetched into L2 a ring's depth ahead of their load.
-        auto prefetch = [&](int j) {
-          for (int ch = 0; ch < DH / 64; ++ch) tc::tma_prefetch_2d(&tm_kv, col + ch * 64, row0 + j * BK);
-        };
-        for (int j = 0; j < nst && j < nkb; ++j) prefetch(j);
-        for (int j = 0; j < nkb; ++j, ++J) {
-          const int st = J % nst;
-          const uint32_t ph = (J / nst) & 1;
-          if (j + nst < nkb) prefetch(j + nst);
-          if (!tc::mbar_wait(&empty[st], ph ^ 1, abort, p.status)) { ok = false; break; }
-          tc::mbar_expect_tx(&full[st], L::TILE);
+        const int g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
+        const int64_t pair0 = ((int64_t)tl.b * p.Hq + tl.h) * p.npairs + (int64_t)tl.qb * (tl.qb + 1) / 2;
+        for (int kb = 0; kb < nkb; ++kb, ++J) {
+          const int st = J % NST;
+          const uint32_t ph = (J / NST) & 1;
+          if (!tc::mbar_wait(&bars->empty[st], ph ^ 1, abort, p.status)) { ok = false; break; }
+          uint8_t* sb = smem + st * L::STAGE;
+          tc::mbar_expect_tx(&bars->full[st], L::STAGE);
+          const int32_t y = (int32_t)((pair0 + kb) * BK);
+          tc::tma_load_2d(sb, &tm_ds, &bars->full[st], 0, y);
+          tc::tma_load_2d(sb + L::CHUNK, &tm_ds, &bars->full[st], 64, y);
           for (int ch = 0; ch < DH / 64; ++ch)
-            tc::tma_load_2d(ring + st * L::TILE + ch * L::CHUNK, &tm_kv, &full[st], col + ch * 64,
-                            row0 + j * BK);
+            tc::tma_load_2d(sb + L::DS_TILE + ch * L::CHUNK, &tm_kv, &bars->full[st],
+                            p.kcol0 + g * DH + ch * 64, tl.b * p.T + kb * BK);
           iss |= 1u << st;
           par = (par & ~(1u << st)) | (ph << st);
         }
       }
-      if (*abort) {
-        if (stg_issued) drain_wait(&bars->stg_full, stg_par);
-        for (int st = 0; st < nst; ++st)
-          if (iss & (1u << st)) drain_wait(&full[st], (par >> st) & 1);
-      }
+      if (*abort)
+        for (int st = 0; st < NST; ++st)
+          if (iss & (1u << st)) drain_wait(&bars->full[st], (par >> st) & 1);
     }
   } else if (warp == 1) {
-    if (lane == 0) {  // ------------------------------------------------------------- UMMA
-      constexpr uint32_t ID_S = tc::idesc_f16(false, BQ, BK);
-      constexpr uint32_t ID_G = tc::idesc_f16(false, BQ, DH) | (1u << 16);  // B = K, MN-major
-      const uint32_t stg_base = tc::smem_u32(smem + L::STG_OFF);
-      const uint64_t dsd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::DS_OFF));
+    if (lane == 0) {  // ---------------------------------------------------------------- UMMA
+      // A = dS (M = queries, K = keys) and B = K (N = d_h, K = keys) are both MN-major tiles
+      constexpr uint32_t ID_Q = tc::idesc_f16(false, BQ, DH) | (1u << 15) | (1u << 16);
+      uint32_t J = 0;
       bool ok = true;
-      uint32_t Js = 0, Jg = 0, U = 0;  // S/dP blocks, dQ blocks, staging uses so far (all tiles)
       int n = 0;
-      tc::Watchdog wd;
-      auto copy_in = [&](uint32_t col) -> bool {  // staging tile -> TMEM columns [col, col + DH/2)
-        if (!tc::mbar_wait(&bars->stg_full, U & 1, abort, p.status)) return false;
-        tc::fence_after_sync();
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk)
-          tc::tmem_cp_128x256b(tmem + col + kk * 8,
-                               tc::sdesc_kmajor_sw128(stg_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
-        tc::umma_commit(&bars->stg_empty);
-        ++U;
-        return true;
-      };
       for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
            tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
         const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
-        const int nkb = n_kb_of(tl);
-        // Q and dO of this tile into TMEM once every S / dP of the previous tile (which read the old
-        // Q and dO) has completed.
-        if (Js > 0 && !tc::mbar_wait(&bars->s_full, (Js - 1) & 1, abort, p.status)) break;
-        if (!copy_in(L::Q_COL) || !copy_in(L::DO_COL)) break;
-        // Event-driven issue: S/dP of block ns once K_ns, V_ns have landed and the elementwise
-        // warps have read the previous S/dP; dQ of block ng once its dS is written (and, for the
-        // tile's first, once the previous tile's dQ has been read out).
-        int ns = 0, ng = 0;
-        while (ok && ng < nkb) {
-          bool prog = false;
-          if (ns < nkb && ns <= ng + 1 && tc::mbar_ready(&bars->k_full[Js % KST], (Js / KST) & 1) &&
-              tc::mbar_ready(&bars->v_full[Js % VST], (Js / VST) & 1) &&
-              tc::mbar_ready(&bars->s_empty, (Js & 1) ^ 1)) {
-            tc::fence_after_sync();
-            const uint64_t kd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF + (Js % KST) * L::TILE));
-            const uint64_t vd = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::V_OFF + (Js % VST) * L::TILE));
+        const int nkb = n_kb_of(tl), ob = n & 1;
+        // the buffer's previous tile (n - 2) must have been read out by the epilogue
+        if (n >= 2 && !tc::mbar_wait(&bars->o_empty[ob], ((n >> 1) - 1) & 1, abort, p.status)) break;
+        for (int kb = 0; kb < nkb; ++kb, ++J) {
+          const int st = J % NST;
+          if (!tc::mbar_wait(&bars->full[st], (J / NST) & 1, abort, p.status)) { ok = false; break; }
+          tc::fence_after_sync();
+          const uint32_t sb = tc::smem_u32(smem + st * L::STAGE);
+          const uint64_t ad = tc::sdesc_mnmajor_sw128(sb, L::CHUNK, 1024);
+          const uint64_t bd = tc::sdesc_mnmajor_sw128(sb + L::DS_TILE, L::CHUNK, 1024);
 #pragma unroll
-            for (int k = 0; k < DH / 16; ++k) {
-              const uint32_t off = (k >> 2) * L::CHUNK + (k & 3) * 32;
-              tc::umma_f16_ts(tmem + L::S_COL, tmem + L::Q_COL + k * 8, tc::sdesc_advance(kd, off), ID_S,
-                              k > 0 ? 1u : 0u);
-              tc::umma_f16_ts(tmem + L::DP_COL, tmem + L::DO_COL + k * 8, tc::sdesc_advance(vd, off), ID_S,
-                              k > 0 ? 1u : 0u);
-            }
-            tc::umma_commit(&bars->s_full);
-            tc::umma_commit(&bars->v_empty[Js % VST]);
-            ++ns;
-            ++Js;
-            prog = true;
-          }
-          if (ng < ns && tc::mbar_ready(&bars->p_full, Jg & 1) &&
-              (ng > 0 || n == 0 || tc::mbar_ready(&bars->o_empty, (n - 1) & 1))) {
-            tc::fence_after_sync();
-            const uint64_t kd = tc::sdesc_mnmajor_sw128(
-                tc::smem_u32(smem + L::K_OFF + (Jg % KST) * L::TILE), L::CHUNK, 1024);
-#pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-              tc::umma_f16(tmem + L::DQ_COL, tc::sdesc_advance(dsd, (k >> 2) * (BQ * 128) + (k & 3) * 32),
-                           tc::sdesc_advance(kd, k * 16 * 128), ID_G, (ng > 0 || k > 0) ? 1u : 0u);
-            tc::umma_commit(&bars->k_empty[Jg % KST]);
-            tc::umma_commit(&bars->p_empty);
-            ++ng;
-            ++Jg;
-            if (ng == nkb) tc::umma_commit(&bars->o_full);
-            prog = true;
-          }
-          if (prog)
-            wd.progress();
-          else if (!wd.tick(abort, p.status))
-            ok = false;
+          for (int k = 0; k < BK / 16; ++k)
+            tc::umma_f16(tmem + ob * L::DQ_STRIDE, tc::sdesc_advance(ad, k * 16 * 128),
+                         tc::sdesc_advance(bd, k * 16 * 128), ID_Q, (kb > 0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&bars->empty[st]);
         }
+        if (!ok) break;
+        tc::umma_commit(&bars->o_full[ob]);
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else if (warp == DQ_STORE_WARP) {  // ------------------------------------- dQKV^T stores
-    // The staged tile of each tile in turn, once the elementwise warps have written it; the buffer
-    // is handed back before the same warps write the next tile's first dS into it.
-    const bf16_t* stage = reinterpret_cast<const bf16_t*>(smem + L::DS_OFF);
-    int n = 0;
-    for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
-         tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
-      const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
-      const int q0 = tl.qb * BQ;
-      if (!tc::mbar_wait(&bars->out_full, n & 1, abort, p.status)) break;
-      store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
-                     (int64_t)tl.b * p.T + q0, min(BQ, p.T - q0), lane, 32);
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->out_free);
-    }
-  } else {  // ------------------------------------------------ elementwise: row = query, 64 keys
+  } else {  // ----------------------------------------------------- epilogue, 16 rows per warp
     const int quarter = warp & 3;
     const int half = (warp - 2) >> 2;
-    const int row = quarter * 32 + lane;
-    const int col0 = half * 64;
-    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
-    uint8_t* dsrow = smem + L::DS_OFF + half * (BQ * 128) + row * 128;  // one 64-key swizzle chunk
-    bf16_t* stage = reinterpret_cast<bf16_t*>(smem + L::DS_OFF);
-    bool ok = true;
-    uint32_t J = 0;
+    const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
+    const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
+    bf16_t* stage = reinterpret_cast<bf16_t*>(smem + L::STG_OFF);
     int n = 0;
     for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
          tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
       const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
-      const int nkb = n_kb_of(tl);
-      const int q0 = tl.qb * BQ, t = q0 + row;
-      const bool valid_row = t < p.T;
-      const int64_t lrow = ((int64_t)tl.b * p.Hq + tl.h) * p.lse_pitch + (valid_row ? t : 0);
-      const float lse2 = valid_row ? p.lse[lrow] : INFINITY;  // P = 0 on rows past T
-      const float drow = valid_row ? p.dvec[lrow] : 0.f;
-      for (int j = 0; ok && j < nkb; ++j, ++J) {
-        if (!tc::mbar_wait(&bars->s_full, J & 1, abort, p.status)) {
-          ok = false;
-          break;
-        }
+      const int ob = n & 1, q0 = tl.qb * BQ;
+      const bool have = tc::mbar_wait(&bars->o_full[ob], (n >> 1) & 1, abort, p.status);
+      if (have) {
         tc::fence_after_sync();
-        float sv[64], dp[64];
-#pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
-          uint32_t rs[32], rd[32];
-          __syncwarp();
-          tc::tmem_ld32(tmem + lane_base + L::S_COL + col0 + ch * 32, rs);
-          tc::tmem_ld32(tmem + lane_base + L::DP_COL + col0 + ch * 32, rd);
-          tc::tmem_ld_wait();
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            sv[ch * 32 + e] = __uint_as_float(rs[e]);
-            dp[ch * 32 + e] = __uint_as_float(rd[e]);
-          }
-        }
-        tc::fence_before_sync();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->s_empty);
-        const int k0 = j * BK + col0;
-        {  // packed FP32 pairs; one loop per mask case keeps the per-element work minimal
-          const float2 sl2 = make_float2(p.sl2, p.sl2);
-          const float2 nl = make_float2(tc::neg_bits(lse2), tc::neg_bits(lse2));
-          const float2 d2 = make_float2(drow, drow);
-          if (k0 + 63 <= q0) {  // every key of this slice is visible to every row of the tile
-#pragma unroll
-            for (int c = 0; c < 64; c += 2) {
-              const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
-              const float2 ds = tc::mul2(make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y)),
-                                         tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
-              dp[c] = ds.x;
-              dp[c + 1] = ds.y;
-            }
-          } else {
-#pragma unroll
-            for (int c = 0; c < 64; c += 2) {
-              const float2 a = tc::fma2(make_float2(sv[c], sv[c + 1]), sl2, nl);
-              const float2 ds = tc::mul2(make_float2(tc::fast_exp2(a.x), tc::fast_exp2(a.y)),
-                                         tc::sub2(make_float2(dp[c], dp[c + 1]), d2));
-              dp[c] = (k0 + c <= t) ? ds.x : 0.f;
-              dp[c + 1] = (k0 + c + 1 <= t) ? ds.y : 0.f;
-            }
-          }
-        }
-        if (!tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status) ||
-            (j == 0 && n > 0 && !tc::mbar_wait(&bars->out_free, (n - 1) & 1, abort, p.status))) {
-          ok = false;  // (the first dS of a tile waits until the previous tile's dQ is stored)
-          break;
-        }
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          uint4 u;
-          __half2* hp = reinterpret_cast<__half2*>(&u);
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            hp[e] = __floats2half2_rn(dp[c8 * 8 + 2 * e], dp[c8 * 8 + 2 * e + 1]);
-          *reinterpret_cast<uint4*>(dsrow + ((c8 ^ (row & 7)) << 4)) = u;
-        }
-        tc::fence_proxy_async_smem();
-        tc::fence_before_sync();
-        __syncwarp();
-        if (lane == 0) tc::mbar_arrive(&bars->p_full);
-      }
-      if (!ok) break;
-      // Epilogue: dQ rows (transpose of RoPE) staged transposed in the dS buffer (free until this
-      // tile's successor writes its first dS, which waits for the store warp), stored by the store
-      // warp as dQKV^T columns.
-      if (!tc::mbar_wait(&bars->o_full, n & 1, abort, p.status) ||
-          !tc::mbar_wait(&bars->p_empty, (J & 1) ^ 1, abort, p.status)) {
-        ok = false;
-        break;
-      }
-      tc::fence_after_sync();
-      {
-        const int ra = quarter * 32 + half * 16 + (lane >> 2);  // 16x256b rows of this thread
-        const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
         const int ta = q0 + ra, tb = ta + 8;
-        stage_grad_16<DH>(tmem + lane16 + L::DQ_COL, p.scale, p.use_rope != 0, ta < p.T ? ta : 0,
-                          tb < p.T ? tb : 0, p.cos_t, p.sin_t, stage, ra);
+        stage_grad_16<DH>(tmem + lane16 + ob * L::DQ_STRIDE, p.scale, p.use_rope != 0,
+                          ta < p.T ? ta : 0, tb < p.T ? tb : 0, p.cos_t, p.sin_t, stage, ra);
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&bars->o_empty[ob]);  // the dQ buffer is free again
       }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) {
-        tc::mbar_arrive(&bars->o_empty);   // dQ accumulator reusable
-        tc::mbar_arrive(&bars->out_full);  // this warp's share of the staged tile is written
-      }
+      tc::named_bar_sync(1, EW_WARPS * 32);  // every epilogue warp reaches this once per tile
+      if (have)
+        store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
+                       (int64_t)tl.b * p.T + q0, min(BQ, p.T - q0), threadIdx.x - 64,
+                       EW_WARPS * 32);
+      // One snapshot of the abort flag between the two barriers, so that all epilogue warps leave
+      // together (a warp left behind would wait on the named barrier of the next tile).
+      if (threadIdx.x == 64) reinterpret_cast<volatile int*>(&bars->stop)[0] = *abort;
+      tc::named_bar_sync(1, EW_WARPS * 32);  // the staging tile is read before it is rewritten
+      if (reinterpret_cast<volatile int*>(&bars->stop)[0]) break;
     }
   }
   tc::fence_before_sync();
@@ -861,7 +715,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
   tc::fence_after_sync();
   if (warp == 1) {
     __syncwarp();
-    tc::tmem_dealloc(tmem, 512);
+    tc::tmem_dealloc(tmem, 256);
   }
 }
 
@@ -902,9 +756,13 @@ cudaError_t set_smem(K kernel, int bytes, bool& done) {
 template <int DH>
 cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   const int64_t N = (int64_t)L.B * L.T;
-  CUtensorMap kv128, do128;
+  // dS^T tiles as a 2-D fp16 tensor of 128-query rows, one 128-row block per (sequence, head,
+  // query block, key block)
+  const uint64_t ds_rows = (uint64_t)L.B * L.Hq * p.npairs * 128;
+  CUtensorMap kv128, do128, ds128;
   if (!tmap_rows(&kv128, L.qkv, L.ldq, N, 128) ||
-      !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128))
+      !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128) ||
+      !tmap_rows(&ds128, L.ds, 128, ds_rows, 128) || ds_rows >= (1ull << 31))
     return cudaErrorInvalidValue;
   static bool a1 = false, a2 = false;
   cudaError_t e = set_smem(attn_bwd_dkdv_tc_kernel<DH>, DkdvLayout<DH>::SMEM, a1);
@@ -912,7 +770,8 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   e = set_smem(attn_bwd_dq_tc_kernel<DH>, DqLayout<DH>::SMEM, a2);
   if (e != cudaSuccess) return e;
   dim3 g1((unsigned)L.Hkv, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
-  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128, p);
+  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128,
+                                                                                     ds128, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -920,7 +779,7 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int64_t dq_tiles = (int64_t)((L.T + 127) / 128) * L.Hq * L.B;
   const unsigned g2 = (unsigned)std::min<int64_t>(dq_tiles, sms > 0 ? sms : 1);
-  attn_bwd_dq_tc_kernel<DH><<<g2, DQ_THREADS, DqLayout<DH>::SMEM, L.stream>>>(kv128, kv128, do128, p);
+  attn_bwd_dq_tc_kernel<DH><<<g2, DQ_THREADS, DqLayout<DH>::SMEM, L.stream>>>(ds128, kv128, p);
   return cudaGetLastError();
 }
 
@@ -938,6 +797,8 @@ cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const fl
   p.kcol0 = L.Hq * L.dh;
   p.vcol0 = (L.Hq + L.Hkv) * L.dh;
   p.ldt = L.ldt;
+  const int nq = (L.T + 127) / 128;
+  p.npairs = nq * (nq + 1) / 2;
   p.scale = L.scale;
   p.sl2 = L.scale * kLog2e;
   p.lse = L.lse;
@@ -948,7 +809,7 @@ cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const fl
   p.dqkvt = static_cast<bf16_t*>(dqkvt);
   p.status = L.status;
   if ((reinterpret_cast<uintptr_t>(L.lse) & 15u) || (reinterpret_cast<uintptr_t>(L.dvec) & 15u) ||
-      (L.lse_pitch % 128) != 0)
+      (L.lse_pitch % 128) != 0 || L.ds == nullptr || (reinterpret_cast<uintptr_t>(L.ds) & 15u))
     return cudaErrorInvalidValue;
   return L.dh == 128 ? launch_bwd<128>(L, p) : launch_bwd<64>(L, p);
 }

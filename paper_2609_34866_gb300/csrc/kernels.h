@@ -20,6 +20,7 @@ struct AttnLaunch {
   float* dvec;          // fp32 [B, Hq, T] (backward)
   int64_t ldt;          // row pitch of the transposed dQKV^T (backward)
   int lse_pitch;        // row pitch of lse and dvec ([B, Hq, lse_pitch])
+  void* ds;             // fp16 dS^T tiles (backward): [B, Hq, nq (nq + 1) / 2, 128 keys, 128 queries]
   int* status;
   cudaStream_t stream;
 };

@@ -26,6 +26,8 @@ struct Workspace {
   size_t lse;      // fp32 [B, Hq, Tp]       student log-sum-exp in log2 units (Tp = T rounded to 128)
   size_t dvec;     // fp32 [B, Hq, Tp]       rowsum(dO * O)
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
+  size_t ds;       // fp16 [B, Hq, nq (nq + 1) / 2, 128, 128]   dS^T tile of every (query block,
+                   //                        key block <= query block) pair, nq = ceil(T / 128)
   int64_t ldt;     // row pitch (elements) of dqkvt: N rounded up to 64
   int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 128
   size_t total;
@@ -63,8 +65,10 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
     w.lse = take((size_t)B * d->n_q_heads * w.tp * 4);
     w.dvec = take((size_t)B * d->n_q_heads * w.tp * 4);
     w.dqkvt = take((size_t)D * w.ldt * 2);
+    const int64_t nq = (T + 127) / 128;
+    w.ds = take((size_t)B * d->n_q_heads * (nq * (nq + 1) / 2) * 128 * 128 * 2);
   } else {
-    w.d_o = w.lse = w.dvec = w.dqkvt = SIZE_MAX;
+    w.d_o = w.lse = w.dvec = w.dqkvt = w.ds = SIZE_MAX;
   }
   w.total = off;
   return w;
