@@ -26,6 +26,7 @@ namespace {
 
 constexpr int NUM_THREADS = 352;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise, warp 10 dS^T stores
 constexpr int EW_WARPS = 8;
+constexpr int kSuperGroup = 8;  // (KV head, sequence) pairs whose dK/dV CTAs are interleaved
 constexpr float kLog2e = 1.4426950408889634f;
 
 struct BwdParams {
@@ -182,9 +183,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
 
-  const int kb = blockIdx.z, g = blockIdx.x, b = blockIdx.y;  // key block slowest: longest first
   const int r = p.Hq / p.Hkv;
   const int nq = (p.T + BQ - 1) / BQ;
+  // CTA order: super-groups of kSuperGroup (KV head, sequence) pairs, key block slowest inside one,
+  // so that the CTAs which stream the same Q and dO blocks run at the same time (their reads hit
+  // L2) and the longest CTAs of a super-group start first.
+  int kb, g, b;
+  {
+    const int pairs = p.Hkv * p.B;
+    const int sg = blockIdx.x / (kSuperGroup * nq);
+    const int sgs = min(kSuperGroup, pairs - sg * kSuperGroup);
+    const int rem = blockIdx.x - sg * kSuperGroup * nq;
+    kb = rem / sgs;
+    const int pr = sg * kSuperGroup + rem % sgs;
+    g = pr % p.Hkv;
+    b = pr / p.Hkv;
+  }
   const int per_head = nq - kb;  // query blocks kb .. nq - 1 see keys of block kb
   const int n_it = r * per_head;
   const int row0 = b * p.T;
@@ -563,12 +577,15 @@ struct DqBars {
 struct DqTile {
   int qb, h, b;
 };
-// Tile n of the most-work-first order: query blocks from the last (most keys) to the first, then
-// query heads (the heads of a KV group next to each other: K tiles shared in L2) and sequences.
-__device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int B) {
-  const int per_qb = Hq * B;
-  const int r = n % per_qb;
-  return DqTile{nqb - 1 - n / per_qb, r % Hq, r / Hq};
+// Tile n: grouped by (sequence, KV group), so that all tiles which read the K blocks of one KV head
+// run close together (K read from HBM once); inside a group query blocks from the last (most keys)
+// to the first, the query heads of the group next to each other.
+__device__ __forceinline__ DqTile dq_tile(int n, int nqb, int Hq, int Hkv) {
+  const int r = Hq / Hkv;
+  const int per_group = r * nqb;
+  const int grp = n / per_group, rem = n - grp * per_group;
+  const int g = grp % Hkv, b = grp / Hkv;
+  return DqTile{nqb - 1 - rem / r, g * r + rem % r, b};
 }
 
 template <int DH>
@@ -622,7 +639,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       bool ok = true;
       for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
            tile = sched_tile(++it, gridDim.x, blockIdx.x)) {
-        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.Hkv);
         const int g = tl.h / (p.Hq / p.Hkv), nkb = n_kb_of(tl);
         const int64_t pair0 = ((int64_t)tl.b * p.Hq + tl.h) * p.npairs + (int64_t)tl.qb * (tl.qb + 1) / 2;
         for (int kb = 0; kb < nkb; ++kb, ++J) {
@@ -654,7 +671,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       int n = 0;
       for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); ok && tile < n_tiles;
            tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
-        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+        const DqTile tl = dq_tile(tile, nqb, p.Hq, p.Hkv);
         const int nkb = n_kb_of(tl), ob = n & 1;
         // the buffer's previous tile (n - 2) must have been read out by the epilogue
         if (n >= 2 && !tc::mbar_wait(&bars->o_empty[ob], ((n >> 1) - 1) & 1, abort, p.status)) break;
@@ -686,7 +703,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
     int n = 0;
     for (int it = 0, tile = sched_tile(0, gridDim.x, blockIdx.x); tile < n_tiles;
          tile = sched_tile(++it, gridDim.x, blockIdx.x), ++n) {
-      const DqTile tl = dq_tile(tile, nqb, p.Hq, p.B);
+      const DqTile tl = dq_tile(tile, nqb, p.Hq, p.Hkv);
       const int ob = n & 1, q0 = tl.qb * BQ;
       const bool have = tc::mbar_wait(&bars->o_full[ob], (n >> 1) & 1, abort, p.status);
       if (have) {
@@ -769,7 +786,9 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   if (e != cudaSuccess) return e;
   e = set_smem(attn_bwd_dq_tc_kernel<DH>, DqLayout<DH>::SMEM, a2);
   if (e != cudaSuccess) return e;
-  dim3 g1((unsigned)L.Hkv, (unsigned)L.B, (unsigned)((L.T + 127) / 128));
+  const int64_t n_dkdv = (int64_t)L.Hkv * L.B * ((L.T + 127) / 128);
+  if (n_dkdv >= (1ll << 31)) return cudaErrorInvalidValue;
+  const dim3 g1((unsigned)n_dkdv);
   attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128,
                                                                                      ds128, p);
   e = cudaGetLastError();

@@ -126,10 +126,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &bars->abort;
 
-  const int qb = p.nqb - 1 - (int)blockIdx.z;  // slowest grid index: longest rows start first
-  const int h = blockIdx.x;
-  const int b = (int)blockIdx.y % p.B, c = (int)blockIdx.y / p.B;
-  const int g = h / (p.Hq / p.Hkv);
+  // CTA order: grouped by (sequence x candidate, KV group), so that the CTAs which stream the K blocks
+  // of one KV head run close together (read from HBM about once); inside a group query blocks from
+  // the last (most keys) to the first, the query heads of the group next to each other.
+  const int ratio = p.Hq / p.Hkv;
+  const int per_group = ratio * p.nqb;
+  const int grp = (int)blockIdx.x / per_group, rem = (int)blockIdx.x - grp * per_group;
+  const int qb = p.nqb - 1 - rem / ratio;
+  const int g = grp % p.Hkv;
+  const int h = g * ratio + rem % ratio;
+  const int b = (grp / p.Hkv) % p.B, c = (grp / p.Hkv) / p.B;
   const int q0 = qb * BQ;
   const int nkb = min(qb + 1, (p.T + BK - 1) / BK);
   const int row0 = b * p.T;
@@ -407,7 +413,9 @@ cudaError_t launch_kl(const CUtensorMap& ts, const CUtensorMap& tt, const KlPara
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((unsigned)p.Hq, (unsigned)(p.B * p.C), (unsigned)p.nqb);
+  const int64_t n = (int64_t)p.Hq * p.B * p.C * p.nqb;
+  if (n >= (1ll << 31)) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)n);
   attn_kl_tc_kernel<DH><<<grid, NUM_THREADS, KlLayout<DH>::SMEM, st>>>(ts, tt, p);
   return cudaGetLastError();
 }

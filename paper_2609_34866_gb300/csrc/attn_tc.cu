@@ -102,13 +102,18 @@ struct StackTile {
   int hu, bc, qb, nkb;  // head unit (HPT consecutive query heads), sequence x candidate, row block
 };
 
-// Tile k of the most-work-first order: query blocks from the last (most key blocks) to the first,
-// then sequences and head units. rph = query rows per head in a tile.
-__device__ __forceinline__ StackTile stack_tile(int k, int units, int BC, int nqb, int T, int rph) {
+// Tile k: grouped by (sequence x candidate, KV group), so that the tiles which stream the K and V
+// blocks of one KV head run close together (K and V read from HBM about once); inside a group query
+// blocks from the last (most key blocks) to the first, the head units of the group next to each
+// other. rph = query rows per head in a tile; units (query heads / HPT) is a multiple of Hkv.
+__device__ __forceinline__ StackTile stack_tile(int k, int units, int Hkv, int nqb, int T, int rph) {
+  const int upg = units / Hkv;  // head units per KV group
+  const int per_group = upg * nqb;
+  const int grp = k / per_group, rem = k - grp * per_group;
   StackTile t;
-  t.hu = k % units;
-  t.bc = (k / units) % BC;
-  t.qb = nqb - 1 - k / (units * BC);
+  t.hu = (grp % Hkv) * upg + rem % upg;
+  t.bc = grp / Hkv;
+  t.qb = nqb - 1 - rem / upg;
   t.nkb = (min((t.qb + 1) * rph, T) + SKB - 1) / SKB;
   return t;
 }
@@ -180,7 +185,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       const int NST = is_v ? SV_ST : SK_ST;
       for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
            k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
-        const StackTile tl = stack_tile(k, units, BC, nqb, p.T, RPH);
+        const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
         const int b = tl.bc % p.B, c = tl.bc / p.B, h0 = HPT * tl.hu, g = h0 / ratio;
         const int row0 = b * p.T, q0 = tl.qb * RPH;
         const int col = c * p.D + (is_v ? p.Hq + p.Hkv + g : p.Hq + g) * DH;
@@ -262,7 +267,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       };
       for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
            k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
-        const StackTile tl = stack_tile(k, units, BC, nqb, p.T, RPH);
+        const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
         // Q of this tile into TMEM once the previous tile's last S (which read the old Q) is done.
         if (g0 > 0 && !tc::mbar_wait(&bars->s_full, (g0 - 1) & 1, abort, p.status)) break;
         if (!tc::mbar_wait(&bars->q_full, tc_ & 1, abort, p.status)) break;
@@ -299,7 +304,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
-      const StackTile tl = stack_tile(k, units, BC, nqb, p.T, RPH);
+      const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
       const int q0 = tl.qb * RPH;
       const int tA = q0 + (rA & (RPH - 1)), tB = q0 + (rB & (RPH - 1));
       const uint32_t o_col = L::O_COL + (tc_ & 1) * DH;
@@ -461,7 +466,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
-      const StackTile tl = stack_tile(k, units, BC, nqb, p.T, RPH);
+      const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
       const int b = tl.bc % p.B, c = tl.bc / p.B;
       const int h = HPT * tl.hu + row / RPH;
       const int q0 = tl.qb * RPH;
