@@ -476,8 +476,20 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.k_blocks = (int)((N + BK - 1) / BK);
   const int tiles = p.num_m * p.num_n;
   const int sms = sm_count();
-  int splits = 1;  // enough units for >= 4 waves, each at least 16 k-blocks long
-  while (tiles * splits < 4 * sms && p.k_blocks / (splits * 2) >= 16) splits *= 2;
+  // Split K so that the units (tile x K range) fill whole waves of the persistent grid: the
+  // makespan in k-blocks is ceil(tiles * s / sms) * (k_blocks / s + kFill), kFill standing for a
+  // unit's pipeline fill and drain. (768 tiles on 152 SMs without a split leave 8 SMs a sixth
+  // full-K unit while the others idle.) Each unit keeps at least 16 k-blocks.
+  constexpr double kFill = 8.0;
+  int splits = 1;
+  double best = (double)((tiles + sms - 1) / sms) * ((double)p.k_blocks + kFill);
+  for (int s = 2; s <= 32 && p.k_blocks / s >= 16; ++s) {
+    const double t = (double)(((int64_t)tiles * s + sms - 1) / sms) * ((double)p.k_blocks / s + kFill);
+    if (t < best * 0.995) {  // fewer splits on near-ties: fewer atomics and unit boundaries
+      best = t;
+      splits = s;
+    }
+  }
   p.splits = splits;
   p.group_m = 8;
   p.status = status;
