@@ -615,9 +615,12 @@ jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int3
   const int D = (int)block_rows(desc), dm = desc->d_model;
   const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
   if (grad_sqnorm_dev) JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_sqnorm_dev, 0, sizeof(double), st));
+  // the projection output is dead once the attention backward has run: scratch for a split K
   JAB_SITE("wgrad_store", 1, launch_wgrad_store_tc(w + wp.dqkvt, wp.ldt, X_dev, N, D, dm,
                                                    (float)(2.0 / n_el), grad_w_dev, grad_sqnorm_dev,
-                                                   status, st));
+                                                   reinterpret_cast<float*>(w + wp.qkv),
+                                                   (int64_t)(N * D * 2 / 4),
+                                                   reinterpret_cast<double*>(w + wp.red), status, st));
   if (grad_w_dev)
     JAB_SITE("check_finite", 1, launch_check_finite(grad_w_dev, (int64_t)D * dm, status, st));
   return JAB_OK;

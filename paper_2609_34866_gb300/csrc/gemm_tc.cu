@@ -16,6 +16,9 @@
 //               with the LSQ factor r of Eq. 13 recomputed from w and s; G is never stored. X is
 //               read as it is stored, [tokens, features], as the MN-major B operand (four 64-feature
 //               TMA boxes per stage), so no transposed copy of X is needed.
+//   store       coef * dQKV^T X as fp32 dW (STE weight gradient) and / or its squared norm; with a
+//               split K the partial tiles are added into a zeroed dW with vector atomics and the
+//               norm is reduced from dW afterwards in fixed order.
 #include <cudaTypedefs.h>
 
 #include "kernels.h"
@@ -50,7 +53,7 @@ struct GemmParams {
   int d, G, bits;
   float coef;
   float* ds;
-  // weight-gradient store epilogue (one unit covers the whole K range)
+  // weight-gradient store epilogue (a split K adds partial tiles into a zeroed dw)
   float* dw;
   double* sqnorm;
 };
@@ -164,9 +167,10 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
 }
 
 // STE weight gradient (App. B: d w_hat / d w = 1, so dL/dW = dL/dw_hat = coef * dQKV^T X): the
-// tile times coef stored as fp32 rows of dw (when set) and its squared Frobenius norm added to
-// *sqnorm (when set; fp64 atomics, one per warp and tile). Packed FP32 pairs, as this runs beside
-// the next tile's UMMAs.
+// tile times coef stored as fp32 rows of dw (when set; with a split K each unit's partial tile is
+// added with vector atomics) and, without a split, its squared Frobenius norm added to *sqnorm
+// (when set; fp64 atomics, one per warp and tile). Packed FP32 pairs, as this runs beside the next
+// tile's UMMAs.
 __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, int mb, int nb,
                                           int row) {
   const int64_t o = (int64_t)mb * BM + row;  // M = D is a multiple of 128: every row is valid
@@ -190,11 +194,17 @@ __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, i
     }
     if (p.dw != nullptr) {
       float4* d = reinterpret_cast<float4*>(p.dw + o * p.Nn + i0);
+      if (p.splits > 1) {  // a K range: add the partial tile into the zeroed dw
 #pragma unroll
-      for (int v = 0; v < 8; ++v) d[v] = make_float4(g[4 * v], g[4 * v + 1], g[4 * v + 2], g[4 * v + 3]);
+        for (int v = 0; v < 8; ++v)
+          atomicAdd(d + v, make_float4(g[4 * v], g[4 * v + 1], g[4 * v + 2], g[4 * v + 3]));
+      } else {
+#pragma unroll
+        for (int v = 0; v < 8; ++v) d[v] = make_float4(g[4 * v], g[4 * v + 1], g[4 * v + 2], g[4 * v + 3]);
+      }
     }
   }
-  if (p.sqnorm != nullptr) {
+  if (p.sqnorm != nullptr && p.splits == 1) {  // with a split K the caller reduces dw afterwards
     const double t = warp_sum((double)sq.x + (double)sq.y);
     if ((threadIdx.x & 31) == 0) atomicAdd(p.sqnorm, t);
   }
@@ -461,6 +471,25 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
   return launch_gemm<kEpiRope, false, false>(ta, tb, p, st);
 }
 
+// Split K so that the units (tile x K range) fill whole waves of the persistent grid: the makespan
+// in k-blocks is ceil(tiles * s / sms) * (k_blocks / s + kFill), kFill standing for a unit's pipeline
+// fill and drain. (768 tiles on 152 SMs without a split leave 8 SMs a sixth full-K unit while the
+// others idle.) Each unit keeps at least 16 k-blocks; near-ties go to fewer splits (fewer atomics
+// and unit boundaries).
+int choose_splits(int tiles, int k_blocks, int sms) {
+  constexpr double kFill = 8.0;
+  int splits = 1;
+  double best = (double)((tiles + sms - 1) / sms) * ((double)k_blocks + kFill);
+  for (int s = 2; s <= 32 && k_blocks / s >= 16; ++s) {
+    const double t = (double)(((int64_t)tiles * s + sms - 1) / sms) * ((double)k_blocks / s + kFill);
+    if (t < best * 0.995) {
+      best = t;
+      splits = s;
+    }
+  }
+  return splits;
+}
+
 cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st) {
@@ -474,23 +503,7 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.num_m = D / BM;
   p.num_n = (d + BN - 1) / BN;
   p.k_blocks = (int)((N + BK - 1) / BK);
-  const int tiles = p.num_m * p.num_n;
-  const int sms = sm_count();
-  // Split K so that the units (tile x K range) fill whole waves of the persistent grid: the
-  // makespan in k-blocks is ceil(tiles * s / sms) * (k_blocks / s + kFill), kFill standing for a
-  // unit's pipeline fill and drain. (768 tiles on 152 SMs without a split leave 8 SMs a sixth
-  // full-K unit while the others idle.) Each unit keeps at least 16 k-blocks.
-  constexpr double kFill = 8.0;
-  int splits = 1;
-  double best = (double)((tiles + sms - 1) / sms) * ((double)p.k_blocks + kFill);
-  for (int s = 2; s <= 32 && p.k_blocks / s >= 16; ++s) {
-    const double t = (double)(((int64_t)tiles * s + sms - 1) / sms) * ((double)p.k_blocks / s + kFill);
-    if (t < best * 0.995) {  // fewer splits on near-ties: fewer atomics and unit boundaries
-      best = t;
-      splits = s;
-    }
-  }
-  p.splits = splits;
+  p.splits = choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count());
   p.group_m = 8;
   p.status = status;
   p.w = static_cast<const bf16_t*>(w);
@@ -504,8 +517,8 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
 }
 
 cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
-                                  int d, float coef, float* dw, double* sqnorm, int* status,
-                                  cudaStream_t st) {
+                                  int d, float coef, float* dw, double* sqnorm, float* scratch,
+                                  int64_t scratch_elems, double* red, int* status, cudaStream_t st) {
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, x, true, d, N, d, BK))
     return cudaErrorInvalidValue;
@@ -516,13 +529,27 @@ cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x,
   p.num_m = D / BM;
   p.num_n = (d + BN - 1) / BN;
   p.k_blocks = (int)((N + BK - 1) / BK);
-  p.splits = 1;  // the stored tile and its squared norm need the whole sum over tokens
   p.group_m = 8;
   p.status = status;
   p.coef = coef;
-  p.dw = dw;
-  p.sqnorm = sqnorm;
-  return launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
+  // With a split K the partial tiles are added into a zeroed dw (the caller's, or the scratch when
+  // only the norm is wanted) and the squared norm is reduced from dw afterwards; without a place
+  // for dw the whole K range stays in one unit.
+  const int64_t n_w = (int64_t)D * d;
+  float* target = dw != nullptr ? dw : (scratch_elems >= n_w ? scratch : nullptr);
+  p.splits = target != nullptr && red != nullptr ? choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count()) : 1;
+  if (p.splits == 1) {
+    p.dw = dw;
+    p.sqnorm = sqnorm;
+    return launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
+  }
+  p.dw = target;
+  p.sqnorm = nullptr;
+  cudaError_t e = cudaMemsetAsync(target, 0, (size_t)n_w * sizeof(float), st);
+  if (e != cudaSuccess) return e;
+  e = launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
+  if (e != cudaSuccess || sqnorm == nullptr) return e;
+  return launch_sumsq(target, n_w, red, sqnorm, st);
 }
 
 }  // namespace jab

@@ -44,11 +44,14 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
 cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
                                 float coef, float* ds, int* status, cudaStream_t st);
-// coef * dQKV^T X stored fp32 [D, d] (dw may be NULL) and its squared norm added to *sqnorm (may be
-// NULL; the caller zeroes it)
+// coef * dQKV^T X stored fp32 [D, d] (dw may be NULL) and its squared norm in *sqnorm (may be NULL;
+// the caller zeroes it). With a split K the tile partials go through dw, or through scratch (fp32,
+// scratch_elems >= D d, may be NULL) when dw is NULL; red is fp64 [kRedBlocks] for the norm.
 cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
-                                  int d, float coef, float* dw, double* sqnorm, int* status,
-                                  cudaStream_t st);
+                                  int d, float coef, float* dw, double* sqnorm, float* scratch,
+                                  int64_t scratch_elems, double* red, int* status, cudaStream_t st);
+// split count of a K-split GEMM: whole waves of units on the persistent grid
+int choose_splits(int tiles, int k_blocks, int sms);
 // attn_tc.cu
 int attn_fwd_tc_rows(int Hq, int Hkv);  // query rows per loss partial of the forward kernel
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);
@@ -90,5 +93,7 @@ cudaError_t launch_omega_finish(const double* part, int nblocks, int C, const do
                                 double layers_after, double* c1, double* c2, cudaStream_t st);
 cudaError_t launch_mean(const double* x, int n, double* out, cudaStream_t st);
 cudaError_t launch_check_finite(const float* x, int64_t n, int* status, cudaStream_t st);
+// *out = sum of x[i]^2 in fp64, fixed order (part: fp64 [kRedBlocks])
+cudaError_t launch_sumsq(const float* x, int64_t n, double* part, double* out, cudaStream_t st);
 
 }  // namespace jab

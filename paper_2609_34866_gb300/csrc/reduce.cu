@@ -2,6 +2,7 @@
 // and L = SSE / (B T Hq d_h). Fixed summation order, so repeated calls give identical bits.
 #include "common.cuh"
 #include "kernels.h"
+#include "workspace.h"
 
 namespace jab {
 
@@ -64,6 +65,30 @@ __global__ void check_finite_kernel(const float* __restrict__ x, int64_t n, int*
   if (__syncthreads_or(bad) && threadIdx.x == 0) report(status, JAB_ERR_NONFINITE);
 }
 
+// Sum of squares in fp64: block b sums its contiguous chunk (fixed per-thread order, fixed tree),
+// then one thread adds the kRedBlocks partials in order.
+__global__ void __launch_bounds__(256) sumsq_partial_kernel(const float* __restrict__ x, int64_t n,
+                                                            double* __restrict__ part) {
+  __shared__ double red[8];
+  const int64_t chunk = (n + gridDim.x - 1) / gridDim.x;
+  const int64_t lo = blockIdx.x * chunk, hi = lo + chunk < n ? lo + chunk : n;
+  double acc = 0.0;
+  for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    const double v = x[i];
+    acc += v * v;
+  }
+  const double t = block_sum<256>(acc, red);
+  if (threadIdx.x == 0) part[blockIdx.x] = t;
+}
+
+__global__ void sum_in_order_kernel(const double* __restrict__ part, int n, double* __restrict__ out) {
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int i = 0; i < n; ++i) t += part[i];
+    *out = t;
+  }
+}
+
 cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
                                double* out, double* parts_out, int* status, cudaStream_t st) {
   loss_reduce_kernel<<<C, 256, 0, st>>>(part, B, Hq, nP, inv_n, out, parts_out, status);
@@ -84,6 +109,14 @@ cudaError_t launch_omega_finish(const double* part, int nblocks, int C, const do
 
 cudaError_t launch_mean(const double* x, int n, double* out, cudaStream_t st) {
   mean_kernel<<<1, 32, 0, st>>>(x, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sumsq(const float* x, int64_t n, double* part, double* out, cudaStream_t st) {
+  sumsq_partial_kernel<<<kRedBlocks, 256, 0, st>>>(x, n, part);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  sum_in_order_kernel<<<1, 32, 0, st>>>(part, kRedBlocks, out);
   return cudaGetLastError();
 }
 

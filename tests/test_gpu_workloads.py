@@ -196,3 +196,43 @@ def test_backward_full_size(name, k):
         comb = (f1 * g1 + f2 * g2).cpu().numpy()
         assert cosine(g_full.cpu().numpy(), comb) >= 0.99999
     assert J().jab_get_device_status() == 0
+
+
+def test_weight_gradient_split_k_full_shape():
+    """The STE weight gradient (App. B) on the Mistral-7B-shaped block at 8 and 4 sequences, where
+    the weight-gradient GEMM splits the token range (2-3 parts, partial tiles added with atomics):
+    the gradient is additive over sequences (halves recombined by their size), and the norm-only
+    call (through the workspace scratch) matches the stored gradient's norm."""
+    wl, desc, X, W = _setup("mistral_block")
+    B = 8
+    X = X[:B].contiguous()
+    bits = wl.bits[0]
+    s = _scales(desc, wl, W, bits)
+
+    def grad(Xb, nb):
+        ws = J().Workspace(desc, nb, wl.seq_len, 1, True)
+        A = torch.empty((nb, wl.seq_len, wl.shape.n_q_heads * wl.shape.head_dim),
+                        dtype=torch.float32, device="cuda")
+        J().jab_reference_forward(desc, nb, wl.seq_len, Xb, W, A, ws)
+        loss = torch.empty(1, dtype=torch.float64, device="cuda")
+        gw = torch.empty(W.shape, dtype=torch.float32, device="cuda")
+        sq = torch.empty(1, dtype=torch.float64, device="cuda")
+        J().jab_loss_backward_weights(desc, nb, wl.seq_len, Xb, W, A, bits, s, loss, grad_w=gw,
+                                      grad_sqnorm=sq, ws=ws)
+        sq2 = torch.empty(1, dtype=torch.float64, device="cuda")
+        J().jab_loss_backward_weights(desc, nb, wl.seq_len, Xb, W, A, bits, s, loss, grad_sqnorm=sq2,
+                                      ws=ws)
+        g = gw.double()
+        np.testing.assert_allclose(sq.item(), (g * g).sum().item(), rtol=1e-5)
+        np.testing.assert_allclose(sq2.item(), sq.item(), rtol=1e-5)
+        return g
+
+    g_full = grad(X, B)
+    h = B // 2
+    g1 = grad(X[:h].contiguous(), h)
+    g2 = grad(X[h:].contiguous(), B - h)
+    comb = 0.5 * (g1 + g2)
+    cos = (g_full * comb).sum() / (g_full.norm() * comb.norm())
+    assert cos.item() >= 0.99999, cos.item()
+    np.testing.assert_allclose(g_full.norm().item(), comb.norm().item(), rtol=1e-4)
+    assert J().jab_get_device_status() == 0
