@@ -3,10 +3,12 @@
 //   C[m, n] = sum_k A[m, k] B[n, k]        A K-major 16-bit, fp32 accumulation in TMEM; B K-major
 //                                          (stored [n][k]) or MN-major (stored [k][n])
 //
-// Persistent, warp-specialised kernel, one CTA per SM:
-//   warp 0      TMA producer: 128x64 A tile and 256x64 B tile per stage, 4-stage mbarrier ring
-//   warp 1      TMEM owner and UMMA issuer (one thread): 4 x tcgen05.mma M128 N256 K16 per stage
-//   warps 2..5  epilogue: tcgen05.ld of the 128 x 256 fp32 accumulator, one TMEM lane per thread
+// Persistent, warp-specialised kernel on CTA pairs (clusters of two CTAs on two SMs, cta_group::2):
+// a pair computes a 256 x 256 tile with M256 N256 K16 UMMAs issued by its even CTA; each CTA holds
+// 128 rows of A, half of the B tile and 128 lanes of the accumulator (details above the kernel).
+//   warp 0      TMA producer: the CTA's 128x64 A tile and 128x64 half of B per stage, 6-stage ring
+//   warp 1      TMEM owner (512 columns, allocated by the pair) and, in the even CTA, UMMA issuer
+//   warps 2..5  epilogue: tcgen05.ld of the CTA's 128 x 256 fp32 accumulator, one lane per thread
 // Two accumulators (2 x 256 TMEM columns) let the epilogue of one tile overlap the next mainloop.
 //
 // Epilogues:
@@ -14,8 +16,8 @@
 //               lives in the same thread's row), fp16 store.
 //   wgrad       G = dQKV^T X (K = tokens, split-K): ds[o, g] += coef * sum_{i in g} G[o,i] r[o,i]
 //               with the LSQ factor r of Eq. 13 recomputed from w and s; G is never stored. X is
-//               read as it is stored, [tokens, features], as the MN-major B operand (four 64-feature
-//               TMA boxes per stage), so no transposed copy of X is needed.
+//               read as it is stored, [tokens, features], as the MN-major B operand (two 64-feature
+//               TMA boxes per CTA and stage), so no transposed copy of X is needed.
 //   store       coef * dQKV^T X as fp32 dW (STE weight gradient) and / or its squared norm; with a
 //               split K the partial tiles are added into a zeroed dW with vector atomics and the
 //               norm is reduced from dW afterwards in fixed order.
@@ -27,13 +29,10 @@
 namespace jab {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BM = 128, BN = 256, BK = 64;  // BM: rows of one CTA (an epilogue's 128 TMEM lanes)
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int NUM_THREADS = 192;
 constexpr uint32_t TMEM_COLS = 2 * BN;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
 
 enum EpiKind { kEpiRope = 0, kEpiLsq = 1, kEpiStore = 2 };
 
@@ -56,12 +55,6 @@ struct GemmParams {
   // weight-gradient store epilogue (a split K adds partial tiles into a zeroed dw)
   float* dw;
   double* sqnorm;
-};
-
-struct Bars {
-  uint64_t full[STAGES], empty[STAGES], tfull[2], tempty[2], drain;
-  uint32_t tmem_base;
-  int abort;
 };
 
 __device__ __forceinline__ void decode_unit(const GemmParams& p, int unit, int& mb, int& nb,
@@ -248,26 +241,58 @@ __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int
   if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
 }
 
+// ------------------------------------------------------------------ CTA-pair variant (cta_group::2)
+// Two CTAs of a cluster on two SMs share one 256 x 256 tile: CTA r holds rows 128 r .. 128 r + 127
+// of A and rows 128 r .. of the B tile (the N half it loads), and its 128 accumulator lanes. One
+// M256 N256 K16 UMMA per 16-deep K step, issued by the even CTA, reads A and B from both CTAs' shared
+// memory. Each SM then stages 16 KB of A and 16 KB of B per K block instead of the 16 + 32 KB of a
+// one-CTA 128 x 256 tile, so six stages fit where four did and the operand loads have 1.7x the
+// look-ahead (the one-CTA layout was bound by it: three stages instead of four cost it 10-26 %).
+//   warp 0      TMA producer (both CTAs): its rows of A and its half of B, completion counted on the
+//               even CTA's stage barrier, which expects both CTAs' bytes
+//   warp 1      TMEM owner (both CTAs, allocated collectively); UMMA issuer (even CTA, one thread);
+//               each stage's commit releases the stage in both CTAs, each tile's commit wakes both
+//               CTAs' epilogues
+//   warps 2..5  epilogue (both CTAs): this CTA's 128 rows, as in the single-CTA kernel; the
+//               accumulator is free again once all eight epilogue warps of the pair have arrived on
+//               the even CTA's barrier
+constexpr int STAGES2 = 6;
+constexpr int BM2 = 2 * BM;                 // rows of A per pair tile
+constexpr int B2_ROWS = BN / 2;             // rows (K-major) or columns (MN-major) of B per CTA
+constexpr int B2_BYTES = B2_ROWS * BK * 2;  // 16 KB
+constexpr int STAGE2_BYTES = A_BYTES + B2_BYTES;
+constexpr int SMEM2_BYTES = STAGES2 * STAGE2_BYTES + 1024 + 256;
+
+struct Bars2 {
+  uint64_t full[STAGES2], empty[STAGES2], tfull[2], tempty[2], drain;
+  uint32_t tmem_base;
+  int abort;
+};
+static_assert(STAGES2 * STAGE2_BYTES + (int)sizeof(Bars2) <= SMEM2_BYTES - 1024, "shared memory");
+
 template <int EPI, bool BF16, bool B_MN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmParams p) {
+    gemm2_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  Bars* bars = reinterpret_cast<Bars*>(smem + STAGES * STAGE_BYTES);
+  Bars2* bars = reinterpret_cast<Bars2*>(smem + STAGES2 * STAGE2_BYTES);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int total = p.num_m * p.num_n * p.splits;
+  const uint32_t rank = tc::cluster_ctarank();  // 0: issues the pair's UMMAs
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const int total = p.num_m * p.num_n * p.splits;  // num_m counts 256-row blocks here
   volatile int* abort = &bars->abort;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < STAGES2; ++s) {
       tc::mbar_init(&bars->full[s], 1);
       tc::mbar_init(&bars->empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(&bars->tfull[a], 1);
-      tc::mbar_init(&bars->tempty[a], 4);
+      tc::mbar_init(&bars->tempty[a], 2 * 4);  // the epilogue warps of both CTAs
     }
     tc::mbar_init(&bars->drain, 1);
     bars->abort = 0;
@@ -276,58 +301,63 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc::prefetch_tmap(&tmB);
   }
   if (warp == 1) {
-    tc::tmem_alloc(&bars->tmem_base, TMEM_COLS);
-    tc::tmem_relinquish();
+    tc::tmem_alloc2(&bars->tmem_base, TMEM_COLS);
+    tc::tmem_relinquish2();
   }
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
+  // both CTAs' barriers are initialised and their tensor memory allocated before any signal crosses
+  tc::cluster_sync();
   const uint32_t tmem = bars->tmem_base;
+  const uint32_t full_lead = tc::mapa_shared(tc::smem_u32(&bars->full[0]), 0);
+  const uint32_t tempty_lead = tc::mapa_shared(tc::smem_u32(&bars->tempty[0]), 0);
 
   if (warp == 0) {
     if (lane == 0) {  // ---------------- TMA producer
       int stage = 0;
       uint32_t phase = 0;
-      uint32_t issued = 0, last_parity = 0;  // per-stage bitmasks for the exit drain
-      for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x) {
+      uint32_t issued = 0, last_parity = 0;  // per-stage bitmasks for the exit drain (even CTA)
+      for (int unit = pair; unit < total && !*abort; unit += npairs) {
         int mb, nb, ks, kb0, kb1;
         decode_unit(p, unit, mb, nb, ks);
         k_range(p, ks, kb0, kb1);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!tc::mbar_wait(&bars->empty[stage], phase ^ 1, abort, p.status)) break;
-          uint8_t* sa = smem + stage * STAGE_BYTES;
-          tc::mbar_expect_tx(&bars->full[stage], STAGE_BYTES);
-          tc::tma_load_2d(sa, &tmA, &bars->full[stage], kb * BK, mb * BM);
-          if (B_MN)  // B stored [k][n]: four boxes of BK rows x 64 columns
-            for (int c = 0; c < BN / 64; ++c)
-              tc::tma_load_2d(sa + A_BYTES + c * (BK * 128), &tmB, &bars->full[stage],
-                              nb * BN + c * 64, kb * BK);
+          uint8_t* sa = smem + stage * STAGE2_BYTES;
+          const uint32_t bar = full_lead + stage * 8;
+          if (leader) tc::mbar_expect_tx(&bars->full[stage], 2 * STAGE2_BYTES);
+          tc::tma_load_2d_pair(sa, &tmA, bar, kb * BK, mb * BM2 + (int)rank * BM);
+          if (B_MN)  // B stored [k][n]: this CTA's two boxes of BK rows x 64 columns
+            for (int c = 0; c < B2_ROWS / 64; ++c)
+              tc::tma_load_2d_pair(sa + A_BYTES + c * (BK * 128), &tmB, bar,
+                                   nb * BN + (int)rank * B2_ROWS + c * 64, kb * BK);
           else
-            tc::tma_load_2d(sa + A_BYTES, &tmB, &bars->full[stage], kb * BK, nb * BN);
+            tc::tma_load_2d_pair(sa + A_BYTES, &tmB, bar, kb * BK, nb * BN + (int)rank * B2_ROWS);
           issued |= 1u << stage;
           last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) {
+          if (++stage == STAGES2) {
             stage = 0;
             phase ^= 1;
           }
         }
       }
-      if (*abort)  // let every issued copy land before the CTA's shared memory is released
-        for (int s = 0; s < STAGES; ++s)
+      if (*abort && leader)  // let every issued copy of the pair land before shared memory goes
+        for (int s = 0; s < STAGES2; ++s)
           if (issued & (1u << s)) drain_wait(&bars->full[s], (last_parity >> s) & 1);
     }
   } else if (warp == 1) {
-    if (lane == 0) {  // ---------------- UMMA issuer
-      constexpr uint32_t IDESC = tc::idesc_f16(BF16, BM, BN) | (B_MN ? (1u << 16) : 0u);
+    if (lane == 0 && leader) {  // ---------------- UMMA issuer of the pair
+      constexpr uint32_t IDESC = tc::idesc_f16(BF16, BM2, BN) | (B_MN ? (1u << 16) : 0u);
       int stage = 0, it = 0;
       uint32_t phase = 0;
-      for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x, ++it) {
+      for (int unit = pair; unit < total && !*abort; unit += npairs, ++it) {
         int mb, nb, ks, kb0, kb1;
         decode_unit(p, unit, mb, nb, ks);
         k_range(p, ks, kb0, kb1);
         const int acc = it & 1;
         const uint32_t aphase = (it >> 1) & 1;
-        if (!tc::mbar_wait(&bars->tempty[acc], aphase ^ 1, abort, p.status)) break;
+        if (!tc::mbar_wait_cluster(&bars->tempty[acc], aphase ^ 1, abort, p.status)) break;
         tc::fence_after_sync();
         const uint32_t d_tmem = tmem + acc * BN;
         bool ok = true;
@@ -337,31 +367,31 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           tc::fence_after_sync();
-          const uint32_t a0 = tc::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t a0 = tc::smem_u32(smem + stage * STAGE2_BYTES);
           const uint32_t b0 = a0 + A_BYTES;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            tc::umma_f16(d_tmem, tc::sdesc_kmajor_sw128(a0 + k * 32),
-                         B_MN ? tc::sdesc_mnmajor_sw128(b0 + k * 16 * 128, BK * 128, 1024)
-                              : tc::sdesc_kmajor_sw128(b0 + k * 32),
-                         IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
-          tc::umma_commit(&bars->empty[stage]);
-          if (++stage == STAGES) {
+            tc::umma2_f16(d_tmem, tc::sdesc_kmajor_sw128(a0 + k * 32),
+                          B_MN ? tc::sdesc_mnmajor_sw128(b0 + k * 16 * 128, BK * 128, 1024)
+                               : tc::sdesc_kmajor_sw128(b0 + k * 32),
+                          IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+          tc::umma2_commit_mc(&bars->empty[stage], 0x3);
+          if (++stage == STAGES2) {
             stage = 0;
             phase ^= 1;
           }
         }
         if (!ok) break;
-        tc::umma_commit(&bars->tfull[acc]);
+        tc::umma2_commit_mc(&bars->tfull[acc], 0x3);
       }
-      tc::umma_commit(&bars->drain);  // every MMA of this CTA has completed once this flips
+      tc::umma2_commit_mc(&bars->drain, 0x1);  // every UMMA of the pair has completed once this flips
       drain_wait(&bars->drain, 0);
     }
-  } else {  // ---------------- epilogue warps 2..5
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+  } else {  // ---------------- epilogue warps 2..5 (both CTAs)
+    const int q = warp & 3;
     const int row = q * 32 + lane;
     int it = 0;
-    for (int unit = blockIdx.x; unit < total && !*abort; unit += gridDim.x, ++it) {
+    for (int unit = pair; unit < total && !*abort; unit += npairs, ++it) {
       int mb, nb, ks;
       decode_unit(p, unit, mb, nb, ks);
       const int acc = it & 1;
@@ -369,23 +399,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!tc::mbar_wait(&bars->tfull[acc], aphase, abort, p.status)) break;
       tc::fence_after_sync();
       const uint32_t taddr = tmem + ((uint32_t)(q * 32) << 16) + acc * BN;
+      const int mb128 = 2 * mb + (int)rank;  // this CTA's 128-row block
       if (EPI == kEpiRope)
-        epi_rope(p, taddr, mb, nb, row);
-      else if (EPI == kEpiLsq)
-        epi_lsq(p, taddr, mb, nb, row);
-      else
-        epi_store(p, taddr, mb, nb, row);
+        epi_rope(p, taddr, mb128, nb, row);  // masks rows past M itself
+      else if ((int64_t)mb128 * BM < p.M) {  // M is a multiple of 128: whole halves are valid or not
+        if (EPI == kEpiLsq)
+          epi_lsq(p, taddr, mb128, nb, row);
+        else
+          epi_store(p, taddr, mb128, nb, row);
+      }
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&bars->tempty[acc]);
+      if (lane == 0) {
+        if (leader)
+          tc::mbar_arrive(&bars->tempty[acc]);
+        else
+          tc::mbar_arrive_cluster(tempty_lead + acc * 8);
+      }
     }
   }
   tc::fence_before_sync();
   __syncthreads();
+  // the pair's UMMAs have completed (the issuer drained) and no arrival is in flight to the other
+  // CTA before either frees its tensor memory or exits
+  tc::cluster_sync();
   tc::fence_after_sync();
   if (warp == 1) {
     __syncwarp();
-    tc::tmem_dealloc(tmem, TMEM_COLS);
+    tc::tmem_dealloc2(tmem, TMEM_COLS);
   }
 }
 
@@ -427,20 +468,38 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
+// CTA-pair launch: clusters of two, one pair per two SMs (as many pairs as fit at once).
 template <int EPI, bool BF16, bool B_MN>
-cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmParams& p,
-                        cudaStream_t st) {
+cudaError_t launch_gemm2(const CUtensorMap& ta, const CUtensorMap& tb, GemmParams& p,
+                         cudaStream_t st) {
+  auto kern = gemm2_tc_kernel<EPI, BF16, B_MN>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI, BF16, B_MN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int total = p.num_m * p.num_n * p.splits;
-  const int grid = std::min(total, sm_count());
-  gemm_tc_kernel<EPI, BF16, B_MN><<<grid, NUM_THREADS, SMEM_BYTES, st>>>(ta, tb, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = SMEM2_BYTES;
+  cfg.stream = st;
+  const int sms = sm_count();
+  cfg.gridDim = dim3((unsigned)(sms / 2 * 2));
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess || clusters < 1)
+    clusters = sms / 2;
+  const int64_t total = (int64_t)p.num_m * p.num_n * p.splits;
+  const int pairs = (int)std::min<int64_t>(total, std::min(clusters, sms / 2));
+  cfg.gridDim = dim3((unsigned)(2 * pairs));
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
 }
 
 }  // namespace
@@ -449,13 +508,13 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
                                 int D, int n_rot, int dh, int T, const float* cos_t,
                                 const float* sin_t, int* status, cudaStream_t st) {
   CUtensorMap ta, tb;
-  if (!make_tmap(&ta, A, false, K, M, K, BM) || !make_tmap(&tb, Bw, false, K, Nn, K, BN))
+  if (!make_tmap(&ta, A, false, K, M, K, BM) || !make_tmap(&tb, Bw, false, K, Nn, K, B2_ROWS))
     return cudaErrorInvalidValue;
   GemmParams p{};
   p.M = M;
   p.Nn = Nn;
   p.K = K;
-  p.num_m = (int)((M + BM - 1) / BM);
+  p.num_m = (int)((M + BM2 - 1) / BM2);  // 256-row blocks: CTA pairs
   p.num_n = (Nn + BN - 1) / BN;
   p.splits = 1;
   p.k_blocks = K / BK;
@@ -468,7 +527,7 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
   p.T = T;
   p.cos_t = cos_t;
   p.sin_t = sin_t;
-  return launch_gemm<kEpiRope, false, false>(ta, tb, p, st);
+  return launch_gemm2<kEpiRope, false, false>(ta, tb, p, st);
 }
 
 // Split K so that the units (tile x K range) fill whole waves of the persistent grid: the makespan
@@ -500,10 +559,10 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.M = D;
   p.Nn = d;
   p.K = (int)std::min<int64_t>(N, INT32_MAX);
-  p.num_m = D / BM;
+  p.num_m = (D + BM2 - 1) / BM2;  // 256-row blocks: CTA pairs
   p.num_n = (d + BN - 1) / BN;
   p.k_blocks = (int)((N + BK - 1) / BK);
-  p.splits = choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count());
+  p.splits = choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count() / 2);
   p.group_m = 8;
   p.status = status;
   p.w = static_cast<const bf16_t*>(w);
@@ -513,7 +572,7 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.bits = bits;
   p.coef = coef;
   p.ds = ds;
-  return launch_gemm<kEpiLsq, true, true>(ta, tb, p, st);
+  return launch_gemm2<kEpiLsq, true, true>(ta, tb, p, st);
 }
 
 cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
@@ -526,7 +585,7 @@ cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x,
   p.M = D;
   p.Nn = d;
   p.K = (int)std::min<int64_t>(N, INT32_MAX);
-  p.num_m = D / BM;
+  p.num_m = (D + BM2 - 1) / BM2;  // 256-row blocks: CTA pairs
   p.num_n = (d + BN - 1) / BN;
   p.k_blocks = (int)((N + BK - 1) / BK);
   p.group_m = 8;
@@ -537,17 +596,17 @@ cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x,
   // for dw the whole K range stays in one unit.
   const int64_t n_w = (int64_t)D * d;
   float* target = dw != nullptr ? dw : (scratch_elems >= n_w ? scratch : nullptr);
-  p.splits = target != nullptr && red != nullptr ? choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count()) : 1;
+  p.splits = target != nullptr && red != nullptr ? choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count() / 2) : 1;
   if (p.splits == 1) {
     p.dw = dw;
     p.sqnorm = sqnorm;
-    return launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
+    return launch_gemm2<kEpiStore, true, true>(ta, tb, p, st);
   }
   p.dw = target;
   p.sqnorm = nullptr;
   cudaError_t e = cudaMemsetAsync(target, 0, (size_t)n_w * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  e = launch_gemm<kEpiStore, true, true>(ta, tb, p, st);
+  e = launch_gemm2<kEpiStore, true, true>(ta, tb, p, st);
   if (e != cudaSuccess || sqnorm == nullptr) return e;
   return launch_sumsq(target, n_w, red, sqnorm, st);
 }
