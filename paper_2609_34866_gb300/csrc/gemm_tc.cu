@@ -518,7 +518,7 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
   p.num_n = (Nn + BN - 1) / BN;
   p.splits = 1;
   p.k_blocks = K / BK;
-  p.group_m = 32;
+  p.group_m = 16;  // 16 pair rows = 4096 rows of X and all of W in L2 while the N tiles pass
   p.status = status;
   p.C = static_cast<half_t*>(C);
   p.D = D;
