@@ -173,7 +173,9 @@ jab_status jab_omega_scores(const jab_block_desc* desc, const void* W_dev, int32
  * v = w / s.
  *   grad_scales_dev out fp32 [(Hq+2Hkv)*d_h, d_model/G] = kappa * sum_{i in group} dL/dw_hat[o,i] * r[o,i]
  *   kappa          <= 0 selects the LSQ factor (G * qmax)^(-1/2); 1 gives the raw rule
- *   loss_dev       out fp64 [1] */
+ *   loss_dev       out fp64 [1]
+ * The gradient's sums (over tokens in the GEMM, then over the GEMM's K splits) run in a fixed order:
+ * repeated calls with identical inputs return identical bits. */
 jab_status jab_loss_backward_scales(const jab_block_desc* desc, int32_t B, int32_t T,
                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
                                     int32_t bits, const float* scales_dev, float kappa,
@@ -203,8 +205,11 @@ jab_status jab_loss_backward_scales_prepared(const jab_block_desc* desc, int32_t
  * of App. B "Fisher-coupling" when called with bits = 2 and round-to-nearest scales
  * (jab_init_scales mode 0).
  *   grad_w_dev      out fp32 [(Hq+2Hkv)*d_h, d_model] or NULL   dL/dw_hat = (2/n) dQKV^T X, n = B*T*Hq*d_h
- *   grad_sqnorm_dev out fp64 [1] or NULL                        ||dL/dw_hat||_F^2 (fp64 atomics: the
- *                                                               last bits may differ between calls)
+ *   grad_sqnorm_dev out fp64 [1] or NULL                        ||dL/dw_hat||_F^2, reduced from the
+ *                                                               stored gradient in a fixed order
+ * The weight-gradient GEMM may split the token range and add the partial tiles with atomics, so the
+ * last bits of grad_w (and of its norm) may differ between calls; in the deterministic-reduction
+ * mode (jab_set_deterministic) each tile is one unit and repeated calls are bit-identical.
  *   loss_dev        out fp64 [1]
  * At least one of grad_w_dev and grad_sqnorm_dev must be non-NULL. Uses the with_bwd workspace of
  * jab_workspace_size. */
@@ -286,6 +291,15 @@ jab_status jab_loss_forward_noalloc(const jab_block_desc* desc, int32_t B, int32
  * 2-second limit the kernel sets JAB_ERR_TIMEOUT in the device status and returns; the context
  * stays usable. Read the result with jab_get_device_status. */
 jab_status jab_selftest_wait_timeout(jab_stream_t stream);
+
+/* Deterministic-reduction mode (the boundary's "bit-identical results" convention), process-wide,
+ * read when a call is issued: on = 1 makes every floating-point reduction of the library run in a
+ * fixed order, so that two calls with identical inputs return bit-identical results; on = 0 (the
+ * default) lets the weight-gradient GEMM of jab_loss_backward_weights split the token range and add
+ * its partial tiles with atomics (faster on large batches; the last bits of grad_w may then differ).
+ * Every other result (losses, scale gradients, KL, Hutchinson and Omega sums, norms) is reduced in a
+ * fixed order in both modes. Returns JAB_ERR_INVALID_ARG for other values of on. Host only. */
+jab_status jab_set_deterministic(int32_t on);
 
 /* Synchronises `stream`, then returns and clears the device-side status of the current device
  * (JAB_OK if no kernel reported a problem since the last call). */

@@ -91,6 +91,7 @@ def lib() -> ctypes.CDLL:
     L.jab_allocate_bits.argtypes = [_P, _P, _P, i32, i32, ctypes.c_double, i32, _P]
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
     L.jab_get_device_status.argtypes = [_P]
+    L.jab_set_deterministic.argtypes = [i32]
     L.jab_selftest_wait_timeout.argtypes = [_P]
     L.jab_status_string.argtypes = [i32]
     L.jab_status_string.restype = ctypes.c_char_p
@@ -107,7 +108,7 @@ def lib() -> ctypes.CDLL:
                "jab_reference_projection", "jab_loss_forward_kl", "jab_hutchinson_trace",
                "jab_omega_scores", "jab_rademacher_probes",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
-               "jab_selftest_wait_timeout",
+               "jab_selftest_wait_timeout", "jab_set_deterministic",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
         getattr(L, fn).restype = i32
     _LIB = L
@@ -352,6 +353,13 @@ def jab_init_scales(desc, bits, mode, W, scales, stream=None):
 def jab_selftest_wait_timeout(stream=None):
     """Launches the bounded-wait self-test kernel (its wait runs out after 2 s)."""
     _check(lib().jab_selftest_wait_timeout(_stream(stream)), "jab_selftest_wait_timeout")
+
+
+def jab_set_deterministic(on: bool):
+    """Deterministic-reduction mode, process-wide: every floating-point reduction in a fixed order
+    (repeated calls bit-identical). Off by default: the STE weight gradient may then split its GEMM's
+    token range and add the partial tiles with atomics."""
+    _check(lib().jab_set_deterministic(int(on)), "jab_set_deterministic")
 
 
 def jab_get_device_status(stream=None) -> int:

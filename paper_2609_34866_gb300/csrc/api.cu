@@ -17,6 +17,9 @@
 
 namespace jab {
 
+// Deterministic-reduction mode (jab_set_deterministic): process-wide, read when a call is issued.
+int g_deterministic = 0;
+
 __device__ int g_status;  // one per device context: first device-side problem since the last read
 
 namespace {
@@ -536,9 +539,10 @@ static jab_status backward_scales(const jab_block_desc* desc, int32_t B, int32_t
   const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
   const double k = kappa > 0.f ? (double)kappa : 1.0 / sqrt((double)G * qmax_of(bits));
   const float coef = (float)(k * 2.0 / n_el);
-  JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_scales_dev, 0, (size_t)D * (dm / G) * sizeof(float), st));
+  // per-split partials summed in order: the scale gradient is bit-identical between calls
   JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, wp.ldt, X_dev, W_dev, scales_dev, N, D,
-                                               dm, G, bits, coef, grad_scales_dev, status, st));
+                                               dm, G, bits, coef, grad_scales_dev,
+                                               reinterpret_cast<float*>(w + wp.gpart), status, st));
   JAB_SITE("check_finite", 1, launch_check_finite(grad_scales_dev, (int64_t)D * (dm / G), status, st));
   return JAB_OK;
 }
@@ -614,13 +618,11 @@ jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int3
   const int64_t N = (int64_t)B * T;
   const int D = (int)block_rows(desc), dm = desc->d_model;
   const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
-  if (grad_sqnorm_dev) JAB_SITE("memset_grad", 0, cudaMemsetAsync(grad_sqnorm_dev, 0, sizeof(double), st));
-  // the projection output is dead once the attention backward has run: scratch for a split K
   JAB_SITE("wgrad_store", 1, launch_wgrad_store_tc(w + wp.dqkvt, wp.ldt, X_dev, N, D, dm,
                                                    (float)(2.0 / n_el), grad_w_dev, grad_sqnorm_dev,
-                                                   reinterpret_cast<float*>(w + wp.qkv),
-                                                   (int64_t)(N * D * 2 / 4),
-                                                   reinterpret_cast<double*>(w + wp.red), status, st));
+                                                   reinterpret_cast<float*>(w + wp.dwscr),
+                                                   reinterpret_cast<double*>(w + wp.red),
+                                                   g_deterministic != 0, status, st));
   if (grad_w_dev)
     JAB_SITE("check_finite", 1, launch_check_finite(grad_w_dev, (int64_t)D * dm, status, st));
   return JAB_OK;
@@ -653,6 +655,12 @@ jab_status jab_init_scales(const jab_block_desc* desc, int32_t bits, int32_t mod
     return JAB_ERR_INVALID_ARG;
   JAB_TRY(launch_init_scales(W_dev, (int)block_rows(desc), desc->d_model, desc->group_size, bits,
                              mode, scales_dev, reinterpret_cast<cudaStream_t>(stream)));
+  return JAB_OK;
+}
+
+jab_status jab_set_deterministic(int32_t on) {
+  if (on != 0 && on != 1) return JAB_ERR_INVALID_ARG;
+  jab::g_deterministic = on;
   return JAB_OK;
 }
 

@@ -52,9 +52,9 @@ struct GemmParams {
   int d, G, bits;
   float coef;
   float* ds;
+  float* dspart;  // fp32 [splits, M, d/G]: each unit's partial, summed over the splits in order
   // weight-gradient store epilogue (a split K adds partial tiles into a zeroed dw)
   float* dw;
-  double* sqnorm;
 };
 
 __device__ __forceinline__ void decode_unit(const GemmParams& p, int unit, int& mb, int& nb,
@@ -160,15 +160,12 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
 }
 
 // STE weight gradient (App. B: d w_hat / d w = 1, so dL/dW = dL/dw_hat = coef * dQKV^T X): the
-// tile times coef stored as fp32 rows of dw (when set; with a split K each unit's partial tile is
-// added with vector atomics) and, without a split, its squared Frobenius norm added to *sqnorm
-// (when set; fp64 atomics, one per warp and tile). Packed FP32 pairs, as this runs beside the next
-// tile's UMMAs.
+// tile times coef stored as fp32 rows of dw (with a split K each unit's partial tile is added with
+// vector atomics). Packed FP32 pairs, as this runs beside the next tile's UMMAs.
 __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, int mb, int nb,
                                           int row) {
   const int64_t o = (int64_t)mb * BM + row;  // M = D is a multiple of 128: every row is valid
   const float2 c2 = make_float2(p.coef, p.coef);
-  float2 sq = make_float2(0.f, 0.f);
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
     const int i0 = nb * BN + c * 32;
@@ -183,7 +180,6 @@ __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, i
       const float2 v = tc::mul2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), c2);
       g[i] = v.x;
       g[i + 1] = v.y;
-      sq = tc::fma2(v, v, sq);
     }
     if (p.dw != nullptr) {
       float4* d = reinterpret_cast<float4*>(p.dw + o * p.Nn + i0);
@@ -197,17 +193,15 @@ __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, i
       }
     }
   }
-  if (p.sqnorm != nullptr && p.splits == 1) {  // with a split K the caller reduces dw afterwards
-    const double t = warp_sum((double)sq.x + (double)sq.y);
-    if ((threadIdx.x & 31) == 0) atomicAdd(p.sqnorm, t);
-  }
 }
 
 __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int mb, int nb,
-                                        int row) {
+                                        int ks, int row) {
   const int o = mb * BM + row;  // M = D is a multiple of 128: every row is valid
   const int qmax = qmax_of(p.bits);
   const int ng = p.d / p.G;
+  // one value per (split, row, group): this unit's tile covers whole groups (BN is a multiple of G)
+  float* part_out = p.dspart + ((int64_t)ks * p.M + o) * ng;
   float part = 0.f;
   int cur = -1;
 #pragma unroll 1
@@ -232,13 +226,13 @@ __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int
                    acc);
     }
     if (g != cur) {
-      if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
+      if (cur >= 0) part_out[cur] = p.coef * part;
       part = 0.f;
       cur = g;
     }
     part += acc;
   }
-  if (cur >= 0) atomicAdd(p.ds + (int64_t)o * ng + cur, p.coef * part);
+  if (cur >= 0) part_out[cur] = p.coef * part;
 }
 
 // ------------------------------------------------------------------ CTA-pair variant (cta_group::2)
@@ -404,7 +398,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         epi_rope(p, taddr, mb128, nb, row);  // masks rows past M itself
       else if ((int64_t)mb128 * BM < p.M) {  // M is a multiple of 128: whole halves are valid or not
         if (EPI == kEpiLsq)
-          epi_lsq(p, taddr, mb128, nb, row);
+          epi_lsq(p, taddr, mb128, nb, ks, row);
         else
           epi_store(p, taddr, mb128, nb, row);
       }
@@ -551,7 +545,7 @@ int choose_splits(int tiles, int k_blocks, int sms) {
 
 cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
-                                float coef, float* ds, int* status, cudaStream_t st) {
+                                float coef, float* ds, float* dspart, int* status, cudaStream_t st) {
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, x, true, d, N, d, BK))
     return cudaErrorInvalidValue;
@@ -572,12 +566,17 @@ cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, c
   p.bits = bits;
   p.coef = coef;
   p.ds = ds;
-  return launch_gemm2<kEpiLsq, true, true>(ta, tb, p, st);
+  p.dspart = dspart;
+  // every (split, row, group) partial is written once; the splits are summed in order: the scale
+  // gradient is bit-identical between calls
+  cudaError_t e = launch_gemm2<kEpiLsq, true, true>(ta, tb, p, st);
+  if (e != cudaSuccess) return e;
+  return launch_split_sum(dspart, p.splits, (int64_t)D * (d / G), ds, st);
 }
 
 cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
                                   int d, float coef, float* dw, double* sqnorm, float* scratch,
-                                  int64_t scratch_elems, double* red, int* status, cudaStream_t st) {
+                                  double* red, bool deterministic, int* status, cudaStream_t st) {
   CUtensorMap ta, tb;
   if (!make_tmap(&ta, dqkvt, true, N, D, ldt, BM) || !make_tmap(&tb, x, true, d, N, d, BK))
     return cudaErrorInvalidValue;
@@ -591,24 +590,21 @@ cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x,
   p.group_m = 8;
   p.status = status;
   p.coef = coef;
-  // With a split K the partial tiles are added into a zeroed dw (the caller's, or the scratch when
-  // only the norm is wanted) and the squared norm is reduced from dw afterwards; without a place
-  // for dw the whole K range stays in one unit.
+  // dW goes to the caller's buffer, or to the scratch when only the norm is asked for. A split K
+  // adds the partial tiles into a zeroed dW with atomics (the last bits depend on their order);
+  // the deterministic mode keeps one unit per tile.
   const int64_t n_w = (int64_t)D * d;
-  float* target = dw != nullptr ? dw : (scratch_elems >= n_w ? scratch : nullptr);
-  p.splits = target != nullptr && red != nullptr ? choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count() / 2) : 1;
-  if (p.splits == 1) {
-    p.dw = dw;
-    p.sqnorm = sqnorm;
-    return launch_gemm2<kEpiStore, true, true>(ta, tb, p, st);
-  }
+  float* target = dw != nullptr ? dw : scratch;
+  p.splits = deterministic ? 1 : choose_splits(p.num_m * p.num_n, p.k_blocks, sm_count() / 2);
   p.dw = target;
-  p.sqnorm = nullptr;
-  cudaError_t e = cudaMemsetAsync(target, 0, (size_t)n_w * sizeof(float), st);
-  if (e != cudaSuccess) return e;
+  cudaError_t e;
+  if (p.splits > 1) {
+    e = cudaMemsetAsync(target, 0, (size_t)n_w * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+  }
   e = launch_gemm2<kEpiStore, true, true>(ta, tb, p, st);
   if (e != cudaSuccess || sqnorm == nullptr) return e;
-  return launch_sumsq(target, n_w, red, sqnorm, st);
+  return launch_sumsq(target, n_w, red, sqnorm, st);  // fixed order
 }
 
 }  // namespace jab

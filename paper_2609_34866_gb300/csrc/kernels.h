@@ -41,15 +41,16 @@ cudaError_t launch_proj_gemm_tc(const void* A, const void* Bw, void* C, int64_t 
                                 int D, int n_rot, int dh, int T, const float* cos_t,
                                 const float* sin_t, int* status, cudaStream_t st);
 // x: bf16 [N, d] as the caller stores it (no transposed copy)
+// ds: the scale gradient, written (fp32 [D, d/G]); dspart: fp32 [kMaxSplits, D, d/G] scratch
 cudaError_t launch_wgrad_lsq_tc(const void* dqkvt, int64_t ldt, const void* x, const void* w,
                                 const float* s, int64_t N, int D, int d, int G, int bits,
-                                float coef, float* ds, int* status, cudaStream_t st);
-// coef * dQKV^T X stored fp32 [D, d] (dw may be NULL) and its squared norm in *sqnorm (may be NULL;
-// the caller zeroes it). With a split K the tile partials go through dw, or through scratch (fp32,
-// scratch_elems >= D d, may be NULL) when dw is NULL; red is fp64 [kRedBlocks] for the norm.
+                                float coef, float* ds, float* dspart, int* status, cudaStream_t st);
+// coef * dQKV^T X stored fp32 [D, d] in dw, or in scratch (fp32 [D, d]) when dw is NULL, and its
+// squared norm in *sqnorm (may be NULL) by a fixed-order reduction (red: fp64 [kRedBlocks]). A split
+// K adds partial tiles with atomics; deterministic keeps one unit per tile (bit-identical dW).
 cudaError_t launch_wgrad_store_tc(const void* dqkvt, int64_t ldt, const void* x, int64_t N, int D,
                                   int d, float coef, float* dw, double* sqnorm, float* scratch,
-                                  int64_t scratch_elems, double* red, int* status, cudaStream_t st);
+                                  double* red, bool deterministic, int* status, cudaStream_t st);
 // split count of a K-split GEMM: whole waves of units on the persistent grid
 int choose_splits(int tiles, int k_blocks, int sms);
 // attn_tc.cu
@@ -95,5 +96,7 @@ cudaError_t launch_mean(const double* x, int n, double* out, cudaStream_t st);
 cudaError_t launch_check_finite(const float* x, int64_t n, int* status, cudaStream_t st);
 // *out = sum of x[i]^2 in fp64, fixed order (part: fp64 [kRedBlocks])
 cudaError_t launch_sumsq(const float* x, int64_t n, double* part, double* out, cudaStream_t st);
+// out[i] = sum over s < splits of part[s n + i], in order of s (fp64 sum, fp32 result)
+cudaError_t launch_split_sum(const float* part, int splits, int64_t n, float* out, cudaStream_t st);
 
 }  // namespace jab

@@ -89,6 +89,17 @@ __global__ void sum_in_order_kernel(const double* __restrict__ part, int n, doub
   }
 }
 
+// Sum of the K-split partials of a gradient in the order of the splits (one thread per element).
+__global__ void split_sum_kernel(const float* __restrict__ part, int splits, int64_t n,
+                                 float* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    double t = 0.0;
+    for (int s = 0; s < splits; ++s) t += part[(int64_t)s * n + i];
+    out[i] = (float)t;
+  }
+}
+
 cudaError_t launch_loss_reduce(const double* part, int C, int B, int Hq, int nP, double inv_n,
                                double* out, double* parts_out, int* status, cudaStream_t st) {
   loss_reduce_kernel<<<C, 256, 0, st>>>(part, B, Hq, nP, inv_n, out, parts_out, status);
@@ -117,6 +128,14 @@ cudaError_t launch_sumsq(const float* x, int64_t n, double* part, double* out, c
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   sum_in_order_kernel<<<1, 32, 0, st>>>(part, kRedBlocks, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_split_sum(const float* part, int splits, int64_t n, float* out, cudaStream_t st) {
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  split_sum_kernel<<<(unsigned)blocks, 256, 0, st>>>(part, splits, n, out);
   return cudaGetLastError();
 }
 

@@ -10,6 +10,7 @@ namespace jab {
 
 constexpr int kPartRows = 64;  // query rows per loss partial (one partial per (c, b, h, 64 rows))
 constexpr int kRedBlocks = 1024;  // blocks of a grid-stride reduction over the weights
+constexpr int kMaxSplits = 32;    // K splits of the weight-gradient GEMMs at most
 
 struct Workspace {
   // byte offsets into ws; SIZE_MAX when absent
@@ -28,6 +29,8 @@ struct Workspace {
   size_t dqkvt;    // bf16 [D, ldt]          dL/d[Q|K|V] (pre-RoPE), transposed
   size_t ds;       // fp16 [B, Hq, nq (nq + 1) / 2, 128, 128]   dS^T tile of every (query block,
                    //                        key block <= query block) pair, nq = ceil(T / 128)
+  size_t gpart;    // fp32 [kMaxSplits, D, d/G]  scale-gradient partial of every K split (summed in order)
+  size_t dwscr;    // fp32 [D, d]            dW when only its squared norm is asked for
   int64_t ldt;     // row pitch (elements) of dqkvt: N rounded up to 64
   int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 128
   size_t total;
@@ -67,8 +70,10 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
     w.dqkvt = take((size_t)D * w.ldt * 2);
     const int64_t nq = (T + 127) / 128;
     w.ds = take((size_t)B * d->n_q_heads * (nq * (nq + 1) / 2) * 128 * 128 * 2);
+    w.gpart = take((size_t)kMaxSplits * D * (dm / d->group_size) * 4);
+    w.dwscr = take((size_t)D * dm * 4);
   } else {
-    w.d_o = w.lse = w.dvec = w.dqkvt = w.ds = SIZE_MAX;
+    w.d_o = w.lse = w.dvec = w.dqkvt = w.ds = w.gpart = w.dwscr = SIZE_MAX;
   }
   w.total = off;
   return w;
