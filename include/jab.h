@@ -54,8 +54,10 @@ typedef enum {
   JAB_ERR_TIMEOUT = 6,       /* device: a bounded wait in a pipelined kernel gave up             */
   JAB_ERR_SCRATCH_LIMIT = 7, /* jab_loss_forward_noalloc: the problem needs more scratch than the
                                 fixed JAB_NOALLOC_SCRATCH_BYTES                                    */
-  JAB_ERR_INTERNAL = 8       /* device: an internal invariant did not hold (e.g. the alignment of
+  JAB_ERR_INTERNAL = 8,      /* device: an internal invariant did not hold (e.g. the alignment of
                                 a kernel's shared memory); the kernel returned without work     */
+  JAB_ERR_DEVICE_ASSERT = 9  /* device, checked build only (libjab_checked.so): an index was
+                                outside its buffer; the access was skipped                       */
 } jab_status;
 
 /* One attention block. Section 2.1 (d, d_head), App. C (Mistral-7B: GQA, RoPE theta = 1e4). */
@@ -300,6 +302,13 @@ jab_status jab_selftest_wait_timeout(jab_stream_t stream);
  * Every other result (losses, scale gradients, KL, Hutchinson and Omega sums, norms) is reduced in a
  * fixed order in both modes. Returns JAB_ERR_INVALID_ARG for other values of on. Host only. */
 jab_status jab_set_deterministic(int32_t on);
+
+/* Self-test of the checked build's bounds checks: a one-block kernel writes buf_dev[i] = i for
+ * i = 0 .. n, one index past the n-element extent it is given, each write behind the check. In the
+ * checked build the last write is skipped and the device status becomes JAB_ERR_DEVICE_ASSERT
+ * (buf_dev[n] keeps its value: give the buffer n + 1 elements to see it). The normal build launches
+ * nothing and returns JAB_ERR_UNSUPPORTED. JAB_ERR_INVALID_ARG for a NULL buffer or n < 1. */
+jab_status jab_selftest_bounds_check(int32_t* buf_dev, int32_t n, jab_stream_t stream);
 
 /* Synchronises `stream`, then returns and clears the device-side status of the current device
  * (JAB_OK if no kernel reported a problem since the last call). */

@@ -16,13 +16,15 @@ import torch
 JAB_OK = 0
 _STATUS_NAMES = {0: "JAB_OK", 1: "JAB_ERR_INVALID_ARG", 2: "JAB_ERR_UNSUPPORTED", 3: "JAB_ERR_CUDA",
                  4: "JAB_ERR_NONFINITE", 5: "JAB_ERR_RANGE", 6: "JAB_ERR_TIMEOUT",
-                 7: "JAB_ERR_SCRATCH_LIMIT", 8: "JAB_ERR_INTERNAL"}
+                 7: "JAB_ERR_SCRATCH_LIMIT", 8: "JAB_ERR_INTERNAL", 9: "JAB_ERR_DEVICE_ASSERT"}
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
 
 def lib_path() -> str:
-    return os.path.join(_HERE, "libjab.so")
+    """libjab.so, or the checked build libjab_checked.so when the environment sets JAB_CHECKED=1."""
+    name = "libjab_checked.so" if os.environ.get("JAB_CHECKED", "0") == "1" else "libjab.so"
+    return os.path.join(_HERE, name)
 
 
 class JabError(RuntimeError):
@@ -92,6 +94,7 @@ def lib() -> ctypes.CDLL:
     L.jab_init_scales.argtypes = [D, i32, i32, _P, _P, _P]
     L.jab_get_device_status.argtypes = [_P]
     L.jab_set_deterministic.argtypes = [i32]
+    L.jab_selftest_bounds_check.argtypes = [_P, i32, _P]
     L.jab_selftest_wait_timeout.argtypes = [_P]
     L.jab_status_string.argtypes = [i32]
     L.jab_status_string.restype = ctypes.c_char_p
@@ -108,7 +111,7 @@ def lib() -> ctypes.CDLL:
                "jab_reference_projection", "jab_loss_forward_kl", "jab_hutchinson_trace",
                "jab_omega_scores", "jab_rademacher_probes",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
-               "jab_selftest_wait_timeout", "jab_set_deterministic",
+               "jab_selftest_wait_timeout", "jab_set_deterministic", "jab_selftest_bounds_check",
                "jab_timing_collect", "jab_timing_get", "jab_timing_reset"):
         getattr(L, fn).restype = i32
     _LIB = L
@@ -360,6 +363,13 @@ def jab_set_deterministic(on: bool):
     (repeated calls bit-identical). Off by default: the STE weight gradient may then split its GEMM's
     token range and add the partial tiles with atomics."""
     _check(lib().jab_set_deterministic(int(on)), "jab_set_deterministic")
+
+
+def jab_selftest_bounds_check(buf, n: int, stream=None) -> int:
+    """Checked build only: writes buf[0..n] behind bounds checks against an n-element extent (the
+    last write is skipped, JAB_ERR_DEVICE_ASSERT raised on the device). Returns the call's status
+    (JAB_ERR_UNSUPPORTED from the normal build, which launches nothing)."""
+    return int(lib().jab_selftest_bounds_check(_ptr(buf, torch.int32, "buf"), int(n), _stream(stream)))
 
 
 def jab_get_device_status(stream=None) -> int:

@@ -1,7 +1,8 @@
 """Builds the C-ABI library libjab.so in-tree with nvcc for sm_103a (GB300).
 
-Usage: python -m paper_2609_34866_gb300.build [--force] [--verbose]
-Object files go to _build/ at the repository root; the library lands next to this file.
+Usage: python -m paper_2609_34866_gb300.build [--force] [--verbose] [--checked]
+Object files go to _build/ (_build_checked/ for the checked build) at the repository root; the
+library (libjab.so, or libjab_checked.so) lands next to this file.
 """
 from __future__ import annotations
 
@@ -19,6 +20,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_PATH = os.path.join(HERE, "libjab.so")
+CHECKED_BUILD_DIR = os.path.join(ROOT, "_build_checked")
+CHECKED_LIB_PATH = os.path.join(HERE, "libjab_checked.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
@@ -36,9 +39,9 @@ def _sources():
     return sorted(glob.glob(os.path.join(CSRC, "*.cu")))
 
 
-def _fingerprint() -> str:
+def _fingerprint(flags) -> str:
     h = hashlib.sha256()
-    h.update(" ".join(ARCH + CFLAGS).encode())
+    h.update(" ".join(ARCH + flags).encode())
     files = sorted(glob.glob(os.path.join(CSRC, "*")) + glob.glob(os.path.join(INCLUDE, "*.h")))
     for f in files:
         if os.path.isfile(f):
@@ -48,21 +51,26 @@ def _fingerprint() -> str:
     return h.hexdigest()
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile every .cu of csrc/ in parallel and link libjab.so. Returns the library path."""
-    os.makedirs(BUILD_DIR, exist_ok=True)
-    stamp = os.path.join(BUILD_DIR, "libjab.stamp")
-    fp = _fingerprint()
-    if not force and os.path.exists(LIB_PATH) and os.path.exists(stamp):
+def build(force: bool = False, verbose: bool = False, checked: bool = False) -> str:
+    """Compile every .cu of csrc/ in parallel and link libjab.so (checked=True: libjab_checked.so,
+    built with -DJAB_CHECKED=1: bounds checks that report JAB_ERR_DEVICE_ASSERT and skip the access).
+    Returns the library path."""
+    build_dir = CHECKED_BUILD_DIR if checked else BUILD_DIR
+    lib_path = CHECKED_LIB_PATH if checked else LIB_PATH
+    flags = CFLAGS + (["-DJAB_CHECKED=1"] if checked else [])
+    os.makedirs(build_dir, exist_ok=True)
+    stamp = os.path.join(build_dir, "libjab.stamp")
+    fp = _fingerprint(flags)
+    if not force and os.path.exists(lib_path) and os.path.exists(stamp):
         with open(stamp) as f:
             if f.read().strip() == fp:
-                return LIB_PATH
+                return lib_path
     nvcc = _nvcc()
     objs = []
 
     def compile_one(src):
-        obj = os.path.join(BUILD_DIR, os.path.basename(src)[:-3] + ".o")
-        cmd = [nvcc, *ARCH, *CFLAGS, "-c", src, "-o", obj]
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
+        cmd = [nvcc, *ARCH, *flags, "-c", src, "-o", obj]
         if verbose:
             cmd.insert(1, "-Xptxas=-v")
         r = subprocess.run(cmd, capture_output=True, text=True)
@@ -75,15 +83,16 @@ def build(force: bool = False, verbose: bool = False) -> str:
     srcs = _sources()
     with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, min(len(srcs), os.cpu_count() or 4))) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB_PATH + ".tmp"
+    tmp = lib_path + ".tmp"
     r = subprocess.run([nvcc, *ARCH, "-shared", "-o", tmp, *objs], capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
+    os.replace(tmp, lib_path)
     with open(stamp, "w") as f:
         f.write(fp)
-    return LIB_PATH
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose="--verbose" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose="--verbose" in sys.argv,
+                checked="--checked" in sys.argv))

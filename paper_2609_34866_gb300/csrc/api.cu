@@ -688,6 +688,7 @@ const char* jab_status_string(jab_status status) {
     case JAB_ERR_TIMEOUT: return "device wait timed out";
     case JAB_ERR_SCRATCH_LIMIT: return "problem larger than the fixed no-allocation scratch";
     case JAB_ERR_INTERNAL: return "internal device invariant failed";
+    case JAB_ERR_DEVICE_ASSERT: return "index outside its buffer (checked build)";
   }
   return "unknown status";
 }

@@ -106,12 +106,15 @@ __device__ __forceinline__ void stage_grad_16(uint32_t taddr, float mul, bool ro
 // the token offset is 8-aligned (consecutive threads cover consecutive 16-byte chunks of a dim
 // row), element-wise otherwise.
 template <int DH>
+// (checked build: every store is tested against [base, base + extent) of dQKV^T)
 __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int64_t ldt, int64_t n0,
-                                           int nvalid, int tid, int nthreads) {
+                                           int nvalid, int tid, int nthreads, const bf16_t* base,
+                                           int64_t extent, int* status) {
   if ((n0 & 7) == 0) {
     for (int idx = tid; idx < DH * 16; idx += nthreads) {
       const int d = idx >> 4, r0 = (idx & 15) * 8;
       bf16_t* o = dst + (int64_t)d * ldt + n0 + r0;
+      if (!in_bounds((o - base) + min(8, nvalid - r0) - 1, extent, status)) continue;
       if (r0 + 8 <= nvalid)
         *reinterpret_cast<uint4*>(o) = *reinterpret_cast<const uint4*>(tile + d * 128 + r0);
       else
@@ -120,7 +123,8 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
   } else {
     for (int idx = tid; idx < DH * 128; idx += nthreads) {
       const int d = idx >> 7, r = idx & 127;
-      if (r < nvalid) dst[(int64_t)d * ldt + n0 + r] = tile[d * 128 + r];
+      if (r < nvalid && in_bounds((dst - base) + (int64_t)d * ldt + n0 + r, extent, status))
+        dst[(int64_t)d * ldt + n0 + r] = tile[d * 128 + r];
     }
   }
 }
@@ -272,8 +276,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                           h * DH + ch * 64, row0 + i * BQ);
         }
         const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + i * BQ;
-        tc::bulk_load(sbase + L::ST_LSE, p.lse + lrow, BQ * 4, &bars->ld_full[st]);
-        tc::bulk_load(sbase + L::ST_D, p.dvec + lrow, BQ * 4, &bars->ld_full[st]);
+        // (checked build: a failed test leaves the stage incomplete; its consumers' bounded waits
+        // then give up and the kernel returns with the status raised)
+        if (in_bounds(lrow + BQ - 1, (int64_t)p.B * p.Hq * p.lse_pitch, p.status)) {
+          tc::bulk_load(sbase + L::ST_LSE, p.lse + lrow, BQ * 4, &bars->ld_full[st]);
+          tc::bulk_load(sbase + L::ST_D, p.dvec + lrow, BQ * 4, &bars->ld_full[st]);
+        }
         issued |= 1u << st;
         last_par = (last_par & ~(1u << st)) | (ph << st);
       }
@@ -524,11 +532,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (have) {
       const int nvalid = min(BK, p.T - kb * BK);
       const int64_t n0 = (int64_t)row0 + kb * BK;
+      const int64_t ext_t = (int64_t)(p.Hq + 2 * p.Hkv) * DH * p.ldt;  // dQKV^T elements
       const int tid = threadIdx.x - 64;
       store_tile<DH>(tv, p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
-                     EW_WARPS * 32);
+                     EW_WARPS * 32, p.dqkvt, ext_t, p.status);
       store_tile<DH>(tk, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
-                     EW_WARPS * 32);
+                     EW_WARPS * 32, p.dqkvt, ext_t, p.status);
     }
   }
   tc::fence_before_sync();
@@ -719,7 +728,7 @@ __global__ void __launch_bounds__(DQ_THREADS, 1)
       if (have)
         store_tile<DH>(stage, p.dqkvt + (int64_t)(p.qcol0 + tl.h * DH) * p.ldt, p.ldt,
                        (int64_t)tl.b * p.T + q0, min(BQ, p.T - q0), threadIdx.x - 64,
-                       EW_WARPS * 32);
+                       EW_WARPS * 32, p.dqkvt, (int64_t)(p.Hq + 2 * p.Hkv) * DH * p.ldt, p.status);
       // One snapshot of the abort flag between the two barriers, so that all epilogue warps leave
       // together (a warp left behind would wait on the named barrier of the next tile).
       if (threadIdx.x == 64) reinterpret_cast<volatile int*>(&bars->stop)[0] = *abort;

@@ -374,7 +374,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (warp == 2 && lane == 0 && ok) {
       double tot = 0.0;
       for (int w = 0; w < EW_WARPS; ++w) tot += bars->red[w];
-      p.part[((int64_t)b * p.Hq + h) * p.nP + qb] = tot;
+      const int64_t pi = ((int64_t)b * p.Hq + h) * p.nP + qb;
+      if (in_bounds(pi, (int64_t)p.B * p.Hq * p.nP, p.status)) p.part[pi] = tot;
     }
   }
   tc::fence_before_sync();

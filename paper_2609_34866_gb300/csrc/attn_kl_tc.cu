@@ -348,13 +348,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           kLn2 * (__fdiv_rn(rb.a, rb.lt) + (rb.ms - rb.mt) + log2f(__fdiv_rn(rb.ls, rb.lt)));
       if (cq == 0) {
         const int64_t rbase = (((int64_t)c * p.B + b) * p.Hq + h) * p.T;
+        const int64_t ext_r = (int64_t)p.C * p.B * p.Hq * p.T;
         if (tA < p.T) {
           acc += (double)klA;
-          if (p.kl_rows) p.kl_rows[rbase + tA] = klA;
+          if (p.kl_rows && in_bounds(rbase + tA, ext_r, p.status)) p.kl_rows[rbase + tA] = klA;
         }
         if (tB < p.T) {
           acc += (double)klB;
-          if (p.kl_rows) p.kl_rows[rbase + tB] = klB;
+          if (p.kl_rows && in_bounds(rbase + tB, ext_r, p.status)) p.kl_rows[rbase + tB] = klB;
         }
       }
     }
@@ -364,7 +365,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (warp == 2 && lane == 0 && ok) {
       double tot = 0.0;
       for (int w = 0; w < EW_WARPS; ++w) tot += bars->red[w];
-      p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb] = tot;
+      const int64_t pi = (((int64_t)c * p.B + b) * p.Hq + h) * p.nP + qb;
+      if (in_bounds(pi, (int64_t)p.C * p.B * p.Hq * p.nP, p.status)) p.part[pi] = tot;
     }
   }
   tc::fence_before_sync();

@@ -463,6 +463,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     const int c4 = lane & 7;
     int tc_ = 0;
     uint32_t range_bits = 0;  // mode 2: an fp16 dO value out of range (inf) or NaN
+    const int64_t ext_a = (int64_t)p.B * p.T * p.Hq * DH;         // A_ref, A, dO elements
+    const int64_t ext_p = (int64_t)p.C * p.B * p.Hq * p.nP;       // loss partials
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
@@ -493,9 +495,9 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
               const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & (RPH - 1));
-              if (tt < p.T)
-                av[i] = __ldg(reinterpret_cast<const float4*>(
-                    p.a_ref + ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col));
+              const int64_t aoff = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
+              if (tt < p.T && in_bounds(aoff + 3, ext_a, p.status))
+                av[i] = __ldg(reinterpret_cast<const float4*>(p.a_ref + aoff));
             }
           }
           float o[32];
@@ -529,6 +531,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             const int tt = q0 + ((rbase + rr) & (RPH - 1));
             if (tt >= p.T) continue;
             const int64_t off = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
+            if (!in_bounds(off + 3, ext_a, p.status)) continue;
             if (MODE == 0) {
               *reinterpret_cast<float4*>(p.a_out + off) = ov;
               const float2 v01 = make_float2(ov.x, ov.y), v23 = make_float2(ov.z, ov.w);
@@ -562,7 +565,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
             __syncwarp();
           }
         }
-        if (t < p.T) {
+        if (t < p.T && in_bounds(((int64_t)b * p.Hq + h) * p.lse_pitch + t,
+                                 (int64_t)p.B * p.Hq * p.lse_pitch, p.status)) {
           const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + t;
           if (MODE != 1 && p.lse != nullptr)
             p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
@@ -578,11 +582,13 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         // head hd = row >> 6 has lane quarters 2 hd and 2 hd + 1; quarter q is epilogue warp (q + 1) & 3
         const int hd = row >> 6;
         const double v = red[(2 * hd + 1) & 3] + red[(2 * hd + 2) & 3];
-        p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] = v;
+        const int64_t pi = (((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb;
+        if (in_bounds(pi, ext_p, p.status)) p.part[pi] = v;
       }
-      if (HPT == 1 && lane == 0 && quarter == 0 && have)  // one head: all four lane quarters
-        p.part[(((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb] =
-            ((red[0] + red[1]) + red[2]) + red[3];
+      if (HPT == 1 && lane == 0 && quarter == 0 && have) {  // one head: all four lane quarters
+        const int64_t pi = (((int64_t)c * p.B + b) * p.Hq + h) * p.nP + tl.qb;
+        if (in_bounds(pi, ext_p, p.status)) p.part[pi] = ((red[0] + red[1]) + red[2]) + red[3];
+      }
       if (!have) break;
     }
     if (MODE == 2 && range_bits) report(p.status, JAB_ERR_RANGE);

@@ -18,6 +18,26 @@ __device__ __forceinline__ void report(int* status, int code) {
   if (status != nullptr) atomicCAS(status, 0, code);
 }
 
+// Checked build (nvcc -DJAB_CHECKED=1, libjab_checked.so): the kernels test the last index of each
+// computed global access against its buffer's extent before making it; a failed test reports
+// JAB_ERR_DEVICE_ASSERT and the caller skips the access (no trap, no fault). Compiled out otherwise.
+#ifndef JAB_CHECKED
+#define JAB_CHECKED 0
+#endif
+__device__ __forceinline__ bool in_bounds(int64_t last, int64_t extent, int* status) {
+#if JAB_CHECKED
+  if (last < 0 || last >= extent) {
+    report(status, JAB_ERR_DEVICE_ASSERT);
+    return false;
+  }
+#else
+  (void)last;
+  (void)extent;
+  (void)status;
+#endif
+  return true;
+}
+
 // Non-zero when either half of a packed fp16 pair has every exponent bit set: an infinity (the
 // rounded value was outside the fp16 range) or a NaN. Integer SIMD compare, no FP instructions.
 __device__ __forceinline__ uint32_t half2_exp_all_ones(uint32_t h2) {

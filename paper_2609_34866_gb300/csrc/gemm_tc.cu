@@ -108,7 +108,8 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
       b[i] = __uint_as_float(rb[i]);
     }
     const int o = col1 % p.D;
-    if (p.n_rot > 0 && o < p.n_rot) {
+    if (p.n_rot > 0 && o < p.n_rot &&
+        in_bounds((int64_t)t * half + o % p.dh + 31, (int64_t)p.T * half, p.status)) {
       const int jj0 = o % p.dh;
       const float4* cp = reinterpret_cast<const float4*>(p.cos_t + (int64_t)t * half + jj0);
       const float4* sp = reinterpret_cast<const float4*>(p.sin_t + (int64_t)t * half + jj0);
@@ -133,7 +134,7 @@ __device__ __forceinline__ void epi_rope(const GemmParams& p, uint32_t taddr, in
         }
       }
     }
-    if (row_ok) {
+    if (row_ok && in_bounds(m * p.Nn + col1 + half + 31, p.M * (int64_t)p.Nn, p.status)) {
       uint4* d1 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1);
       uint4* d2 = reinterpret_cast<uint4*>(p.C + m * p.Nn + col1 + half);
       uint32_t inf_bits = 0;  // a half with all exponent bits set: inf (out of fp16 range) or NaN
@@ -181,7 +182,7 @@ __device__ __forceinline__ void epi_store(const GemmParams& p, uint32_t taddr, i
       g[i] = v.x;
       g[i + 1] = v.y;
     }
-    if (p.dw != nullptr) {
+    if (p.dw != nullptr && in_bounds(o * p.Nn + i0 + 31, p.M * (int64_t)p.Nn, p.status)) {
       float4* d = reinterpret_cast<float4*>(p.dw + o * p.Nn + i0);
       if (p.splits > 1) {  // a K range: add the partial tile into the zeroed dw
 #pragma unroll
@@ -202,6 +203,7 @@ __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int
   const int ng = p.d / p.G;
   // one value per (split, row, group): this unit's tile covers whole groups (BN is a multiple of G)
   float* part_out = p.dspart + ((int64_t)ks * p.M + o) * ng;
+  const int64_t part_extent = (int64_t)p.splits * p.M * ng;
   float part = 0.f;
   int cur = -1;
 #pragma unroll 1
@@ -213,26 +215,31 @@ __device__ __forceinline__ void epi_lsq(const GemmParams& p, uint32_t taddr, int
     tc::tmem_ld32(taddr + c * 32, r);
     tc::tmem_ld_wait();
     const int g = i0 / p.G;
-    const float sc = __ldg(p.s + (int64_t)o * ng + g);
-    const uint4* wp = reinterpret_cast<const uint4*>(p.w + (int64_t)o * p.d + i0);
     float acc = 0.f;
+    if (in_bounds((int64_t)o * p.d + i0 + 31, (int64_t)p.M * p.d, p.status) &&
+        in_bounds((int64_t)o * ng + g, (int64_t)p.M * ng, p.status)) {
+      const float sc = __ldg(p.s + (int64_t)o * ng + g);
+      const uint4* wp = reinterpret_cast<const uint4*>(p.w + (int64_t)o * p.d + i0);
 #pragma unroll
-    for (int v = 0; v < 4; ++v) {
-      const uint4 u = __ldg(wp + v);
-      const bf16_t* wb = reinterpret_cast<const bf16_t*>(&u);
+      for (int v = 0; v < 4; ++v) {
+        const uint4 u = __ldg(wp + v);
+        const bf16_t* wb = reinterpret_cast<const bf16_t*>(&u);
 #pragma unroll
-      for (int e = 0; e < 8; ++e)
-        acc = fmaf(__uint_as_float(r[v * 8 + e]), lsq_factor(__bfloat162float(wb[e]), sc, qmax),
-                   acc);
+        for (int e = 0; e < 8; ++e)
+          acc = fmaf(__uint_as_float(r[v * 8 + e]), lsq_factor(__bfloat162float(wb[e]), sc, qmax),
+                     acc);
+      }
     }
     if (g != cur) {
-      if (cur >= 0) part_out[cur] = p.coef * part;
+      if (cur >= 0 && in_bounds(((int64_t)ks * p.M + o) * ng + cur, part_extent, p.status))
+        part_out[cur] = p.coef * part;
       part = 0.f;
       cur = g;
     }
     part += acc;
   }
-  if (cur >= 0) part_out[cur] = p.coef * part;
+  if (cur >= 0 && in_bounds(((int64_t)ks * p.M + o) * ng + cur, part_extent, p.status))
+    part_out[cur] = p.coef * part;
 }
 
 // ------------------------------------------------------------------ CTA-pair variant (cta_group::2)

@@ -64,6 +64,8 @@ def test_host_side_checks_without_gpu(libjab):
     assert st == 1
     assert L.jab_prepare_x(ctypes.byref(good), 2, 130, None, None, 0, None) == 1
     assert L.jab_flip_rate(None, None, 16, None, None) == 1
+    assert L.jab_selftest_bounds_check(None, 4, None) == 1
+    assert L.jab_set_deterministic(2) == 1 and L.jab_set_deterministic(0) == 0
     st = L.jab_quantize(ctypes.byref(bad_dh), 3, None, None, None, None, None)
     assert st == 2
     assert L.jab_status_string(4).decode() == "non-finite or non-positive value"
