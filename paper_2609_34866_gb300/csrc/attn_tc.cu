@@ -452,8 +452,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
   } else if (warp < EPI_WARP0 + EPI_WARPS) {  // ------------------------------------- epilogue
     // Coalesced pass: the warp's 32 rows x 32 columns of O go through shared memory; lane l then
     // handles 16 bytes of rows 4 i + l / 8 (i < 8), eight lanes per 128-byte row segment. In mode 2
-    // the fp16-rounded error goes back through the same slots to the row's owner, which accumulates
-    // D = rowsum(dO * O).
+    // each lane accumulates its share of D = rowsum(dO * O) for its rows in this layout and the
+    // eight lanes of a row add them at the end of the tile (no second pass through the slots).
     const int quarter = warp & 3;
     const int ew = warp - EPI_WARP0;
     const int row = quarter * 32 + lane;  // stacked row = TMEM lane
@@ -485,49 +485,51 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         if (lane == 0) tc::mbar_arrive(&bars->st_empty[ob]);
         tc::fence_after_sync();
         const float inv_l = __fdiv_rn(1.f, lt);
-        float2 sq = make_float2(0.f, 0.f), dsum = make_float2(0.f, 0.f);  // packed partial sums
+        float2 sq = make_float2(0.f, 0.f);  // packed partial sum of squares
+        float dpart[8];                     // mode 2: this lane's share of D for rows 4 i + lane / 8
+#pragma unroll
+        for (int i = 0; i < 8; ++i) dpart[i] = 0.f;
         const float2 il2 = make_float2(inv_l, inv_l);
+        // A_ref rows of this lane in the coalesced layout (loading them a chunk ahead costs more in
+        // register spills than it hides)
+        float4 av[8];
+        auto load_aref = [&](int ch, float4 (&dst)[8]) {
+          const int col = h * DH + ch * 32 + c4 * 4;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & (RPH - 1));
+            const int64_t aoff = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
+            if (tt < p.T && in_bounds(aoff + 3, ext_a, p.status))
+              dst[i] = __ldg(reinterpret_cast<const float4*>(p.a_ref + aoff));
+          }
+        };
 #pragma unroll 1
         for (int ch = 0; ch < DH / 32; ++ch) {
           const int col = h * DH + ch * 32 + c4 * 4;
-          float4 av[8];
-          if (MODE != 0) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int tt = q0 + ((rbase + 4 * i + (lane >> 3)) & (RPH - 1));
-              const int64_t aoff = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
-              if (tt < p.T && in_bounds(aoff + 3, ext_a, p.status))
-                av[i] = __ldg(reinterpret_cast<const float4*>(p.a_ref + aoff));
-            }
-          }
-          float o[32];
+          if (MODE != 0) load_aref(ch, av);
           {
             uint32_t r[32];
             __syncwarp();
             tc::tmem_ld32(tmem + lane_base + L::O_COL + ob * DH + ch * 32, r);
             tc::tmem_ld_wait();
+            if (ch == DH / 32 - 1) {  // O of this buffer is read out: the next-but-one tile may use it
+              tc::fence_before_sync();
+              __syncwarp();
+              if (lane == 0) tc::mbar_arrive(&bars->o_empty[ob]);
+            }
 #pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-              const float2 v = tc::mul2(make_float2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), il2);
-              o[i] = v.x;
-              o[i + 1] = v.y;
+            for (int v = 0; v < 8; ++v) {
+              const float2 lo = tc::mul2(make_float2(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1])), il2);
+              const float2 hi = tc::mul2(make_float2(__uint_as_float(r[4 * v + 2]), __uint_as_float(r[4 * v + 3])), il2);
+              *reinterpret_cast<float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2)) =
+                  make_float4(lo.x, lo.y, hi.x, hi.y);
             }
           }
-          if (ch == DH / 32 - 1) {  // O of this buffer is read out: the next-but-one tile may use it
-            tc::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) tc::mbar_arrive(&bars->o_empty[ob]);
-          }
-#pragma unroll
-          for (int v = 0; v < 8; ++v)
-            *reinterpret_cast<float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2)) =
-                make_float4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
           __syncwarp();
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int rr = 4 * i + (lane >> 3);
-            float4* slot = reinterpret_cast<float4*>(stg + rr * 32 + ((c4 ^ (rr & 7)) << 2));
-            const float4 ov = *slot;
+            const float4 ov = *reinterpret_cast<const float4*>(stg + rr * 32 + ((c4 ^ (rr & 7)) << 2));
             const int tt = q0 + ((rbase + rr) & (RPH - 1));
             if (tt >= p.T) continue;
             const int64_t off = ((int64_t)row0 + tt) * (int64_t)(p.Hq * DH) + col;
@@ -540,37 +542,43 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
               const float4 a = av[i];
               const float2 e01 = tc::sub2(make_float2(ov.x, ov.y), make_float2(a.x, a.y));
               const float2 e23 = tc::sub2(make_float2(ov.z, ov.w), make_float2(a.z, a.w));
-              const float e0 = e01.x, e1 = e01.y, e2 = e23.x, e3 = e23.y;
               sq = tc::fma2(e23, e23, tc::fma2(e01, e01, sq));
               if (MODE == 2) {
-                const __half2 a01 = __floats2half2_rn(e0, e1), a23 = __floats2half2_rn(e2, e3);
+                const __half2 a01 = __floats2half2_rn(e01.x, e01.y), a23 = __floats2half2_rn(e23.x, e23.y);
                 uint2 u;
                 u.x = *reinterpret_cast<const uint32_t*>(&a01);
                 u.y = *reinterpret_cast<const uint32_t*>(&a23);
                 *reinterpret_cast<uint2*>(p.d_o + off) = u;
                 range_bits |= half2_exp_all_ones(u.x) | half2_exp_all_ones(u.y);
+                // D = rowsum(dO * O) with dO as stored (fp16-rounded)
                 const float2 f01 = __half22float2(a01), f23 = __half22float2(a23);
-                *slot = make_float4(f01.x, f01.y, f23.x, f23.y);
+                const float2 d2 = tc::fma2(f23, make_float2(ov.z, ov.w),
+                                           tc::mul2(f01, make_float2(ov.x, ov.y)));
+                dpart[i] += d2.x + d2.y;
               }
             }
           }
-          __syncwarp();
-          if (MODE == 2) {
+          __syncwarp();  // the staging slots are rewritten by the next chunk
+        }
+        if (MODE == 2) {  // the eight lanes of a row (lane / 8 equal) add their shares, fixed tree
 #pragma unroll
-            for (int v = 0; v < 8; ++v) {
-              const float4 e = *reinterpret_cast<const float4*>(stg + lane * 32 + ((v ^ (lane & 7)) << 2));
-              dsum = tc::fma2(make_float2(e.x, e.y), make_float2(o[4 * v], o[4 * v + 1]), dsum);
-              dsum = tc::fma2(make_float2(e.z, e.w), make_float2(o[4 * v + 2], o[4 * v + 3]), dsum);
-            }
-            __syncwarp();
+          for (int i = 0; i < 8; ++i) {
+            float v = dpart[i];
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            const int rr = 4 * i + (lane >> 3);
+            const int tt = q0 + ((rbase + rr) & (RPH - 1));
+            const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + tt;
+            if ((lane & 7) == 0 && tt < p.T && in_bounds(li, (int64_t)p.B * p.Hq * p.lse_pitch, p.status))
+              p.dvec[li] = v;
           }
         }
-        if (t < p.T && in_bounds(((int64_t)b * p.Hq + h) * p.lse_pitch + t,
-                                 (int64_t)p.B * p.Hq * p.lse_pitch, p.status)) {
+        if (MODE != 1 && p.lse != nullptr && t < p.T &&
+            in_bounds(((int64_t)b * p.Hq + h) * p.lse_pitch + t, (int64_t)p.B * p.Hq * p.lse_pitch,
+                      p.status)) {
           const int64_t li = ((int64_t)b * p.Hq + h) * p.lse_pitch + t;
-          if (MODE != 1 && p.lse != nullptr)
-            p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
-          if (MODE == 2) p.dvec[li] = dsum.x + dsum.y;
+          p.lse[li] = MODE == 2 ? m + log2f(lt) : (m + log2f(lt)) * kLn2;  // mode 2: log2 units
         }
         acc = (double)sq.x + (double)sq.y;
       }
