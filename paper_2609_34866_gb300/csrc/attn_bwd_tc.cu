@@ -8,8 +8,9 @@
 // Two kernels, no atomics:
 //   dkdv  one CTA per (128-key block, KV head, sequence); loops over the query heads of the group and
 //         over 128-query blocks: S^T = K Q^T, dP^T = V dO^T into TMEM, P^T and dS^T (fp16) written
-//         back over them, dV += P^T dO and dK += dS^T Q (A operands in TMEM) accumulated in TMEM.
-//         Each dS^T tile is also staged in shared memory and stored to HBM by TMA (a store warp).
+//         back over them by 16 elementwise warps (16 key rows x 64 queries each), dV += P^T dO and
+//         dK += dS^T Q (A operands in TMEM) accumulated in TMEM. Each dS^T tile is also staged in
+//         shared memory and stored to HBM by TMA (a store warp).
 //   dq    persistent, (128 query rows, query head, sequence) tiles: dQ = scale * sum_kb dS K from the
 //         stored dS^T tiles, a plain tensor-core product per key block (no recomputation of S, P or
 //         dP: two of the three products and all elementwise work of a recomputing dq are saved, for
@@ -24,8 +25,9 @@
 namespace jab {
 namespace {
 
-constexpr int NUM_THREADS = 352;  // warp 0 TMA, warp 1 UMMA, warps 2..9 elementwise, warp 10 dS^T stores
-constexpr int EW_WARPS = 8;
+constexpr int EW_WARPS = 8;       // dq: epilogue warps
+constexpr int DKDV_EW = 16;       // dK/dV: elementwise warps, 16 key rows x 64 queries each
+constexpr int DKDV_THREADS = (2 + DKDV_EW + 1) * 32;  // warp 0 TMA, 1 UMMA, 2..17 elementwise, 18 stores
 constexpr int kSuperGroup = 8;  // (KV head, sequence) pairs whose dK/dV CTAs are interleaved
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -171,7 +173,7 @@ struct DkdvBars {
 };
 
 template <int DH>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(DKDV_THREADS, 1)
     attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
                             const __grid_constant__ CUtensorMap tm_do,
                             const __grid_constant__ CUtensorMap tm_ds, const BwdParams p) {
@@ -215,13 +217,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     tc::mbar_init(&bars->s_full, 1);
     tc::mbar_init(&bars->dp_full, 1);
-    tc::mbar_init(&bars->p_full, EW_WARPS);
-    tc::mbar_init(&bars->ds_full, EW_WARPS);
+    tc::mbar_init(&bars->p_full, DKDV_EW);
+    tc::mbar_init(&bars->ds_full, DKDV_EW);
     tc::mbar_init(&bars->dv_done, 1);
     tc::mbar_init(&bars->dk_done, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
-    tc::mbar_init(&bars->dss_full, EW_WARPS);  // the block's dS^T is in the staging tile
+    tc::mbar_init(&bars->dss_full, DKDV_EW);  // the block's dS^T is in the staging tile
     tc::mbar_init(&bars->dss_free, 1);         // the store warp's TMA stores have read it
     bars->abort = 0;
     tc::fence_mbar_init();
@@ -372,7 +374,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
     }
-  } else if (warp == 10) {
+  } else if (warp == 2 + DKDV_EW) {
     if (lane == 0) {  // ------------------------------------------ dS^T tiles to global memory
       // Tile (sequence b, head h, query block i, key block kb) is row block
       // (b Hq + h) npairs + i (i + 1) / 2 + kb of the dS^T buffer: 128 key rows of 128 queries.
@@ -388,9 +390,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       tc::bulk_wait_group<0>();
     }
-  } else {  // ------------------------------------ elementwise: 16 key rows x 128 queries per warp
+  } else {  // ------------------------------------ elementwise: 16 key rows x 64 queries per warp
+    // Warp w (2..17) may access TMEM lane quarter w % 4; the four warps of a quarter take its two
+    // 16-row groups x the block's two 64-query halves. Nothing is reduced across queries here (the
+    // row log-sum-exp and D come with the block), so a warp needs only its half.
     const int quarter = warp & 3;
-    const int half = (warp - 2) >> 2;
+    const int idx = (warp - 2) >> 2;
+    const int half = idx & 1;   // 16-row group of the quarter
+    const int chalf = idx >> 1; // 64-query half of the block
     const int cq = lane & 3;
     const int rA = quarter * 32 + half * 16 + (lane >> 2);  // key rows rA and rA + 8 of the block
     const int keyA = kb * BK + rA, keyB = keyA + 8;
@@ -399,65 +406,59 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int it = 0; it < n_it; ++it) {
       const int st = it % STAGES;
       const int i = kb + it % per_head;
-      const float* lse_s = reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_LSE);
-      const float* d_s = reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_D);
+      const float* lse_s =
+          reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_LSE) + 64 * chalf;
+      const float* d_s =
+          reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_D) + 64 * chalf;
       if (!tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status) ||
           !tc::mbar_wait(&bars->s_full, it & 1, abort, p.status)) {
         ok = false;
         break;
       }
       tc::fence_after_sync();
-      // x[hh][4n + e] (e < 2): row A, query column 64 hh + 8n + 2 cq + e; e = 2, 3: row B.
-      float x[2][32];
+      // x[4n + e] (e < 2): row A, query 64 chalf + 8n + 2 cq + e; e = 2, 3: row B
+      float x[32];
       {
-        uint32_t r0[32], r1[32];
+        uint32_t r0[32];
         __syncwarp();
-        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL, r0);
-        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + 64, r1);
+        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::S_COL + 64 * chalf, r0);
         tc::tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          x[0][c] = __uint_as_float(r0[c]);
-          x[1][c] = __uint_as_float(r1[c]);
-        }
+        for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(r0[c]);
       }
-      const int qc0 = i * BQ + 2 * cq;  // query of x[0][0]
+      const int qc0 = i * BQ + 64 * chalf + 2 * cq;  // query of x[0]
       const bool full = i > kb && i * BQ + BQ <= p.T;
       const float2 sl2 = make_float2(p.sl2, p.sl2);
 #pragma unroll
-      for (int hh = 0; hh < 2; ++hh)
+      for (int n = 0; n < 8; ++n) {
+        const float2 l2 = *reinterpret_cast<const float2*>(lse_s + 8 * n + 2 * cq);
+        const float2 nl = make_float2(tc::neg_bits(l2.x), tc::neg_bits(l2.y));
+        const float2 ea = tc::fma2(make_float2(x[4 * n], x[4 * n + 1]), sl2, nl);
+        const float2 eb = tc::fma2(make_float2(x[4 * n + 2], x[4 * n + 3]), sl2, nl);
+        float pa[2] = {tc::fast_exp2(ea.x), tc::fast_exp2(ea.y)};
+        float pb[2] = {tc::fast_exp2(eb.x), tc::fast_exp2(eb.y)};
+        if (!full) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int q = qc0 + 8 * n + e;
+            if (q >= p.T || q < keyA) pa[e] = 0.f;
+            if (q >= p.T || q < keyB) pb[e] = 0.f;
+          }
+        }
+        x[4 * n] = pa[0];
+        x[4 * n + 1] = pa[1];
+        x[4 * n + 2] = pb[0];
+        x[4 * n + 3] = pb[1];
+      }
+      {
+        uint32_t pw[16];  // pw[2n] row A, pw[2n + 1] row B: packed column 32 chalf + 4n + cq
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
-          const float2 l2 = *reinterpret_cast<const float2*>(lse_s + 64 * hh + 8 * n + 2 * cq);
-          const float2 nl = make_float2(tc::neg_bits(l2.x), tc::neg_bits(l2.y));
-          const float2 ea = tc::fma2(make_float2(x[hh][4 * n], x[hh][4 * n + 1]), sl2, nl);
-          const float2 eb = tc::fma2(make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]), sl2, nl);
-          float pa[2] = {tc::fast_exp2(ea.x), tc::fast_exp2(ea.y)};
-          float pb[2] = {tc::fast_exp2(eb.x), tc::fast_exp2(eb.y)};
-          if (!full) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int q = qc0 + 64 * hh + 8 * n + e;
-              if (q >= p.T || q < keyA) pa[e] = 0.f;
-              if (q >= p.T || q < keyB) pb[e] = 0.f;
-            }
-          }
-          x[hh][4 * n] = pa[0];
-          x[hh][4 * n + 1] = pa[1];
-          x[hh][4 * n + 2] = pb[0];
-          x[hh][4 * n + 3] = pb[1];
+          pw[2 * n] = tc::pack_half2(x[4 * n], x[4 * n + 1]);
+          pw[2 * n + 1] = tc::pack_half2(x[4 * n + 2], x[4 * n + 3]);
         }
-      {
-        uint32_t pw[32];  // pw[2m] row A, pw[2m + 1] row B, packed column 4m + cq
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-          for (int n = 0; n < 8; ++n) {
-            pw[2 * (8 * hh + n)] = tc::pack_half2(x[hh][4 * n], x[hh][4 * n + 1]);
-            pw[2 * (8 * hh + n) + 1] = tc::pack_half2(x[hh][4 * n + 2], x[hh][4 * n + 3]);
-          }
         __syncwarp();
-        tc::tmem_st_16x128b_x16(tmem + lane16 + L::S_COL, pw);
+        tc::tmem_st_16x128b_x8(tmem + lane16 + L::S_COL + 32 * chalf, pw);
         tc::tmem_st_wait();
       }
       tc::fence_before_sync();
@@ -468,76 +469,80 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         break;
       }
       tc::fence_after_sync();
-      uint32_t dw[32];
-#pragma unroll
-      for (int hh = 0; hh < 2; ++hh) {
+      uint32_t dw[16];
+      {
         uint32_t rd[32];
         __syncwarp();
-        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::DP_COL + 64 * hh, rd);
+        tc::tmem_ld_16x256b_x8(tmem + lane16 + L::DP_COL + 64 * chalf, rd);
         tc::tmem_ld_wait();
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
-          const float2 d2 = *reinterpret_cast<const float2*>(d_s + 64 * hh + 8 * n + 2 * cq);
+          const float2 d2 = *reinterpret_cast<const float2*>(d_s + 8 * n + 2 * cq);
           const float2 ta = tc::sub2(make_float2(__uint_as_float(rd[4 * n]), __uint_as_float(rd[4 * n + 1])), d2);
           const float2 tb = tc::sub2(make_float2(__uint_as_float(rd[4 * n + 2]), __uint_as_float(rd[4 * n + 3])), d2);
-          float2 da = tc::mul2(make_float2(x[hh][4 * n], x[hh][4 * n + 1]), ta);
-          float2 db = tc::mul2(make_float2(x[hh][4 * n + 2], x[hh][4 * n + 3]), tb);
+          float2 da = tc::mul2(make_float2(x[4 * n], x[4 * n + 1]), ta);
+          float2 db = tc::mul2(make_float2(x[4 * n + 2], x[4 * n + 3]), tb);
           if (!full) {  // masked entries (P = 0; D past T is not written): dS = 0
-            if (x[hh][4 * n] == 0.f) da.x = 0.f;
-            if (x[hh][4 * n + 1] == 0.f) da.y = 0.f;
-            if (x[hh][4 * n + 2] == 0.f) db.x = 0.f;
-            if (x[hh][4 * n + 3] == 0.f) db.y = 0.f;
+            if (x[4 * n] == 0.f) da.x = 0.f;
+            if (x[4 * n + 1] == 0.f) da.y = 0.f;
+            if (x[4 * n + 2] == 0.f) db.x = 0.f;
+            if (x[4 * n + 3] == 0.f) db.y = 0.f;
           }
-          dw[2 * (8 * hh + n)] = tc::pack_half2(da.x, da.y);
-          dw[2 * (8 * hh + n) + 1] = tc::pack_half2(db.x, db.y);
+          dw[2 * n] = tc::pack_half2(da.x, da.y);
+          dw[2 * n + 1] = tc::pack_half2(db.x, db.y);
         }
       }
       __syncwarp();
-      tc::tmem_st_16x128b_x16(tmem + lane16 + L::DP_COL, dw);
+      tc::tmem_st_16x128b_x8(tmem + lane16 + L::DP_COL + 32 * chalf, dw);
       tc::tmem_st_wait();
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->ds_full);
-      // The same dS^T words into the staging tile (two 64-query halves, 128-byte swizzle) for the
-      // store warp, once it has stored the previous block's: packed column c = 4m + cq (queries
-      // 2c, 2c + 1) is 16-byte unit m % 8 of half m / 8 of its key row.
+      // The same dS^T words into the staging tile for the store warp, once it has stored the
+      // previous block's: packed word n (queries 64 chalf + 8n + 2cq, +1) is 16-byte unit n of the
+      // 64-query half chalf of its key row (128-byte swizzle).
       if (it > 0 && !tc::mbar_wait(&bars->dss_free, (it - 1) & 1, abort, p.status)) {
         ok = false;
         break;
       }
+      {
+        uint8_t* hb = smem + L::DSS_OFF + chalf * L::CHUNK;
 #pragma unroll
-      for (int m = 0; m < 16; ++m) {
-        uint8_t* hb = smem + L::DSS_OFF + (m >> 3) * L::CHUNK;
-        *reinterpret_cast<uint32_t*>(hb + rA * 128 + (((m & 7) ^ (rA & 7)) << 4) + cq * 4) = dw[2 * m];
-        *reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + (((m & 7) ^ ((rA + 8) & 7)) << 4) + cq * 4) =
-            dw[2 * m + 1];
+        for (int n = 0; n < 8; ++n) {
+          *reinterpret_cast<uint32_t*>(hb + rA * 128 + ((n ^ (rA & 7)) << 4) + cq * 4) = dw[2 * n];
+          *reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + ((n ^ ((rA + 8) & 7)) << 4) + cq * 4) =
+              dw[2 * n + 1];
+        }
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&bars->dss_full);
     }
-    // Epilogue: dV and dK rows (transpose of RoPE on dK) staged transposed in the now idle stage
-    // buffers, then stored as dQKV^T columns with coalesced 16-byte stores.
+    // Epilogue: dV rows (warps of query half 0) and dK rows (half 1; transpose of RoPE) staged
+    // transposed in the now idle stage buffers, then stored as dQKV^T columns with coalesced
+    // 16-byte stores by all elementwise warps.
     const bool have = ok && tc::mbar_wait(&bars->o_full, 0, abort, p.status);
     bf16_t* tv = reinterpret_cast<bf16_t*>(smem + L::ST_OFF);
     bf16_t* tk = tv + DH * 128;
     if (have) {
       tc::fence_after_sync();
       const int kA = keyA < p.T ? keyA : 0, kB = keyB < p.T ? keyB : 0;
-      stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, rA);
-      stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, kA, kB, p.cos_t,
-                        p.sin_t, tk, rA);
+      if (chalf == 0)
+        stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, rA);
+      else
+        stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, kA, kB, p.cos_t,
+                          p.sin_t, tk, rA);
     }
-    tc::named_bar_sync(1, EW_WARPS * 32);  // every elementwise warp reaches this exactly once
+    tc::named_bar_sync(1, DKDV_EW * 32);  // every elementwise warp reaches this exactly once
     if (have) {
       const int nvalid = min(BK, p.T - kb * BK);
       const int64_t n0 = (int64_t)row0 + kb * BK;
       const int64_t ext_t = (int64_t)(p.Hq + 2 * p.Hkv) * DH * p.ldt;  // dQKV^T elements
       const int tid = threadIdx.x - 64;
       store_tile<DH>(tv, p.dqkvt + (int64_t)(p.vcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
-                     EW_WARPS * 32, p.dqkvt, ext_t, p.status);
+                     DKDV_EW * 32, p.dqkvt, ext_t, p.status);
       store_tile<DH>(tk, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
-                     EW_WARPS * 32, p.dqkvt, ext_t, p.status);
+                     DKDV_EW * 32, p.dqkvt, ext_t, p.status);
     }
   }
   tc::fence_before_sync();
@@ -798,7 +803,7 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
   const int64_t n_dkdv = (int64_t)L.Hkv * L.B * ((L.T + 127) / 128);
   if (n_dkdv >= (1ll << 31)) return cudaErrorInvalidValue;
   const dim3 g1((unsigned)n_dkdv);
-  attn_bwd_dkdv_tc_kernel<DH><<<g1, NUM_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128,
+  attn_bwd_dkdv_tc_kernel<DH><<<g1, DKDV_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128,
                                                                                      ds128, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
