@@ -493,10 +493,14 @@ cudaError_t launch_gemm2(const CUtensorMap& ta, const CUtensorMap& tb, GemmParam
   cfg.dynamicSmemBytes = SMEM2_BYTES;
   cfg.stream = st;
   const int sms = sm_count();
-  cfg.gridDim = dim3((unsigned)(sms / 2 * 2));
-  int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess || clusters < 1)
-    clusters = sms / 2;
+  // The pairs that fit at once depend only on the kernel and the device: asked once, so that a
+  // launch makes no occupancy query (a launch-bound loop pays for every host call).
+  static int clusters = 0;
+  if (clusters < 1) {
+    cfg.gridDim = dim3((unsigned)(sms / 2 * 2));
+    if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess || clusters < 1)
+      clusters = sms / 2;
+  }
   const int64_t total = (int64_t)p.num_m * p.num_n * p.splits;
   const int pairs = (int)std::min<int64_t>(total, std::min(clusters, sms / 2));
   cfg.gridDim = dim3((unsigned)(2 * pairs));

@@ -412,6 +412,44 @@ def test_ste_scale_fitting_loop_lowers_the_loss():
     assert count.item() == O.flip_count(codes1.cpu().numpy(), codes0.cpu().numpy()) > 0
 
 
+def test_fit_step_replays_from_a_cuda_graph():
+    """The fit step launches only on the caller's stream and never synchronises the host, so one
+    call captures whole into a CUDA graph. A replay gives the eager call's bits, and reads the
+    scales afresh: after an in-place update of them, a replay equals a new eager call."""
+    c = case("mistral_G64_T70")
+    ws = c.workspace()
+    A, _, _ = c.gpu_teacher(ws)
+    s = c.gpu_scales(2, mode=1)
+    J().jab_prepare_x(c.desc, c.B, c.T, c.X, ws)
+    loss = torch.empty(1, dtype=torch.float64, device="cuda")
+    grad = torch.empty_like(s)
+
+    def step():
+        J().jab_loss_backward_scales_prepared(c.desc, c.B, c.T, c.X, c.W, A, 2, s, 0.0, loss, grad,
+                                              ws)
+
+    step()
+    l_eager, g_eager = loss.clone(), grad.clone()
+    loss.zero_()
+    grad.zero_()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    torch.cuda.synchronize()
+    assert loss.item() == 0.0 and not grad.any()       # captured, not run
+    graph.replay()
+    torch.cuda.synchronize()
+    assert loss.item() == l_eager.item() and torch.equal(grad, g_eager)
+    s.mul_(1.1)
+    graph.replay()
+    torch.cuda.synchronize()
+    l_replay, g_replay = loss.clone(), grad.clone()
+    step()
+    assert l_replay.item() == loss.item() != l_eager.item()
+    assert torch.equal(g_replay, grad)
+    assert J().jab_get_device_status() == 0
+
+
 def test_flip_rate_is_an_exact_count():
     """Eq. 15: the number of changed grid positions, bit-exact against the oracle's count, on a
     length with a ragged tail (not a multiple of 16 bytes) and on an empty range."""
