@@ -56,9 +56,8 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 // may overwrite it), O double-buffered by tile parity at 128 / 128 + DH, Q (DH / 2 columns) and P
 // (64 columns) after them. With two O buffers the epilogue of tile i runs on its own warps while the
 // softmax warps already work on tile i + 1.
-//   warp 0       TMA: Q tile (and an L2 prefetch of the tile's A_ref rows), K ring (3 stages: a K
-//                load is issued once S two blocks back has completed and must land before S of
-//                the block after next)
+//   warp 0       TMA: Q tile, K ring (3 stages: a K load is issued once S two blocks back has
+//                completed and must land before S of the block after next)
 //   warp 1       TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
 //   warps 2..9   softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
 //                16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
@@ -67,7 +66,8 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 //   warp 10      TMA: V ring (2 stages), so that K loads never queue behind a V stage that is busy
 //   warps 11..14 epilogue, one TMEM lane quarter each (32x32b shape, one row per thread, 32 columns
 //                at a time): O is staged through shared memory so that A_ref loads and dO / A
-//                stores are coalesced; per-mode outputs and the SSE partials.
+//                stores are coalesced; per-mode outputs and the SSE partials. Each thread
+//                prefetches its row of the next tile's A_ref into L2 a whole tile ahead.
 constexpr int SQ = 64, SKB = 128, SK_ST = 3, SV_ST = 2;
 constexpr int PAIR_THREADS = 480;
 constexpr int EPI_WARPS = 4, EPI_WARP0 = 11;
@@ -198,12 +198,6 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
                               c * p.D + (h0 + hd) * DH + ch * 64, row0 + q0);
           qiss = 1;
           qpar = tc_ & 1;
-          if (MODE != 0) {  // the epilogue reads these A_ref rows (HPT heads: HPT DH fp32, contiguous)
-            const int nr = min(RPH, p.T - q0);
-            for (int r = 0; r < nr; ++r)
-              tc::prefetch_l2(p.a_ref + ((int64_t)row0 + q0 + r) * (int64_t)(p.Hq * DH) + h0 * DH,
-                              HPT * DH * 4);
-          }
         }
         for (int j = 0; j < tl.nkb; ++j, ++gi) {
           const int st = gi % NST;
@@ -265,30 +259,43 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
         tc::umma_commit(&bars->v_empty[vs]);
         return true;
       };
-      for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); ok && k < ntiles;
-           k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
-        const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
-        // Q of this tile into TMEM once the previous tile's last S (which read the old Q) is done.
-        if (g0 > 0 && !tc::mbar_wait(&bars->s_full, (g0 - 1) & 1, abort, p.status)) break;
-        if (!tc::mbar_wait(&bars->q_full, tc_ & 1, abort, p.status)) break;
+      // Q of tile t into TMEM (its TMA load landed; the previous Q is no longer read).
+      auto load_q = [&](int t) -> bool {
+        if (!tc::mbar_wait(&bars->q_full, t & 1, abort, p.status)) return false;
         tc::fence_after_sync();
-        {
-          const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
+        const uint32_t q_base = tc::smem_u32(smem + L::Q_OFF);
 #pragma unroll
-          for (int kk = 0; kk < DH / 16; ++kk)
-            tc::tmem_cp_128x256b(tmem + L::Q_COL + kk * 8,
-                                 tc::sdesc_kmajor_sw128(q_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
-          tc::umma_commit(&bars->q_empty);
-        }
-        // S runs one block ahead of P V.
-        ok = issue_s(g0);
+        for (int kk = 0; kk < DH / 16; ++kk)
+          tc::tmem_cp_128x256b(tmem + L::Q_COL + kk * 8,
+                               tc::sdesc_kmajor_sw128(q_base + (kk >> 2) * L::CHUNK + (kk & 3) * 32));
+        tc::umma_commit(&bars->q_empty);
+        return true;
+      };
+      // S runs one block ahead of P V, across tile boundaries too: the next tile's Q and first S
+      // are issued before this tile's last P V, so the softmax finds S ready when it starts the
+      // next tile. The new Q may replace the old one once the softmax has read this tile's last S
+      // (that S has then completed).
+      int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x);
+      if (k < ntiles) ok = load_q(0) && issue_s(0);
+      while (ok && k < ntiles) {
+        const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
+        const int kn = sched_tile(it + 1, gridDim.x, blockIdx.x);
         for (int j = 0; ok && j < tl.nkb; ++j) {
-          if (j + 1 < tl.nkb && !issue_s(g0 + j + 1)) { ok = false; break; }
-          if (!issue_pv(g0 + j, j == 0)) { ok = false; break; }
+          const int gg = g0 + j;
+          if (j + 1 < tl.nkb) {
+            ok = issue_s(gg + 1);
+          } else if (kn < ntiles) {
+            ok = tc::mbar_wait(&bars->s_empty, gg & 1, abort, p.status) && load_q(tc_ + 1) &&
+                 issue_s(gg + 1);
+          }
+          ok = ok && issue_pv(gg, j == 0);
         }
         if (!ok) break;
         tc::umma_commit(&bars->o_full[tc_ & 1]);
         g0 += tl.nkb;
+        ++tc_;
+        k = kn;
+        ++it;
       }
       tc::umma_commit(&bars->drain);
       drain_wait(&bars->drain, 0);
@@ -465,6 +472,16 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
     uint32_t range_bits = 0;  // mode 2: an fp16 dO value out of range (inf) or NaN
     const int64_t ext_a = (int64_t)p.B * p.T * p.Hq * DH;         // A_ref, A, dO elements
     const int64_t ext_p = (int64_t)p.C * p.B * p.Hq * p.nP;       // loss partials
+    // A_ref row segment (DH fp32) of this thread's stacked row of tile k into L2, one line at a time
+    auto prefetch_aref = [&](int k) {
+      const StackTile tn = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
+      const int tt = tn.qb * RPH + (row & (RPH - 1));
+      if (tt >= p.T) return;
+      const float* src = p.a_ref + ((int64_t)(tn.bc % p.B) * p.T + tt) * (int64_t)(p.Hq * DH) +
+                         (HPT * tn.hu + row / RPH) * DH;
+#pragma unroll
+      for (int l = 0; l < DH / 32; ++l) tc::prefetch_line_l2(src + 32 * l);
+    };
     for (int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x); k < ntiles;
          k = sched_tile(++it, gridDim.x, blockIdx.x), ++tc_) {
       if (*abort) break;
@@ -474,6 +491,11 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       const int q0 = tl.qb * RPH;
       const int t = q0 + (row & (RPH - 1));
       const int row0 = b * p.T;
+      if (MODE != 0) {  // A_ref of this tile (the first one) and of the next, a whole tile ahead
+        if (it == 0) prefetch_aref(k);
+        const int kn = sched_tile(it + 1, gridDim.x, blockIdx.x);
+        if (kn < ntiles) prefetch_aref(kn);
+      }
       const int ob = tc_ & 1;
       const uint32_t ph = (tc_ >> 1) & 1;
       double acc = 0.0;

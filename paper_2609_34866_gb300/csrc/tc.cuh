@@ -391,6 +391,12 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
+// Hint: bring the 128-byte line holding `src` into L2 (an ordinary load-store-unit prefetch: it
+// does not queue in the TMA unit behind, or ahead of, the bulk tensor copies).
+__device__ __forceinline__ void prefetch_line_l2(const void* src) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(src)));
+}
+
 // Hint: bring `bytes` (a multiple of 16, 16-byte aligned source) of global memory into L2.
 __device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)),
