@@ -58,7 +58,9 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 // softmax warps already work on tile i + 1.
 //   warp 0       TMA: Q tile, K ring (3 stages: a K load is issued once S two blocks back has
 //                completed and must land before S of the block after next)
-//   warp 1       TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread)
+//   warp 1       TMEM owner, tcgen05.cp of Q, UMMA issuer (one thread): S, and for d_h = 64 also
+//                P V; for d_h = 128 warp 15 issues P V (two issuers, so that S of the next block
+//                is not held back behind the issue of P V, and vice versa)
 //   warps 2..9   softmax: warp (quarter q, half h) owns the 16 rows at lanes 32 q + 16 h; with the
 //                16x256b TMEM shape four threads share a row (32 of its 128 scores each, two rows per
 //                thread), so row maxima and sums need only warp shuffles. Lazy rescaling as in the
@@ -69,13 +71,19 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 //                stores are coalesced; per-mode outputs and the SSE partials. Each thread
 //                prefetches its row of the next tile's A_ref into L2 a whole tile ahead.
 constexpr int SQ = 64, SKB = 128, SK_ST = 3, SV_ST = 2;
-constexpr int PAIR_THREADS = 480;
+// d_h = 128: S and P V are issued by two threads (warp 1 and PV_WARP), so that S of the next block
+// never waits behind the issue of the current P V. d_h = 64: one issuer (measured faster there).
+template <int DH> struct Issue {
+  static constexpr bool kSplit = DH == 128;
+  static constexpr int kThreads = kSplit ? 512 : 480;
+};
+constexpr int PV_WARP = 15;
 constexpr int EPI_WARPS = 4, EPI_WARP0 = 11;
 
 struct StackBars {
   uint64_t q_full, q_empty, k_full[SK_ST], k_empty[SK_ST], v_full[SV_ST], v_empty[SV_ST];
   uint64_t s_full, s_empty, p_full, pv_done, o_full[2], o_empty[2], st_full[2], st_empty[2];
-  uint64_t drain;
+  uint64_t drain, drain_pv;
   uint32_t tmem_base;
   int abort;
   double red[2][EPI_WARPS];         // [tile parity][epilogue warp]
@@ -121,7 +129,7 @@ __device__ __forceinline__ StackTile stack_tile(int k, int units, int Hkv, int n
 // HPT = query heads per tile: 2 stacks 64 rows of two heads of one KV group (even GQA ratio), 1
 // takes 128 rows of one head (any ratio, e.g. GPT-2's separate heads).
 template <int DH, int MODE, int HPT>
-__global__ void __launch_bounds__(PAIR_THREADS, 1)
+__global__ void __launch_bounds__(Issue<DH>::kThreads, 1)
     attn_fwd_pair_kernel(const __grid_constant__ CUtensorMap tm_q,
                          const __grid_constant__ CUtensorMap tm_kv, const FwdParams p) {
   using L = StackLayout<DH>;
@@ -159,6 +167,7 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       tc::mbar_init(&bars->st_empty[i], EPI_WARPS);
     }
     tc::mbar_init(&bars->drain, 1);
+    tc::mbar_init(&bars->drain_pv, 1);
     bars->abort = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_q);
@@ -217,8 +226,8 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
           if (iss & (1u << st)) drain_wait(&full[st], (par >> st) & 1);
       }
     }
-  } else if (warp == 1) {
-    if (lane == 0) {  // ---------------------------------------------------------------- UMMA
+  } else if (warp == 1 || (Issue<DH>::kSplit && warp == PV_WARP)) {
+    if (lane == 0) {  // ------------------------------------------ UMMA: S (warp 1), P V (PV_WARP)
       constexpr uint32_t ID_S = tc::idesc_f16(false, 128, SKB);
       constexpr uint32_t ID_PV = tc::idesc_f16(false, 128, DH) | (1u << 16);  // B = V, MN-major
       int g0 = 0, tc_ = 0;
@@ -276,29 +285,42 @@ __global__ void __launch_bounds__(PAIR_THREADS, 1)
       // next tile. The new Q may replace the old one once the softmax has read this tile's last S
       // (that S has then completed).
       int it = 0, k = sched_tile(0, gridDim.x, blockIdx.x);
-      if (k < ntiles) ok = load_q(0) && issue_s(0);
-      while (ok && k < ntiles) {
-        const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
-        const int kn = sched_tile(it + 1, gridDim.x, blockIdx.x);
-        for (int j = 0; ok && j < tl.nkb; ++j) {
-          const int gg = g0 + j;
-          if (j + 1 < tl.nkb) {
-            ok = issue_s(gg + 1);
-          } else if (kn < ntiles) {
-            ok = tc::mbar_wait(&bars->s_empty, gg & 1, abort, p.status) && load_q(tc_ + 1) &&
-                 issue_s(gg + 1);
+      if (warp == 1) {
+        if (k < ntiles) ok = load_q(0) && issue_s(0);
+        while (ok && k < ntiles) {
+          const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
+          const int kn = sched_tile(it + 1, gridDim.x, blockIdx.x);
+          for (int j = 0; ok && j < tl.nkb; ++j) {
+            const int gg = g0 + j;
+            if (j + 1 < tl.nkb) {
+              ok = issue_s(gg + 1);
+            } else if (kn < ntiles) {
+              ok = tc::mbar_wait(&bars->s_empty, gg & 1, abort, p.status) && load_q(tc_ + 1) &&
+                   issue_s(gg + 1);
+            }
+            if (!Issue<DH>::kSplit) ok = ok && issue_pv(gg, j == 0);
           }
-          ok = ok && issue_pv(gg, j == 0);
+          if (!ok) break;
+          if (!Issue<DH>::kSplit) tc::umma_commit(&bars->o_full[tc_ & 1]);
+          g0 += tl.nkb;
+          ++tc_;
+          k = kn;
+          ++it;
         }
-        if (!ok) break;
-        tc::umma_commit(&bars->o_full[tc_ & 1]);
-        g0 += tl.nkb;
-        ++tc_;
-        k = kn;
-        ++it;
+      } else {
+        while (ok && k < ntiles) {
+          const StackTile tl = stack_tile(k, units, p.Hkv, nqb, p.T, RPH);
+          for (int j = 0; ok && j < tl.nkb; ++j) ok = issue_pv(g0 + j, j == 0);
+          if (!ok) break;
+          tc::umma_commit(&bars->o_full[tc_ & 1]);
+          g0 += tl.nkb;
+          ++tc_;
+          k = sched_tile(++it, gridDim.x, blockIdx.x);
+        }
       }
-      tc::umma_commit(&bars->drain);
-      drain_wait(&bars->drain, 0);
+      uint64_t* dr = warp == 1 ? &bars->drain : &bars->drain_pv;
+      tc::umma_commit(dr);
+      drain_wait(dr, 0);
     }
   } else if (warp < EPI_WARP0) {  // ------------------------------------------------------ softmax
     const int quarter = warp & 3;
@@ -656,7 +678,8 @@ cudaError_t launch_fwd_pair(const CUtensorMap& tq, const CUtensorMap& tkv, const
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  attn_fwd_pair_kernel<DH, MODE, HPT><<<grid, PAIR_THREADS, StackLayout<DH>::SMEM, st>>>(tq, tkv, p);
+  attn_fwd_pair_kernel<DH, MODE, HPT><<<grid, Issue<DH>::kThreads, StackLayout<DH>::SMEM, st>>>(tq,
+                                                                                      tkv, p);
   return cudaGetLastError();
 }
 
