@@ -27,7 +27,9 @@ namespace {
 
 constexpr int EW_WARPS = 8;       // dq: epilogue warps
 constexpr int DKDV_EW = 16;       // dK/dV: elementwise warps, 16 key rows x 64 queries each
-constexpr int DKDV_THREADS = (2 + DKDV_EW + 1) * 32;  // warp 0 TMA, 1 UMMA, 2..17 elementwise, 18 stores
+// warp 0 TMA, 1 UMMA (S^T, dP^T), 2..17 elementwise, 18 stores, 19 UMMA (dV, dK)
+constexpr int DKDV_THREADS = (2 + DKDV_EW + 2) * 32;
+constexpr int DKDV_GRAD_WARP = 3 + DKDV_EW;
 constexpr int kSuperGroup = 8;  // (KV head, sequence) pairs whose dK/dV CTAs are interleaved
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -136,12 +138,19 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
 // 128-query blocks, so that every UMMA runs at N = 128 (an N = 64 UMMA costs the tensor pipe as much
 // time as an N = 128 one). Tensor memory: S^T = K Q^T at column 0 and dP^T = V dO^T at 128 (SS form:
 // K and V stay in shared memory for the whole tile), dV at 256, dK at 256 + DH. The elementwise warps
-// write P^T and dS^T back as packed fp16 over the first 64 columns of S^T and dP^T, where the TS-form
-// gradient UMMAs dV += P^T dO and dK += dS^T Q read them as their A operand. With no room for a second
-// S^T / dP^T buffer, the issuer orders the tensor pipe as
-//   dV(j), S^T(j+1), dK(j), dP^T(j+1), dV(j+1), ...
-// S^T(j+1) going out once dV(j) has completed (it overwrites the P^T(j) columns) and dP^T(j+1) once
-// dK(j) has; the elementwise warps compute P^T(j+1) while dK(j) and dP^T(j+1) run.
+// write P^T and dS^T back as packed fp16 into S^T and dP^T, where the TS-form gradient UMMAs
+// dV += P^T dO and dK += dS^T Q read them as their A operand: the 64 queries of half h (whose fp32
+// scores are columns 64 h .. 64 h + 63, read by the warps of that half) go to packed columns
+// 64 h .. 64 h + 31, so a warp writes only columns that it has itself read (warps of the two halves
+// are not synchronised with each other). With no room for a second
+// S^T / dP^T buffer, S^T(j+1) goes out once dV(j) has completed (it overwrites the P^T(j) columns)
+// and dP^T(j+1) once dK(j) has; the elementwise warps compute P^T(j+1) while dK(j) and dP^T(j+1)
+// run. The score products (S^T, dP^T) and the gradient products (dV, dK) are issued by two threads,
+// so that neither waits behind the issue of the other.
+
+// TMEM column of the K-step k (queries 16 k .. 16 k + 15) of packed P^T or dS^T.
+__device__ __forceinline__ uint32_t pk_col(int k) { return (uint32_t)((k >> 2) * 64 + (k & 3) * 8); }
+
 template <int DH>
 struct DkdvLayout {
   static constexpr int BK = 128, BQ = 128, STAGES = 2;
@@ -167,7 +176,7 @@ struct DkdvLayout {
 
 struct DkdvBars {
   uint64_t kv_full, ld_full[2], ld_empty[2], s_full, dp_full, p_full, ds_full, dv_done, dk_done;
-  uint64_t o_full, drain, dss_full, dss_free;
+  uint64_t o_full, drain, drain_g, dss_full, dss_free;
   uint32_t tmem_base;
   int abort;
 };
@@ -223,6 +232,7 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
     tc::mbar_init(&bars->dk_done, 1);
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
+    tc::mbar_init(&bars->drain_g, 1);
     tc::mbar_init(&bars->dss_full, DKDV_EW);  // the block's dS^T is in the staging tile
     tc::mbar_init(&bars->dss_free, 1);         // the store warp's TMA stores have read it
     bars->abort = 0;
@@ -293,25 +303,27 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
           if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
       }
     }
-  } else if (warp == 1) {
-    if (lane == 0) {  // ------------------------------------------------------------- UMMA
+  } else if (warp == 1 || warp == DKDV_GRAD_WARP) {
+    if (lane == 0) {  // ---------------------- UMMA: S^T, dP^T (warp 1); dV, dK (DKDV_GRAD_WARP)
+      // Two issuing threads, so that the score products of the next block are never held back
+      // behind the issue of this block's gradient products, nor the other way round. Every
+      // dependency between them goes through a barrier: S^T(j) overwrites P^T(j - 1), so it waits
+      // for dV(j - 1); dP^T(j) overwrites dS^T(j - 1), so it waits for dK(j - 1).
       constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
       constexpr uint32_t ID_G = tc::idesc_f16(false, BK, DH) | (1u << 16);  // B MN-major
-      const uint64_t ka = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF));
-      const uint64_t va = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::V_OFF));
       bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
-      // Event-driven issue in the order dV(j), S^T(j+1), dK(j), dP^T(j+1): ns, nd, nv, nk count
-      // the S^T, dP^T, dV and dK UMMA groups issued so far.
-      int ns = 0, nd = 0, nv = 0, nk = 0;
-      tc::Watchdog wd;
-      while (ok && nk < n_it) {
-        bool prog = false;
-        // S^T(ns): its Q has landed and dV(ns - 1) has read P^T(ns - 1) out of the S^T columns.
-        if (ns < n_it && nv == ns && tc::mbar_ready(&bars->ld_full[ns % STAGES], (ns / STAGES) & 1) &&
-            (ns == 0 || tc::mbar_ready(&bars->dv_done, (ns - 1) & 1))) {
+      if (warp == 1) {
+        const uint64_t ka = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::K_OFF));
+        const uint64_t va = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::V_OFF));
+        for (int j = 0; ok && j < n_it; ++j) {
+          const int st = j % STAGES;
+          // S^T(j) = K Q(j)^T: its Q has landed and dV(j - 1) has read P^T(j - 1).
+          ok = tc::mbar_wait(&bars->ld_full[st], (j / STAGES) & 1, abort, p.status) &&
+               (j == 0 || tc::mbar_wait(&bars->dv_done, (j - 1) & 1, abort, p.status));
+          if (!ok) break;
           tc::fence_after_sync();
           const uint64_t bq = tc::sdesc_kmajor_sw128(
-              tc::smem_u32(smem + L::ST_OFF + (ns % STAGES) * L::ST_STRIDE + L::ST_Q));
+              tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_Q));
 #pragma unroll
           for (int k = 0; k < DH / 16; ++k) {
             const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
@@ -319,14 +331,12 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
                          k > 0 ? 1u : 0u);
           }
           tc::umma_commit(&bars->s_full);
-          ++ns;
-          prog = true;
-        }
-        // dP^T(nd): after S^T(nd) (same stage) and once dK(nd - 1) has read dS^T(nd - 1).
-        if (nd < ns && nk == nd && (nd == 0 || tc::mbar_ready(&bars->dk_done, (nd - 1) & 1))) {
+          // dP^T(j) = V dO(j)^T once dK(j - 1) has read dS^T(j - 1).
+          ok = j == 0 || tc::mbar_wait(&bars->dk_done, (j - 1) & 1, abort, p.status);
+          if (!ok) break;
           tc::fence_after_sync();
           const uint64_t bd = tc::sdesc_kmajor_sw128(
-              tc::smem_u32(smem + L::ST_OFF + (nd % STAGES) * L::ST_STRIDE + L::ST_DO));
+              tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_DO));
 #pragma unroll
           for (int k = 0; k < DH / 16; ++k) {
             const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
@@ -334,45 +344,41 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
                          k > 0 ? 1u : 0u);
           }
           tc::umma_commit(&bars->dp_full);
-          ++nd;
-          prog = true;
         }
-        // dV(nv) += P^T(nv) dO(nv) once the elementwise warps have written P^T(nv).
-        if (nv < ns && tc::mbar_ready(&bars->p_full, nv & 1)) {
+      } else {
+        for (int j = 0; ok && j < n_it; ++j) {
+          const int st = j % STAGES;
+          // dV += P^T(j) dO(j) once the elementwise warps have written P^T(j).
+          ok = tc::mbar_wait(&bars->p_full, j & 1, abort, p.status);
+          if (!ok) break;
           tc::fence_after_sync();
           const uint64_t bd = tc::sdesc_mnmajor_sw128(
-              tc::smem_u32(smem + L::ST_OFF + (nv % STAGES) * L::ST_STRIDE + L::ST_DO), L::CHUNK, 1024);
+              tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_DO), L::CHUNK, 1024);
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k)
-            tc::umma_f16_ts(tmem + L::DV_COL, tmem + L::S_COL + k * 8, tc::sdesc_advance(bd, k * 16 * 128),
-                            ID_G, (nv > 0 || k > 0) ? 1u : 0u);
+            tc::umma_f16_ts(tmem + L::DV_COL, tmem + L::S_COL + pk_col(k), tc::sdesc_advance(bd, k * 16 * 128),
+                            ID_G, (j > 0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->dv_done);
-          ++nv;
-          prog = true;
-        }
-        // dK(nk) += dS^T(nk) Q(nk) once dS^T(nk) is written, behind S^T(nk + 1) in the pipe.
-        if (nk < nd && (ns > nk + 1 || ns == n_it) && tc::mbar_ready(&bars->ds_full, nk & 1)) {
+          // dK += dS^T(j) Q(j) once dS^T(j) is written.
+          ok = tc::mbar_wait(&bars->ds_full, j & 1, abort, p.status);
+          if (!ok) break;
           tc::fence_after_sync();
-          const int st = nk % STAGES;
           const uint64_t bq = tc::sdesc_mnmajor_sw128(
               tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE + L::ST_Q), L::CHUNK, 1024);
 #pragma unroll
           for (int k = 0; k < BQ / 16; ++k)
-            tc::umma_f16_ts(tmem + L::DK_COL, tmem + L::DP_COL + k * 8, tc::sdesc_advance(bq, k * 16 * 128),
-                            ID_G, (nk > 0 || k > 0) ? 1u : 0u);
+            tc::umma_f16_ts(tmem + L::DK_COL, tmem + L::DP_COL + pk_col(k), tc::sdesc_advance(bq, k * 16 * 128),
+                            ID_G, (j > 0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->dk_done);
-          tc::umma_commit(&bars->ld_empty[st]);  // dV(nk) and dK(nk) were the stage's last readers
-          if (nk == n_it - 1) tc::umma_commit(&bars->o_full);
-          ++nk;
-          prog = true;
+          // dV(j) and dK(j) are the stage's last readers (S^T(j) and dP^T(j) completed before the
+          // elementwise warps released P^T(j) and dS^T(j))
+          tc::umma_commit(&bars->ld_empty[st]);
+          if (j == n_it - 1) tc::umma_commit(&bars->o_full);
         }
-        if (prog)
-          wd.progress();
-        else if (!wd.tick(abort, p.status))
-          ok = false;
       }
-      tc::umma_commit(&bars->drain);
-      drain_wait(&bars->drain, 0);
+      uint64_t* dr = warp == 1 ? &bars->drain : &bars->drain_g;
+      tc::umma_commit(dr);
+      drain_wait(dr, 0);
     }
   } else if (warp == 2 + DKDV_EW) {
     if (lane == 0) {  // ------------------------------------------ dS^T tiles to global memory
@@ -451,14 +457,14 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
         x[4 * n + 3] = pb[1];
       }
       {
-        uint32_t pw[16];  // pw[2n] row A, pw[2n + 1] row B: packed column 32 chalf + 4n + cq
+        uint32_t pw[16];  // pw[2n] row A, pw[2n + 1] row B: packed column 64 chalf + 4n + cq
 #pragma unroll
         for (int n = 0; n < 8; ++n) {
           pw[2 * n] = tc::pack_half2(x[4 * n], x[4 * n + 1]);
           pw[2 * n + 1] = tc::pack_half2(x[4 * n + 2], x[4 * n + 3]);
         }
         __syncwarp();
-        tc::tmem_st_16x128b_x8(tmem + lane16 + L::S_COL + 32 * chalf, pw);
+        tc::tmem_st_16x128b_x8(tmem + lane16 + L::S_COL + 64 * chalf, pw);
         tc::tmem_st_wait();
       }
       tc::fence_before_sync();
@@ -493,7 +499,7 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
         }
       }
       __syncwarp();
-      tc::tmem_st_16x128b_x8(tmem + lane16 + L::DP_COL + 32 * chalf, dw);
+      tc::tmem_st_16x128b_x8(tmem + lane16 + L::DP_COL + 64 * chalf, dw);
       tc::tmem_st_wait();
       tc::fence_before_sync();
       __syncwarp();

@@ -52,40 +52,6 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Non-blocking test of a barrier phase (never suspends the thread): for issuers that poll several
-// barriers and act on whichever is ready.
-__device__ __forceinline__ bool mbar_ready(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Progress watchdog of a polling issuer: call tick() once per idle pass; it returns false (and
-// raises JAB_ERR_TIMEOUT, sets *abort) once no progress was made for kWaitLimitNs.
-struct Watchdog {
-  uint64_t t0;
-  uint32_t idle;
-  __device__ __forceinline__ Watchdog() : t0(globaltimer()), idle(0) {}
-  __device__ __forceinline__ void progress() { idle = 0; }
-  __device__ __forceinline__ bool tick(volatile int* abort, int* status) {
-    if (idle++ == 0) t0 = globaltimer();
-    if ((idle & 63u) == 0) {
-      if (*abort) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
-        *abort = 1;
-        report(status, JAB_ERR_TIMEOUT);
-        return false;
-      }
-    }
-    return true;
-  }
-};
 
 // Bounded wait. Returns false (and sets *abort) when the barrier did not flip within the limit or
 // another role of the CTA already aborted.
