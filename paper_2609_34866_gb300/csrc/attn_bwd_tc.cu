@@ -146,7 +146,8 @@ __device__ __forceinline__ void store_tile(const bf16_t* tile, bf16_t* dst, int6
 // S^T / dP^T buffer, S^T(j+1) goes out once dV(j) has completed (it overwrites the P^T(j) columns)
 // and dP^T(j+1) once dK(j) has; the elementwise warps compute P^T(j+1) while dK(j) and dP^T(j+1)
 // run. The score products (S^T, dP^T) and the gradient products (dV, dK) are issued by two threads,
-// so that neither waits behind the issue of the other.
+// so that neither waits behind the issue of the other; dK(j) enters the pipe only after S^T(j+1)
+// has been issued, since the elementwise warps wait for S^T(j+1) and nothing waits for dK(j) sooner.
 
 // TMEM column of the K-step k (queries 16 k .. 16 k + 15) of packed P^T or dS^T.
 __device__ __forceinline__ uint32_t pk_col(int k) { return (uint32_t)((k >> 2) * 64 + (k & 3) * 8); }
@@ -176,7 +177,7 @@ struct DkdvLayout {
 
 struct DkdvBars {
   uint64_t kv_full, ld_full[2], ld_empty[2], s_full, dp_full, p_full, ds_full, dv_done, dk_done;
-  uint64_t o_full, drain, drain_g, dss_full, dss_free;
+  uint64_t o_full, drain, drain_g, dss_full, dss_free, s_issued;
   uint32_t tmem_base;
   int abort;
 };
@@ -233,6 +234,7 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
     tc::mbar_init(&bars->o_full, 1);
     tc::mbar_init(&bars->drain, 1);
     tc::mbar_init(&bars->drain_g, 1);
+    tc::mbar_init(&bars->s_issued, 1);
     tc::mbar_init(&bars->dss_full, DKDV_EW);  // the block's dS^T is in the staging tile
     tc::mbar_init(&bars->dss_free, 1);         // the store warp's TMA stores have read it
     bars->abort = 0;
@@ -331,6 +333,7 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
                          k > 0 ? 1u : 0u);
           }
           tc::umma_commit(&bars->s_full);
+          tc::mbar_arrive(&bars->s_issued);  // dK(j - 1) may now queue behind S^T(j)
           // dP^T(j) = V dO(j)^T once dK(j - 1) has read dS^T(j - 1).
           ok = j == 0 || tc::mbar_wait(&bars->dk_done, (j - 1) & 1, abort, p.status);
           if (!ok) break;
@@ -360,7 +363,9 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
                             ID_G, (j > 0 || k > 0) ? 1u : 0u);
           tc::umma_commit(&bars->dv_done);
           // dK += dS^T(j) Q(j) once dS^T(j) is written.
-          ok = tc::mbar_wait(&bars->ds_full, j & 1, abort, p.status);
+          // dK(j) goes into the pipe behind S^T(j + 1), which the elementwise warps wait for
+          ok = tc::mbar_wait(&bars->ds_full, j & 1, abort, p.status) &&
+               (j + 1 == n_it || tc::mbar_wait(&bars->s_issued, (j + 1) & 1, abort, p.status));
           if (!ok) break;
           tc::fence_after_sync();
           const uint64_t bq = tc::sdesc_mnmajor_sw128(
