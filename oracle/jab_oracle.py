@@ -22,7 +22,8 @@ Readings of points the paper leaves open (each is stated where it is used):
   R1  w/s is the IEEE fp32 quotient and round() is round-half-to-even.
   R2  the code range is symmetric [-qmax, qmax], qmax = 2^(b-1) - 1.
   R3  the MSE term is an element-wise mean over B*T*(Hq*d_h) entries; SSE is also returned.
-  R4  only the MSE term (lambda_KL = 0) is on this path.
+  R4  the hot path's loss is the MSE term (lambda_KL = 0); jab_loss_joint and
+      jab_loss_joint_and_grad add lambda_KL times the KL term (R18) and its gradient.
   R5  the LSQ branch tests |v| <= qmax on the unrounded quotient v.
   R6  n_w in (n_w * qmax)^(-1/2) is the group size G; it is exposed as kappa.
   R7  RoPE is the rotate-half convention with inv_freq_j = theta^(-2j/d_h).
@@ -304,11 +305,13 @@ def jab_loss_joint(x, w, s, bits: int, desc: dict, lam_kl: float = 0.1):
 # 6. Backward: attention VJP, STE on w_hat, LSQ rule on s (App. B "Joint STE fine-tuning", Eq. 13)
 # --------------------------------------------------------------------------------------------
 
-def attention_vjp(q, k, v, P, dO, scale: float):
+def attention_vjp(q, k, v, P, dO, scale: float, dS_extra=None):
     """Vector-Jacobian product of causal GQA attention.
 
     dV = P^T dO, dP = dO V^T, dS = P * (dP - rowsum(dP * P)), dQ = dS K * scale,
     dK = dS^T Q * scale; key/value gradients are summed over the query heads of a group.
+    dS_extra [B, Hq, T, T] (optional) is a gradient of the loss with respect to the scaled scores
+    S = Q K^T * scale that does not pass through O (the KL term of Eq. 3); it is added to dS.
     """
     B, T, Hq, dh = q.shape
     Hkv = k.shape[2]
@@ -323,6 +326,8 @@ def attention_vjp(q, k, v, P, dO, scale: float):
             dv[b, :, g, :] += Ph.T @ dOh
             dP = dOh @ v[b, :, g, :].T
             dS = Ph * (dP - (dP * Ph).sum(axis=1, keepdims=True))
+            if dS_extra is not None:
+                dS = dS + dS_extra[b, h]
             dq[b, :, h, :] = (dS @ k[b, :, g, :]) * scale
             dk[b, :, g, :] += (dS.T @ q[b, :, h, :]) * scale
     return dq, dk, dv
@@ -375,6 +380,50 @@ def jab_loss_and_grad(x, w, s, bits: int, desc: dict, a_ref=None, kappa: float =
     grad_s = kappa * (grad_w_hat * r).reshape(D, d // G, G).sum(axis=2)
     return dict(loss=sse / n_el, sse=sse, grad_s=grad_s, grad_w_hat=grad_w_hat, codes=codes,
                 w_hat=w_hat, a_ref=a_ref, a_hat=a_hat, lse=parts["lse"])
+
+
+def jab_loss_joint_and_grad(x, w, s, bits: int, desc: dict, lam_kl: float = 0.1, kappa: float = 1.0):
+    """Eq. 3 with both terms (readings R3, R18) and its STE / LSQ gradient w.r.t. the scales.
+
+    L = MSE + lam_kl * KL with KL = sum over (sequence, query head, query row) of
+    D_KL(P_row || Q_row) / B, P the teacher's map and Q the student's. Q_row = softmax(s_row) of the
+    student's scaled scores s = Q K^T * scale, so d KL_row / d s_row = Q_row - P_row (the gradient
+    of log-sum-exp minus the P-weighted scores); the KL term reaches the weights only through the
+    student's scores, and adds (lam_kl / B) (Q - P) to the score gradient of the MSE term's
+    attention VJP. Then the transpose of RoPE, dL/dw_hat = dQKV^T X and the LSQ rule (Eq. 13) as in
+    jab_loss_and_grad. Returns dict(loss, mse, kl, grad_s, grad_w_hat).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    G = desc["group_size"]
+    Hq, Hkv, dh = desc["n_q_heads"], desc["n_kv_heads"], desc["head_dim"]
+    B, T, d = x.shape
+    codes, w_hat, v = quantize(w, s, bits, G)
+    a_ref, teacher = block_forward(x, w, desc, return_parts=True)
+    a_hat, student = block_forward(x, w_hat, desc, return_parts=True)
+    n_el = B * T * Hq * dh
+    diff = a_hat - a_ref
+    mse = float((diff ** 2).sum()) / n_el
+    P, Qs = teacher["P"], student["P"]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        kl = float(np.where(P > 0, P * (np.log(P) - np.log(Qs)), 0.0).sum()) / B
+    dO = (2.0 / n_el) * diff.reshape(B, T, Hq, dh)
+    dS_kl = (lam_kl / B) * (Qs - P)
+    dq, dk, dv = attention_vjp(student["q"], student["k"], student["v"], Qs, dO,
+                               _softmax_scale(desc), dS_extra=dS_kl)
+    if desc.get("use_rope", False):
+        cos, sin = rope_tables(T, dh, float(desc.get("rope_theta", 10000.0)))
+        dq = apply_rope_transpose(dq, cos, sin)
+        dk = apply_rope_transpose(dk, cos, sin)
+    dqkv = np.concatenate([dq.reshape(B, T, Hq * dh), dk.reshape(B, T, Hkv * dh),
+                           dv.reshape(B, T, Hkv * dh)], axis=2)
+    grad_w_hat = dqkv.reshape(B * T, -1).T @ x.reshape(B * T, d)
+    r = lsq_factor(v, bits)
+    if kappa is None or kappa <= 0:
+        kappa = default_kappa(bits, G)
+    D = grad_w_hat.shape[0]
+    grad_s = kappa * (grad_w_hat * r).reshape(D, d // G, G).sum(axis=2)
+    return dict(loss=mse + lam_kl * kl, mse=mse, kl=kl, grad_s=grad_s, grad_w_hat=grad_w_hat,
+                codes=codes, w_hat=w_hat, a_ref=a_ref, lse_ref=teacher["lse"])
 
 
 # --------------------------------------------------------------------------------------------

@@ -413,6 +413,84 @@ def test_scale_gradient_matches_lsq_surrogate_finite_differences(bits):
             np.testing.assert_allclose(g["grad_s"][o, gi], fd, rtol=2e-5, atol=1e-12)
 
 
+def _joint_at_w_hat(x, w_hat, desc, a_ref, P_teacher, lam):
+    """MSE + lam * KL at given quantized weights, the KL from scipy's elementwise relative entropy."""
+    special = pytest.importorskip("scipy.special")
+    a_hat, parts = O.block_forward(x, w_hat, desc, return_parts=True)
+    mse = ((a_hat - a_ref) ** 2).sum() / a_ref.size
+    kl = special.rel_entr(P_teacher, parts["P"]).sum() / x.shape[0]
+    return mse + lam * kl
+
+
+@pytest.mark.parametrize("rope,Hq,Hkv,lam", [(False, 2, 2, 0.1), (True, 2, 1, 0.1),
+                                             (True, 2, 1, 3e-4)])
+def test_joint_weight_gradient_matches_finite_differences(rope, Hq, Hkv, lam):
+    """dL/dw_hat of MSE + lam * KL (Eq. 3 with both terms, readings R3 and R18) against central
+    differences; lam = 3e-4 puts the two terms' gradients at comparable size on this block."""
+    desc, x, w = _tiny(rope=rope, Hq=Hq, Hkv=Hkv, T=5)
+    s = O.init_scales_absmax(w, 2, 4)
+    g = O.jab_loss_joint_and_grad(x, w, s, 2, desc, lam_kl=lam, kappa=1.0)
+    a_ref, w_hat = g["a_ref"], g["w_hat"]
+    _, teacher = O.block_forward(x, w, desc, return_parts=True)
+    P = teacher["P"]
+    np.testing.assert_allclose(g["loss"], _joint_at_w_hat(x, w_hat, desc, a_ref, P, lam), rtol=1e-12)
+    h = 1e-6
+    rng = np.random.default_rng(11)
+    idx = [tuple(i) for i in rng.integers(0, [w.shape[0], w.shape[1]], size=(24, 2))]
+    for i in idx:
+        wp, wm = w_hat.copy(), w_hat.copy()
+        wp[i] += h
+        wm[i] -= h
+        fd = (_joint_at_w_hat(x, wp, desc, a_ref, P, lam) -
+              _joint_at_w_hat(x, wm, desc, a_ref, P, lam)) / (2 * h)
+        np.testing.assert_allclose(g["grad_w_hat"][i], fd, rtol=1e-5, atol=1e-11)
+
+
+def test_joint_scale_gradient_matches_lsq_surrogate_finite_differences():
+    """The LSQ rule (Eq. 13) on the joint objective: central differences of the frozen-code
+    surrogate (as for the MSE term) of MSE + 0.1 KL equal grad_s (kappa = 1)."""
+    desc, x, w = _tiny(rope=True, T=5)
+    G, bits, lam = 4, 2, 0.1
+    s = O.init_scales_absmax(w, bits, G) * np.float32(0.8)
+    g = O.jab_loss_joint_and_grad(x, w, s, bits, desc, lam_kl=lam, kappa=1.0)
+    codes, w_hat, v = O.quantize(w, s, bits, G)
+    inside = np.abs(v) <= 1
+    a_ref = g["a_ref"]
+    _, teacher = O.block_forward(x, w, desc, return_parts=True)
+    h = 1e-7
+    for o in range(0, w.shape[0], 3):
+        for gi in range(w.shape[1] // G):
+            cols = slice(gi * G, (gi + 1) * G)
+
+            def surrogate(sp):
+                wh = w_hat.copy()
+                wh[o, cols] = np.where(inside[o, cols],
+                                       sp * codes[o, cols] + w[o, cols] * (1 - sp / float(s[o, gi])),
+                                       sp * np.sign(v[o, cols]))
+                return _joint_at_w_hat(x, wh, desc, a_ref, teacher["P"], lam)
+
+            s0 = float(s[o, gi])
+            fd = (surrogate(s0 + h) - surrogate(s0 - h)) / (2 * h)
+            np.testing.assert_allclose(g["grad_s"][o, gi], fd, rtol=2e-5, atol=1e-12)
+
+
+def test_joint_gradient_reduces_to_the_mse_gradient_and_splits_into_its_terms():
+    """lam = 0 gives the MSE term's loss and gradient; the KL value is kl_attention_term's; and the
+    gradient is linear in lam (the KL term's gradient does not depend on lam)."""
+    desc, x, w = _tiny(rope=True, T=6)
+    s = O.init_scales_absmax(w, 3, 4)
+    g0 = O.jab_loss_joint_and_grad(x, w, s, 3, desc, lam_kl=0.0)
+    ref = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=1.0)
+    np.testing.assert_allclose(g0["loss"], ref["loss"], rtol=1e-13)
+    np.testing.assert_allclose(g0["grad_s"], ref["grad_s"], rtol=1e-11, atol=1e-16)
+    g1 = O.jab_loss_joint_and_grad(x, w, s, 3, desc, lam_kl=0.1)
+    g2 = O.jab_loss_joint_and_grad(x, w, s, 3, desc, lam_kl=0.2)
+    np.testing.assert_allclose(g1["kl"], O.kl_attention_term(x, w, s, 3, desc)["kl"], rtol=1e-13)
+    np.testing.assert_allclose(g2["grad_s"] - g1["grad_s"], g1["grad_s"] - g0["grad_s"],
+                               rtol=1e-9, atol=1e-15)
+    assert np.abs(g1["grad_s"] - g0["grad_s"]).max() > 1e-3 * np.abs(g0["grad_s"]).max()
+
+
 def test_kappa_is_a_pure_multiplier_and_default():
     desc, x, w = _tiny(rope=True)
     s = O.init_scales_absmax(w, 3, 4)
