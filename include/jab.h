@@ -202,6 +202,31 @@ jab_status jab_loss_backward_scales_prepared(const jab_block_desc* desc, int32_t
                                              double* loss_dev, float* grad_scales_dev, void* ws,
                                              size_t ws_bytes, jab_stream_t stream);
 
+/* The STE / LSQ scale gradient of the joint objective of Eq. 3, L = MSE + lambda_kl * KL, with the
+ * KL term D_KL(P || Q) between the teacher's attention map P and the student's Q in the batchmean
+ * normalisation (App. B "Effective weight of the KL term"; the paper's default lambda_kl = 0.1,
+ * Section 3). The KL term adds (lambda_kl / B)(Q - P) to the gradient with respect to the student's
+ * scaled scores (P, Q: post-softmax maps), which then flows through the same dQ / dK products,
+ * the transpose of RoPE, the weight-gradient GEMM and the LSQ rule (Eq. 13) as the MSE term's.
+ *   QKV_ref_dev    fp16 [B, T, (Hq + 2 Hkv) * d_h] from jab_reference_projection (same X and W),
+ *                  16-byte aligned
+ *   lse_ref_dev    fp32 [B, Hq, T]: the teacher's row log-sum-exp from jab_reference_forward
+ *                  (natural log, scaled scores)
+ *   lambda_kl      >= 0 (0 gives jab_loss_backward_scales' gradient through the KL code path)
+ *   loss_dev       out fp64 [1]   MSE + lambda_kl * KL
+ *   kl_dev         out fp64 [1] or NULL   the KL term (nats, batchmean)
+ * Other arguments, layouts and errors as for jab_loss_backward_scales (X is converted by the call);
+ * ws of jab_workspace_size(desc, B, T, 1, 1) bytes. The score gradient is held in fp16 tiles as
+ * a P (dP - D) + b (P - P_teacher) with b / a = lambda_kl B T Hq d_h / (2 B) and b <= 1024, so
+ * where the KL term dominates, the MSE term's share below the fp16 resolution of the sum is lost. */
+jab_status jab_loss_backward_scales_kl(const jab_block_desc* desc, int32_t B, int32_t T,
+                                       const void* X_dev, const void* W_dev,
+                                       const float* A_ref_dev, const void* QKV_ref_dev,
+                                       const float* lse_ref_dev, int32_t bits,
+                                       const float* scales_dev, float kappa, float lambda_kl,
+                                       double* loss_dev, double* kl_dev, float* grad_scales_dev,
+                                       void* ws, size_t ws_bytes, jab_stream_t stream);
+
 /* Forward L_JAB and the STE weight gradient for one candidate (App. B "Joint STE fine-tuning":
  * d w_hat / d w = 1, so dL/dW = dL/dw_hat), and its squared Frobenius norm: the Fisher-coupling score
  * of App. B "Fisher-coupling" when called with bits = 2 and round-to-nearest scales

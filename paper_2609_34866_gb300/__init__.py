@@ -14,5 +14,5 @@ from .binding import (  # noqa: F401
     jab_timing_reset, jab_timing_read, jab_selftest_wait_timeout, jab_prepare_x,
     jab_loss_backward_scales_prepared, jab_flip_rate, jab_reference_projection,
     jab_loss_forward_kl, jab_hutchinson_trace, jab_omega_scores, jab_rademacher_probes,
-    jab_set_deterministic, jab_selftest_bounds_check,
+    jab_set_deterministic, jab_selftest_bounds_check, jab_loss_backward_scales_kl,
 )

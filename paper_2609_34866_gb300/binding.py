@@ -80,6 +80,8 @@ def lib() -> ctypes.CDLL:
     L.jab_prepare_x.argtypes = [D, i32, i32, _P, _P, sz, _P]
     L.jab_loss_backward_scales_prepared.argtypes = [D, i32, i32, _P, _P, _P, i32, _P, f32, _P, _P,
                                                     _P, sz, _P]
+    L.jab_loss_backward_scales_kl.argtypes = [D, i32, i32, _P, _P, _P, _P, _P, i32, _P, f32, f32,
+                                              _P, _P, _P, _P, sz, _P]
     L.jab_flip_rate.argtypes = [_P, _P, ctypes.c_int64, _P, _P]
     L.jab_reference_projection.argtypes = [D, i32, i32, _P, _P, _P, _P, sz, _P]
     L.jab_hutchinson_trace.argtypes = [D, i32, i32, _P, _P, _P, _P, i32, ctypes.c_uint64, _P, _P,
@@ -108,6 +110,7 @@ def lib() -> ctypes.CDLL:
     for fn in ("jab_reference_forward", "jab_loss_forward", "jab_loss_forward_noalloc",
                "jab_loss_backward_scales", "jab_loss_backward_weights", "jab_allocate_bits",
                "jab_prepare_x", "jab_loss_backward_scales_prepared", "jab_flip_rate",
+               "jab_loss_backward_scales_kl",
                "jab_reference_projection", "jab_loss_forward_kl", "jab_hutchinson_trace",
                "jab_omega_scores", "jab_rademacher_probes",
                "jab_quantize", "jab_init_scales", "jab_get_device_status", "jab_timing_enable",
@@ -295,6 +298,21 @@ def jab_loss_backward_scales_prepared(desc, B, T, X, W, A_ref, bits: int, scales
         float(kappa), _ptr(loss, torch.float64, "loss"),
         _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "jab_loss_backward_scales_prepared")
+
+
+def jab_loss_backward_scales_kl(desc, B, T, X, W, A_ref, QKV_ref, lse_ref, bits: int, scales,
+                                kappa: float, lambda_kl: float, loss, grad_scales, ws: Workspace,
+                                kl=None, stream=None):
+    """Scale gradient of MSE + lambda_kl * KL (Eq. 3 with both terms); the teacher's projection and
+    log-sum-exp from jab_reference_projection / jab_reference_forward."""
+    st = lib().jab_loss_backward_scales_kl(
+        ctypes.byref(desc), B, T, _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(A_ref, torch.float32, "A_ref"), _ptr(QKV_ref, torch.float16, "QKV_ref"),
+        _ptr(lse_ref, torch.float32, "lse_ref"), int(bits), _ptr(scales, torch.float32, "scales"),
+        float(kappa), float(lambda_kl), _ptr(loss, torch.float64, "loss"),
+        _ptr(kl, torch.float64, "kl"), _ptr(grad_scales, torch.float32, "grad_scales"), ws.ptr,
+        ws.nbytes, _stream(stream))
+    _check(st, "jab_loss_backward_scales_kl")
 
 
 def jab_flip_rate(codes_a, codes_b, count, stream=None):

@@ -458,14 +458,28 @@ jab_status jab_omega_scores(const jab_block_desc* desc, const void* W_dev, int32
   return JAB_OK;
 }
 
+// The KL term of Eq. 3 in the backward (App. B "Effective weight of the KL term"): the teacher's
+// projection and log-sum-exp, lambda_KL, where the KL value goes, and the two factors of the
+// combined score gradient dS = a P (dP - D) + b (P - P_teacher) (b / a = lambda n / (2 B), with
+// n = B T Hq d_h; a <= 1 keeps b <= 1024 so that the fp16 dS tiles hold the KL part in range).
+struct KlTerm {
+  const void* qkv_ref;
+  const float* lse_ref;
+  double lambda;
+  double* kl_out;
+  float ab[2];
+};
+
 // Steps shared by the backward entry points (App. B, STE): quantise, project (+ RoPE), attention
 // forward in mode 2 (loss partials, dO = A_hat - A_ref, lse, D), the loss, and the attention backward
-// into dQKV^T (bf16 [D, ldt]) in the workspace. Checks the arguments common to both.
+// into dQKV^T (bf16 [D, ldt]) in the workspace; with a KL term also the teacher's probability tiles
+// and the KL value. Checks the arguments common to all.
 static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32_t T,
                                     const void* X_dev, const void* W_dev, const float* A_ref_dev,
                                     int32_t bits, const float* scales_dev, double* loss_dev,
                                     void* ws, size_t ws_bytes, bool x_prepared, cudaStream_t st,
-                                    Workspace* wp_out, int** status_out) {
+                                    Workspace* wp_out, int** status_out,
+                                    const KlTerm* kl = nullptr) {
   jab_status s = check_desc(desc);
   if (s != JAB_OK) return s;
   if ((s = check_bt(B, T)) != JAB_OK) return s;
@@ -508,7 +522,23 @@ static jab_status backward_to_dqkvt(const jab_block_desc* desc, int32_t B, int32
   const double n_el = (double)N * desc->n_q_heads * dh;
   JAB_SITE("loss_reduce", 1, launch_loss_reduce(L.part, 1, B, desc->n_q_heads, L.nP, 1.0 / n_el,
                                                 loss_dev, nullptr, status, st));
-  JAB_SITE("attn_bwd", 2, launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt));
+  const float* kl_ab = nullptr;
+  if (kl != nullptr) {
+    const int Hq = desc->n_q_heads, Hkv = desc->n_kv_heads;
+    float* lse_t = reinterpret_cast<float*>(w + wp.lse_t);
+    double* klpart = reinterpret_cast<double*>(w + wp.klpart);
+    double* klv = kl->kl_out ? kl->kl_out : reinterpret_cast<double*>(w + wp.scal) + 1;
+    JAB_SITE("lse_log2", 1, launch_lse_to_log2(kl->lse_ref, B * Hq, T, (int)wp.tp, lse_t, st));
+    JAB_SITE("teacher_p", 1, launch_attn_teacher_p_tc(w + wp.qkv, D, kl->qkv_ref, D, B, T, Hq, Hkv,
+                                                      dh, L.scale, lse_t, L.lse, (int)wp.tp, L.ds,
+                                                      klpart, status, st));
+    // batchmean (reading R18): the sum over sequences, heads, rows and keys divided by B
+    JAB_SITE("kl_reduce", 1, launch_sum_scaled(klpart, Hkv * B * ((T + 127) / 128), 1.0 / B, klv,
+                                               st));
+    JAB_SITE("loss_combine", 1, launch_loss_combine(loss_dev, klv, kl->lambda, 1, loss_dev, st));
+    kl_ab = kl->ab;
+  }
+  JAB_SITE("attn_bwd", 2, launch_attn_bwd_tc(L, cos_t, sin_t, desc->use_rope, w + wp.dqkvt, kl_ab));
   *wp_out = wp;
   *status_out = status;
   return JAB_OK;
@@ -522,7 +552,8 @@ static jab_status backward_scales(const jab_block_desc* desc, int32_t B, int32_t
                                   const void* X_dev, const void* W_dev, const float* A_ref_dev,
                                   int32_t bits, const float* scales_dev, float kappa,
                                   double* loss_dev, float* grad_scales_dev, void* ws,
-                                  size_t ws_bytes, bool x_prepared, jab_stream_t stream) {
+                                  size_t ws_bytes, bool x_prepared, jab_stream_t stream,
+                                  const KlTerm* kl = nullptr) {
   if (!grad_scales_dev || !aligned16(grad_scales_dev)) {
     const jab_status s = check_desc(desc);
     return s != JAB_OK ? s : JAB_ERR_INVALID_ARG;
@@ -531,14 +562,15 @@ static jab_status backward_scales(const jab_block_desc* desc, int32_t B, int32_t
   Workspace wp;
   int* status;
   jab_status s = backward_to_dqkvt(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, loss_dev,
-                                   ws, ws_bytes, x_prepared, st, &wp, &status);
+                                   ws, ws_bytes, x_prepared, st, &wp, &status, kl);
   if (s != JAB_OK) return s;
   char* w = static_cast<char*>(ws);
   const int64_t N = (int64_t)B * T;
   const int D = (int)block_rows(desc), dm = desc->d_model, G = desc->group_size;
   const double n_el = (double)N * desc->n_q_heads * desc->head_dim;
   const double k = kappa > 0.f ? (double)kappa : 1.0 / sqrt((double)G * qmax_of(bits));
-  const float coef = (float)(k * 2.0 / n_el);
+  // with the KL term the attention backward's dQKV^T is a times the MSE term's units
+  const float coef = (float)(k * 2.0 / n_el / (kl ? (double)kl->ab[0] : 1.0));
   // per-split partials summed in order: the scale gradient is bit-identical between calls
   JAB_SITE("wgrad_lsq", 1, launch_wgrad_lsq_tc(w + wp.dqkvt, wp.ldt, X_dev, W_dev, scales_dev, N, D,
                                                dm, G, bits, coef, grad_scales_dev,
@@ -597,6 +629,27 @@ jab_status jab_flip_rate(const int8_t* codes_a_dev, const int8_t* codes_b_dev, i
   JAB_TRY(launch_flip_count(codes_a_dev, codes_b_dev, n, count_dev, sms,
                             reinterpret_cast<cudaStream_t>(stream)));
   return JAB_OK;
+}
+
+jab_status jab_loss_backward_scales_kl(const jab_block_desc* desc, int32_t B, int32_t T,
+                                       const void* X_dev, const void* W_dev,
+                                       const float* A_ref_dev, const void* QKV_ref_dev,
+                                       const float* lse_ref_dev, int32_t bits,
+                                       const float* scales_dev, float kappa, float lambda_kl,
+                                       double* loss_dev, double* kl_dev, float* grad_scales_dev,
+                                       void* ws, size_t ws_bytes, jab_stream_t stream) {
+  jab_status s = check_desc(desc);
+  if (s != JAB_OK) return s;
+  if ((s = check_bt(B, T)) != JAB_OK) return s;
+  if (!QKV_ref_dev || !aligned16(QKV_ref_dev) || !lse_ref_dev ||
+      (reinterpret_cast<uintptr_t>(lse_ref_dev) & 3u) || !(lambda_kl >= 0.f) || !isfinite(lambda_kl))
+    return JAB_ERR_INVALID_ARG;
+  const double n_el = (double)B * T * desc->n_q_heads * desc->head_dim;
+  const double c = (double)lambda_kl * n_el / (2.0 * B);
+  const double a = c > 1024.0 ? 1024.0 / c : 1.0;
+  KlTerm kl{QKV_ref_dev, lse_ref_dev, (double)lambda_kl, kl_dev, {(float)a, (float)(a * c)}};
+  return backward_scales(desc, B, T, X_dev, W_dev, A_ref_dev, bits, scales_dev, kappa, loss_dev,
+                         grad_scales_dev, ws, ws_bytes, false, stream, &kl);
 }
 
 jab_status jab_loss_backward_weights(const jab_block_desc* desc, int32_t B, int32_t T,

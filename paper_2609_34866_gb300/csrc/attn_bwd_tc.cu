@@ -32,6 +32,7 @@ constexpr int DKDV_THREADS = (2 + DKDV_EW + 2) * 32;
 constexpr int DKDV_GRAD_WARP = 3 + DKDV_EW;
 constexpr int kSuperGroup = 8;  // (KV head, sequence) pairs whose dK/dV CTAs are interleaved
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr double kLn2 = 0.6931471805599453;
 
 struct BwdParams {
   int T, B, Hq, Hkv, lse_pitch;
@@ -39,6 +40,9 @@ struct BwdParams {
   int64_t ldt;
   int npairs;  // (query block, key block) pairs of one (sequence, head): nq (nq + 1) / 2
   float scale, sl2;
+  // KL term of Eq. 3 (dK/dV kernel with KL): dS = a_mse P (dP - D) + b_kl (P - P_teacher), dV times
+  // a_mse; the caller's coefficient of the whole gradient is divided by a_mse
+  float a_mse, b_kl;
   const float* lse;
   const float* dvec;
   const float* cos_t;
@@ -177,12 +181,16 @@ struct DkdvLayout {
 
 struct DkdvBars {
   uint64_t kv_full, ld_full[2], ld_empty[2], s_full, dp_full, p_full, ds_full, dv_done, dk_done;
-  uint64_t o_full, drain, drain_g, dss_full, dss_free, s_issued;
+  uint64_t o_full, drain, drain_g, dss_full, dss_free, s_issued, pt_full;
   uint32_t tmem_base;
   int abort;
 };
 
-template <int DH>
+// KL: the teacher's probabilities P^T of each (query block, key block) tile were stored in the dS^T
+// tile buffer (attn_teacher_p_tc_kernel); the store warp loads the tile into the staging buffer
+// before the block's dS, the elementwise warps add b_kl (P - P^T) to a_mse P (dP - D) and write
+// dS^T over it, and the tile goes back to the same place.
+template <int DH, bool KL>
 __global__ void __launch_bounds__(DKDV_THREADS, 1)
     attn_bwd_dkdv_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
                             const __grid_constant__ CUtensorMap tm_do,
@@ -237,6 +245,7 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
     tc::mbar_init(&bars->s_issued, 1);
     tc::mbar_init(&bars->dss_full, DKDV_EW);  // the block's dS^T is in the staging tile
     tc::mbar_init(&bars->dss_free, 1);         // the store warp's TMA stores have read it
+    tc::mbar_init(&bars->pt_full, 1);          // KL: the block's P^T tile is in the staging tile
     bars->abort = 0;
     tc::fence_mbar_init();
     tc::prefetch_tmap(&tm_qkv);
@@ -273,6 +282,11 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
         const int64_t lrow = ((int64_t)b * p.Hq + hj) * p.lse_pitch + ij * BQ;
         tc::prefetch_l2(p.lse + lrow, BQ * 4);
         tc::prefetch_l2(p.dvec + lrow, BQ * 4);
+        if constexpr (KL) {
+          const int64_t tile = ((int64_t)b * p.Hq + hj) * p.npairs + (int64_t)ij * (ij + 1) / 2 + kb;
+          tc::tma_prefetch_2d(&tm_ds, 0, (int32_t)(tile * BK));
+          tc::tma_prefetch_2d(&tm_ds, 64, (int32_t)(tile * BK));
+        }
       };
       for (int j = STAGES; j < STAGES + L::PREFETCH - 1 && j < n_it; ++j) prefetch(j);
       for (int it = 0; it < n_it; ++it) {
@@ -389,17 +403,35 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
     if (lane == 0) {  // ------------------------------------------ dS^T tiles to global memory
       // Tile (sequence b, head h, query block i, key block kb) is row block
       // (b Hq + h) npairs + i (i + 1) / 2 + kb of the dS^T buffer: 128 key rows of 128 queries.
+      auto tile_of = [&](int it) {
+        const int h = g * r + it / per_head, i = kb + it % per_head;
+        return ((int64_t)b * p.Hq + h) * p.npairs + (int64_t)i * (i + 1) / 2 + kb;
+      };
+      int pt_issued = 0;  // KL: P^T tiles loaded into the staging tile so far
+      auto load_pt = [&](int it) {  // KL: block it's P^T tile into the staging tile
+        const int32_t y = (int32_t)(tile_of(it) * BK);
+        tc::mbar_expect_tx(&bars->pt_full, 2 * L::CHUNK);
+        tc::tma_load_2d(smem + L::DSS_OFF, &tm_ds, &bars->pt_full, 0, y);
+        tc::tma_load_2d(smem + L::DSS_OFF + L::CHUNK, &tm_ds, &bars->pt_full, 64, y);
+        ++pt_issued;
+      };
+      if constexpr (KL) load_pt(0);
       for (int it = 0; it < n_it; ++it) {
         if (!tc::mbar_wait(&bars->dss_full, it & 1, abort, p.status)) break;
-        const int h = g * r + it / per_head, i = kb + it % per_head;
-        const int64_t tile = ((int64_t)b * p.Hq + h) * p.npairs + (int64_t)i * (i + 1) / 2 + kb;
+        const int64_t tile = tile_of(it);
         tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF, 0, (int32_t)(tile * BK));
         tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF + L::CHUNK, 64, (int32_t)(tile * BK));
         tc::bulk_commit_group();
         tc::bulk_wait_group_read<0>();  // the staging tile may be rewritten
-        tc::mbar_arrive(&bars->dss_free);
+        if constexpr (KL) {
+          if (it + 1 < n_it) load_pt(it + 1);
+        } else {
+          tc::mbar_arrive(&bars->dss_free);
+        }
       }
       tc::bulk_wait_group<0>();
+      // KL: a P^T load that nobody waited for (the loop gave up) lands before shared memory goes
+      if (KL && pt_issued > 0) drain_wait(&bars->pt_full, (pt_issued - 1) & 1);
     }
   } else {  // ------------------------------------ elementwise: 16 key rows x 64 queries per warp
     // Warp w (2..17) may access TMEM lane quarter w % 4; the four warps of a quarter take its two
@@ -481,6 +513,16 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
       }
       tc::fence_after_sync();
       uint32_t dw[16];
+      // The staging tile's words of this thread: packed word n of key rows rA and rA + 8 of the
+      // 64-query half chalf (128-byte swizzle).
+      uint8_t* hb = smem + L::DSS_OFF + chalf * L::CHUNK;
+      uint32_t* wa_p = reinterpret_cast<uint32_t*>(hb + rA * 128 + cq * 4);
+      uint32_t* wb_p = reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + cq * 4);
+      const int swa = rA & 7, swb = (rA + 8) & 7;
+      if (KL && !tc::mbar_wait(&bars->pt_full, it & 1, abort, p.status)) {
+        ok = false;
+        break;
+      }
       {
         uint32_t rd[32];
         __syncwarp();
@@ -491,9 +533,28 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
           const float2 d2 = *reinterpret_cast<const float2*>(d_s + 8 * n + 2 * cq);
           const float2 ta = tc::sub2(make_float2(__uint_as_float(rd[4 * n]), __uint_as_float(rd[4 * n + 1])), d2);
           const float2 tb = tc::sub2(make_float2(__uint_as_float(rd[4 * n + 2]), __uint_as_float(rd[4 * n + 3])), d2);
-          float2 da = tc::mul2(make_float2(x[4 * n], x[4 * n + 1]), ta);
-          float2 db = tc::mul2(make_float2(x[4 * n + 2], x[4 * n + 3]), tb);
-          if (!full) {  // masked entries (P = 0; D past T is not written): dS = 0
+          const float2 pa = make_float2(x[4 * n], x[4 * n + 1]);
+          const float2 pb = make_float2(x[4 * n + 2], x[4 * n + 3]);
+          float2 da = tc::mul2(pa, ta);
+          float2 db = tc::mul2(pb, tb);
+          if constexpr (KL) {
+            // + b_kl (P - P^T): the teacher's probabilities of the same entries (0 where masked)
+            const float2 qa = __half22float2(
+                *reinterpret_cast<const __half2*>(&wa_p[(n ^ swa) << 2]));
+            const float2 qb = __half22float2(
+                *reinterpret_cast<const __half2*>(&wb_p[(n ^ swb) << 2]));
+            const float2 am = make_float2(p.a_mse, p.a_mse), bk = make_float2(p.b_kl, p.b_kl);
+            const float2 ka = tc::mul2(tc::sub2(pa, qa), bk), kb2 = tc::mul2(tc::sub2(pb, qb), bk);
+            float2 ea = tc::fma2(da, am, ka), eb = tc::fma2(db, am, kb2);
+            if (!full) {  // masked entries (P = P^T = 0; D past T is not written): dS = 0
+              if (pa.x == 0.f && qa.x == 0.f) ea.x = 0.f;
+              if (pa.y == 0.f && qa.y == 0.f) ea.y = 0.f;
+              if (pb.x == 0.f && qb.x == 0.f) eb.x = 0.f;
+              if (pb.y == 0.f && qb.y == 0.f) eb.y = 0.f;
+            }
+            da = ea;
+            db = eb;
+          } else if (!full) {  // masked entries (P = 0; D past T is not written): dS = 0
             if (x[4 * n] == 0.f) da.x = 0.f;
             if (x[4 * n + 1] == 0.f) da.y = 0.f;
             if (x[4 * n + 2] == 0.f) db.x = 0.f;
@@ -511,19 +572,16 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
       if (lane == 0) tc::mbar_arrive(&bars->ds_full);
       // The same dS^T words into the staging tile for the store warp, once it has stored the
       // previous block's: packed word n (queries 64 chalf + 8n + 2cq, +1) is 16-byte unit n of the
-      // 64-query half chalf of its key row (128-byte swizzle).
-      if (it > 0 && !tc::mbar_wait(&bars->dss_free, (it - 1) & 1, abort, p.status)) {
+      // 64-query half chalf of its key row (128-byte swizzle). With KL they go over this thread's
+      // own P^T words, loaded only after the previous block's store had read the tile.
+      if (!KL && it > 0 && !tc::mbar_wait(&bars->dss_free, (it - 1) & 1, abort, p.status)) {
         ok = false;
         break;
       }
-      {
-        uint8_t* hb = smem + L::DSS_OFF + chalf * L::CHUNK;
 #pragma unroll
-        for (int n = 0; n < 8; ++n) {
-          *reinterpret_cast<uint32_t*>(hb + rA * 128 + ((n ^ (rA & 7)) << 4) + cq * 4) = dw[2 * n];
-          *reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + ((n ^ ((rA + 8) & 7)) << 4) + cq * 4) =
-              dw[2 * n + 1];
-        }
+      for (int n = 0; n < 8; ++n) {
+        wa_p[(n ^ swa) << 2] = dw[2 * n];
+        wb_p[(n ^ swb) << 2] = dw[2 * n + 1];
       }
       tc::fence_proxy_async_smem();
       __syncwarp();
@@ -539,7 +597,8 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
       tc::fence_after_sync();
       const int kA = keyA < p.T ? keyA : 0, kB = keyB < p.T ? keyB : 0;
       if (chalf == 0)
-        stage_grad_16<DH>(tmem + lane16 + L::DV_COL, 1.f, false, 0, 0, p.cos_t, p.sin_t, tv, rA);
+        stage_grad_16<DH>(tmem + lane16 + L::DV_COL, KL ? p.a_mse : 1.f, false, 0, 0, p.cos_t,
+                          p.sin_t, tv, rA);
       else
         stage_grad_16<DH>(tmem + lane16 + L::DK_COL, p.scale, p.use_rope != 0, kA, kB, p.cos_t,
                           p.sin_t, tk, rA);
@@ -554,6 +613,310 @@ __global__ void __launch_bounds__(DKDV_THREADS, 1)
                      DKDV_EW * 32, p.dqkvt, ext_t, p.status);
       store_tile<DH>(tk, p.dqkvt + (int64_t)(p.kcol0 + g * DH) * p.ldt, p.ldt, n0, nvalid, tid,
                      DKDV_EW * 32, p.dqkvt, ext_t, p.status);
+    }
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// ================================================================================ teacher P tiles
+// The KL term of Eq. 3 (D_KL(P || Q), P the teacher's map) for the STE gradient: its gradient with
+// respect to the student's scaled scores is (lambda / B)(Q - P), so the backward needs the teacher's
+// probabilities P of every (query, key) entry that the dS tiles hold. This kernel writes P^T into
+// the dS^T tile buffer in the dS^T layout (the dK/dV kernel then reads each tile, forms dS and
+// stores it back over it), and the KL value itself, using the two softmax normalisers of the
+// forward passes (teacher: jab_reference_forward; student: the loss+backward forward):
+//   KL_row i = sum_j P_ij (s^T_ij - s^S_ij) + lse^S_i - lse^T_i,  s = scale Q K^T (natural units),
+//   P_ij = exp(s^T_ij - lse^T_i).
+// Per CTA (128-key block, KV head, sequence), as the dK/dV kernel's walk over the group's query
+// heads and query blocks: S_t^T = K_t Q_t^T and S_s^T = K_s Q_s^T into one of two TMEM buffers
+// (the next block's products run while the elementwise warps read this one), P^T = exp2(s_t^T sl2 -
+// lse2_t) with the causal mask, the CTA's partial sum of P (s_t - s_s) (and, in the key-block-0 CTAs
+// that see every query row once, of lse^S - lse^T), and P^T staged and stored by TMA.
+//   warp 0      TMA: K_t, K_s once; per block Q_t, Q_s and the two rows of lse (log2 units)
+//   warp 1      TMEM owner, UMMA issuer
+//   warps 2..17 elementwise, 16 key rows x 64 queries each (the dK/dV kernel's layout)
+//   warp 18     P^T tiles to global memory
+constexpr int TP_THREADS = (2 + DKDV_EW + 1) * 32;
+
+struct TpParams {
+  int T, B, Hq, Hkv, lse_pitch, npairs;
+  int qcol0, kcol0;  // column offsets of the Q and K heads (the same in both projections)
+  float scale, sl2;
+  const float* lse2_t;  // teacher log-sum-exp, log2 units, [B, Hq, lse_pitch]
+  const float* lse2_s;  // student log-sum-exp, log2 units, [B, Hq, lse_pitch]
+  double* part;         // [gridDim.x] KL partial of each CTA (natural units)
+  int* status;
+};
+
+template <int DH>
+struct TpLayout {
+  static constexpr int BK = 128, BQ = 128, STAGES = 2;
+  static constexpr int CHUNK = 128 * 128;
+  static constexpr int NCH = DH / 64;
+  static constexpr int KT_OFF = 0, KS_OFF = NCH * CHUNK;
+  static constexpr int ST_OFF = 2 * NCH * CHUNK;
+  static constexpr int ST_QT = 0, ST_QS = NCH * CHUNK, ST_LT = 2 * NCH * CHUNK,
+                       ST_LS = ST_LT + BQ * 4, ST_BYTES = ST_LS + BQ * 4;
+  static constexpr int ST_STRIDE = (ST_BYTES + 1023) / 1024 * 1024;
+  static constexpr int DSS_OFF = ST_OFF + STAGES * ST_STRIDE;
+  static constexpr int BAR_OFF = DSS_OFF + 2 * CHUNK;
+  static constexpr int USED = BAR_OFF + 512;  // base alignment checked in the kernel
+  static constexpr int SMEM = USED > 118 * 1024 ? USED : 118 * 1024;
+  static_assert(USED <= 227 * 1024, "shared memory budget");
+};
+
+struct TpBars {
+  uint64_t kv_full, ld_full[2], ld_empty[2], s_full[2], s_free[2], dss_full, dss_free, drain;
+  uint32_t tmem_base;
+  int abort;
+  double red[DKDV_EW];
+};
+
+template <int DH>
+__global__ void __launch_bounds__(TP_THREADS, 1)
+    attn_teacher_p_tc_kernel(const __grid_constant__ CUtensorMap tm_s,
+                             const __grid_constant__ CUtensorMap tm_t,
+                             const __grid_constant__ CUtensorMap tm_ds, const TpParams p) {
+  using L = TpLayout<DH>;
+  constexpr int BK = L::BK, BQ = L::BQ, STAGES = L::STAGES;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  if (tc::smem_u32(smem_raw) & 1023u) {
+    if (threadIdx.x == 0) report(p.status, JAB_ERR_INTERNAL);
+    return;
+  }
+  uint8_t* smem = smem_raw;
+  TpBars* bars = reinterpret_cast<TpBars*>(smem + L::BAR_OFF);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &bars->abort;
+
+  const int r = p.Hq / p.Hkv;
+  const int nq = (p.T + BQ - 1) / BQ;
+  int kb, g, b;  // the dK/dV kernel's CTA order
+  {
+    const int pairs = p.Hkv * p.B;
+    const int sg = blockIdx.x / (kSuperGroup * nq);
+    const int sgs = min(kSuperGroup, pairs - sg * kSuperGroup);
+    const int rem = blockIdx.x - sg * kSuperGroup * nq;
+    kb = rem / sgs;
+    const int pr = sg * kSuperGroup + rem % sgs;
+    g = pr % p.Hkv;
+    b = pr / p.Hkv;
+  }
+  const int per_head = nq - kb;
+  const int n_it = r * per_head;
+  const int row0 = b * p.T;
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bars->kv_full, 1);
+    for (int i = 0; i < STAGES; ++i) {
+      tc::mbar_init(&bars->ld_full[i], 1);
+      tc::mbar_init(&bars->ld_empty[i], 1 + DKDV_EW);  // the products and the lse readers
+      tc::mbar_init(&bars->s_full[i], 1);
+      tc::mbar_init(&bars->s_free[i], DKDV_EW);
+    }
+    tc::mbar_init(&bars->dss_full, DKDV_EW);
+    tc::mbar_init(&bars->dss_free, 1);
+    tc::mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    tc::fence_mbar_init();
+    tc::prefetch_tmap(&tm_s);
+    tc::prefetch_tmap(&tm_t);
+    tc::prefetch_tmap(&tm_ds);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(&bars->tmem_base, 512);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = bars->tmem_base;
+
+  if (warp == 0) {
+    if (lane == 0) {  // ------------------------------------------------------------- TMA
+      uint32_t issued = 0, last_par = 0;
+      tc::mbar_expect_tx(&bars->kv_full, 2 * BK * DH * 2);
+      for (int ch = 0; ch < L::NCH; ++ch) {
+        tc::tma_load_2d(smem + L::KT_OFF + ch * L::CHUNK, &tm_t, &bars->kv_full,
+                        p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
+        tc::tma_load_2d(smem + L::KS_OFF + ch * L::CHUNK, &tm_s, &bars->kv_full,
+                        p.kcol0 + g * DH + ch * 64, row0 + kb * BK);
+      }
+      for (int it = 0; it < n_it; ++it) {
+        const int st = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        const int h = g * r + it / per_head, i = kb + it % per_head;
+        if (!tc::mbar_wait(&bars->ld_empty[st], ph ^ 1, abort, p.status)) break;
+        uint8_t* sbase = smem + L::ST_OFF + st * L::ST_STRIDE;
+        tc::mbar_expect_tx(&bars->ld_full[st], L::ST_BYTES);
+        for (int ch = 0; ch < L::NCH; ++ch) {
+          tc::tma_load_2d(sbase + L::ST_QT + ch * L::CHUNK, &tm_t, &bars->ld_full[st],
+                          p.qcol0 + h * DH + ch * 64, row0 + i * BQ);
+          tc::tma_load_2d(sbase + L::ST_QS + ch * L::CHUNK, &tm_s, &bars->ld_full[st],
+                          p.qcol0 + h * DH + ch * 64, row0 + i * BQ);
+        }
+        const int64_t lrow = ((int64_t)b * p.Hq + h) * p.lse_pitch + i * BQ;
+        if (in_bounds(lrow + BQ - 1, (int64_t)p.B * p.Hq * p.lse_pitch, p.status)) {
+          tc::bulk_load(sbase + L::ST_LT, p.lse2_t + lrow, BQ * 4, &bars->ld_full[st]);
+          tc::bulk_load(sbase + L::ST_LS, p.lse2_s + lrow, BQ * 4, &bars->ld_full[st]);
+        }
+        issued |= 1u << st;
+        last_par = (last_par & ~(1u << st)) | (ph << st);
+      }
+      if (*abort) {
+        drain_wait(&bars->kv_full, 0);
+        for (int st = 0; st < STAGES; ++st)
+          if (issued & (1u << st)) drain_wait(&bars->ld_full[st], (last_par >> st) & 1);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {  // ---------------------------------------------------------------- UMMA
+      constexpr uint32_t ID_S = tc::idesc_f16(false, BK, BQ);
+      bool ok = tc::mbar_wait(&bars->kv_full, 0, abort, p.status);
+      const uint64_t kt = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::KT_OFF));
+      const uint64_t ks = tc::sdesc_kmajor_sw128(tc::smem_u32(smem + L::KS_OFF));
+      for (int j = 0; ok && j < n_it; ++j) {
+        const int st = j % STAGES, bf = j & 1;
+        // the stage has landed and the elementwise warps have read block j - 2's scores
+        ok = tc::mbar_wait(&bars->ld_full[st], (j / STAGES) & 1, abort, p.status) &&
+             (j < 2 || tc::mbar_wait(&bars->s_free[bf], ((j >> 1) - 1) & 1, abort, p.status));
+        if (!ok) break;
+        tc::fence_after_sync();
+        const uint32_t sb = tc::smem_u32(smem + L::ST_OFF + st * L::ST_STRIDE);
+        const uint64_t bt = tc::sdesc_kmajor_sw128(sb + L::ST_QT);
+        const uint64_t bs = tc::sdesc_kmajor_sw128(sb + L::ST_QS);
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
+          tc::umma_f16(tmem + 256 * bf, tc::sdesc_advance(kt, o), tc::sdesc_advance(bt, o), ID_S,
+                       k > 0 ? 1u : 0u);
+        }
+#pragma unroll
+        for (int k = 0; k < DH / 16; ++k) {
+          const uint32_t o = (k >> 2) * L::CHUNK + (k & 3) * 32;
+          tc::umma_f16(tmem + 256 * bf + 128, tc::sdesc_advance(ks, o), tc::sdesc_advance(bs, o),
+                       ID_S, k > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&bars->s_full[bf]);
+        tc::umma_commit(&bars->ld_empty[st]);
+      }
+      tc::umma_commit(&bars->drain);
+      drain_wait(&bars->drain, 0);
+    }
+  } else if (warp == 2 + DKDV_EW) {
+    if (lane == 0) {  // ------------------------------------------------- P^T tiles to global
+      for (int it = 0; it < n_it; ++it) {
+        if (!tc::mbar_wait(&bars->dss_full, it & 1, abort, p.status)) break;
+        const int h = g * r + it / per_head, i = kb + it % per_head;
+        const int64_t tile = ((int64_t)b * p.Hq + h) * p.npairs + (int64_t)i * (i + 1) / 2 + kb;
+        tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF, 0, (int32_t)(tile * BK));
+        tc::tma_store_2d(&tm_ds, smem + L::DSS_OFF + L::CHUNK, 64, (int32_t)(tile * BK));
+        tc::bulk_commit_group();
+        tc::bulk_wait_group_read<0>();
+        tc::mbar_arrive(&bars->dss_free);
+      }
+      tc::bulk_wait_group<0>();
+    }
+  } else {  // ------------------------------------ elementwise: 16 key rows x 64 queries per warp
+    const int quarter = warp & 3;
+    const int idx = (warp - 2) >> 2;
+    const int half = idx & 1;
+    const int chalf = idx >> 1;
+    const int cq = lane & 3;
+    const int rA = quarter * 32 + half * 16 + (lane >> 2);
+    const int keyA = kb * BK + rA, keyB = keyA + 8;
+    const uint32_t lane16 = (uint32_t)(quarter * 32 + half * 16) << 16;
+    float2 acc = make_float2(0.f, 0.f);  // sum of P (s_t - s_s) in raw score units (times scale later)
+    double rows = 0.0;                   // key-block-0 CTAs, warp 2: sum of lse2_s - lse2_t
+    for (int it = 0; it < n_it; ++it) {
+      const int st = it % STAGES, bf = it & 1;
+      const int i = kb + it % per_head;
+      const float* sbase = reinterpret_cast<const float*>(smem + L::ST_OFF + st * L::ST_STRIDE);
+      const float* lt = sbase + L::ST_LT / 4;
+      const float* ls = sbase + L::ST_LS / 4;
+      if (!tc::mbar_wait(&bars->ld_full[st], (it / STAGES) & 1, abort, p.status) ||
+          !tc::mbar_wait(&bars->s_full[bf], (it >> 1) & 1, abort, p.status))
+        break;
+      tc::fence_after_sync();
+      uint32_t rt[32], rs[32];
+      __syncwarp();
+      tc::tmem_ld_16x256b_x8(tmem + lane16 + 256 * bf + 64 * chalf, rt);
+      tc::tmem_ld_16x256b_x8(tmem + lane16 + 256 * bf + 128 + 64 * chalf, rs);
+      tc::tmem_ld_wait();
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->s_free[bf]);  // the products of block it + 2 may start
+      const int qc0 = i * BQ + 64 * chalf + 2 * cq;
+      const bool full = i > kb && i * BQ + BQ <= p.T;
+      const float2 sl2 = make_float2(p.sl2, p.sl2);
+      uint32_t pw[16];
+#pragma unroll
+      for (int n = 0; n < 8; ++n) {
+        const float2 l2 = *reinterpret_cast<const float2*>(lt + 64 * chalf + 8 * n + 2 * cq);
+        const float2 nl = make_float2(tc::neg_bits(l2.x), tc::neg_bits(l2.y));
+        const float2 ta = make_float2(__uint_as_float(rt[4 * n]), __uint_as_float(rt[4 * n + 1]));
+        const float2 tb = make_float2(__uint_as_float(rt[4 * n + 2]), __uint_as_float(rt[4 * n + 3]));
+        const float2 sa = make_float2(__uint_as_float(rs[4 * n]), __uint_as_float(rs[4 * n + 1]));
+        const float2 sb = make_float2(__uint_as_float(rs[4 * n + 2]), __uint_as_float(rs[4 * n + 3]));
+        const float2 ea = tc::fma2(ta, sl2, nl), eb = tc::fma2(tb, sl2, nl);
+        float pa[2] = {tc::fast_exp2(ea.x), tc::fast_exp2(ea.y)};
+        float pb[2] = {tc::fast_exp2(eb.x), tc::fast_exp2(eb.y)};
+        if (!full) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int q = qc0 + 8 * n + e;
+            if (q >= p.T || q < keyA) pa[e] = 0.f;
+            if (q >= p.T || q < keyB) pb[e] = 0.f;
+          }
+        }
+        acc = tc::fma2(make_float2(pa[0], pa[1]), tc::sub2(ta, sa), acc);
+        acc = tc::fma2(make_float2(pb[0], pb[1]), tc::sub2(tb, sb), acc);
+        pw[2 * n] = tc::pack_half2(pa[0], pa[1]);
+        pw[2 * n + 1] = tc::pack_half2(pb[0], pb[1]);
+      }
+      if (kb == 0 && warp == 2) {  // lse^S - lse^T of the block's query rows (each row once)
+        float t = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int qi = lane * 4 + e;
+          if (i * BQ + qi < p.T) t += ls[qi] - lt[qi];
+        }
+        rows += t;
+      }
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->ld_empty[st]);  // this warp has read the lse rows
+      if (it > 0 && !tc::mbar_wait(&bars->dss_free, (it - 1) & 1, abort, p.status)) break;
+      {
+        uint8_t* hb = smem + L::DSS_OFF + chalf * L::CHUNK;
+#pragma unroll
+        for (int n = 0; n < 8; ++n) {
+          *reinterpret_cast<uint32_t*>(hb + rA * 128 + ((n ^ (rA & 7)) << 4) + cq * 4) = pw[2 * n];
+          *reinterpret_cast<uint32_t*>(hb + (rA + 8) * 128 + ((n ^ ((rA + 8) & 7)) << 4) + cq * 4) =
+              pw[2 * n + 1];
+        }
+      }
+      tc::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&bars->dss_full);
+    }
+    // The CTA's partial: the warps' sums in a fixed order (natural units).
+    float v = acc.x + acc.y;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) rows += __shfl_xor_sync(0xffffffffu, rows, o);
+    if (lane == 0) bars->red[warp - 2] = (double)v * p.scale + rows * (double)kLn2;
+    tc::named_bar_sync(1, DKDV_EW * 32);
+    if (threadIdx.x == 64) {
+      double t = 0.0;
+      for (int w = 0; w < DKDV_EW; ++w) t += bars->red[w];
+      p.part[blockIdx.x] = t;
     }
   }
   tc::fence_before_sync();
@@ -796,7 +1159,7 @@ cudaError_t set_smem(K kernel, int bytes, bool& done) {
 }
 
 template <int DH>
-cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
+cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p, bool kl) {
   const int64_t N = (int64_t)L.B * L.T;
   // dS^T tiles as a 2-D fp16 tensor of 128-query rows, one 128-row block per (sequence, head,
   // query block, key block)
@@ -806,16 +1169,22 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
       !tmap_rows(&do128, L.d_o, (uint64_t)L.Hq * DH, N, 128) ||
       !tmap_rows(&ds128, L.ds, 128, ds_rows, 128) || ds_rows >= (1ull << 31))
     return cudaErrorInvalidValue;
-  static bool a1 = false, a2 = false;
-  cudaError_t e = set_smem(attn_bwd_dkdv_tc_kernel<DH>, DkdvLayout<DH>::SMEM, a1);
+  static bool a1 = false, a2 = false, a3 = false;
+  cudaError_t e = set_smem(attn_bwd_dkdv_tc_kernel<DH, false>, DkdvLayout<DH>::SMEM, a1);
+  if (e != cudaSuccess) return e;
+  e = set_smem(attn_bwd_dkdv_tc_kernel<DH, true>, DkdvLayout<DH>::SMEM, a3);
   if (e != cudaSuccess) return e;
   e = set_smem(attn_bwd_dq_tc_kernel<DH>, DqLayout<DH>::SMEM, a2);
   if (e != cudaSuccess) return e;
   const int64_t n_dkdv = (int64_t)L.Hkv * L.B * ((L.T + 127) / 128);
   if (n_dkdv >= (1ll << 31)) return cudaErrorInvalidValue;
   const dim3 g1((unsigned)n_dkdv);
-  attn_bwd_dkdv_tc_kernel<DH><<<g1, DKDV_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(kv128, do128,
-                                                                                     ds128, p);
+  if (kl)
+    attn_bwd_dkdv_tc_kernel<DH, true><<<g1, DKDV_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(
+        kv128, do128, ds128, p);
+  else
+    attn_bwd_dkdv_tc_kernel<DH, false><<<g1, DKDV_THREADS, DkdvLayout<DH>::SMEM, L.stream>>>(
+        kv128, do128, ds128, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
@@ -830,7 +1199,7 @@ cudaError_t launch_bwd(const AttnLaunch& L, const BwdParams& p) {
 }  // namespace
 
 cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
-                               int use_rope, void* dqkvt) {
+                               int use_rope, void* dqkvt, const float* kl_ab) {
   BwdParams p{};
   p.T = L.T;
   p.B = L.B;
@@ -845,6 +1214,8 @@ cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const fl
   p.npairs = nq * (nq + 1) / 2;
   p.scale = L.scale;
   p.sl2 = L.scale * kLog2e;
+  p.a_mse = kl_ab ? kl_ab[0] : 1.f;
+  p.b_kl = kl_ab ? kl_ab[1] : 0.f;
   p.lse = L.lse;
   p.dvec = L.dvec;
   p.cos_t = cos_t;
@@ -855,7 +1226,56 @@ cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const fl
   if ((reinterpret_cast<uintptr_t>(L.lse) & 15u) || (reinterpret_cast<uintptr_t>(L.dvec) & 15u) ||
       (L.lse_pitch % 128) != 0 || L.ds == nullptr || (reinterpret_cast<uintptr_t>(L.ds) & 15u))
     return cudaErrorInvalidValue;
-  return L.dh == 128 ? launch_bwd<128>(L, p) : launch_bwd<64>(L, p);
+  return L.dh == 128 ? launch_bwd<128>(L, p, kl_ab != nullptr)
+                     : launch_bwd<64>(L, p, kl_ab != nullptr);
+}
+
+namespace {
+template <int DH>
+cudaError_t launch_tp(const CUtensorMap& ms, const CUtensorMap& mt, const CUtensorMap& md,
+                      const TpParams& p, cudaStream_t st) {
+  static bool attr = false;
+  cudaError_t e = set_smem(attn_teacher_p_tc_kernel<DH>, TpLayout<DH>::SMEM, attr);
+  if (e != cudaSuccess) return e;
+  const int64_t n = (int64_t)p.Hkv * p.B * ((p.T + 127) / 128);
+  if (n >= (1ll << 31)) return cudaErrorInvalidValue;
+  attn_teacher_p_tc_kernel<DH><<<(unsigned)n, TP_THREADS, TpLayout<DH>::SMEM, st>>>(ms, mt, md, p);
+  return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_attn_teacher_p_tc(const void* qkv_s, int64_t ldq_s, const void* qkv_t,
+                                     int64_t ldq_t, int B, int T, int Hq, int Hkv, int dh,
+                                     float scale, const float* lse2_t, const float* lse2_s,
+                                     int lse_pitch, void* ds, double* part, int* status,
+                                     cudaStream_t st) {
+  const int64_t N = (int64_t)B * T;
+  const int nq = (T + 127) / 128;
+  TpParams p{};
+  p.T = T;
+  p.B = B;
+  p.Hq = Hq;
+  p.Hkv = Hkv;
+  p.lse_pitch = lse_pitch;
+  p.npairs = nq * (nq + 1) / 2;
+  p.qcol0 = 0;
+  p.kcol0 = Hq * dh;
+  p.scale = scale;
+  p.sl2 = scale * kLog2e;
+  p.lse2_t = lse2_t;
+  p.lse2_s = lse2_s;
+  p.part = part;
+  p.status = status;
+  if ((reinterpret_cast<uintptr_t>(lse2_t) & 15u) || (reinterpret_cast<uintptr_t>(lse2_s) & 15u) ||
+      (lse_pitch % 128) != 0 || ds == nullptr || (reinterpret_cast<uintptr_t>(ds) & 15u) ||
+      part == nullptr || (dh != 64 && dh != 128))
+    return cudaErrorInvalidValue;
+  const uint64_t ds_rows = (uint64_t)B * Hq * p.npairs * 128;
+  CUtensorMap ms, mt, md;
+  if (!tmap_rows(&ms, qkv_s, ldq_s, N, 128) || !tmap_rows(&mt, qkv_t, ldq_t, N, 128) ||
+      !tmap_rows(&md, ds, 128, ds_rows, 128) || ds_rows >= (1ull << 31))
+    return cudaErrorInvalidValue;
+  return dh == 128 ? launch_tp<128>(ms, mt, md, p, st) : launch_tp<64>(ms, mt, md, p, st);
 }
 
 }  // namespace jab

@@ -56,8 +56,25 @@ int choose_splits(int tiles, int k_blocks, int sms);
 // attn_tc.cu
 int attn_fwd_tc_rows(int Hq, int Hkv);  // query rows per loss partial of the forward kernel
 cudaError_t launch_attn_fwd_tc(const AttnLaunch& L, int mode);
+// kl_ab: null for the MSE term alone; else {a, b}: dS = a P (dP - D) + b (P - P_teacher) with the
+// teacher's probabilities read from the dS^T tile buffer (launch_attn_teacher_p_tc), dV times a
 cudaError_t launch_attn_bwd_tc(const AttnLaunch& L, const float* cos_t, const float* sin_t,
-                               int use_rope, void* dqkvt);
+                               int use_rope, void* dqkvt, const float* kl_ab = nullptr);
+// The teacher's probabilities P^T of every (query block, key block <= query block) tile into the
+// dS^T tile buffer `ds` (layout of AttnLaunch::ds) and one KL partial per CTA in part
+// [Hkv, B, ceil(T / 128)]: the sum of P (s_t - s_s) over its entries plus, in key block 0, of
+// lse_s - lse_t over its query rows (natural units). qkv_s / qkv_t: student and teacher projections,
+// fp16 [B*T, ldq]; lse2_t / lse2_s: log-sum-exp in log2 units, [B, Hq, lse_pitch].
+cudaError_t launch_attn_teacher_p_tc(const void* qkv_s, int64_t ldq_s, const void* qkv_t,
+                                     int64_t ldq_t, int B, int T, int Hq, int Hkv, int dh,
+                                     float scale, const float* lse2_t, const float* lse2_s,
+                                     int lse_pitch, void* ds, double* part, int* status,
+                                     cudaStream_t st);
+// out[b, h, t] = in[b, h, t] * log2(e) for t < T: [B, Hq, T] -> [B, Hq, pitch]
+cudaError_t launch_lse_to_log2(const float* in, int BH, int T, int pitch, float* out,
+                               cudaStream_t st);
+// *out = scale * sum of part[0 .. n - 1], in order (fp64)
+cudaError_t launch_sum_scaled(const double* part, int n, double scale, double* out, cudaStream_t st);
 
 // attn_kl_tc.cu: KL attention-map term (Eq. 3). qkv_s: student fp16 [B*T, ldq] (candidate c at
 // column c * D); qkv_t: teacher fp16 [B*T, D]. part [C, B, Hq, nP] (nP >= ceil(T / rows)), kl_rows

@@ -89,6 +89,26 @@ __global__ void sum_in_order_kernel(const double* __restrict__ part, int n, doub
   }
 }
 
+__global__ void sum_scaled_kernel(const double* __restrict__ part, int n, double scale,
+                                  double* __restrict__ out) {
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int i = 0; i < n; ++i) t += part[i];
+    *out = scale * t;
+  }
+}
+
+// Natural-log log-sum-exp rows [BH, T] to log2 units with the row pitch of the backward workspace.
+__global__ void lse_to_log2_kernel(const float* __restrict__ in, int BH, int T, int pitch,
+                                   float* __restrict__ out) {
+  const int64_t n = (int64_t)BH * T;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / T, t = i - r * T;
+    out[r * pitch + t] = in[i] * 1.4426950408889634f;
+  }
+}
+
 // Sum of the K-split partials of a gradient in the order of the splits (one thread per element).
 __global__ void split_sum_kernel(const float* __restrict__ part, int splits, int64_t n,
                                  float* __restrict__ out) {
@@ -136,6 +156,20 @@ cudaError_t launch_split_sum(const float* part, int splits, int64_t n, float* ou
   if (blocks > 4096) blocks = 4096;
   if (blocks < 1) blocks = 1;
   split_sum_kernel<<<(unsigned)blocks, 256, 0, st>>>(part, splits, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sum_scaled(const double* part, int n, double scale, double* out, cudaStream_t st) {
+  sum_scaled_kernel<<<1, 32, 0, st>>>(part, n, scale, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lse_to_log2(const float* in, int BH, int T, int pitch, float* out,
+                               cudaStream_t st) {
+  int64_t blocks = ((int64_t)BH * T + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  lse_to_log2_kernel<<<(unsigned)blocks, 256, 0, st>>>(in, BH, T, pitch, out);
   return cudaGetLastError();
 }
 

@@ -31,6 +31,8 @@ struct Workspace {
                    //                        key block <= query block) pair, nq = ceil(T / 128)
   size_t gpart;    // fp32 [kMaxSplits, D, d/G]  scale-gradient partial of every K split (summed in order)
   size_t dwscr;    // fp32 [D, d]            dW when only its squared norm is asked for
+  size_t lse_t;    // fp32 [B, Hq, Tp]       teacher log-sum-exp in log2 units (KL term's gradient)
+  size_t klpart;   // fp64 [Hkv, B, nq]      KL partial sum of every teacher-probability CTA
   int64_t ldt;     // row pitch (elements) of dqkvt: N rounded up to 64
   int64_t tp;      // row pitch (elements) of lse and dvec: T rounded up to 128
   size_t total;
@@ -72,8 +74,10 @@ inline Workspace plan_workspace(const jab_block_desc* d, int64_t B, int64_t T, i
     w.ds = take((size_t)B * d->n_q_heads * (nq * (nq + 1) / 2) * 128 * 128 * 2);
     w.gpart = take((size_t)kMaxSplits * D * (dm / d->group_size) * 4);
     w.dwscr = take((size_t)D * dm * 4);
+    w.lse_t = take((size_t)B * d->n_q_heads * w.tp * 4);
+    w.klpart = take((size_t)d->n_kv_heads * B * nq * 8);
   } else {
-    w.d_o = w.lse = w.dvec = w.dqkvt = w.ds = w.gpart = w.dwscr = SIZE_MAX;
+    w.d_o = w.lse = w.dvec = w.dqkvt = w.ds = w.gpart = w.dwscr = w.lse_t = w.klpart = SIZE_MAX;
   }
   w.total = off;
   return w;

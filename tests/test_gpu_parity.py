@@ -232,6 +232,61 @@ def test_backward_parity(name, bits):
     assert J().jab_get_device_status() == 0
 
 
+# ------------------------------------------------------------------ STE / LSQ backward with the KL term
+def _kl_teacher(c, ws):
+    """Teacher output, its log-sum-exp and its projection (the KL term's inputs)."""
+    A, lse, _ = c.gpu_teacher(ws)
+    qkv_ref = torch.empty((c.B, c.T, c.D), dtype=torch.float16, device="cuda")
+    J().jab_reference_projection(c.desc, c.B, c.T, c.X, c.W, qkv_ref, ws)
+    return A, lse, qkv_ref
+
+
+@pytest.mark.parametrize("name,bits", [("gpt2_T200", 3), ("mistral_T130", 3),
+                                       ("mistral_G64_T70", 2), ("gqa2_T257", 3),
+                                       ("dh64_gqa4_T65", 4), ("dh64_gqa4_B64_T256", 3),
+                                       ("gpt2_T1", 3)])
+@pytest.mark.parametrize("regime", ["default", "balanced"])
+def test_backward_kl_parity(name, bits, regime):
+    """Scale gradient of MSE + lambda KL (Eq. 3, both terms) against the oracle's
+    jab_loss_joint_and_grad: lambda = 0.1 (the paper's default; the KL term dominates) and a lambda
+    at which the two terms' score gradients have the same weight (lambda n / (2 B) = 1)."""
+    c = case(name)
+    ws = c.workspace()
+    A, lse, qkv_ref = _kl_teacher(c, ws)
+    n = c.B * c.T * c.Hq * c.dh
+    lam = float(np.float32(0.1 if regime == "default" else 2.0 * c.B / n))
+    s = c.gpu_scales(bits)
+    loss, kl = (torch.empty(1, dtype=torch.float64, device="cuda") for _ in range(2))
+    grad = torch.empty_like(s)
+    J().jab_loss_backward_scales_kl(c.desc, c.B, c.T, c.X, c.W, A, qkv_ref, lse, bits, s, 1.0, lam,
+                                    loss, grad, ws, kl=kl)
+    assert J().jab_get_device_status() == 0
+    r = O.jab_loss_joint_and_grad(c.x64, c.w64, s.cpu().numpy(), bits, c.odesc, lam_kl=lam,
+                                  kappa=1.0)
+    floor = KL_ROW_ATOL * c.Hq * c.T
+    assert abs(kl.item() - r["kl"]) <= KL_TOL[bits] * r["kl"] + floor, (kl.item(), r["kl"])
+    assert abs(loss.item() - r["loss"]) <= L_TOL * r["loss"], (loss.item(), r["loss"])
+    cos = cosine(grad.cpu().numpy(), r["grad_s"])
+    assert cos >= COS_MIN, cos
+
+
+def test_backward_kl_with_zero_lambda_is_the_mse_gradient():
+    """lambda_KL = 0 through the KL code path (teacher tiles, combined score gradient) gives the
+    MSE term's loss and scale gradient bit for bit."""
+    c = case("gqa2_T257")
+    ws = c.workspace()
+    A, lse, qkv_ref = _kl_teacher(c, ws)
+    s = c.gpu_scales(3)
+    l0, l1 = (torch.empty(1, dtype=torch.float64, device="cuda") for _ in range(2))
+    g0, g1 = torch.empty_like(s), torch.empty_like(s)
+    J().jab_loss_backward_scales(c.desc, c.B, c.T, c.X, c.W, A, 3, s, 1.0, l0, g0, ws)
+    J().jab_loss_backward_scales_kl(c.desc, c.B, c.T, c.X, c.W, A, qkv_ref, lse, 3, s, 1.0, 0.0, l1,
+                                    g1, ws)
+    assert J().jab_get_device_status() == 0
+    assert l0.item() == l1.item()
+    assert torch.equal(g0, g1)
+
+
 # ------------------------------------------------------------------ STE weight gradient, Fisher score
 @pytest.mark.parametrize("name,bits", [("gpt2_T200", 2), ("mistral_T130", 2), ("gqa2_T257", 3),
                                        ("dh64_gqa4_B64_T256", 2)])
