@@ -613,8 +613,28 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
 
     kl_ms, _ = timed(J, kl_step, args.steps, max(1, args.warmup), st, barrier, sites=False)
     kl_ms = max_over_ranks(kl_ms, dev)
-    del qkv_ref
     kl_f = fwd_f + work_of(wl)["attn_kl"][1]
+
+    # ---- STE step on both terms of Eq. 3 (lambda_KL = 0.1): the scale gradient of MSE + 0.1 KL;
+    # the teacher's projection and log-sum-exp are made once per calibration batch, like A_ref;
+    # the call converts X itself
+    lse_ref = torch.empty((B, s.n_q_heads, T), dtype=torch.float32, device=dev)
+    J.jab_reference_forward(desc, B, T, X, W, A, ws, lse=lse_ref)
+
+    def kl_bwd_step():
+        J.jab_loss_backward_scales_kl(desc, B, T, X, W, A, qkv_ref, lse_ref, bits, scales, 0.0, 0.1,
+                                      loss, grad, ws)
+        if world > 1:
+            combine_shards(loss, grad, B, B * world)
+
+    n_klb = max(1, min(args.steps, 5))
+    klb_ms, _ = timed(J, kl_bwd_step, n_klb, max(1, min(args.warmup, 2)), st, barrier, sites=False)
+    klb_ms = max_over_ranks(klb_ms, dev)
+    if J.jab_get_device_status() != 0:
+        raise RuntimeError("device status set in the KL-term backward")
+    J.jab_prepare_x(desc, B, T, X, ws)  # the headline's prepared X for what follows
+    del qkv_ref, lse_ref
+    klb_f = fwd_f + bwd_f + work_of(wl)["attn_kl"][1]
 
     # ---- Fisher-coupling probe (App. B): the loss and ||dL/dw_hat||^2 at 2 bits with round-to-
     # nearest (absmax) scales, one fwd + bwd per evaluation; reported beside the main metric
@@ -728,6 +748,11 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
         "fwd_kl": {"value": world * args.steps / (kl_ms / 1e3), "unit": "evals/s",
                    "ms_per_eval": kl_ms / args.steps, "lambda_kl": 0.1,
                    "achieved_tflops": kl_f / (kl_ms / args.steps / 1e3) / 1e12},
+        "fwd_bwd_kl": {"value": world * n_klb / (klb_ms / 1e3), "unit": "evals/s",
+                       "ms_per_eval": klb_ms / n_klb, "lambda_kl": 0.1,
+                       "achieved_tflops": klb_f / (klb_ms / n_klb / 1e3) / 1e12,
+                       "note": "scale gradient of MSE + 0.1 KL (jab_loss_backward_scales_kl), "
+                               "X converted by the call"},
         "fisher_probe": {"value": world * n_fis / (fis_ms / 1e3), "unit": "evals/s", "bits": 2,
                          "ms_per_eval": fis_ms / n_fis,
                          "achieved_tflops": (fwd_f + bwd_f) / (fis_ms / n_fis / 1e3) / 1e12},

@@ -53,10 +53,11 @@ def test_normal_build_has_no_bounds_checks():
 
 
 def test_parity_cases_raise_no_check_in_the_checked_build():
-    """Forward (teacher, loss), KL, Hutchinson, backward, weight gradient and the CTA-pair GEMMs on
+    """Forward (teacher, loss), KL, Hutchinson, backward (with and without the KL term), weight
+    gradient and the CTA-pair GEMMs on
     small cases, each test asserting its parity bar and device status 0, on libjab_checked.so."""
     r = _child([sys.executable, "-m", "pytest", "-x", "-q", "-m", "gpu", "-p", "no:cacheprovider",
                 os.path.join("tests", "test_gpu_parity.py"), "-k",
-                "teacher_output_parity or loss_forward_parity or backward_parity or "
+                "teacher_output_parity or loss_forward_parity or backward_parity or backward_kl or "
                 "weight_gradient_and_fisher or kl_forward or hutchinson or bit_identical"])
     assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-3000:]

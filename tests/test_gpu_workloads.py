@@ -198,6 +198,47 @@ def test_backward_full_size(name, k):
     assert J().jab_get_device_status() == 0
 
 
+def test_backward_kl_full_size():
+    """The STE backward of both terms of Eq. 3 (lambda_KL = 0.1) on the Mistral-7B-shaped block at
+    its full size (the launch bench.py times): a one-sequence sub-batch against the oracle's joint
+    gradient, and the full batch against its two halves (the batchmean KL is the mean of the
+    halves', the loss and the gradient their size-weighted sums)."""
+    wl, desc, X, W = _setup("mistral_block")
+    bits, lam = wl.bits[0], float(np.float32(0.1))
+    s = _scales(desc, wl, W, bits)
+    T = wl.seq_len
+
+    def run(Xb, nb):
+        ws = J().Workspace(desc, nb, T, 1, True)
+        A = torch.empty((nb, T, wl.shape.n_q_heads * wl.shape.head_dim), dtype=torch.float32,
+                        device="cuda")
+        lse = torch.empty((nb, wl.shape.n_q_heads, T), dtype=torch.float32, device="cuda")
+        J().jab_reference_forward(desc, nb, T, Xb, W, A, ws, lse=lse)
+        qkv_ref = torch.empty((nb, T, wl.shape.d_out), dtype=torch.float16, device="cuda")
+        J().jab_reference_projection(desc, nb, T, Xb, W, qkv_ref, ws)
+        loss, kl = (torch.empty(1, dtype=torch.float64, device="cuda") for _ in range(2))
+        g = torch.empty_like(s)
+        J().jab_loss_backward_scales_kl(desc, nb, T, Xb, W, A, qkv_ref, lse, bits, s, 1.0, lam,
+                                        loss, g, ws, kl=kl)
+        assert J().jab_get_device_status() == 0
+        return loss.item(), kl.item(), g
+
+    l_full, kl_full, g_full = run(X, wl.batch)
+    l1, kl1, g1 = run(X[:1].contiguous(), 1)
+    r = O.jab_loss_joint_and_grad(np64(X[:1]), np64(W), s.cpu().numpy(), bits,
+                                  oracle_desc(wl.shape, wl.group_size), lam_kl=lam, kappa=1.0)
+    assert abs(kl1 - r["kl"]) <= L_TOL * r["kl"], (kl1, r["kl"])
+    assert abs(l1 - r["loss"]) <= L_TOL * r["loss"], (l1, r["loss"])
+    assert cosine(g1.cpu().numpy(), r["grad_s"]) >= COS_MIN
+    h = wl.batch // 2
+    la, kla, ga = run(X[:h].contiguous(), h)
+    lb, klb, gb = run(X[h:].contiguous(), wl.batch - h)
+    np.testing.assert_allclose(kl_full, 0.5 * (kla + klb), rtol=1e-9)
+    np.testing.assert_allclose(l_full, 0.5 * (la + lb), rtol=1e-9)
+    comb = (0.5 * (ga + gb)).cpu().numpy()
+    assert cosine(g_full.cpu().numpy(), comb) >= 0.99999
+
+
 def test_weight_gradient_split_k_full_shape():
     """The STE weight gradient (App. B) on the Mistral-7B-shaped block at 8 and 4 sequences, where
     the weight-gradient GEMM splits the token range (2-3 parts, partial tiles added with atomics):
