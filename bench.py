@@ -628,7 +628,7 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
             combine_shards(loss, grad, B, B * world)
 
     n_klb = max(1, min(args.steps, 5))
-    klb_ms, _ = timed(J, kl_bwd_step, n_klb, max(1, min(args.warmup, 2)), st, barrier, sites=False)
+    klb_ms, klb_sites = timed(J, kl_bwd_step, n_klb, max(1, min(args.warmup, 2)), st, barrier)
     klb_ms = max_over_ranks(klb_ms, dev)
     if J.jab_get_device_status() != 0:
         raise RuntimeError("device status set in the KL-term backward")
@@ -752,7 +752,10 @@ def headline(J, args, wl, dev, pk, st, world, rank, barrier):
                        "ms_per_eval": klb_ms / n_klb, "lambda_kl": 0.1,
                        "achieved_tflops": klb_f / (klb_ms / n_klb / 1e3) / 1e12,
                        "note": "scale gradient of MSE + 0.1 KL (jab_loss_backward_scales_kl), "
-                               "X converted by the call"},
+                               "X converted by the call",
+                       "kernels": {k: {"ms_per_step": v[0] / n_klb,
+                                       "launches_per_step": v[2] / n_klb}
+                                   for k, v in klb_sites.items()}},
         "fisher_probe": {"value": world * n_fis / (fis_ms / 1e3), "unit": "evals/s", "bits": 2,
                          "ms_per_eval": fis_ms / n_fis,
                          "achieved_tflops": (fwd_f + bwd_f) / (fis_ms / n_fis / 1e3) / 1e12},

@@ -89,13 +89,17 @@ __global__ void sum_in_order_kernel(const double* __restrict__ part, int n, doub
   }
 }
 
-__global__ void sum_scaled_kernel(const double* __restrict__ part, int n, double scale,
-                                  double* __restrict__ out) {
-  if (threadIdx.x == 0) {
-    double t = 0.0;
-    for (int i = 0; i < n; ++i) t += part[i];
-    *out = scale * t;
-  }
+// One block: thread t adds its contiguous chunk in order, then a fixed tree (block_sum), so the
+// result is the same on every call.
+__global__ void __launch_bounds__(256) sum_scaled_kernel(const double* __restrict__ part, int n,
+                                                         double scale, double* __restrict__ out) {
+  __shared__ double red[8];
+  const int chunk = (n + blockDim.x - 1) / blockDim.x;
+  const int lo = threadIdx.x * chunk, hi = min(lo + chunk, n);
+  double t = 0.0;
+  for (int i = lo; i < hi; ++i) t += part[i];
+  const double tot = block_sum<256>(t, red);
+  if (threadIdx.x == 0) *out = scale * tot;
 }
 
 // Natural-log log-sum-exp rows [BH, T] to log2 units with the row pitch of the backward workspace.
@@ -160,7 +164,7 @@ cudaError_t launch_split_sum(const float* part, int splits, int64_t n, float* ou
 }
 
 cudaError_t launch_sum_scaled(const double* part, int n, double scale, double* out, cudaStream_t st) {
-  sum_scaled_kernel<<<1, 32, 0, st>>>(part, n, scale, out);
+  sum_scaled_kernel<<<1, 256, 0, st>>>(part, n, scale, out);
   return cudaGetLastError();
 }
 
