@@ -63,6 +63,24 @@ def test_host_side_checks_without_gpu(libjab):
                                              1.0, None, None, None, 0, None)
     assert st == 1
     assert L.jab_prepare_x(ctypes.byref(good), 2, 130, None, None, 0, None) == 1
+    # the KL-term backward: no teacher projection / log-sum-exp, a negative or NaN lambda, an
+    # unsupported block, each refused before any CUDA call
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: the checks fail first
+    st = L.jab_loss_backward_scales_kl(ctypes.byref(good), 2, 130, fake, fake, fake, None, fake, 3,
+                                       fake, 1.0, 0.1, fake, None, fake, fake, 1 << 40, None)
+    assert st == 1
+    st = L.jab_loss_backward_scales_kl(ctypes.byref(good), 2, 130, fake, fake, fake, fake, None, 3,
+                                       fake, 1.0, 0.1, fake, None, fake, fake, 1 << 40, None)
+    assert st == 1
+    for lam in (-0.1, float("nan")):
+        st = L.jab_loss_backward_scales_kl(ctypes.byref(good), 2, 130, fake, fake, fake, fake, fake,
+                                           3, fake, 1.0, lam, fake, None, fake, fake, 1 << 40, None)
+        assert st == 1
+    st = L.jab_loss_backward_scales_kl(ctypes.byref(bad_dh), 2, 130, fake, fake, fake, fake, fake,
+                                       3, fake, 1.0, 0.1, fake, None, fake, fake, 1 << 40, None)
+    assert st == 2
+    # the backward workspace holds the KL term's teacher log-sum-exp and partials too
+    assert J.jab_workspace_size(good, 2, 130, 1, True) > J.jab_workspace_size(good, 2, 130, 1, False)
     assert L.jab_flip_rate(None, None, 16, None, None) == 1
     assert L.jab_selftest_bounds_check(None, 4, None) == 1
     assert L.jab_set_deterministic(2) == 1 and L.jab_set_deterministic(0) == 0
