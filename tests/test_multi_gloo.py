@@ -1,7 +1,8 @@
 """Multi-process host logic on CPU with the gloo backend, world size 2: sequence sharding of one
 evaluation (size-weighted all-reduce equals the full batch, computed here with the oracle on each
-shard), the Fisher-coupling score of a sharded evaluation (norm of the combined weight gradient),
-and the max-over-ranks timing reduction used by bench.py."""
+shard, for the MSE term and for the joint MSE + KL objective), the Fisher-coupling score of a
+sharded evaluation (norm of the combined weight gradient), and the max-over-ranks timing reduction
+used by bench.py."""
 import os
 import socket
 
@@ -44,8 +45,17 @@ def _worker(rank, world, port, out):
         combine_shards(loss, grad, b - a, B)
         gw = torch.tensor(r["grad_w_hat"], dtype=torch.float64)
         score = fisher_score_from_shards(gw, b - a, B)
+        # the joint objective (MSE + 0.1 KL, Eq. 3): the KL batchmean shards like the MSE mean
+        rj = O.jab_loss_joint_and_grad(x[a:b], w, s, 3, desc, lam_kl=0.1, kappa=1.0)
+        jloss = torch.tensor([rj["loss"]], dtype=torch.float64)
+        jgrad = torch.tensor(rj["grad_s"], dtype=torch.float64)
+        combine_shards(jloss, jgrad, b - a, B)
         t = max_over_ranks(10.0 + rank)
         if rank == 0:
+            jfull = O.jab_loss_joint_and_grad(x, w, s, 3, desc, lam_kl=0.1, kappa=1.0)
+            out["jloss"] = (jloss.item(), jfull["loss"])
+            out["jgrad"] = float(np.abs(jgrad.numpy() - jfull["grad_s"]).max() /
+                                 np.abs(jfull["grad_s"]).max())
             full = O.jab_loss_and_grad(x, w, s, 3, desc, kappa=1.0)
             out["loss"] = (loss.item(), full["loss"])
             out["grad"] = float(np.abs(grad.numpy() - full["grad_s"]).max() /
@@ -78,3 +88,6 @@ def test_sharded_evaluation_matches_full_batch_gloo_world2():
         assert out["tmax"] == 11.0
         score_sharded, score_full = out["score"]
         np.testing.assert_allclose(score_sharded, score_full, rtol=1e-12)
+        jl_sharded, jl_full = out["jloss"]
+        np.testing.assert_allclose(jl_sharded, jl_full, rtol=1e-12)
+        assert out["jgrad"] < 1e-12
